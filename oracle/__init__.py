@@ -1,0 +1,189 @@
+"""fp64 CPU oracle for the FPO pseudogradient update (test infrastructure only).
+
+Only ``tests/``, ``__graft_entry__.smoke()`` and ``bench.py``'s CPU-baseline
+and reference legs import this package.  It wraps ``oracle.c`` (plain C, fp64,
+OpenMP over independent tokens) through ctypes and numpy; it shares no code
+with the CUDA library and never imports it.
+
+Each function follows one passage of the paper:
+
+* :func:`error_signal`  Sec. 3.1 steps 2-4, Eq. (gproj), App. E Eq. (rmsnorm-vjp)
+  with the min-RMS clamp.
+* :func:`pseudograd`    Sec. 3.1 step 5, Eq. (w3update).
+* :func:`sgd_update`    App. A, fp32 master weights cast to bf16.
+* :func:`cosine`        Sec. 2.2, Eq. (cosine).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "oracle.c")
+_LIB_PATH = os.path.join(_HERE, "liboracle.so")
+
+F32, BF16, F64 = 0, 1, 2
+
+_lib = None
+
+
+def build(force: bool = False) -> str:
+    """Compile oracle.c into liboracle.so with gcc (-O2, OpenMP)."""
+    if (not force and os.path.exists(_LIB_PATH)
+            and os.path.getmtime(_LIB_PATH) >= os.path.getmtime(_SRC)):
+        return _LIB_PATH
+    tmp = _LIB_PATH + f".tmp{os.getpid()}"
+    cmd = ["gcc", "-O2", "-std=c11", "-fopenmp", "-fPIC", "-shared", _SRC,
+           "-o", tmp, "-lm"]
+    subprocess.run(cmd, check=True)
+    os.replace(tmp, _LIB_PATH)
+    return _LIB_PATH
+
+
+def _load():
+    global _lib
+    if _lib is not None:
+        return _lib
+    build()
+    lib = ctypes.CDLL(_LIB_PATH)
+    vp, i64, dbl, i32 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_double, ctypes.c_int
+    lib.oracle_error_signal.argtypes = [i64, i64, i64, i32, vp, vp, vp, vp, dbl, dbl, dbl,
+                                        vp, i64, vp, vp, vp, vp, vp, vp]
+    lib.oracle_error_signal.restype = i32
+    lib.oracle_pseudograd.argtypes = [i64, i64, i64, i32, vp, i32, vp, vp, vp, i64, vp]
+    lib.oracle_pseudograd.restype = i32
+    lib.oracle_sgd_update.argtypes = [i64, vp, vp, dbl, vp, vp]
+    lib.oracle_sgd_update.restype = None
+    lib.oracle_f32_to_bf16.argtypes = [i64, vp, vp]
+    lib.oracle_f32_to_bf16.restype = None
+    lib.oracle_cosine.argtypes = [i64, i32, vp, vp, vp]
+    lib.oracle_cosine.restype = None
+    lib.oracle_mean_ce.argtypes = [i64, vp, vp]
+    lib.oracle_mean_ce.restype = dbl
+    _lib = lib
+    return lib
+
+
+def _typed(a: np.ndarray):
+    """Return (dtype code, contiguous array) for fp32 / fp64 / bf16-as-uint16."""
+    a = np.ascontiguousarray(a)
+    if a.dtype == np.float64:
+        return F64, a
+    if a.dtype == np.float32:
+        return F32, a
+    if a.dtype == np.uint16:  # raw bf16 bit patterns
+        return BF16, a
+    raise TypeError(f"oracle inputs must be float64, float32 or uint16 (bf16 bits), got {a.dtype}")
+
+
+def _ptr(a):
+    return None if a is None else a.ctypes.data_as(ctypes.c_void_p)
+
+
+def error_signal(h, w, W_U, y, *, eps=1e-6, min_rms=0.5, s=1.0, rows=None, want_e=False):
+    """Steps 1-5 of the FPO error signal for every token (or the listed rows).
+
+    ``h`` [T,d], ``w`` [d], ``W_U`` [V,d] share one dtype (float32/float64, or
+    uint16 holding bf16 bits); ``y`` int32 [T].  Returns a dict of fp64 arrays:
+    rho, lse, zy (target logit), g (= e W_U, Eq. gproj), g_tilde (after the
+    final-norm VJP) and optionally e.
+    """
+    dt, h = _typed(h)
+    dtw, w = _typed(w)
+    dtu, W_U = _typed(W_U)
+    if not (dt == dtw == dtu):
+        raise TypeError("h, w and W_U must share one dtype")
+    T, d = h.shape
+    V = W_U.shape[0]
+    y = np.ascontiguousarray(y, dtype=np.int32)
+    if rows is None:
+        n = T
+        rows_arr = None
+    else:
+        rows_arr = np.ascontiguousarray(rows, dtype=np.int64)
+        n = rows_arr.shape[0]
+    out = {k: np.zeros(n) for k in ("rho", "lse", "zy")}
+    out["g"] = np.zeros((n, d))
+    out["g_tilde"] = np.zeros((n, d))
+    e = np.zeros((n, V)) if want_e else None
+    rc = _load().oracle_error_signal(T, d, V, dt, _ptr(h), _ptr(w), _ptr(W_U), _ptr(y),
+                                     eps, min_rms, s, _ptr(rows_arr), n,
+                                     _ptr(out["rho"]), _ptr(out["lse"]), _ptr(out["zy"]),
+                                     _ptr(out["g"]), _ptr(out["g_tilde"]), _ptr(e))
+    if rc == -2:
+        raise ValueError("target or row index out of range")
+    if rc != 0:
+        raise ValueError(f"oracle_error_signal failed ({rc})")
+    if want_e:
+        out["e"] = e
+    return out
+
+
+def pseudograd(g_tilde, A, pairs=None):
+    """Eq. (w3update): G = g~^T A, [d, d_ff] fp64 (or the listed (i, j) entries)."""
+    dtg, g_tilde = _typed(g_tilde)
+    dta, A = _typed(A)
+    T, d = g_tilde.shape
+    d_ff = A.shape[1]
+    if A.shape[0] != T:
+        raise ValueError("g_tilde and A must have the same number of tokens")
+    if pairs is None:
+        G = np.zeros((d, d_ff))
+        rc = _load().oracle_pseudograd(T, d, d_ff, dtg, _ptr(g_tilde), dta, _ptr(A),
+                                       None, None, 0, _ptr(G))
+    else:
+        ii = np.ascontiguousarray(pairs[0], dtype=np.int64)
+        jj = np.ascontiguousarray(pairs[1], dtype=np.int64)
+        G = np.zeros(ii.shape[0])
+        rc = _load().oracle_pseudograd(T, d, d_ff, dtg, _ptr(g_tilde), dta, _ptr(A),
+                                       _ptr(ii), _ptr(jj), ii.shape[0], _ptr(G))
+    if rc != 0:
+        raise ValueError(f"oracle_pseudograd failed ({rc})")
+    return G
+
+
+def sgd_update(W_master, G, lr):
+    """App. A: returns (W_new fp32, W_bf16 bits uint16) for W_master -= lr * G."""
+    W = np.ascontiguousarray(W_master, dtype=np.float32)
+    G = np.ascontiguousarray(G, dtype=np.float64)
+    if W.shape != G.shape:
+        raise ValueError("W_master and G must have the same shape")
+    W_new = np.empty_like(W)
+    W_b = np.empty(W.shape, dtype=np.uint16)
+    _load().oracle_sgd_update(W.size, _ptr(W), _ptr(G), float(lr), _ptr(W_new), _ptr(W_b))
+    return W_new, W_b
+
+
+def f32_to_bf16_bits(x):
+    """Round-to-nearest-even fp32 -> bf16, returned as uint16 bit patterns."""
+    x = np.ascontiguousarray(x, dtype=np.float32)
+    out = np.empty(x.shape, dtype=np.uint16)
+    _load().oracle_f32_to_bf16(x.size, _ptr(x), _ptr(out))
+    return out
+
+
+def bf16_bits_to_f64(b):
+    """Exact value of bf16 bit patterns as fp64 (plain bit placement)."""
+    b = np.ascontiguousarray(b, dtype=np.uint16)
+    return (b.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+
+
+def cosine(X, Y):
+    """Eq. (cosine): returns (<X,Y>, |X|^2, |Y|^2, cos) in fp64."""
+    dtx, X = _typed(X)
+    dty, Y = _typed(Y)
+    if dtx != dty or X.size != Y.size:
+        raise TypeError("X and Y must have the same dtype and size")
+    out = np.zeros(4)
+    _load().oracle_cosine(X.size, dtx, _ptr(X.reshape(-1)), _ptr(Y.reshape(-1)), _ptr(out))
+    return tuple(out)
+
+
+def mean_ce(lse, zy):
+    """(1/T) sum_t (lse_t - z_{t,y_t}): the mean cross-entropy."""
+    lse = np.ascontiguousarray(lse, dtype=np.float64)
+    zy = np.ascontiguousarray(zy, dtype=np.float64)
+    return _load().oracle_mean_ce(lse.size, _ptr(lse), _ptr(zy))

@@ -1,0 +1,242 @@
+/*
+ * oracle.c -- plain, slow, fp64 CPU oracle for the FPO pseudogradient update.
+ *
+ * TEST INFRASTRUCTURE ONLY.  Only tests/, __graft_entry__.smoke() and the
+ * cpu_baseline / reference legs of bench.py may load this library.  The
+ * product path (libfpo.so and its Python binding) never calls it, and this
+ * file shares no code, header, table or helper with the CUDA sources.
+ *
+ * Every function is the plain definition of one step of the method of
+ * "Forward Pass Domain Adaptation (Without Cross-Layer Backpropagation)"
+ * written out in fp64, with no blocking, fusion or reordering:
+ *
+ *   oracle_error_signal  Sec. 3.1 steps 2-4, Eq. (gproj), App. E Eq. (rmsnorm-vjp)
+ *                        and the min-RMS clamp (Sec. 3.2 / App. E)
+ *   oracle_pseudograd    Sec. 3.1 step 5, Eq. (w3update): G = g~^T h_mid
+ *   oracle_sgd_update    App. A (fp32 master weights, cast to bf16)
+ *   oracle_cosine        Sec. 2.2, Eq. (cosine)
+ *
+ * Inputs are the exact stored values (fp32, bf16 or fp64) upcast to fp64 as
+ * they are read.  OpenMP parallelises only over independent tokens / output
+ * rows; every sum runs in index order inside one thread.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+enum { ORC_F32 = 0, ORC_BF16 = 1, ORC_F64 = 2 };
+
+/* Upcast element i of a typed array to fp64.  bf16 is the upper half of an
+ * IEEE binary32, so its value is that binary32 with a zero lower half. */
+static inline double orc_load(int dt, const void* p, int64_t i) {
+    if (dt == ORC_F64) return ((const double*)p)[i];
+    if (dt == ORC_F32) return (double)((const float*)p)[i];
+    uint32_t bits = (uint32_t)((const uint16_t*)p)[i] << 16;
+    float f;
+    memcpy(&f, &bits, sizeof f);
+    return (double)f;
+}
+
+int oracle_abi_version(void) { return 1; }
+
+/*
+ * Steps 1-5 of the error signal, one token at a time (tokens are independent
+ * until the contraction over T in Eq. (w3update)).
+ *
+ * For token t (rows[r] when rows != NULL, else r):
+ *   rho   = sqrt(mean_j h_tj^2 + eps)                       App. E, below Eq. (rmsnorm-vjp)
+ *   xhat  = h_t / rho ;  yhat = w (.) xhat                  final RMSNorm forward
+ *   z_v   = <yhat, W_U[v,:]>                                logits (Sec. 3.1 step 2)
+ *   lse   = m + log sum_v exp(z_v - m),  m = max_v z_v
+ *   e_v   = s * (exp(z_v - lse) - [v == y_t])              softmax(z) - 1_y, loss scale s
+ *   g_j   = sum_v e_v W_U[v,j]                              Eq. (gproj)
+ *   c     = <xhat, w (.) g>
+ *   g~_j  = (w_j g_j - xhat_j c / d) / max(rho, rho_min)    Eq. (rmsnorm-vjp) + min-RMS clamp
+ *
+ * The clamp replaces rho only in the 1/rho prefactor; xhat keeps the true rho
+ * (the reading under which the clamp "caps the 1/rho amplification" and the
+ * projection term stays exact).
+ *
+ * Outputs (each optional, NULL to skip) are indexed by r, the position in the
+ * row list: rho[r], lse[r], zy[r] = z_{t,y_t}, g[r*d + j], g_tilde[r*d + j],
+ * e[r*V + v].  Returns 0, or -1 for a bad argument, or -2 when a target is
+ * outside [0, V) (that token's outputs are left untouched).
+ */
+int oracle_error_signal(int64_t T, int64_t d, int64_t V, int dt,
+                        const void* h, const void* w, const void* W_U,
+                        const int32_t* y, double eps, double min_rms, double s,
+                        const int64_t* rows, int64_t n_rows,
+                        double* rho, double* lse, double* zy, double* g,
+                        double* g_tilde, double* e) {
+    if (T < 0 || d <= 0 || V <= 0 || !h || !w || !W_U || !y) return -1;
+    if (!rows) n_rows = T;
+    int bad_target = 0;
+#pragma omp parallel for schedule(dynamic, 1) reduction(| : bad_target)
+    for (int64_t r = 0; r < n_rows; ++r) {
+        int64_t t = rows ? rows[r] : r;
+        if (t < 0 || t >= T) { bad_target = 1; continue; }
+        int32_t yt = y[t];
+        if (yt < 0 || yt >= V) { bad_target = 1; continue; }
+
+        double* xhat = (double*)malloc(sizeof(double) * (size_t)d);
+        double* yhat = (double*)malloc(sizeof(double) * (size_t)d);
+        double* z = (double*)malloc(sizeof(double) * (size_t)V);
+        double* gt = (double*)malloc(sizeof(double) * (size_t)d);
+
+        double ss = 0.0;
+        for (int64_t j = 0; j < d; ++j) {
+            double x = orc_load(dt, h, t * d + j);
+            ss += x * x;
+        }
+        double rh = sqrt(ss / (double)d + eps);
+        for (int64_t j = 0; j < d; ++j) {
+            xhat[j] = orc_load(dt, h, t * d + j) / rh;
+            yhat[j] = orc_load(dt, w, j) * xhat[j];
+        }
+
+        double m = -INFINITY;
+        for (int64_t v = 0; v < V; ++v) {
+            double acc = 0.0;
+            for (int64_t j = 0; j < d; ++j) acc += yhat[j] * orc_load(dt, W_U, v * d + j);
+            z[v] = acc;
+            if (acc > m) m = acc;
+        }
+        double se = 0.0;
+        for (int64_t v = 0; v < V; ++v) se += exp(z[v] - m);
+        double l = m + log(se);
+
+        /* e overwrites z in place: e_v = s (p_v - [v == y]). */
+        for (int64_t v = 0; v < V; ++v) {
+            double p = exp(z[v] - l);
+            if (v == yt) {
+                if (zy) zy[r] = z[v];
+                p -= 1.0;
+            }
+            z[v] = s * p;
+        }
+        if (e) memcpy(e + r * V, z, sizeof(double) * (size_t)V);
+
+        for (int64_t j = 0; j < d; ++j) gt[j] = 0.0;
+        for (int64_t v = 0; v < V; ++v) {
+            double ev = z[v];
+            for (int64_t j = 0; j < d; ++j) gt[j] += ev * orc_load(dt, W_U, v * d + j);
+        }
+        if (g) memcpy(g + r * d, gt, sizeof(double) * (size_t)d);
+
+        if (g_tilde) {
+            double c = 0.0;
+            for (int64_t j = 0; j < d; ++j) c += xhat[j] * orc_load(dt, w, j) * gt[j];
+            double denom = rh > min_rms ? rh : min_rms;
+            for (int64_t j = 0; j < d; ++j)
+                g_tilde[r * d + j] =
+                    (orc_load(dt, w, j) * gt[j] - xhat[j] * c / (double)d) / denom;
+        }
+        if (rho) rho[r] = rh;
+        if (lse) lse[r] = l;
+
+        free(xhat);
+        free(yhat);
+        free(z);
+        free(gt);
+    }
+    return bad_target ? -2 : 0;
+}
+
+/*
+ * Eq. (w3update): G[i,j] = sum_t g~[t,i] * A[t,j]  (g~ is [T,d], A is [T,d_ff],
+ * G is [d,d_ff], the nn.Linear layout of the down-projection weight).
+ * With ii == NULL every entry is written to G[i*d_ff + j]; otherwise only the
+ * n_pairs entries (ii[k], jj[k]) are computed, into G[k].
+ */
+int oracle_pseudograd(int64_t T, int64_t d, int64_t d_ff, int dt_g, const void* gt,
+                      int dt_a, const void* A, const int64_t* ii, const int64_t* jj,
+                      int64_t n_pairs, double* G) {
+    if (T < 0 || d <= 0 || d_ff <= 0 || !G || (T > 0 && (!gt || !A))) return -1;
+    if (!ii) {
+#pragma omp parallel for schedule(static)
+        for (int64_t i = 0; i < d; ++i) {
+            double* row = G + i * d_ff;
+            for (int64_t j = 0; j < d_ff; ++j) row[j] = 0.0;
+            for (int64_t t = 0; t < T; ++t) {
+                double gi = orc_load(dt_g, gt, t * d + i);
+                for (int64_t j = 0; j < d_ff; ++j) row[j] += gi * orc_load(dt_a, A, t * d_ff + j);
+            }
+        }
+        return 0;
+    }
+    int bad = 0;
+#pragma omp parallel for schedule(static) reduction(| : bad)
+    for (int64_t k = 0; k < n_pairs; ++k) {
+        int64_t i = ii[k], j = jj[k];
+        if (i < 0 || i >= d || j < 0 || j >= d_ff) { bad = 1; continue; }
+        double acc = 0.0;
+        for (int64_t t = 0; t < T; ++t)
+            acc += orc_load(dt_g, gt, t * d + i) * orc_load(dt_a, A, t * d_ff + j);
+        G[k] = acc;
+    }
+    return bad ? -1 : 0;
+}
+
+/* IEEE binary64 -> binary32, round to nearest even (the C cast does this under
+ * the default rounding mode). */
+static inline float orc_to_f32(double x) { return (float)x; }
+
+/* binary32 -> bfloat16, round to nearest even, from the definition: keep the
+ * upper 16 bits; round up when the discarded half is above one half ulp, or
+ * exactly one half ulp and the kept part is odd.  NaN stays a quiet NaN. */
+static inline uint16_t orc_f32_to_bf16(float f) {
+    uint32_t u;
+    memcpy(&u, &f, sizeof u);
+    if ((u & 0x7f800000u) == 0x7f800000u && (u & 0x007fffffu)) return (uint16_t)((u >> 16) | 0x40u);
+    uint32_t upper = u >> 16, lower = u & 0xffffu;
+    if (lower > 0x8000u || (lower == 0x8000u && (upper & 1u))) upper += 1u;
+    return (uint16_t)upper;
+}
+
+/*
+ * App. A: the fp32 master copy receives the step and the bf16 working weight
+ * is its cast.  W_new = RN32(W - lr * G) evaluated in fp64, W_bf16 = RNE16(W_new).
+ * Either output may be NULL.
+ */
+void oracle_sgd_update(int64_t n, const float* W, const double* G, double lr,
+                       float* W_new, uint16_t* W_bf16) {
+#pragma omp parallel for schedule(static)
+    for (int64_t k = 0; k < n; ++k) {
+        float wn = orc_to_f32((double)W[k] - lr * G[k]);
+        if (W_new) W_new[k] = wn;
+        if (W_bf16) W_bf16[k] = orc_f32_to_bf16(wn);
+    }
+}
+
+/* Plain RNE conversion of an fp32 array to bf16 bits (test helper for the
+ * update's bf16 output). */
+void oracle_f32_to_bf16(int64_t n, const float* x, uint16_t* out) {
+    for (int64_t k = 0; k < n; ++k) out[k] = orc_f32_to_bf16(x[k]);
+}
+
+/*
+ * Eq. (cosine): out = { <X,Y>, ||X||^2, ||Y||^2, <X,Y> / (||X|| ||Y||) }.
+ * Sequential fp64 sums in index order.
+ */
+void oracle_cosine(int64_t n, int dt, const void* X, const void* Y, double* out) {
+    double xy = 0.0, xx = 0.0, yy = 0.0;
+    for (int64_t k = 0; k < n; ++k) {
+        double a = orc_load(dt, X, k), b = orc_load(dt, Y, k);
+        xy += a * b;
+        xx += a * a;
+        yy += b * b;
+    }
+    out[0] = xy;
+    out[1] = xx;
+    out[2] = yy;
+    out[3] = (xx > 0.0 && yy > 0.0) ? xy / (sqrt(xx) * sqrt(yy)) : 0.0;
+}
+
+/* Mean cross-entropy over tokens, (1/T) sum_t (lse_t - z_{t,y_t}), from the
+ * per-token values returned by oracle_error_signal. */
+double oracle_mean_ce(int64_t n, const double* lse, const double* zy) {
+    double acc = 0.0;
+    for (int64_t k = 0; k < n; ++k) acc += lse[k] - zy[k];
+    return n > 0 ? acc / (double)n : 0.0;
+}

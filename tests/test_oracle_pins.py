@@ -1,0 +1,308 @@
+"""Pins for the fp64 oracle: checks against things other than the oracle itself.
+
+Each test fixes one step of the oracle by a fact the paper or the mathematics
+determines -- finite differences of the forward loss, an exact invariant, a
+special case that reduces to a textbook routine, or a hand-derived closed
+form -- chosen so that a dropped term, a wrong sign or index, or a transposed
+operand in the oracle fails at least one of them.
+"""
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+
+import oracle
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+# ---------------------------------------------------------------------------
+# Independent forward model: the loss the error signal is the gradient of.
+# L(h) = s * sum_t CE(RMSNorm(h_t) W_U^T, y_t)   (Sec. 3.1, App. E)
+# ---------------------------------------------------------------------------
+def forward_loss(h, w, W_U, y, eps, s):
+    rho = np.sqrt(np.mean(h * h, axis=1, keepdims=True) + eps)
+    z = (h / rho * w) @ W_U.T
+    m = z.max(axis=1, keepdims=True)
+    lse = (m + np.log(np.exp(z - m).sum(axis=1, keepdims=True)))[:, 0]
+    return s * float(np.sum(lse - z[np.arange(len(y)), y]))
+
+
+def fd_grad(f, x, step=1e-6):
+    gr = np.zeros_like(x)
+    it = np.nditer(x, flags=["multi_index"])
+    for _ in it:
+        i = it.multi_index
+        old = x[i]
+        x[i] = old + step
+        fp = f(x)
+        x[i] = old - step
+        fm = f(x)
+        x[i] = old
+        gr[i] = (fp - fm) / (2 * step)
+    return gr
+
+
+def rel_err(a, b):
+    return float(np.linalg.norm(a - b) / max(np.linalg.norm(b), 1e-300))
+
+
+def _toy(T=4, d=8, V=16, seed=0, scale_h=1.0):
+    rng = np.random.default_rng(seed)
+    h = rng.standard_normal((T, d)) * scale_h
+    w = 1.0 + 0.1 * rng.standard_normal(d)
+    W_U = 0.5 * rng.standard_normal((V, d))
+    y = rng.integers(0, V, T).astype(np.int32)
+    return h, w, W_U, y
+
+
+def test_error_signal_matches_finite_differences():
+    """g~ = dL/dh exactly when the clamp is inactive (Eq. gproj + Eq. rmsnorm-vjp)."""
+    h, w, W_U, y = _toy()
+    s = 1.0 / len(y)
+    out = oracle.error_signal(h, w, W_U, y, eps=1e-6, min_rms=0.5, s=s)
+    assert np.all(out["rho"] > 0.5)
+    fd = fd_grad(lambda x: forward_loss(x, w, W_U, y, 1e-6, s), h.copy())
+    assert rel_err(out["g_tilde"], fd) < 1e-7
+
+
+def test_error_signal_loss_scale_is_linear():
+    h, w, W_U, y = _toy(seed=3)
+    a = oracle.error_signal(h, w, W_U, y, s=1.0)["g_tilde"]
+    b = oracle.error_signal(h, w, W_U, y, s=0.25)["g_tilde"]
+    assert rel_err(0.25 * a, b) < 1e-14
+
+
+def test_pre_vjp_signal_is_gradient_wrt_unembedding_input():
+    """Eq. (gproj): g = e W_U is the exact gradient w.r.t. the unembedding input yhat."""
+    h, w, W_U, y = _toy(seed=1)
+    out = oracle.error_signal(h, w, W_U, y, s=1.0)
+    rho = np.sqrt(np.mean(h * h, axis=1, keepdims=True) + 1e-6)
+    yhat = h / rho * w
+
+    def loss_of_yhat(yh):
+        z = yh @ W_U.T
+        m = z.max(axis=1, keepdims=True)
+        lse = (m + np.log(np.exp(z - m).sum(axis=1, keepdims=True)))[:, 0]
+        return float(np.sum(lse - z[np.arange(len(y)), y]))
+
+    fd = fd_grad(loss_of_yhat, yhat.copy())
+    assert rel_err(out["g"], fd) < 1e-7
+
+
+def test_min_rms_clamp_scales_only_the_prefactor():
+    """A token with rho < rho_min: g~ = (rho / rho_min) * dL/dh (clamp on 1/rho only)."""
+    h, w, W_U, y = _toy(T=3, seed=2)
+    h[1] *= 0.2  # rho ~ 0.2 < 0.5
+    out = oracle.error_signal(h, w, W_U, y, eps=1e-6, min_rms=0.5, s=1.0)
+    assert out["rho"][1] < 0.5 and out["rho"][0] > 0.5 and out["rho"][2] > 0.5
+    fd = fd_grad(lambda x: forward_loss(x, w, W_U, y, 1e-6, 1.0), h.copy())
+    expect = fd.copy()
+    expect[1] *= out["rho"][1] / 0.5
+    assert rel_err(out["g_tilde"], expect) < 1e-7
+    # and with the clamp floor at 0 the plain gradient comes back
+    out0 = oracle.error_signal(h, w, W_U, y, eps=1e-6, min_rms=0.0, s=1.0)
+    assert rel_err(out0["g_tilde"], fd) < 1e-7
+
+
+def test_rows_of_error_sum_to_zero():
+    """softmax(z) - 1_y sums to zero over the vocabulary for every token."""
+    h, w, W_U, y = _toy(T=6, V=40, seed=4)
+    out = oracle.error_signal(h, w, W_U, y, s=1.0, want_e=True)
+    assert np.max(np.abs(out["e"].sum(axis=1))) < 1e-12
+    assert np.all(out["e"][np.arange(6), y] < 0)
+
+
+def test_eps0_vjp_orthogonal_to_h():
+    """At eps = 0 the RMSNorm VJP is orthogonal to h, clamped tokens included."""
+    h, w, W_U, y = _toy(T=5, seed=5)
+    h[2] *= 0.1
+    out = oracle.error_signal(h, w, W_U, y, eps=0.0, min_rms=0.5, s=1.0)
+    for t in range(5):
+        gt = out["g_tilde"][t]
+        assert abs(gt @ h[t]) <= 1e-12 * np.linalg.norm(gt) * np.linalg.norm(h[t])
+
+
+def test_vocab_of_one_gives_zero_signal():
+    h, w, W_U, y = _toy(V=1, seed=6)
+    y[:] = 0
+    out = oracle.error_signal(h, w, W_U, y, s=1.0, want_e=True)
+    assert np.all(out["e"] == 0.0)
+    assert np.all(out["g_tilde"] == 0.0)
+    A = np.random.default_rng(0).standard_normal((len(y), 5))
+    assert np.all(oracle.pseudograd(out["g_tilde"], A) == 0.0)
+
+
+def test_equal_unembedding_rows_give_zero_signal():
+    h, w, W_U, y = _toy(V=12, seed=7)
+    W_U[:] = W_U[0]
+    out = oracle.error_signal(h, w, W_U, y, s=1.0)
+    assert np.max(np.abs(out["g"])) < 1e-14
+    assert np.max(np.abs(out["g_tilde"])) < 1e-13
+
+
+def test_logsumexp_and_mean_ce_against_library():
+    scipy_special = pytest.importorskip("scipy.special")
+    h, w, W_U, y = _toy(T=7, V=33, seed=8)
+    out = oracle.error_signal(h, w, W_U, y, eps=1e-6, s=1.0)
+    rho = np.sqrt(np.mean(h * h, axis=1) + 1e-6)
+    z = (h / rho[:, None] * w) @ W_U.T
+    assert np.allclose(out["lse"], scipy_special.logsumexp(z, axis=1), rtol=0, atol=1e-13)
+    assert np.allclose(out["zy"], z[np.arange(7), y], rtol=0, atol=1e-13)
+    assert np.allclose(out["rho"], rho, rtol=1e-15, atol=0)
+    ce = oracle.mean_ce(out["lse"], out["zy"])
+    assert abs(ce - forward_loss(h, w, W_U, y, 1e-6, 1.0 / 7)) < 1e-13
+
+
+def test_row_subset_equals_full():
+    h, w, W_U, y = _toy(T=9, seed=9)
+    full = oracle.error_signal(h, w, W_U, y, s=0.5)
+    rows = [7, 0, 3]
+    sub = oracle.error_signal(h, w, W_U, y, s=0.5, rows=rows)
+    for k in ("rho", "lse", "zy"):
+        assert np.array_equal(sub[k], full[k][rows])
+    assert np.array_equal(sub["g_tilde"], full["g_tilde"][rows])
+
+
+def test_pseudograd_against_matmul_and_pairs():
+    rng = np.random.default_rng(10)
+    g = rng.standard_normal((13, 6))
+    A = rng.standard_normal((13, 9))
+    G = oracle.pseudograd(g, A)
+    assert G.shape == (6, 9)
+    assert np.allclose(G, g.T @ A, rtol=1e-13, atol=1e-13)
+    ii = np.array([0, 5, 2, 5])
+    jj = np.array([8, 0, 4, 8])
+    Gs = oracle.pseudograd(g, A, pairs=(ii, jj))
+    assert np.array_equal(Gs, G[ii, jj])
+
+
+def test_identity_above_layer_invariant():
+    """With nothing above layer l (h = h0 + A W^T, the MLP output added to the
+    residual and fed straight to the final norm), the pseudogradient is the
+    exact down-projection gradient: dL/dW = g~(h)^T A (Sec. 2.1, Eq. decomp with R = 0)."""
+    rng = np.random.default_rng(11)
+    T, d, d_ff, V = 5, 6, 7, 10
+    h0 = rng.standard_normal((T, d))
+    A = rng.standard_normal((T, d_ff))
+    W = 0.1 * rng.standard_normal((d, d_ff))
+    w = 1.0 + 0.1 * rng.standard_normal(d)
+    W_U = 0.5 * rng.standard_normal((V, d))
+    y = rng.integers(0, V, T).astype(np.int32)
+    s = 1.0 / T
+    h = h0 + A @ W.T
+    out = oracle.error_signal(h, w, W_U, y, eps=1e-6, min_rms=0.5, s=s)
+    assert np.all(out["rho"] > 0.5)
+    G = oracle.pseudograd(out["g_tilde"], A)
+    fd = fd_grad(lambda Wx: forward_loss(h0 + A @ Wx.T, w, W_U, y, 1e-6, s), W.copy())
+    assert rel_err(G, fd) < 1e-7
+
+
+def _ev(expr):
+    return float(eval(expr, {"__builtins__": {}}, {"exp": math.exp, "log": math.log, "sqrt": math.sqrt}))
+
+
+def test_hand_derived_closed_form():
+    fx = json.load(open(os.path.join(GOLDEN, "closed_form_t1_d2_v2.json")))
+    inp = fx["inputs"]
+    w = np.array(inp["w"])
+    W_U = np.array(inp["W_U"])
+    y = np.array(inp["y"], dtype=np.int32)
+    for name, case in fx["cases"].items():
+        h = np.array(case["h"])
+        out = oracle.error_signal(h, w, W_U, y, eps=inp["eps"], min_rms=inp["min_rms"], s=inp["s"])
+        assert abs(out["rho"][0] - _ev(case["rho"])) < 1e-15, name
+        assert abs(out["lse"][0] - _ev(case["lse"])) < 1e-15, name
+        assert np.allclose(out["g"][0], [_ev(e) for e in case["g"]], rtol=0, atol=1e-15), name
+        assert np.allclose(out["g_tilde"][0], [_ev(e) for e in case["g_tilde"]], rtol=0,
+                           atol=1e-15), name
+        if "G" in case:
+            G = oracle.pseudograd(out["g_tilde"], np.array(inp["A"]))
+            assert np.allclose(G, [[_ev(e) for e in r] for r in case["G"]], rtol=0, atol=1e-15)
+            W_new, _ = oracle.sgd_update(np.array(inp["W"], dtype=np.float32), G, inp["lr"])
+            expect = np.array([[_ev(e) for e in r] for r in case["W_new"]]).astype(np.float32)
+            assert np.array_equal(W_new, expect)
+        if "ce" in case:
+            assert abs(oracle.mean_ce(out["lse"], out["zy"]) - _ev(case["ce"])) < 1e-15
+
+
+def test_symbolic_gradient_exact():
+    """Exact symbolic differentiation of the forward loss (sympy) on a 2x3x3 case."""
+    sp = pytest.importorskip("sympy")
+    rng = np.random.default_rng(12)
+    T, d, V = 2, 3, 3
+    hv = np.round(rng.standard_normal((T, d)), 3)
+    wv = np.round(1 + 0.1 * rng.standard_normal(d), 3)
+    Wv = np.round(rng.standard_normal((V, d)), 3)
+    yv = np.array([2, 0], dtype=np.int32)
+    eps = sp.Rational(1, 1000)
+    H = sp.Matrix(T, d, lambda i, j: sp.Symbol(f"h{i}{j}"))
+    L = 0
+    for t in range(T):
+        rho = sp.sqrt(sum(H[t, j] ** 2 for j in range(d)) / d + eps)
+        z = [sum(sp.nsimplify(wv[j]) * H[t, j] / rho * sp.nsimplify(Wv[v, j]) for j in range(d))
+             for v in range(V)]
+        L += sp.log(sum(sp.exp(zv) for zv in z)) - z[int(yv[t])]
+    subs = {H[i, j]: sp.nsimplify(hv[i, j]) for i in range(T) for j in range(d)}
+    grad = np.array([[float(sp.diff(L, H[i, j]).evalf(30, subs=subs)) for j in range(d)]
+                     for i in range(T)])
+    out = oracle.error_signal(hv, wv, Wv, yv, eps=1e-3, min_rms=0.0, s=1.0)
+    assert rel_err(out["g_tilde"], grad) < 1e-13
+
+
+def test_bf16_input_upcast_is_exact():
+    torch = pytest.importorskip("torch")
+    x = torch.randn(257, dtype=torch.float32).to(torch.bfloat16)
+    bits = x.view(torch.int16).numpy().view(np.uint16)
+    assert np.array_equal(oracle.bf16_bits_to_f64(bits), x.to(torch.float64).numpy())
+    # the oracle reads bf16 the same way: a bf16 run equals an fp64 run on the upcast values
+    rng = np.random.default_rng(13)
+    h = torch.tensor(rng.standard_normal((3, 16)), dtype=torch.bfloat16)
+    w = torch.tensor(1 + 0.1 * rng.standard_normal(16), dtype=torch.bfloat16)
+    W_U = torch.tensor(0.3 * rng.standard_normal((20, 16)), dtype=torch.bfloat16)
+    y = np.array([1, 19, 4], dtype=np.int32)
+    as_bits = lambda t: t.view(torch.int16).numpy().view(np.uint16)
+    a = oracle.error_signal(as_bits(h), as_bits(w), as_bits(W_U), y, s=1.0)
+    b = oracle.error_signal(h.double().numpy(), w.double().numpy(), W_U.double().numpy(), y, s=1.0)
+    assert np.array_equal(a["g_tilde"], b["g_tilde"])
+
+
+def test_sgd_update_exact_cases_and_bf16_rounding():
+    torch = pytest.importorskip("torch")
+    rng = np.random.default_rng(14)
+    W = (0.02 * rng.standard_normal(4096)).astype(np.float32)
+    G = rng.standard_normal(4096)
+    W0, b0 = oracle.sgd_update(W, G, 0.0)
+    assert np.array_equal(W0, W)  # lr = 0 leaves the master bit-identical
+    W1, b1 = oracle.sgd_update(W, G, 1e-3)
+    assert np.array_equal(W1, (W.astype(np.float64) - 1e-3 * G).astype(np.float32))
+    # round-to-nearest-even to bf16 agrees with torch's conversion bit for bit
+    ref = torch.from_numpy(W1).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    assert np.array_equal(b1, ref)
+    # ties go to even: 1 + 2^-8 -> 1.0 ; 1 + 3*2^-8 -> 1 + 2^-6
+    ties = np.array([1 + 2 ** -8, 1 + 3 * 2 ** -8, -(1 + 2 ** -8)], dtype=np.float32)
+    assert oracle.f32_to_bf16_bits(ties).tolist() == [0x3F80, 0x3F82, 0xBF80]
+
+
+def test_cosine_closed_forms():
+    th = 0.7
+    X = np.array([1.0, 0.0, 0.0])
+    Y = np.array([math.cos(th), math.sin(th), 0.0]) * 3.0
+    xy, xx, yy, c = oracle.cosine(X, Y)
+    assert abs(c - math.cos(th)) < 1e-15 and abs(yy - 9.0) < 1e-14 and xx == 1.0
+    assert oracle.cosine(X, X)[3] == 1.0
+    assert oracle.cosine(X, np.array([0.0, 2.0, 0.0]))[3] == 0.0
+
+
+def test_cosine_noise_expectation():
+    """cos(G, G + sigma |G| Z / sqrt(n)) -> 1/sqrt(1 + sigma^2) for large n."""
+    rng = np.random.default_rng(15)
+    n = 1 << 20
+    G = rng.standard_normal(n)
+    for sigma in (4.0, 2.5, 1.5):
+        Z = rng.standard_normal(n)
+        Y = G + sigma * np.linalg.norm(G) / math.sqrt(n) * Z
+        c = oracle.cosine(G, Y)[3]
+        assert abs(c - 1.0 / math.sqrt(1.0 + sigma * sigma)) < 3e-3
