@@ -1,0 +1,189 @@
+/*
+ * fpo.h -- C ABI of libfpo, the GB300 (sm_103a) implementation of the
+ * per-step pseudogradient update of Forward-Pass-Only MLP training (FPO) from
+ * "Forward Pass Domain Adaptation (Without Cross-Layer Backpropagation)".
+ *
+ * One FPO step on the down-projections is
+ *
+ *     fpo_error_signal(...)            Sec. 3.1 steps 2-4 + App. E
+ *     for each target layer l:
+ *         fpo_layer_update(...)        Sec. 3.1 step 5, Eq. (w3update), App. A
+ *     (or one fpo_layer_update_grouped call for all target layers)
+ *
+ * and the layer-viability diagnostic of Sec. 2.2 reduces pairs of gradients
+ * with fpo_cosine.
+ *
+ * Conventions (all entry points)
+ * ------------------------------
+ * - Tensor arguments are CUDA device pointers to dense row-major arrays,
+ *   16-byte aligned.  The caller owns every buffer; the library allocates
+ *   and frees no memory and never synchronises, except fpo_get_device_status.
+ * - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).
+ *   Every call only enqueues work on it and returns.
+ * - The return value reports errors the host can see (null pointers, shapes,
+ *   dtype, alignment, workspace size, device architecture, CUDA launch
+ *   errors).  After such an error nothing was enqueued.
+ * - Errors only the device can see (a target id outside [0, V), a bounded
+ *   wait inside a kernel that ran out) set bits of a status word at offset 0
+ *   of the call's workspace.  Each call clears that word when it starts;
+ *   fpo_get_device_status reads it after the call.
+ * - dtype FPO_BF16: every floating-point tensor argument except the fp32
+ *   master weights and lse/loss outputs is bf16; arithmetic is bf16 tensor-core
+ *   MMA with fp32 accumulation and fp32 elementwise math.  d, V and d_ff must be
+ *   multiples of 8 (16-byte rows for the TMA engine).
+ *   dtype FPO_F32: every floating-point tensor is fp32 and all arithmetic is
+ *   fp32 FFMA (no TF32); any positive shape is accepted.
+ * - The library only runs on compute capability 10.3 (GB300); any other
+ *   device returns FPO_ERR_ARCH.
+ */
+#ifndef FPO_H_
+#define FPO_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define FPO_ABI_VERSION 1
+
+/* Largest number of layers one fpo_layer_update_grouped call accepts. */
+#define FPO_MAX_GROUPED_LAYERS 64
+
+typedef enum fpo_dtype {
+    FPO_F32 = 0,
+    FPO_BF16 = 1
+} fpo_dtype;
+
+typedef enum fpo_status {
+    FPO_OK = 0,
+    FPO_ERR_NULL = 1,          /* a required pointer is NULL */
+    FPO_ERR_SHAPE = 2,         /* a size is negative, unsupported, or too large */
+    FPO_ERR_DTYPE = 3,         /* unknown dtype */
+    FPO_ERR_ALIGN = 4,         /* a tensor pointer is not 16-byte aligned */
+    FPO_ERR_WORKSPACE = 5,     /* workspace NULL or smaller than the query returned */
+    FPO_ERR_ARCH = 6,          /* current device is not compute capability 10.3 */
+    FPO_ERR_CUDA = 7,          /* a CUDA runtime/driver call failed */
+    FPO_ERR_TARGET_RANGE = 8,  /* device: a target id was outside [0, V) */
+    FPO_ERR_TIMEOUT = 9,       /* device: a bounded wait inside a kernel ran out */
+    FPO_ERR_ARG = 10           /* any other invalid argument */
+} fpo_status;
+
+/* Error-signal problem description (Sec. 3.1 steps 2-4, App. E). */
+typedef struct fpo_error_signal_desc {
+    int64_t T;          /* tokens (B x L flattened), >= 0; T = 0 enqueues nothing */
+    int64_t d;          /* model width (RMSNorm size, unembedding input)          */
+    int64_t V;          /* vocabulary size                                        */
+    int32_t dtype;      /* fpo_dtype of h, norm_w, W_U and g_out                  */
+    float eps;          /* RMSNorm epsilon, inside the square root (App. E)      */
+    float min_rms;      /* floor on rho in the 1/rho prefactor of the VJP (0.5)  */
+    float loss_scale;   /* s in e = s (softmax(z) - 1_y); 1/T = mean-reduced CE */
+    int64_t t_chunk;    /* tokens per error-matrix chunk; 0 = all T at once       */
+} fpo_error_signal_desc;
+
+/* Bytes of workspace fpo_error_signal needs for `desc` (0 on a bad desc). */
+size_t fpo_error_signal_workspace(const fpo_error_signal_desc* desc);
+
+/*
+ * fpo_error_signal -- output-layer error projected to the residual stream and
+ * through the final RMSNorm's Jacobian (Sec. 3.1 steps 2-4; Eq. (gproj);
+ * App. E Eq. (rmsnorm-vjp) with the min-RMS clamp).
+ *
+ * For every token t:
+ *   rho_t = sqrt(mean_j h_tj^2 + eps),  xhat_t = h_t / rho_t
+ *   z_t   = (norm_w (.) xhat_t) W_U^T                        (logits, never stored)
+ *   e_t   = s (softmax(z_t) - onehot(targets[t]))
+ *   g_t   = e_t W_U                                          (Eq. gproj)
+ *   g~_t  = (norm_w (.) g_t - xhat_t <xhat_t, norm_w (.) g_t> / d) / max(rho_t, min_rms)
+ *
+ * h        [T, d]   final pre-norm residual (dtype)
+ * norm_w   [d]      final RMSNorm weight (dtype)
+ * W_U      [V, d]   unembedding, nn.Linear layout (dtype)
+ * targets  [T]      int32 next-token ids in [0, V); out-of-range ids set
+ *                   FPO_ERR_TARGET_RANGE in the device status
+ * g_out    [T, d]   g~ (dtype)
+ * lse_out  [T]      fp32 log-sum-exp of each token's logits, or NULL
+ * loss_out [1]      fp32 mean cross-entropy (1/T) sum_t (lse_t - z_t,y_t), or NULL
+ * workspace         device scratch of fpo_error_signal_workspace(desc) bytes,
+ *                   256-byte aligned; owned by the caller, must not be shared
+ *                   with a call that runs concurrently
+ */
+int32_t fpo_error_signal(const fpo_error_signal_desc* desc, const void* h, const void* norm_w,
+                         const void* W_U, const int32_t* targets, void* g_out, float* lse_out,
+                         float* loss_out, void* workspace, size_t workspace_bytes, void* stream);
+
+/* Bytes of workspace fpo_layer_update / fpo_layer_update_grouped need. */
+size_t fpo_layer_update_workspace(void);
+
+/*
+ * fpo_layer_update -- pseudogradient of one target layer's down-projection and
+ * its plain-SGD step on the fp32 master copy (Sec. 3.1 step 5, Eq. (w3update);
+ * App. A, fp32 master weights cast to the working dtype).
+ *
+ *   G = g~^T A                    [d, d_ff], fp32 accumulation over T
+ *   W_master <- W_master - lr G   (fp32, one rounding)
+ *   W_out    <- W_master          (rounded to dtype, nearest-even)
+ *
+ * g        [T, d]      g~ from fpo_error_signal (dtype)
+ * A        [T, d_ff]   the layer's cached down-projection input h_mid (dtype)
+ * W_master [d, d_ff]   fp32, updated in place; NULL computes G only
+ * W_out    [d, d_ff]   updated weight in dtype, or NULL; needs W_master
+ * G_out    [d, d_ff]   G in dtype, or NULL
+ * workspace            fpo_layer_update_workspace() bytes (device status word)
+ * At least one of W_master and G_out must be non-NULL.  lr = 0 leaves
+ * W_master bit-identical.
+ */
+int32_t fpo_layer_update(int64_t T, int64_t d, int64_t d_ff, int32_t dtype, const void* g,
+                         const void* A, float lr, float* W_master, void* W_out, void* G_out,
+                         void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * fpo_layer_update_grouped -- fpo_layer_update for n_layers target layers that
+ * share g~ and the shapes, in one launch (1 <= n_layers <= FPO_MAX_GROUPED_LAYERS).
+ * A, W_master, W_out and G_out are HOST arrays of n_layers device pointers;
+ * W_master, W_out or G_out may be NULL as a whole (no such output for any
+ * layer), and individual entries may be NULL with the same meaning per layer.
+ */
+int32_t fpo_layer_update_grouped(int32_t n_layers, int64_t T, int64_t d, int64_t d_ff,
+                                 int32_t dtype, const void* g, const void* const* A, float lr,
+                                 float* const* W_master, void* const* W_out,
+                                 void* const* G_out, void* workspace, size_t workspace_bytes,
+                                 void* stream);
+
+/* Bytes of workspace fpo_cosine needs for n elements. */
+size_t fpo_cosine_workspace(int64_t n);
+
+/*
+ * fpo_cosine -- the layer-viability diagnostic's reduction (Sec. 2.2,
+ * Eq. (cosine)): cos = <X, Y> / (||X|| ||Y||) over n elements.
+ *
+ * X, Y  [n]  dtype (e.g. a pseudogradient and a true gradient, flattened)
+ * out   [4]  device fp64: <X,Y>, ||X||^2, ||Y||^2, cos (cos = 0 if a norm is 0)
+ * Per-thread partial sums are fp32, everything after is fp64, and the
+ * reduction order is fixed, so repeated calls give identical bits.
+ */
+int32_t fpo_cosine(int64_t n, int32_t dtype, const void* X, const void* Y, double* out,
+                   void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * Synchronise `stream`, read the device status word of `workspace` (set by the
+ * last call that used it), clear it, and return FPO_OK, FPO_ERR_TARGET_RANGE
+ * or FPO_ERR_TIMEOUT (the first of the two when both are set).
+ */
+int32_t fpo_get_device_status(void* workspace, void* stream);
+
+/* Upper bound, in nanoseconds, on every wait inside a kernel (default 2 s). */
+void fpo_set_wait_limit_ns(uint64_t ns);
+
+/* Static, human-readable name of a status code. */
+const char* fpo_status_string(int32_t status);
+
+/* FPO_ABI_VERSION of the loaded library. */
+int32_t fpo_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* FPO_H_ */

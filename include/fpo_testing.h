@@ -1,0 +1,34 @@
+/*
+ * fpo_testing.h -- test-only entry points of libfpo.  Not part of the FPO
+ * step; they expose internal building blocks so tests can check them alone.
+ */
+#ifndef FPO_TESTING_H_
+#define FPO_TESTING_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/*
+ * The tensor-core GEMM core of fpo_error_signal / fpo_layer_update with a
+ * plain fp32 store epilogue: C[M, N] = sum_k A(m, k) B(n, k), bf16 inputs,
+ * fp32 accumulation (the contraction of Eq. (gproj) and Eq. (w3update)).
+ *   a_mn = 0: A is [M, K] row-major (K contiguous); a_mn = 1: A is [K, M].
+ *   b_mn = 0: B is [N, K] row-major;                 b_mn = 1: B is [K, N].
+ * Supported (a_mn, b_mn): (0, 0), (0, 1), (1, 1).  M, N, K > 0; the
+ * contiguous extent of each operand must be a multiple of 8.  C is [M, N]
+ * fp32 row-major with N a multiple of 8.  workspace holds the device status
+ * word (>= 256 bytes).  Returns an fpo_status code.
+ */
+int32_t fpo_testing_gemm_bf16(int64_t M, int64_t N, int64_t K, int32_t a_mn, int32_t b_mn,
+                              const void* A, const void* B, float* C, void* workspace,
+                              size_t workspace_bytes, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* FPO_TESTING_H_ */

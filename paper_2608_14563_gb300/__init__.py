@@ -1,0 +1,211 @@
+"""Python binding of libfpo (include/fpo.h): the GB300 pseudogradient update of
+Forward-Pass-Only MLP training.
+
+Argument marshalling only: every function here passes device pointers, sizes
+and the current CUDA stream to the C entry point of the same name; every step
+of the computation runs in libfpo's CUDA kernels.  PyTorch supplies device
+memory and streams.  There is no CPU fallback: importing this package fails
+loudly when ``libfpo.so`` has not been built (``python -m
+paper_2608_14563_gb300.build`` or ``__graft_entry__.build()``).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libfpo.so")
+
+F32, BF16 = 0, 1
+OK = 0
+MAX_GROUPED_LAYERS = 64
+
+if not os.path.exists(LIB_PATH):
+    raise ImportError(f"libfpo.so is not built ({LIB_PATH} missing); run "
+                      "`python -m paper_2608_14563_gb300.build` first")
+_lib = ctypes.CDLL(LIB_PATH)
+
+_vp, _i64, _i32, _f32, _sz = (ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32, ctypes.c_float,
+                              ctypes.c_size_t)
+
+
+class ErrorSignalDesc(ctypes.Structure):
+    """Mirror of fpo_error_signal_desc."""
+    _fields_ = [("T", _i64), ("d", _i64), ("V", _i64), ("dtype", _i32), ("eps", _f32),
+                ("min_rms", _f32), ("loss_scale", _f32), ("t_chunk", _i64)]
+
+
+_lib.fpo_abi_version.restype = _i32
+_lib.fpo_status_string.argtypes = [_i32]
+_lib.fpo_status_string.restype = ctypes.c_char_p
+_lib.fpo_set_wait_limit_ns.argtypes = [ctypes.c_uint64]
+_lib.fpo_set_wait_limit_ns.restype = None
+_lib.fpo_error_signal_workspace.argtypes = [ctypes.POINTER(ErrorSignalDesc)]
+_lib.fpo_error_signal_workspace.restype = _sz
+_lib.fpo_error_signal.argtypes = [ctypes.POINTER(ErrorSignalDesc), _vp, _vp, _vp, _vp, _vp, _vp,
+                                  _vp, _vp, _sz, _vp]
+_lib.fpo_error_signal.restype = _i32
+_lib.fpo_layer_update_workspace.argtypes = []
+_lib.fpo_layer_update_workspace.restype = _sz
+_lib.fpo_layer_update.argtypes = [_i64, _i64, _i64, _i32, _vp, _vp, _f32, _vp, _vp, _vp, _vp,
+                                  _sz, _vp]
+_lib.fpo_layer_update.restype = _i32
+_lib.fpo_layer_update_grouped.argtypes = [_i32, _i64, _i64, _i64, _i32, _vp,
+                                          ctypes.POINTER(_vp), _f32, ctypes.POINTER(_vp),
+                                          ctypes.POINTER(_vp), ctypes.POINTER(_vp), _vp, _sz, _vp]
+_lib.fpo_layer_update_grouped.restype = _i32
+_lib.fpo_cosine_workspace.argtypes = [_i64]
+_lib.fpo_cosine_workspace.restype = _sz
+_lib.fpo_cosine.argtypes = [_i64, _i32, _vp, _vp, _vp, _vp, _sz, _vp]
+_lib.fpo_cosine.restype = _i32
+_lib.fpo_get_device_status.argtypes = [_vp, _vp]
+_lib.fpo_get_device_status.restype = _i32
+
+
+class FpoError(RuntimeError):
+    def __init__(self, code: int, where: str):
+        super().__init__(f"{where}: {status_string(code)}")
+        self.code = code
+
+
+def status_string(code: int) -> str:
+    return _lib.fpo_status_string(int(code)).decode()
+
+
+def abi_version() -> int:
+    return _lib.fpo_abi_version()
+
+
+def set_wait_limit_ns(ns: int) -> None:
+    _lib.fpo_set_wait_limit_ns(int(ns))
+
+
+def _check(code: int, where: str) -> None:
+    if code != OK:
+        raise FpoError(code, where)
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.bfloat16:
+        return BF16
+    if t.dtype == torch.float32:
+        return F32
+    raise TypeError(f"unsupported dtype {t.dtype}; libfpo takes bfloat16 or float32")
+
+
+def _ptr(t):
+    if t is None:
+        return None
+    if not t.is_cuda:
+        raise ValueError("libfpo takes CUDA tensors")
+    if not t.is_contiguous():
+        raise ValueError("libfpo takes contiguous tensors")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _workspace(nbytes: int, device) -> torch.Tensor:
+    return torch.empty(max(int(nbytes), 256), dtype=torch.uint8, device=device)
+
+
+# --------------------------------------------------------------------------- error signal
+def error_signal_desc(T, d, V, dtype=BF16, *, eps=1e-6, min_rms=0.5, loss_scale=None, t_chunk=0):
+    s = (1.0 / T if T > 0 else 1.0) if loss_scale is None else loss_scale
+    return ErrorSignalDesc(int(T), int(d), int(V), int(dtype), float(eps), float(min_rms), float(s),
+                           int(t_chunk))
+
+
+def error_signal_workspace(desc: ErrorSignalDesc) -> int:
+    return int(_lib.fpo_error_signal_workspace(ctypes.byref(desc)))
+
+
+def error_signal(h, norm_w, W_U, targets, g_out, *, eps=1e-6, min_rms=0.5, loss_scale=None,
+                 t_chunk=0, lse_out=None, loss_out=None, workspace=None, stream=None):
+    """fpo_error_signal: g~ = final-RMSNorm VJP of (softmax(z) - 1_y) W_U into ``g_out``.
+
+    Returns the workspace tensor (its first word holds the device status).
+    """
+    T, d = h.shape
+    V = W_U.shape[0]
+    desc = error_signal_desc(T, d, V, _dtype_code(h), eps=eps, min_rms=min_rms,
+                             loss_scale=loss_scale, t_chunk=t_chunk)
+    need = error_signal_workspace(desc)
+    if workspace is None:
+        workspace = _workspace(need, h.device)
+    rc = _lib.fpo_error_signal(ctypes.byref(desc), _ptr(h), _ptr(norm_w), _ptr(W_U), _ptr(targets),
+                               _ptr(g_out), _ptr(lse_out), _ptr(loss_out), _ptr(workspace),
+                               workspace.numel() * workspace.element_size(), _stream(stream))
+    _check(rc, "fpo_error_signal")
+    return workspace
+
+
+# --------------------------------------------------------------------------- layer update
+def layer_update_workspace() -> int:
+    return int(_lib.fpo_layer_update_workspace())
+
+
+def layer_update(g, A, lr, *, W_master=None, W_out=None, G_out=None, workspace=None, stream=None):
+    """fpo_layer_update: G = g~^T A ; W_master -= lr G ; W_out = cast(W_master)."""
+    T, d = g.shape
+    d_ff = A.shape[1]
+    if workspace is None:
+        workspace = _workspace(layer_update_workspace(), g.device)
+    rc = _lib.fpo_layer_update(T, d, d_ff, _dtype_code(g), _ptr(g), _ptr(A), float(lr),
+                               _ptr(W_master), _ptr(W_out), _ptr(G_out), _ptr(workspace),
+                               workspace.numel(), _stream(stream))
+    _check(rc, "fpo_layer_update")
+    return workspace
+
+
+def _ptr_array(ts, n):
+    if ts is None:
+        return None
+    arr = (_vp * n)()
+    for i, t in enumerate(ts):
+        arr[i] = None if t is None else _ptr(t).value
+    return arr
+
+
+def layer_update_grouped(g, As, lr, *, W_masters=None, W_outs=None, G_outs=None, workspace=None,
+                         stream=None):
+    """fpo_layer_update_grouped over len(As) target layers in one launch."""
+    n = len(As)
+    T, d = g.shape
+    d_ff = As[0].shape[1]
+    if workspace is None:
+        workspace = _workspace(layer_update_workspace(), g.device)
+    rc = _lib.fpo_layer_update_grouped(n, T, d, d_ff, _dtype_code(g), _ptr(g), _ptr_array(As, n),
+                                       float(lr), _ptr_array(W_masters, n), _ptr_array(W_outs, n),
+                                       _ptr_array(G_outs, n), _ptr(workspace), workspace.numel(),
+                                       _stream(stream))
+    _check(rc, "fpo_layer_update_grouped")
+    return workspace
+
+
+# --------------------------------------------------------------------------- cosine
+def cosine_workspace(n: int) -> int:
+    return int(_lib.fpo_cosine_workspace(int(n)))
+
+
+def cosine(X, Y, out=None, *, workspace=None, stream=None):
+    """fpo_cosine: returns a device fp64 tensor [<X,Y>, |X|^2, |Y|^2, cos]."""
+    n = X.numel()
+    if out is None:
+        out = torch.empty(4, dtype=torch.float64, device=X.device)
+    if workspace is None:
+        workspace = _workspace(cosine_workspace(n), X.device)
+    rc = _lib.fpo_cosine(n, _dtype_code(X), _ptr(X), _ptr(Y), _ptr(out), _ptr(workspace),
+                         workspace.numel(), _stream(stream))
+    _check(rc, "fpo_cosine")
+    return out
+
+
+def get_device_status(workspace, stream=None) -> int:
+    """fpo_get_device_status: synchronise, read and clear the workspace's status word."""
+    return int(_lib.fpo_get_device_status(_ptr(workspace), _stream(stream)))

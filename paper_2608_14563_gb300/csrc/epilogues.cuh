@@ -1,0 +1,211 @@
+// epilogues.cuh -- per-row epilogues of the tcgen05 GEMM.
+//
+// Each epilogue thread owns one output row of a 128 x BN tile and receives its
+// fp32 accumulator 32 columns at a time: Epi(params, group, row, n0), then
+// chunk(params, v[32], col_of_v0, col_offset_in_tile) for each 32-column chunk
+// in order, then finish(params, n_block).  Rows >= M and columns >= N belong
+// to the zero-filled tile overhang and are never written.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <math.h>
+
+#include "ptx.cuh"
+#include "tc_gemm.cuh"
+
+namespace fpo {
+
+constexpr float kLog2e = 1.4426950408889634f;
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+    __nv_bfloat162 p = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<uint32_t*>(&p);
+}
+
+// ---------------------------------------------------------------------------
+// Logits pass (Sec. 3.1 step 2): per (row, vocabulary tile) the running max and
+// sum of exponentials of z = yhat W_U^T over the tile's valid columns, plus the
+// target logit z_{t, y_t} when the target falls inside the tile.
+struct EpiLsePartial {
+    struct Params {
+        float2* part;      // [M, part_ld]: (max, sum exp(z - max)) per vocabulary tile
+        int part_ld;
+        float* zy;         // [M] target logit, or null
+        const int* y;      // [M] targets
+        int M, N;
+    };
+    float m, s, zt;
+    int yoff;
+    int row;
+    bool valid, has_t;
+
+    __device__ __forceinline__ EpiLsePartial(const Params& p, int, int row_, int n0)
+        : m(-INFINITY), s(0.f), zt(0.f), row(row_), has_t(false) {
+        valid = row_ < p.M;
+        yoff = valid ? __ldg(p.y + row_) - n0 : -1;
+    }
+
+    __device__ __forceinline__ void chunk(const Params& p, const float (&v)[32], int col0, int c0) {
+        const int lim = p.N - col0;  // valid columns in this chunk (may be <= 0)
+        if (lim <= 0) return;
+        float cm = -INFINITY;
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+            if (j < lim) cm = fmaxf(cm, v[j]);
+        const float nm = fmaxf(m, cm);
+        const float nml = nm * kLog2e;
+        float acc = (m == -INFINITY) ? 0.f : s * ex2_approx(m * kLog2e - nml);
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+            if (j < lim) acc += ex2_approx(fmaf(v[j], kLog2e, -nml));
+        s = acc;
+        m = nm;
+        const int r = yoff - c0;
+        if (static_cast<unsigned>(r) < 32u) {
+#pragma unroll
+            for (int j = 0; j < 32; ++j)
+                if (j == r) zt = v[j];
+            has_t = true;
+        }
+    }
+
+    __device__ __forceinline__ void finish(const Params& p, int nb) {
+        if (!valid) return;
+        p.part[static_cast<long long>(row) * p.part_ld + nb] = make_float2(m, s);
+        if (has_t && p.zy) p.zy[row] = zt;
+    }
+};
+
+// ---------------------------------------------------------------------------
+// Recompute pass (Sec. 3.1 step 2): e = s (exp(z - lse) - [col == y]) rounded
+// to bf16 into the error matrix E [M, N] (row stride ldE).
+struct EpiError {
+    struct Params {
+        __nv_bfloat16* E;
+        long long ldE;
+        const float* lse;  // [M]
+        const int* y;      // [M]
+        int M, N;
+        float s;
+    };
+    int row, yt;
+    float lse2;
+    bool valid;
+
+    __device__ __forceinline__ EpiError(const Params& p, int, int row_, int) : row(row_) {
+        valid = row_ < p.M;
+        yt = valid ? __ldg(p.y + row_) : -1;
+        lse2 = valid ? __ldg(p.lse + row_) * kLog2e : 0.f;
+    }
+
+    __device__ __forceinline__ void chunk(const Params& p, const float (&v)[32], int col0, int) {
+        const int lim = p.N - col0;
+        if (!valid || lim <= 0) return;
+        uint32_t w[16];
+#pragma unroll
+        for (int j = 0; j < 32; j += 2) {
+            float e0 = ex2_approx(fmaf(v[j], kLog2e, -lse2)) - (col0 + j == yt ? 1.f : 0.f);
+            float e1 = ex2_approx(fmaf(v[j + 1], kLog2e, -lse2)) - (col0 + j + 1 == yt ? 1.f : 0.f);
+            w[j / 2] = pack_bf16x2(p.s * e0, p.s * e1);
+        }
+        uint4* dst = reinterpret_cast<uint4*>(p.E + row * p.ldE + col0);
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+            if (q * 8 < lim) dst[q] = make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
+    }
+
+    __device__ __forceinline__ void finish(const Params&, int) {}
+};
+
+// ---------------------------------------------------------------------------
+// Plain fp32 store of C [M, N] (row stride ld): the projection g = E W_U (Eq. gproj).
+struct EpiStoreF32 {
+    struct Params {
+        float* C;
+        long long ld;
+        int M, N;
+    };
+    int row;
+    bool valid;
+
+    __device__ __forceinline__ EpiStoreF32(const Params& p, int, int row_, int) : row(row_) {
+        valid = row_ < p.M;
+    }
+
+    __device__ __forceinline__ void chunk(const Params& p, const float (&v)[32], int col0, int) {
+        const int lim = p.N - col0;
+        if (!valid || lim <= 0) return;
+        float4* dst = reinterpret_cast<float4*>(p.C + row * p.ld + col0);
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+            if (q * 4 < lim) dst[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+    }
+
+    __device__ __forceinline__ void finish(const Params&, int) {}
+};
+
+// ---------------------------------------------------------------------------
+// Pseudogradient update (Eq. w3update, App. A): for group (layer) g,
+//   W_master[g] -= lr * G ;  W_out[g] = bf16(W_master[g]) ;  G_out[g] = bf16(G)
+// Any of the three pointers may be null for a layer.
+struct EpiUpdate {
+    struct Params {
+        float* W_master[kMaxGroups];
+        __nv_bfloat16* W_out[kMaxGroups];
+        __nv_bfloat16* G_out[kMaxGroups];
+        long long ld;
+        int M, N;
+        float neg_lr;
+    };
+    int row, g;
+    bool valid;
+
+    __device__ __forceinline__ EpiUpdate(const Params& p, int g_, int row_, int) : row(row_), g(g_) {
+        valid = row_ < p.M;
+    }
+
+    __device__ __forceinline__ void chunk(const Params& p, const float (&v)[32], int col0, int) {
+        const int lim = p.N - col0;
+        if (!valid || lim <= 0) return;
+        const long long off = row * p.ld + col0;
+        float* wm = p.W_master[g];
+        __nv_bfloat16* wo = p.W_out[g];
+        __nv_bfloat16* go = p.G_out[g];
+        if (wm) {
+            float4* wp = reinterpret_cast<float4*>(wm + off);
+            uint4* op = reinterpret_cast<uint4*>(wo + off);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                if (q * 8 >= lim) break;
+                float4 a = wp[2 * q], b = wp[2 * q + 1];
+                a.x = fmaf(p.neg_lr, v[8 * q + 0], a.x);
+                a.y = fmaf(p.neg_lr, v[8 * q + 1], a.y);
+                a.z = fmaf(p.neg_lr, v[8 * q + 2], a.z);
+                a.w = fmaf(p.neg_lr, v[8 * q + 3], a.w);
+                b.x = fmaf(p.neg_lr, v[8 * q + 4], b.x);
+                b.y = fmaf(p.neg_lr, v[8 * q + 5], b.y);
+                b.z = fmaf(p.neg_lr, v[8 * q + 6], b.z);
+                b.w = fmaf(p.neg_lr, v[8 * q + 7], b.w);
+                wp[2 * q] = a;
+                wp[2 * q + 1] = b;
+                if (wo)
+                    op[q] = make_uint4(pack_bf16x2(a.x, a.y), pack_bf16x2(a.z, a.w),
+                                       pack_bf16x2(b.x, b.y), pack_bf16x2(b.z, b.w));
+            }
+        }
+        if (go) {
+            uint4* gp = reinterpret_cast<uint4*>(go + off);
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+                if (q * 8 < lim)
+                    gp[q] = make_uint4(pack_bf16x2(v[8 * q], v[8 * q + 1]),
+                                       pack_bf16x2(v[8 * q + 2], v[8 * q + 3]),
+                                       pack_bf16x2(v[8 * q + 4], v[8 * q + 5]),
+                                       pack_bf16x2(v[8 * q + 6], v[8 * q + 7]));
+        }
+    }
+
+    __device__ __forceinline__ void finish(const Params&, int) {}
+};
+
+}  // namespace fpo

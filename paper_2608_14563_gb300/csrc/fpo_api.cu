@@ -1,0 +1,339 @@
+// fpo_api.cu -- the C ABI declared in include/fpo.h: argument checks,
+// workspace layout and the launch sequence of each entry point.  All device
+// work is enqueued on the caller's stream; nothing here allocates device
+// memory or synchronises (except fpo_get_device_status).
+#include <cuda_runtime.h>
+
+#include <atomic>
+#include <climits>
+#include <mutex>
+
+#include "../../include/fpo.h"
+#include "../../include/fpo_testing.h"
+#include "internal.h"
+
+namespace fpo {
+
+namespace {
+std::atomic<uint64_t> g_wait_limit_ns{2000000000ull};
+
+struct DevCache {
+    std::once_flag once;
+    DevInfo info;
+    bool ok = false;
+};
+DevCache g_dev[64];
+}  // namespace
+
+uint64_t wait_limit_ns() { return g_wait_limit_ns.load(std::memory_order_relaxed); }
+
+bool current_device_info(DevInfo* out) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return false;
+    DevCache& c = g_dev[dev];
+    std::call_once(c.once, [&] {
+        int sms = 0, maj = 0, min = 0;
+        c.ok = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess &&
+               cudaDeviceGetAttribute(&maj, cudaDevAttrComputeCapabilityMajor, dev) == cudaSuccess &&
+               cudaDeviceGetAttribute(&min, cudaDevAttrComputeCapabilityMinor, dev) == cudaSuccess;
+        c.info = DevInfo{sms, maj, min};
+    });
+    if (c.ok) *out = c.info;
+    return c.ok;
+}
+
+}  // namespace fpo
+
+using namespace fpo;
+
+namespace {
+
+constexpr size_t kAlign = 256;
+constexpr size_t kStatusBytes = 256;
+
+size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+int32_t check_arch() {
+    DevInfo di;
+    if (!current_device_info(&di)) return FPO_ERR_CUDA;
+    if (di.major != 10 || di.minor != 3) return FPO_ERR_ARCH;
+    return FPO_OK;
+}
+
+int32_t cuda_status(cudaError_t e) { return e == cudaSuccess ? FPO_OK : FPO_ERR_CUDA; }
+
+#define FPO_TRY(expr)                                \
+    do {                                             \
+        cudaError_t e_ = (expr);                     \
+        if (e_ != cudaSuccess) return FPO_ERR_CUDA;  \
+    } while (0)
+
+// ------------------------------------------------------------------ error signal
+struct EsLayout {
+    size_t yhat, rho, lse, zy, ce, part, g, E, total;
+    int n_tiles;
+    int64_t Tc;
+};
+
+int32_t es_check_desc(const fpo_error_signal_desc* d) {
+    if (!d) return FPO_ERR_NULL;
+    if (d->dtype != FPO_F32 && d->dtype != FPO_BF16) return FPO_ERR_DTYPE;
+    if (d->T < 0 || d->d <= 0 || d->V <= 0 || d->t_chunk < 0) return FPO_ERR_SHAPE;
+    if (d->T > INT_MAX || d->d > INT_MAX || d->V > INT_MAX) return FPO_ERR_SHAPE;
+    if (d->dtype == FPO_BF16 && (d->d % 8 != 0 || d->V % 8 != 0)) return FPO_ERR_SHAPE;
+    if (!(d->eps >= 0.f) || !(d->min_rms >= 0.f)) return FPO_ERR_ARG;
+    return FPO_OK;
+}
+
+EsLayout es_layout(const fpo_error_signal_desc* d) {
+    EsLayout L{};
+    const size_t esz = d->dtype == FPO_BF16 ? 2 : 4;
+    const size_t T = static_cast<size_t>(d->T), D = static_cast<size_t>(d->d),
+                 V = static_cast<size_t>(d->V);
+    const int tile_n = d->dtype == FPO_BF16 ? lse_tile_n_bf16() : kSimtTile;
+    L.n_tiles = static_cast<int>((d->V + tile_n - 1) / tile_n);
+    L.Tc = d->T == 0 ? 0 : (d->t_chunk > 0 && d->t_chunk < d->T ? d->t_chunk : d->T);
+    size_t off = kStatusBytes;
+    L.yhat = off; off = align_up(off + T * D * esz);
+    L.rho = off;  off = align_up(off + T * 4);
+    L.lse = off;  off = align_up(off + T * 4);
+    L.zy = off;   off = align_up(off + T * 4);
+    L.ce = off;   off = align_up(off + T * 4);
+    L.part = off; off = align_up(off + T * static_cast<size_t>(L.n_tiles) * 8);
+    L.g = off;    off = align_up(off + T * D * 4);
+    L.E = off;    off = align_up(off + static_cast<size_t>(L.Tc) * V * esz);
+    L.total = off;
+    return L;
+}
+
+}  // namespace
+
+extern "C" {
+
+int32_t fpo_abi_version(void) { return FPO_ABI_VERSION; }
+
+void fpo_set_wait_limit_ns(uint64_t ns) {
+    g_wait_limit_ns.store(ns > 0 ? ns : 1, std::memory_order_relaxed);
+}
+
+const char* fpo_status_string(int32_t s) {
+    switch (s) {
+        case FPO_OK: return "FPO_OK";
+        case FPO_ERR_NULL: return "FPO_ERR_NULL: a required pointer is NULL";
+        case FPO_ERR_SHAPE: return "FPO_ERR_SHAPE: unsupported or invalid size";
+        case FPO_ERR_DTYPE: return "FPO_ERR_DTYPE: unknown dtype";
+        case FPO_ERR_ALIGN: return "FPO_ERR_ALIGN: tensor pointer not 16-byte aligned";
+        case FPO_ERR_WORKSPACE: return "FPO_ERR_WORKSPACE: workspace missing or too small";
+        case FPO_ERR_ARCH: return "FPO_ERR_ARCH: device is not compute capability 10.3";
+        case FPO_ERR_CUDA: return "FPO_ERR_CUDA: CUDA call failed";
+        case FPO_ERR_TARGET_RANGE: return "FPO_ERR_TARGET_RANGE: a target id is outside [0, V)";
+        case FPO_ERR_TIMEOUT: return "FPO_ERR_TIMEOUT: a bounded wait inside a kernel ran out";
+        case FPO_ERR_ARG: return "FPO_ERR_ARG: invalid argument";
+        default: return "unknown fpo status";
+    }
+}
+
+size_t fpo_error_signal_workspace(const fpo_error_signal_desc* desc) {
+    if (es_check_desc(desc) != FPO_OK) return 0;
+    return es_layout(desc).total;
+}
+
+int32_t fpo_error_signal(const fpo_error_signal_desc* desc, const void* h, const void* norm_w,
+                         const void* W_U, const int32_t* targets, void* g_out, float* lse_out,
+                         float* loss_out, void* workspace, size_t workspace_bytes, void* stream) {
+    int32_t rc = es_check_desc(desc);
+    if (rc != FPO_OK) return rc;
+    if (!workspace) return FPO_ERR_WORKSPACE;
+    if (desc->T > 0 && (!h || !norm_w || !W_U || !targets || !g_out)) return FPO_ERR_NULL;
+    if (!aligned16(h) || !aligned16(norm_w) || !aligned16(W_U) || !aligned16(g_out) ||
+        (reinterpret_cast<uintptr_t>(workspace) % kAlign) != 0 ||
+        (reinterpret_cast<uintptr_t>(targets) & 3u) || (reinterpret_cast<uintptr_t>(lse_out) & 3u) ||
+        (reinterpret_cast<uintptr_t>(loss_out) & 3u))
+        return FPO_ERR_ALIGN;
+    const EsLayout L = es_layout(desc);
+    if (workspace_bytes < L.total) return FPO_ERR_WORKSPACE;
+    if ((rc = check_arch()) != FPO_OK) return rc;
+
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    uint8_t* ws = static_cast<uint8_t*>(workspace);
+    unsigned* status = reinterpret_cast<unsigned*>(ws);
+    FPO_TRY(cudaMemsetAsync(status, 0, sizeof(unsigned), st));
+    const int T = static_cast<int>(desc->T), d = static_cast<int>(desc->d),
+              V = static_cast<int>(desc->V);
+    if (T == 0) {
+        if (loss_out) FPO_TRY(cudaMemsetAsync(loss_out, 0, sizeof(float), st));
+        return FPO_OK;
+    }
+    const bool bf16 = desc->dtype == FPO_BF16;
+    const size_t esz = bf16 ? 2 : 4;
+    void* yhat = ws + L.yhat;
+    float* rho = reinterpret_cast<float*>(ws + L.rho);
+    float* lse = lse_out ? lse_out : reinterpret_cast<float*>(ws + L.lse);
+    float* zy = loss_out ? reinterpret_cast<float*>(ws + L.zy) : nullptr;
+    float* ce = loss_out ? reinterpret_cast<float*>(ws + L.ce) : nullptr;
+    float2* part = reinterpret_cast<float2*>(ws + L.part);
+    float* g = reinterpret_cast<float*>(ws + L.g);
+    void* E = ws + L.E;
+
+    // 1. final RMSNorm forward: rho, yhat (and the target-range check)
+    FPO_TRY(launch_rmsnorm_fwd(desc->dtype, h, norm_w, T, d, desc->eps, yhat, rho, targets, V,
+                               status, st));
+    // 2. logits pass: per-vocabulary-tile (max, sum exp) partials -> lse
+    if (bf16)
+        FPO_TRY(launch_lse_partial_bf16(yhat, W_U, targets, T, d, V, part, L.n_tiles, zy, status,
+                                        st));
+    else
+        FPO_TRY(launch_lse_partial_f32(static_cast<const float*>(yhat),
+                                       static_cast<const float*>(W_U), targets, T, d, V, part,
+                                       L.n_tiles, zy, st));
+    FPO_TRY(launch_lse_combine(part, L.n_tiles, T, zy, lse, ce, st));
+    if (loss_out) FPO_TRY(launch_mean(ce, T, loss_out, st));
+    // 3./4. per token chunk: recompute logits -> E, then g = E W_U
+    for (int64_t c0 = 0; c0 < T; c0 += L.Tc) {
+        const int tc = static_cast<int>(L.Tc < T - c0 ? L.Tc : T - c0);
+        const void* yh = static_cast<const uint8_t*>(yhat) + static_cast<size_t>(c0) * d * esz;
+        if (bf16) {
+            FPO_TRY(launch_error_bf16(yh, W_U, targets + c0, lse + c0, tc, d, V,
+                                      desc->loss_scale, E, status, st));
+            FPO_TRY(launch_proj_bf16(E, W_U, tc, d, V, g + c0 * d, status, st));
+        } else {
+            FPO_TRY(launch_error_f32(static_cast<const float*>(yh), static_cast<const float*>(W_U),
+                                     targets + c0, lse + c0, tc, d, V, desc->loss_scale,
+                                     static_cast<float*>(E), st));
+            FPO_TRY(launch_proj_f32(static_cast<const float*>(E), static_cast<const float*>(W_U),
+                                    tc, d, V, g + c0 * d, st));
+        }
+    }
+    // 5. final-norm VJP with the min-RMS clamp -> g~
+    FPO_TRY(launch_rmsnorm_vjp(desc->dtype, g, h, norm_w, rho, T, d, desc->min_rms, g_out, st));
+    return FPO_OK;
+}
+
+size_t fpo_layer_update_workspace(void) { return kStatusBytes; }
+
+int32_t fpo_layer_update_grouped(int32_t n_layers, int64_t T, int64_t d, int64_t d_ff,
+                                 int32_t dtype, const void* g, const void* const* A, float lr,
+                                 float* const* W_master, void* const* W_out, void* const* G_out,
+                                 void* workspace, size_t workspace_bytes, void* stream) {
+    if (dtype != FPO_F32 && dtype != FPO_BF16) return FPO_ERR_DTYPE;
+    if (n_layers < 1 || n_layers > FPO_MAX_GROUPED_LAYERS) return FPO_ERR_SHAPE;
+    if (T < 0 || d <= 0 || d_ff <= 0 || T > INT_MAX || d > INT_MAX || d_ff > INT_MAX)
+        return FPO_ERR_SHAPE;
+    if (dtype == FPO_BF16 && (d % 8 != 0 || d_ff % 8 != 0)) return FPO_ERR_SHAPE;
+    if (!(lr == lr)) return FPO_ERR_ARG;
+    if (!workspace || workspace_bytes < kStatusBytes) return FPO_ERR_WORKSPACE;
+    if ((reinterpret_cast<uintptr_t>(workspace) % kAlign) != 0) return FPO_ERR_ALIGN;
+    if (!A || (T > 0 && !g)) return FPO_ERR_NULL;
+    if (!aligned16(g)) return FPO_ERR_ALIGN;
+    for (int l = 0; l < n_layers; ++l) {
+        float* wm = W_master ? W_master[l] : nullptr;
+        void* wo = W_out ? W_out[l] : nullptr;
+        void* go = G_out ? G_out[l] : nullptr;
+        if (T > 0 && !A[l]) return FPO_ERR_NULL;
+        if (!wm && !go) return FPO_ERR_NULL;
+        if (wo && !wm) return FPO_ERR_NULL;
+        if (!aligned16(A[l]) || !aligned16(wm) || !aligned16(wo) || !aligned16(go))
+            return FPO_ERR_ALIGN;
+    }
+    int32_t rc = check_arch();
+    if (rc != FPO_OK) return rc;
+
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    unsigned* status = static_cast<unsigned*>(workspace);
+    FPO_TRY(cudaMemsetAsync(status, 0, sizeof(unsigned), st));
+    const int Ti = static_cast<int>(T), di = static_cast<int>(d), fi = static_cast<int>(d_ff);
+    if (T == 0) {
+        // G = 0: the master is unchanged, W_out is its cast, G_out is zero.
+        const size_t n = static_cast<size_t>(d) * static_cast<size_t>(d_ff);
+        for (int l = 0; l < n_layers; ++l) {
+            void* go = G_out ? G_out[l] : nullptr;
+            void* wo = W_out ? W_out[l] : nullptr;
+            if (go) FPO_TRY(cudaMemsetAsync(go, 0, n * (dtype == FPO_BF16 ? 2 : 4), st));
+            if (wo) FPO_TRY(launch_cast_f32(dtype, W_master[l], n, wo, st));
+        }
+        return FPO_OK;
+    }
+    if (dtype == FPO_BF16)
+        return cuda_status(launch_update_bf16(n_layers, Ti, di, fi, g, A, lr, W_master, W_out,
+                                              G_out, status, st));
+    return cuda_status(launch_update_f32(
+        n_layers, Ti, di, fi, static_cast<const float*>(g), reinterpret_cast<const float* const*>(A),
+        lr, W_master, reinterpret_cast<float* const*>(W_out), reinterpret_cast<float* const*>(G_out),
+        st));
+}
+
+int32_t fpo_layer_update(int64_t T, int64_t d, int64_t d_ff, int32_t dtype, const void* g,
+                         const void* A, float lr, float* W_master, void* W_out, void* G_out,
+                         void* workspace, size_t workspace_bytes, void* stream) {
+    const void* As[1] = {A};
+    float* Wm[1] = {W_master};
+    void* Wo[1] = {W_out};
+    void* Go[1] = {G_out};
+    return fpo_layer_update_grouped(1, T, d, d_ff, dtype, g, As, lr, Wm, Wo, Go, workspace,
+                                    workspace_bytes, stream);
+}
+
+size_t fpo_cosine_workspace(int64_t n) {
+    if (n < 0) return 0;
+    return kStatusBytes + align_up(static_cast<size_t>(cosine_blocks(n)) * 3 * sizeof(double));
+}
+
+int32_t fpo_cosine(int64_t n, int32_t dtype, const void* X, const void* Y, double* out,
+                   void* workspace, size_t workspace_bytes, void* stream) {
+    if (dtype != FPO_F32 && dtype != FPO_BF16) return FPO_ERR_DTYPE;
+    if (n < 0) return FPO_ERR_SHAPE;
+    if (!out || (n > 0 && (!X || !Y))) return FPO_ERR_NULL;
+    if (!aligned16(X) || !aligned16(Y) || (reinterpret_cast<uintptr_t>(out) & 7u)) return FPO_ERR_ALIGN;
+    if (!workspace) return FPO_ERR_WORKSPACE;
+    if ((reinterpret_cast<uintptr_t>(workspace) % kAlign) != 0) return FPO_ERR_ALIGN;
+    int32_t rc = check_arch();
+    if (rc != FPO_OK) return rc;
+    const size_t need = fpo_cosine_workspace(n);
+    if (workspace_bytes < need) return FPO_ERR_WORKSPACE;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    uint8_t* ws = static_cast<uint8_t*>(workspace);
+    FPO_TRY(cudaMemsetAsync(ws, 0, sizeof(unsigned), st));
+    if (n == 0) {
+        FPO_TRY(cudaMemsetAsync(out, 0, 4 * sizeof(double), st));
+        return FPO_OK;
+    }
+    const int blocks = cosine_blocks(n);
+    return cuda_status(launch_cosine(dtype, n, X, Y, reinterpret_cast<double*>(ws + kStatusBytes),
+                                     blocks, out, st));
+}
+
+int32_t fpo_testing_gemm_bf16(int64_t M, int64_t N, int64_t K, int32_t a_mn, int32_t b_mn,
+                              const void* A, const void* B, float* C, void* workspace,
+                              size_t workspace_bytes, void* stream) {
+    if (M <= 0 || N <= 0 || K <= 0 || M > INT_MAX || N > INT_MAX || K > INT_MAX) return FPO_ERR_SHAPE;
+    if (a_mn && !b_mn) return FPO_ERR_ARG;
+    if ((a_mn ? M : K) % 8 != 0 || (b_mn ? N : K) % 8 != 0 || N % 8 != 0) return FPO_ERR_SHAPE;
+    if (!A || !B || !C) return FPO_ERR_NULL;
+    if (!aligned16(A) || !aligned16(B) || !aligned16(C)) return FPO_ERR_ALIGN;
+    if (!workspace || workspace_bytes < kStatusBytes) return FPO_ERR_WORKSPACE;
+    int32_t rc = check_arch();
+    if (rc != FPO_OK) return rc;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    unsigned* status = static_cast<unsigned*>(workspace);
+    FPO_TRY(cudaMemsetAsync(status, 0, sizeof(unsigned), st));
+    return cuda_status(launch_test_gemm_bf16(static_cast<int>(M), static_cast<int>(N),
+                                             static_cast<int>(K), a_mn != 0, b_mn != 0, A, B, C,
+                                             status, st));
+}
+
+int32_t fpo_get_device_status(void* workspace, void* stream) {
+    if (!workspace) return FPO_ERR_WORKSPACE;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (cudaStreamSynchronize(st) != cudaSuccess) return FPO_ERR_CUDA;
+    unsigned word = 0;
+    if (cudaMemcpy(&word, workspace, sizeof word, cudaMemcpyDeviceToHost) != cudaSuccess)
+        return FPO_ERR_CUDA;
+    if (cudaMemset(workspace, 0, sizeof word) != cudaSuccess) return FPO_ERR_CUDA;
+    if (word & kDevTargetRange) return FPO_ERR_TARGET_RANGE;
+    if (word & kDevTimeout) return FPO_ERR_TIMEOUT;
+    return FPO_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,187 @@
+// gemm_bf16.cu -- host launchers of the four tcgen05 GEMMs of the FPO step.
+//
+//   logits pass      z = yhat W_U^T      M=T  N=V    K=d   A K-major, B K-major
+//   recompute pass   same GEMM, epilogue writes E = s (softmax - onehot)
+//   projection       g = E W_U           M=T  N=d    K=V   A K-major, B MN-major
+//   update           G = g~^T A_l        M=d  N=d_ff K=T   A MN-major, B MN-major
+//
+// Tensor maps are encoded per call (a few microseconds of host work) through
+// the driver entry point of cuTensorMapEncodeTiled, so the library does not
+// link libcuda directly.
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include <mutex>
+
+#include "epilogues.cuh"
+#include "internal.h"
+#include "tc_gemm.cuh"
+
+namespace fpo {
+namespace {
+
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                   const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                             &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+    });
+    return fn;
+}
+
+// 2-D bf16 tensor [outer, inner] with row stride `ld` elements, box
+// {box_inner, box_outer}, 128-byte swizzle, zero fill outside the tensor.
+bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, uint64_t ld,
+              uint32_t box_inner, uint32_t box_outer) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t dims[2] = {inner, outer};
+    cuuint64_t strides[1] = {ld * 2};
+    cuuint32_t box[2] = {box_inner, box_outer};
+    cuuint32_t es[2] = {1, 1};
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
+              es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// K-major operand [rows, K]: box {64 (K), rows_per_tile}
+bool map_kmajor(CUtensorMap* m, const void* base, int rows, int K, int box_rows) {
+    return make_map(m, base, K, rows, K, kBK, box_rows);
+}
+// MN-major operand [K, mn]: box {64 (MN), 64 (K)}
+bool map_mnmajor(CUtensorMap* m, const void* base, int K, int mn) {
+    return make_map(m, base, mn, K, mn, 64, kBK);
+}
+
+GemmShape make_shape(int M, int N, int K, int BN, int groups, int band) {
+    GemmShape sh;
+    sh.M = M;
+    sh.N = N;
+    sh.K = K;
+    sh.m_blocks = (M + kBM - 1) / kBM;
+    sh.n_blocks = (N + BN - 1) / BN;
+    sh.k_blocks = (K + kBK - 1) / kBK;
+    sh.groups = groups;
+    sh.band = band;
+    sh.tiles = static_cast<long long>(groups) * sh.m_blocks * sh.n_blocks;
+    return sh;
+}
+
+template <int BN, bool A_MN, bool B_MN, int STAGES, int MAXG, class Epi>
+cudaError_t run_gemm(const GemmMaps<MAXG>& maps, const typename Epi::Params& ep,
+                     const GemmShape& sh, unsigned* status, cudaStream_t st) {
+    if (sh.tiles <= 0 || sh.k_blocks <= 0) return cudaSuccess;
+    using L = GemmSmem<BN, STAGES>;
+    auto kern = tc_gemm_kernel<BN, A_MN, B_MN, STAGES, MAXG, Epi>;
+    static cudaError_t attr_err =
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::kBytes);
+    if (attr_err != cudaSuccess) return attr_err;
+    DevInfo di;
+    if (!current_device_info(&di)) return cudaErrorUnknown;
+    const long long grid = sh.tiles < di.sm_count ? sh.tiles : di.sm_count;
+    kern<<<static_cast<unsigned>(grid), kGemmThreads, L::kBytes, st>>>(maps, ep, sh, status,
+                                                                      wait_limit_ns());
+    return cudaGetLastError();
+}
+
+constexpr int kBandM = 16;
+
+}  // namespace
+
+constexpr int kLseBN = 256;
+constexpr int kLseStages = 4;
+int lse_tile_n_bf16() { return kLseBN; }
+
+cudaError_t launch_lse_partial_bf16(const void* yhat, const void* W_U, const int32_t* y, int T,
+                                    int d, int V, float2* part, int part_ld, float* zy,
+                                    unsigned* status, cudaStream_t st) {
+    GemmMaps<1> maps;
+    if (!map_kmajor(&maps.a, yhat, T, d, kBM) || !map_kmajor(&maps.b[0], W_U, V, d, kLseBN))
+        return cudaErrorInvalidValue;
+    EpiLsePartial::Params ep{part, part_ld, zy, y, T, V};
+    return run_gemm<kLseBN, false, false, kLseStages, 1, EpiLsePartial>(
+        maps, ep, make_shape(T, V, d, kLseBN, 1, kBandM), status, st);
+}
+
+cudaError_t launch_error_bf16(const void* yhat, const void* W_U, const int32_t* y, const float* lse,
+                              int Tc, int d, int V, float s, void* E, unsigned* status,
+                              cudaStream_t st) {
+    GemmMaps<1> maps;
+    if (!map_kmajor(&maps.a, yhat, Tc, d, kBM) || !map_kmajor(&maps.b[0], W_U, V, d, kLseBN))
+        return cudaErrorInvalidValue;
+    EpiError::Params ep{static_cast<__nv_bfloat16*>(E), V, lse, y, Tc, V, s};
+    return run_gemm<kLseBN, false, false, kLseStages, 1, EpiError>(
+        maps, ep, make_shape(Tc, V, d, kLseBN, 1, kBandM), status, st);
+}
+
+constexpr int kProjBN = 256;
+constexpr int kProjStages = 4;
+
+cudaError_t launch_proj_bf16(const void* E, const void* W_U, int Tc, int d, int V, float* g,
+                             unsigned* status, cudaStream_t st) {
+    GemmMaps<1> maps;
+    if (!map_kmajor(&maps.a, E, Tc, V, kBM) || !map_mnmajor(&maps.b[0], W_U, V, d))
+        return cudaErrorInvalidValue;
+    EpiStoreF32::Params ep{g, d, Tc, d};
+    return run_gemm<kProjBN, false, true, kProjStages, 1, EpiStoreF32>(
+        maps, ep, make_shape(Tc, d, V, kProjBN, 1, kBandM), status, st);
+}
+
+constexpr int kUpdBN = 256;
+constexpr int kUpdStages = 4;
+
+cudaError_t launch_update_bf16(int n, int T, int d, int d_ff, const void* g, const void* const* A,
+                               float lr, float* const* W_master, void* const* W_out,
+                               void* const* G_out, unsigned* status, cudaStream_t st) {
+    if (n < 1 || n > kMaxGroups) return cudaErrorInvalidValue;
+    static GemmMaps<kMaxGroups> maps;  // host staging; copied into the launch parameters
+    static EpiUpdate::Params ep;
+    static std::mutex mu;
+    std::lock_guard<std::mutex> lock(mu);
+    if (!map_mnmajor(&maps.a, g, T, d)) return cudaErrorInvalidValue;
+    for (int l = 0; l < n; ++l) {
+        if (!map_mnmajor(&maps.b[l], A[l], T, d_ff)) return cudaErrorInvalidValue;
+        ep.W_master[l] = W_master ? W_master[l] : nullptr;
+        ep.W_out[l] = W_out ? static_cast<__nv_bfloat16*>(W_out[l]) : nullptr;
+        ep.G_out[l] = G_out ? static_cast<__nv_bfloat16*>(G_out[l]) : nullptr;
+    }
+    for (int l = n; l < kMaxGroups; ++l) {
+        maps.b[l] = maps.b[0];
+        ep.W_master[l] = nullptr;
+        ep.W_out[l] = nullptr;
+        ep.G_out[l] = nullptr;
+    }
+    ep.ld = d_ff;
+    ep.M = d;
+    ep.N = d_ff;
+    ep.neg_lr = -lr;
+    return run_gemm<kUpdBN, true, true, kUpdStages, kMaxGroups, EpiUpdate>(
+        maps, ep, make_shape(d, d_ff, T, kUpdBN, n, kBandM), status, st);
+}
+
+cudaError_t launch_test_gemm_bf16(int M, int N, int K, bool a_mn, bool b_mn, const void* A,
+                                  const void* B, float* C, unsigned* status, cudaStream_t st) {
+    GemmMaps<1> maps;
+    bool ok = a_mn ? map_mnmajor(&maps.a, A, K, M) : map_kmajor(&maps.a, A, M, K, kBM);
+    ok = ok && (b_mn ? map_mnmajor(&maps.b[0], B, K, N) : map_kmajor(&maps.b[0], B, N, K, 256));
+    if (!ok) return cudaErrorInvalidValue;
+    EpiStoreF32::Params ep{C, N, M, N};
+    const GemmShape sh = make_shape(M, N, K, 256, 1, kBandM);
+    if (!a_mn && !b_mn) return run_gemm<256, false, false, 4, 1, EpiStoreF32>(maps, ep, sh, status, st);
+    if (!a_mn && b_mn) return run_gemm<256, false, true, 4, 1, EpiStoreF32>(maps, ep, sh, status, st);
+    if (a_mn && b_mn) return run_gemm<256, true, true, 4, 1, EpiStoreF32>(maps, ep, sh, status, st);
+    return cudaErrorInvalidValue;
+}
+
+}  // namespace fpo

@@ -1,0 +1,83 @@
+// internal.h -- launchers shared between the C-ABI layer and the kernel
+// translation units.  Every launcher enqueues on `stream` and returns a
+// cudaError_t (cudaSuccess when the launch was accepted).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace fpo {
+
+// Device status bits, OR-ed into the status word at offset 0 of a workspace.
+enum : unsigned int {
+    kDevTargetRange = 1u,
+    kDevTimeout = 2u,
+};
+
+struct DevInfo {
+    int sm_count;
+    int major, minor;
+};
+// Cached properties of the current device; false if the query failed.
+bool current_device_info(DevInfo* out);
+
+uint64_t wait_limit_ns();
+
+// ------------------------------------------------------------ bf16 (tcgen05)
+// Logits pass: part[T, n_tiles] (max, sum exp) and zy[T] (target logits).
+cudaError_t launch_lse_partial_bf16(const void* yhat, const void* W_U, const int32_t* y, int T,
+                                    int d, int V, float2* part, int part_ld, float* zy,
+                                    unsigned* status, cudaStream_t s);
+int lse_tile_n_bf16();
+
+// Recompute pass for rows [0, Tc) of yhat: E[Tc, V] = s (softmax - onehot) in bf16.
+cudaError_t launch_error_bf16(const void* yhat, const void* W_U, const int32_t* y, const float* lse,
+                              int Tc, int d, int V, float s, void* E, unsigned* status,
+                              cudaStream_t st);
+
+// Projection: g[Tc, d] = E[Tc, V] W_U (fp32 out).
+cudaError_t launch_proj_bf16(const void* E, const void* W_U, int Tc, int d, int V, float* g,
+                             unsigned* status, cudaStream_t st);
+
+// Grouped pseudogradient update over n layers.
+cudaError_t launch_update_bf16(int n, int T, int d, int d_ff, const void* g, const void* const* A,
+                               float lr, float* const* W_master, void* const* W_out,
+                               void* const* G_out, unsigned* status, cudaStream_t st);
+
+// Plain GEMM with an fp32 store epilogue (test entry point).
+cudaError_t launch_test_gemm_bf16(int M, int N, int K, bool a_mn, bool b_mn, const void* A,
+                                  const void* B, float* C, unsigned* status, cudaStream_t st);
+
+// ------------------------------------------------------------ row-wise kernels
+cudaError_t launch_rmsnorm_fwd(int dtype, const void* h, const void* w, int T, int d, float eps,
+                               void* yhat, float* rho, const int32_t* y, int V, unsigned* status,
+                               cudaStream_t st);
+cudaError_t launch_lse_combine(const float2* part, int n_tiles, int T, const float* zy,
+                               float* lse, float* ce, cudaStream_t st);
+cudaError_t launch_mean(const float* x, int n, float* out, cudaStream_t st);
+// dst[n] = src[n] rounded to dtype (a plain copy for fp32).
+cudaError_t launch_cast_f32(int dtype, const float* src, size_t n, void* dst, cudaStream_t st);
+cudaError_t launch_rmsnorm_vjp(int dtype, const float* g, const void* h, const void* w,
+                               const float* rho, int T, int d, float min_rms, void* out,
+                               cudaStream_t st);
+
+// ------------------------------------------------------------ cosine
+int cosine_blocks(int64_t n);
+cudaError_t launch_cosine(int dtype, int64_t n, const void* X, const void* Y, double* partial,
+                          int blocks, double* out, cudaStream_t st);
+
+// ------------------------------------------------------------ fp32 SIMT path
+constexpr int kSimtTile = 64;
+cudaError_t launch_lse_partial_f32(const float* yhat, const float* W_U, const int32_t* y, int T,
+                                   int d, int V, float2* part, int part_ld, float* zy,
+                                   cudaStream_t st);
+cudaError_t launch_error_f32(const float* yhat, const float* W_U, const int32_t* y,
+                             const float* lse, int Tc, int d, int V, float s, float* E,
+                             cudaStream_t st);
+cudaError_t launch_proj_f32(const float* E, const float* W_U, int Tc, int d, int V, float* g,
+                            cudaStream_t st);
+cudaError_t launch_update_f32(int n, int T, int d, int d_ff, const float* g,
+                              const float* const* A, float lr, float* const* W_master,
+                              float* const* W_out, float* const* G_out, cudaStream_t st);
+
+}  // namespace fpo

@@ -1,0 +1,280 @@
+// rowwise.cu -- bandwidth-bound per-token kernels of the error signal.
+//
+//   rmsnorm_fwd   rho_t = sqrt(mean_j h_tj^2 + eps), yhat_t = w (.) h_t / rho_t
+//                 (the final RMSNorm forward of App. E), plus the target-range
+//                 check of every token
+//   lse_combine   lse_t from the per-vocabulary-tile (max, sum exp) partials
+//   mean          mean of a vector in a fixed order (the mean cross-entropy)
+//   rmsnorm_vjp   App. E Eq. (rmsnorm-vjp) with the min-RMS clamp:
+//                 g~ = (w (.) g - xhat <xhat, w (.) g> / d) / max(rho, rho_min)
+//
+// One warp per token row, 16-byte vector loads, warp-shuffle reductions.
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <math.h>
+
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace fpo {
+namespace {
+
+__device__ __forceinline__ float warp_sum(float x) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+    return x;
+}
+
+__device__ __forceinline__ float warp_max(float x) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) x = fmaxf(x, __shfl_xor_sync(0xffffffffu, x, o));
+    return x;
+}
+
+// Load / store VEC consecutive elements as floats (VEC * sizeof(T) is 16 bytes
+// for the vector forms, or VEC = 1).
+template <int VEC>
+__device__ __forceinline__ void ld_vec(const float* p, float (&v)[VEC]) {
+    if constexpr (VEC == 4) {
+        float4 a = *reinterpret_cast<const float4*>(p);
+        v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+    } else if constexpr (VEC == 8) {
+        float4 a = *reinterpret_cast<const float4*>(p);
+        float4 b = *reinterpret_cast<const float4*>(p + 4);
+        v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+        v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+    } else {
+#pragma unroll
+        for (int k = 0; k < VEC; ++k) v[k] = p[k];
+    }
+}
+
+template <int VEC>
+__device__ __forceinline__ void ld_vec(const __nv_bfloat16* p, float (&v)[VEC]) {
+    static_assert(VEC == 8, "bf16 rows are read 8 elements (16 bytes) at a time");
+    uint4 a = *reinterpret_cast<const uint4*>(p);
+    const __nv_bfloat162* h2 = reinterpret_cast<const __nv_bfloat162*>(&a);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        float2 f = __bfloat1622float2(h2[k]);
+        v[2 * k] = f.x;
+        v[2 * k + 1] = f.y;
+    }
+}
+
+template <int VEC>
+__device__ __forceinline__ void st_vec(float* p, const float (&v)[VEC]) {
+    if constexpr (VEC == 4) {
+        *reinterpret_cast<float4*>(p) = make_float4(v[0], v[1], v[2], v[3]);
+    } else {
+#pragma unroll
+        for (int k = 0; k < VEC; ++k) p[k] = v[k];
+    }
+}
+
+template <int VEC>
+__device__ __forceinline__ void st_vec(__nv_bfloat16* p, const float (&v)[VEC]) {
+    static_assert(VEC == 8, "bf16 rows are written 8 elements (16 bytes) at a time");
+    uint4 a;
+    __nv_bfloat162* h2 = reinterpret_cast<__nv_bfloat162*>(&a);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) h2[k] = __floats2bfloat162_rn(v[2 * k], v[2 * k + 1]);
+    *reinterpret_cast<uint4*>(p) = a;
+}
+
+constexpr int kRowThreads = 256;  // 8 warps, one row each
+
+template <typename TT, int VEC>
+__global__ void __launch_bounds__(kRowThreads)
+    rmsnorm_fwd_kernel(const TT* __restrict__ h, const TT* __restrict__ w, int T, int d, float eps,
+                       TT* __restrict__ yhat, float* __restrict__ rho, const int32_t* __restrict__ y,
+                       int V, unsigned* status) {
+    const int lane = threadIdx.x & 31;
+    const int wpb = blockDim.x >> 5;
+    for (int row = blockIdx.x * wpb + (threadIdx.x >> 5); row < T; row += gridDim.x * wpb) {
+        const TT* hr = h + static_cast<size_t>(row) * d;
+        float ss = 0.f;
+        for (int j = lane * VEC; j < d; j += 32 * VEC) {
+            float x[VEC];
+            ld_vec<VEC>(hr + j, x);
+#pragma unroll
+            for (int k = 0; k < VEC; ++k) ss = fmaf(x[k], x[k], ss);
+        }
+        ss = warp_sum(ss);
+        const float r = sqrtf(ss / static_cast<float>(d) + eps);
+        const float inv = 1.0f / r;
+        TT* yr = yhat + static_cast<size_t>(row) * d;
+        for (int j = lane * VEC; j < d; j += 32 * VEC) {
+            float x[VEC], wv[VEC], o[VEC];
+            ld_vec<VEC>(hr + j, x);
+            ld_vec<VEC>(w + j, wv);
+#pragma unroll
+            for (int k = 0; k < VEC; ++k) o[k] = wv[k] * (x[k] * inv);
+            st_vec<VEC>(yr + j, o);
+        }
+        if (lane == 0) {
+            rho[row] = r;
+            const int t = y[row];
+            if (t < 0 || t >= V) atomicOr(status, kDevTargetRange);
+        }
+    }
+}
+
+template <typename TT, int VEC>
+__global__ void __launch_bounds__(kRowThreads)
+    rmsnorm_vjp_kernel(const float* __restrict__ g, const TT* __restrict__ h,
+                       const TT* __restrict__ w, const float* __restrict__ rho, int T, int d,
+                       float min_rms, TT* __restrict__ out) {
+    const int lane = threadIdx.x & 31;
+    const int wpb = blockDim.x >> 5;
+    for (int row = blockIdx.x * wpb + (threadIdx.x >> 5); row < T; row += gridDim.x * wpb) {
+        const float r = rho[row];
+        const float inv_r = 1.0f / r;
+        const float* gr = g + static_cast<size_t>(row) * d;
+        const TT* hr = h + static_cast<size_t>(row) * d;
+        float c = 0.f;
+        for (int j = lane * VEC; j < d; j += 32 * VEC) {
+            float gv[VEC], x[VEC], wv[VEC];
+            ld_vec<VEC>(gr + j, gv);
+            ld_vec<VEC>(hr + j, x);
+            ld_vec<VEC>(w + j, wv);
+#pragma unroll
+            for (int k = 0; k < VEC; ++k) c = fmaf(x[k] * inv_r, wv[k] * gv[k], c);
+        }
+        c = warp_sum(c);
+        const float kd = c / static_cast<float>(d);
+        const float pref = 1.0f / fmaxf(r, min_rms);
+        TT* orow = out + static_cast<size_t>(row) * d;
+        for (int j = lane * VEC; j < d; j += 32 * VEC) {
+            float gv[VEC], x[VEC], wv[VEC], o[VEC];
+            ld_vec<VEC>(gr + j, gv);
+            ld_vec<VEC>(hr + j, x);
+            ld_vec<VEC>(w + j, wv);
+#pragma unroll
+            for (int k = 0; k < VEC; ++k) o[k] = (wv[k] * gv[k] - (x[k] * inv_r) * kd) * pref;
+            st_vec<VEC>(orow + j, o);
+        }
+    }
+}
+
+__global__ void __launch_bounds__(kRowThreads)
+    lse_combine_kernel(const float2* __restrict__ part, int n_tiles, int T,
+                       const float* __restrict__ zy, float* __restrict__ lse, float* __restrict__ ce) {
+    const int lane = threadIdx.x & 31;
+    const int wpb = blockDim.x >> 5;
+    for (int row = blockIdx.x * wpb + (threadIdx.x >> 5); row < T; row += gridDim.x * wpb) {
+        const float2* pr = part + static_cast<size_t>(row) * n_tiles;
+        float m = -INFINITY;
+        for (int i = lane; i < n_tiles; i += 32) m = fmaxf(m, pr[i].x);
+        m = warp_max(m);
+        float s = 0.f;
+        for (int i = lane; i < n_tiles; i += 32) {
+            const float2 p = pr[i];
+            if (p.y > 0.f) s += p.y * expf(p.x - m);
+        }
+        s = warp_sum(s);
+        const float l = m + logf(s);
+        if (lane == 0) {
+            lse[row] = l;
+            if (ce) ce[row] = l - zy[row];
+        }
+    }
+}
+
+constexpr int kMeanThreads = 1024;
+
+__global__ void __launch_bounds__(kMeanThreads) mean_kernel(const float* __restrict__ x, int n,
+                                                            float* __restrict__ out) {
+    __shared__ double buf[kMeanThreads];
+    double acc = 0.0;
+    for (int i = threadIdx.x; i < n; i += kMeanThreads) acc += static_cast<double>(x[i]);
+    buf[threadIdx.x] = acc;
+    __syncthreads();
+    for (int s = kMeanThreads / 2; s > 0; s >>= 1) {
+        if (threadIdx.x < s) buf[threadIdx.x] += buf[threadIdx.x + s];
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) out[0] = static_cast<float>(buf[0] / static_cast<double>(n));
+}
+
+__global__ void cast_f32_kernel(const float* __restrict__ src, size_t n, __nv_bfloat16* __restrict__ dst) {
+    for (size_t i = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x; i < n;
+         i += static_cast<size_t>(gridDim.x) * blockDim.x)
+        dst[i] = __float2bfloat16_rn(src[i]);
+}
+
+int row_grid(int T) {
+    DevInfo di;
+    const int sms = current_device_info(&di) ? di.sm_count : 148;
+    const int wpb = kRowThreads / 32;
+    int blocks = (T + wpb - 1) / wpb;
+    const int cap = sms * 8;
+    return blocks < cap ? (blocks > 0 ? blocks : 1) : cap;
+}
+
+}  // namespace
+
+cudaError_t launch_rmsnorm_fwd(int dtype, const void* h, const void* w, int T, int d, float eps,
+                               void* yhat, float* rho, const int32_t* y, int V, unsigned* status,
+                               cudaStream_t st) {
+    if (T <= 0) return cudaSuccess;
+    const int grid = row_grid(T);
+    if (dtype == 1) {
+        rmsnorm_fwd_kernel<__nv_bfloat16, 8><<<grid, kRowThreads, 0, st>>>(
+            static_cast<const __nv_bfloat16*>(h), static_cast<const __nv_bfloat16*>(w), T, d, eps,
+            static_cast<__nv_bfloat16*>(yhat), rho, y, V, status);
+    } else if (d % 4 == 0) {
+        rmsnorm_fwd_kernel<float, 4><<<grid, kRowThreads, 0, st>>>(
+            static_cast<const float*>(h), static_cast<const float*>(w), T, d, eps,
+            static_cast<float*>(yhat), rho, y, V, status);
+    } else {
+        rmsnorm_fwd_kernel<float, 1><<<grid, kRowThreads, 0, st>>>(
+            static_cast<const float*>(h), static_cast<const float*>(w), T, d, eps,
+            static_cast<float*>(yhat), rho, y, V, status);
+    }
+    return cudaGetLastError();
+}
+
+cudaError_t launch_rmsnorm_vjp(int dtype, const float* g, const void* h, const void* w,
+                               const float* rho, int T, int d, float min_rms, void* out,
+                               cudaStream_t st) {
+    if (T <= 0) return cudaSuccess;
+    const int grid = row_grid(T);
+    if (dtype == 1) {
+        rmsnorm_vjp_kernel<__nv_bfloat16, 8><<<grid, kRowThreads, 0, st>>>(
+            g, static_cast<const __nv_bfloat16*>(h), static_cast<const __nv_bfloat16*>(w), rho, T,
+            d, min_rms, static_cast<__nv_bfloat16*>(out));
+    } else if (d % 4 == 0) {
+        rmsnorm_vjp_kernel<float, 4><<<grid, kRowThreads, 0, st>>>(
+            g, static_cast<const float*>(h), static_cast<const float*>(w), rho, T, d, min_rms,
+            static_cast<float*>(out));
+    } else {
+        rmsnorm_vjp_kernel<float, 1><<<grid, kRowThreads, 0, st>>>(
+            g, static_cast<const float*>(h), static_cast<const float*>(w), rho, T, d, min_rms,
+            static_cast<float*>(out));
+    }
+    return cudaGetLastError();
+}
+
+cudaError_t launch_cast_f32(int dtype, const float* src, size_t n, void* dst, cudaStream_t st) {
+    if (n == 0) return cudaSuccess;
+    if (dtype != 1) return cudaMemcpyAsync(dst, src, n * sizeof(float), cudaMemcpyDeviceToDevice, st);
+    cast_f32_kernel<<<row_grid(static_cast<int>((n + 255) / 256 * 8)), kRowThreads, 0, st>>>(
+        src, n, static_cast<__nv_bfloat16*>(dst));
+    return cudaGetLastError();
+}
+
+cudaError_t launch_lse_combine(const float2* part, int n_tiles, int T, const float* zy, float* lse,
+                               float* ce, cudaStream_t st) {
+    if (T <= 0) return cudaSuccess;
+    lse_combine_kernel<<<row_grid(T), kRowThreads, 0, st>>>(part, n_tiles, T, zy, lse, ce);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_mean(const float* x, int n, float* out, cudaStream_t st) {
+    if (n <= 0) return cudaSuccess;
+    mean_kernel<<<1, kMeanThreads, 0, st>>>(x, n, out);
+    return cudaGetLastError();
+}
+
+}  // namespace fpo

@@ -1,0 +1,119 @@
+"""The C-ABI library loads, exports every entry point include/fpo.h declares, and
+rejects bad arguments on the host before touching a device (no GPU needed)."""
+import ctypes
+import os
+import re
+import subprocess
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "fpo.h")
+LIB = os.path.join(ROOT, "paper_2608_14563_gb300", "libfpo.so")
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(fpo_[a-z0-9_]+)\s*\(", text)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for required in ("fpo_error_signal", "fpo_layer_update", "fpo_layer_update_grouped",
+                     "fpo_cosine", "fpo_get_device_status", "fpo_status_string",
+                     "fpo_error_signal_workspace", "fpo_layer_update_workspace",
+                     "fpo_cosine_workspace"):
+        assert required in names
+
+
+def test_library_exports_every_declared_symbol():
+    out = subprocess.run(["nm", "-D", "--defined-only", LIB], capture_output=True, text=True,
+                         check=True).stdout
+    exported = set(re.findall(r"\sT\s+(fpo_\w+)$", out, flags=re.M))
+    missing = [n for n in declared_functions() if n not in exported]
+    assert not missing, missing
+    lib = ctypes.CDLL(LIB)
+    for n in declared_functions():
+        assert hasattr(lib, n)
+
+
+def test_binding_loads_and_reports_version():
+    import paper_2608_14563_gb300 as fpo
+    assert fpo.abi_version() == 1
+    assert fpo.status_string(0) == "FPO_OK"
+    assert "TARGET_RANGE" in fpo.status_string(8)
+    assert fpo.status_string(12345) == "unknown fpo status"
+
+
+class _Lib:
+    def __init__(self):
+        import paper_2608_14563_gb300 as fpo
+        self.fpo = fpo
+        self.lib = fpo._lib
+
+
+@pytest.fixture(scope="module")
+def L():
+    return _Lib()
+
+
+def test_error_signal_workspace_query(L):
+    fpo = L.fpo
+    small = fpo.error_signal_desc(128, 64, 512, fpo.F32)
+    chunked = fpo.error_signal_desc(4096, 4096, 151936, fpo.BF16, t_chunk=1024)
+    full = fpo.error_signal_desc(4096, 4096, 151936, fpo.BF16)
+    assert fpo.error_signal_workspace(small) > 0
+    assert fpo.error_signal_workspace(chunked) < fpo.error_signal_workspace(full)
+    # E chunk is Tc x V bf16: the difference is exactly (4096 - 1024) * V * 2 bytes (256-aligned)
+    diff = fpo.error_signal_workspace(full) - fpo.error_signal_workspace(chunked)
+    assert abs(diff - 3072 * 151936 * 2) < 512
+    bad = fpo.error_signal_desc(16, 12, 512, fpo.BF16)  # d not a multiple of 8
+    assert fpo.error_signal_workspace(bad) == 0
+    assert L.lib.fpo_error_signal_workspace(None) == 0
+
+
+def test_error_signal_host_validation(L):
+    fpo = L.fpo
+    lib = L.lib
+    desc = fpo.error_signal_desc(16, 64, 256, fpo.BF16)
+    ws = fpo.error_signal_workspace(desc)
+    fake = ctypes.c_void_p(1 << 20)   # never dereferenced: validation fails first
+    mis = ctypes.c_void_p((1 << 20) + 8)
+    call = lambda d, h=fake, ws_ptr=fake, ws_n=ws, g=fake: lib.fpo_error_signal(
+        ctypes.byref(d) if d is not None else None, h, fake, fake, fake, g, None, None, ws_ptr, ws_n,
+        None)
+    assert call(None) == 1                                            # FPO_ERR_NULL
+    assert call(fpo.error_signal_desc(16, 64, 256, 7)) == 3           # FPO_ERR_DTYPE
+    assert call(fpo.error_signal_desc(-1, 64, 256, fpo.BF16)) == 2    # FPO_ERR_SHAPE
+    assert call(fpo.error_signal_desc(16, 60, 256, fpo.BF16)) == 2    # d % 8
+    assert call(fpo.error_signal_desc(16, 64, 250, fpo.BF16)) == 2    # V % 8
+    assert call(desc, h=None) == 1
+    assert call(desc, h=mis) == 4                                     # FPO_ERR_ALIGN
+    assert call(desc, ws_ptr=None) == 5                               # FPO_ERR_WORKSPACE
+    assert call(desc, ws_n=ws - 1) == 5
+    assert call(desc, g=mis) == 4
+
+
+def test_layer_update_and_cosine_host_validation(L):
+    lib = L.lib
+    fake = ctypes.c_void_p(1 << 20)
+    mis = ctypes.c_void_p((1 << 20) + 4)
+    ws = L.fpo.layer_update_workspace()
+    assert lib.fpo_layer_update(16, 64, 128, 9, fake, fake, 0.1, fake, None, None, fake, ws, None) == 3
+    assert lib.fpo_layer_update(16, 64, 100, 1, fake, fake, 0.1, fake, None, None, fake, ws, None) == 2
+    assert lib.fpo_layer_update(16, 64, 128, 1, fake, fake, 0.1, None, None, None, fake, ws, None) == 1
+    assert lib.fpo_layer_update(16, 64, 128, 1, fake, fake, 0.1, None, fake, fake, fake, ws, None) == 1
+    assert lib.fpo_layer_update(16, 64, 128, 1, fake, mis, 0.1, fake, None, None, fake, ws, None) == 4
+    assert lib.fpo_layer_update(16, 64, 128, 1, fake, fake, 0.1, fake, None, None, None, ws, None) == 5
+    assert lib.fpo_layer_update(16, 64, 128, 1, fake, fake, 0.1, fake, None, None, fake, 8, None) == 5
+    arr = (ctypes.c_void_p * 1)(fake.value)
+    assert lib.fpo_layer_update_grouped(0, 16, 64, 128, 1, fake, arr, 0.1, arr, None, None, fake,
+                                        ws, None) == 2
+    assert lib.fpo_layer_update_grouped(65, 16, 64, 128, 1, fake, arr, 0.1, arr, None, None, fake,
+                                        ws, None) == 2
+    assert lib.fpo_cosine(-1, 1, fake, fake, fake, fake, 1 << 20, None) == 2
+    assert lib.fpo_cosine(10, 5, fake, fake, fake, fake, 1 << 20, None) == 3
+    assert lib.fpo_cosine(10, 1, None, fake, fake, fake, 1 << 20, None) == 1
+    assert lib.fpo_cosine(10, 1, mis, fake, fake, fake, 1 << 20, None) == 4
+    assert lib.fpo_get_device_status(None, None) == 5
