@@ -1,0 +1,445 @@
+#!/usr/bin/env python
+"""Throughput of the FPO pseudogradient update on GB300.
+
+One step = fpo_error_signal (final RMSNorm forward, logits pass with the
+log-sum-exp, recompute pass writing E = s(softmax - onehot), projection
+g = E W_U, final-norm VJP) + fpo_layer_update_grouped over every target layer
+(G_l = g~^T A_l, W_master -= lr G_l, bf16 weights out), on the synthetic
+OLMo-2-7B-shaped workload by default.  Prints one JSON line on rank 0.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl fpo|reference]
+
+N > 1 runs N independent replicas (one per GPU, launched by torch.distributed.run):
+the path has no exchange step between replicas, so there is no collective on the
+data path; a barrier and a max over ranks bracket the timing.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "FPO update tokens/s and TFLOP/s at 1 GB300; fraction of dense BF16 roofline"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+# --------------------------------------------------------------------------- helpers
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            p = json.load(f)
+        return p, "measured"
+    return dict(FALLBACK_PEAKS), "fallback"
+
+
+def algorithmic_flops(wl):
+    """4 T V d (logits once + projection) + 2 L T d d_ff."""
+    return 4.0 * wl.T * wl.V * wl.d + 2.0 * wl.layers * wl.T * wl.d * wl.d_ff
+
+
+def executed_flops(wl):
+    """Adds the second logits GEMM of the two-pass (recompute) design: + 2 T V d."""
+    return algorithmic_flops(wl) + 2.0 * wl.T * wl.V * wl.d
+
+
+def algorithmic_bytes(wl):
+    esz = 2 if wl.dtype == "bf16" else 4
+    return (wl.T * wl.d * esz + wl.V * wl.d * esz + wl.layers * wl.T * wl.d_ff * esz + wl.T * 4
+            + wl.T * wl.d * esz + wl.layers * wl.d * wl.d_ff * (4 + 4 + esz))
+
+
+class ClockSampler:
+    """nvidia-smi clocks / throttle reasons sampled during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index):
+        self.dev = device_index
+        self.proc = None
+        self.out = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.dev), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, mx, reasons, power = [], None, set(), []
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.strip().splitlines():
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx = float(parts[2])
+                power.append(float(parts[3]))
+            except ValueError:
+                continue
+            for name, val in zip(names, parts[5:9]):
+                if val.lower() == "active":
+                    reasons.add(name)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": mx, "reasons": ["no samples"]}
+        loaded = [s for s, p in zip(sm, power) if p > 0.5 * max(power)] or sm
+        return {"sm_mhz": statistics.median(loaded), "sm_max_mhz": mx,
+                "reasons": sorted(reasons), "samples": len(sm),
+                "power_w_max": max(power) if power else None}
+
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+# --------------------------------------------------------------------------- oracle baseline
+_CPU_INPUTS = {}
+
+
+def _cpu_inputs(wl):
+    """The workload's inputs generated once on the host (seeded, as on the device)."""
+    from paper_2608_14563_gb300 import synth
+    if wl.name not in _CPU_INPUTS:
+        _CPU_INPUTS[wl.name] = {
+            "h": synth.make_h(wl), "w": synth.make_norm_w(wl), "W_U": synth.make_W_U(wl),
+            "y": synth.make_targets(wl), "A0": synth.make_A(wl, 0),
+            "W0": synth.make_W_master(wl, 0).numpy()}
+    return _CPU_INPUTS[wl.name]
+
+
+def oracle_sample(wl, n_tok, seed=0):
+    """Time the fp64 CPU oracle on n_tok tokens of the workload and extrapolate to one
+    step of T tokens: t_step = T * (per-token error signal + per-token G accumulation)
+    + per-step weight update.  Inputs come from the same seeded generators."""
+    import torch
+
+    import oracle
+    from paper_2608_14563_gb300 import synth
+
+    oracle.build()
+    inp = _cpu_inputs(wl)
+    n_tok = min(n_tok, wl.T)
+    gen = torch.Generator().manual_seed(1234 + seed)
+    rows = torch.randperm(wl.T, generator=gen)[:n_tok].sort().values
+    hn = synth.to_numpy_exact(inp["h"][rows])
+    wn = synth.to_numpy_exact(inp["w"])
+    Un = synth.to_numpy_exact(inp["W_U"])
+    An = synth.to_numpy_exact(inp["A0"][rows])
+    yn = inp["y"][rows].numpy()
+
+    t0 = time.perf_counter()
+    es = oracle.error_signal(hn, wn, Un, yn, eps=wl.eps, min_rms=wl.min_rms, s=1.0 / wl.T)
+    t1 = time.perf_counter()
+    G = oracle.pseudograd(es["g_tilde"], An)
+    t2 = time.perf_counter()
+    oracle.sgd_update(inp["W0"], G, wl.lr)
+    t3 = time.perf_counter()
+    per_tok = (t1 - t0) / n_tok + wl.layers * (t2 - t1) / n_tok
+    step_s = wl.T * per_tok + wl.layers * (t3 - t2)
+    return {"sample_s": t3 - t0, "step_s": step_s, "tokens_per_s": wl.T / step_s,
+            "n_tok": n_tok, "es_s": t1 - t0, "G_s": t2 - t1, "upd_s": t3 - t2}
+
+
+def cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count()
+
+
+def sample_text(r, wl):
+    return (f"{r['n_tok']} of {wl.T} tokens through the oracle (error signal {r['es_s']:.2f} s, "
+            f"G for 1 of {wl.layers} layers {r['G_s']:.2f} s, one weight update {r['upd_s']:.2f} s),"
+            f" extrapolated to one {wl.T}-token step of {wl.layers} layers: "
+            f"T*(t_es+L*t_G)/n + L*t_upd")
+
+
+def run_reference(args, wl):
+    world, rank, _ = dist_setup()
+    if rank != 0:
+        return
+    n_tok = args.cpu_tokens
+    steps = []
+    for i in range(args.warmup + args.steps):
+        r = oracle_sample(wl, n_tok, seed=i)
+        if i >= args.warmup:
+            steps.append(r)
+    step_s = statistics.median(r["step_s"] for r in steps)
+    value = wl.T / step_s
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": step_s * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": workload_config(wl, args),
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores(), "kind": "oracle",
+                         "sample": sample_text(steps[-1], wl)},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def workload_config(wl, args):
+    return {"workload": wl.name, "T": wl.T, "d": wl.d, "d_ff": wl.d_ff, "V": wl.V,
+            "target_layers": wl.layers, "targets": "zipf(1.1)" if wl.targets == "zipf" else wl.targets,
+            "lr": wl.lr, "t_chunk": args.t_chunk or wl.T, "global_batch_tokens": wl.T * args.gpus,
+            "l2": "inputs larger than L2 (W_U %.0f MB, A_l %.2f GB per step); no flush"
+                  % (wl.V * wl.d * 2 / 1e6, wl.layers * wl.T * wl.d_ff * 2 / 1e9)}
+
+
+# --------------------------------------------------------------------------- GPU arm
+def run_fpo(args, wl):
+    import torch
+    import torch.distributed as dist
+
+    world, rank, local = dist_setup()
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+
+    import paper_2608_14563_gb300 as fpo
+    from paper_2608_14563_gb300 import synth
+
+    wl_r = synth.Workload(wl.name, T=wl.T, d=wl.d, d_ff=wl.d_ff, V=wl.V, layers=wl.layers,
+                          dtype=wl.dtype, targets=wl.targets, lr=wl.lr, seed=rank)
+    dev = torch.device("cuda", local)
+    h = synth.make_h(wl_r, dev)
+    w = synth.make_norm_w(wl_r, dev)
+    W_U = synth.make_W_U(wl_r, dev)
+    y = synth.make_targets(wl_r, dev)
+    A = [synth.make_A(wl_r, l, dev) for l in range(wl.layers)]
+    Wm = [synth.make_W_master(wl_r, l, dev) for l in range(wl.layers)]
+    Wo = [torch.empty(wl.d, wl.d_ff, dtype=torch.bfloat16, device=dev) for _ in range(wl.layers)]
+    g = torch.empty_like(h)
+    loss = torch.empty(1, dtype=torch.float32, device=dev)
+    desc = fpo.error_signal_desc(wl.T, wl.d, wl.V, fpo.BF16, eps=wl.eps, min_rms=wl.min_rms,
+                                 t_chunk=args.t_chunk)
+    ws_es = torch.empty(fpo.error_signal_workspace(desc), dtype=torch.uint8, device=dev)
+    ws_up = torch.empty(fpo.layer_update_workspace(), dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+
+    n_chunks = -(-wl.T // (args.t_chunk or wl.T))
+    launches_per_step = 4 + 2 * n_chunks + 1 + 1  # fwd, lse, combine, mean, chunks, vjp, update
+
+    def step(stage_events=None, upd_events=None):
+        fpo.error_signal(h, w, W_U, y, g, eps=wl.eps, min_rms=wl.min_rms, t_chunk=args.t_chunk,
+                         loss_out=loss, workspace=ws_es, stage_events=stage_events)
+        if upd_events:
+            upd_events[0].record(stream)
+        fpo.layer_update_grouped(g, A, wl.lr, W_masters=Wm, W_outs=Wo, workspace=ws_up)
+        if upd_events:
+            upd_events[1].record(stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    assert fpo.get_device_status(ws_es) == fpo.OK and fpo.get_device_status(ws_up) == fpo.OK
+
+    # per-stage events for every timed step (recorded once so their handles exist)
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(fpo.STAGE_EVENTS)]
+          for _ in range(args.steps)]
+    uev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(args.steps)]
+    for e in [x for row in ev + uev for x in row]:
+        e.record(stream)
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clocks = ClockSampler(local)
+    clocks.start()
+    time.sleep(0.3)
+    start.record(stream)
+    for i in range(args.steps):
+        step(ev[i], uev[i])
+    end.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    if world > 1:
+        dist.barrier()
+    ms = start.elapsed_time(end) / args.steps
+    status = (fpo.get_device_status(ws_es), fpo.get_device_status(ws_up))
+
+    names = ["rmsnorm_fwd", "logits_lse_pass", "lse_combine", "recompute_error_pass",
+             "projection", "rmsnorm_vjp"]
+    stage_ms = {n: statistics.mean(ev[i][k].elapsed_time(ev[i][k + 1]) for i in range(args.steps))
+                for k, n in enumerate(names)}
+    stage_ms["layer_update"] = statistics.mean(uev[i][0].elapsed_time(uev[i][1])
+                                               for i in range(args.steps))
+
+    # ------------------------------------------------ end to end through the public API
+    e2e = None
+    if not args.no_e2e:
+        h_host = h.cpu().pin_memory()
+        y_host = y.cpu().pin_memory()
+        A_host = [a.cpu().pin_memory() for a in A]
+        loss_host = torch.empty(1, dtype=torch.float32).pin_memory()
+
+        def e2e_step():
+            h.copy_(h_host, non_blocking=True)
+            y.copy_(y_host, non_blocking=True)
+            for a_d, a_h in zip(A, A_host):
+                a_d.copy_(a_h, non_blocking=True)
+            step()
+            loss_host.copy_(loss, non_blocking=True)
+
+        for _ in range(max(1, args.warmup)):
+            e2e_step()
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+        s2, e2 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s2.record(stream)
+        for _ in range(args.steps):
+            e2e_step()
+        e2.record(stream)
+        torch.cuda.synchronize()
+        e2e_ms = s2.elapsed_time(e2) / args.steps
+        if world > 1:
+            t = torch.tensor([e2e_ms], device=dev)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            e2e_ms = t.item()
+        h2d = (h.numel() * h.element_size() + y.numel() * 4
+               + sum(a.numel() * a.element_size() for a in A))
+        e2e = {"value": wl.T * world / (e2e_ms / 1e3), "unit": "tokens/s",
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": 4, "ms_per_step": e2e_ms}
+
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = t.item()
+
+    if rank == 0:
+        peaks, peaks_src = load_peaks()
+        tok_s = wl.T * world / (ms / 1e3)
+        alg_tf = algorithmic_flops(wl) / (ms / 1e3) / 1e12
+        exe_tf = executed_flops(wl) / (ms / 1e3) / 1e12
+        per_kernel_flops = {
+            "logits_lse_pass": 2.0 * wl.T * wl.V * wl.d,
+            "recompute_error_pass": 2.0 * wl.T * wl.V * wl.d,
+            "projection": 2.0 * wl.T * wl.V * wl.d,
+            "layer_update": 2.0 * wl.layers * wl.T * wl.d * wl.d_ff,
+        }
+        # dominant kernel among those whose work is algorithmic (the recompute is overhead)
+        dom = max(("logits_lse_pass", "projection", "layer_update"), key=lambda k: stage_ms[k])
+        peak_sus = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
+        achieved = per_kernel_flops[dom] / (stage_ms[dom] / 1e3) / 1e12
+        roofline = {"bound": "tensor", "achieved": achieved, "peak": peak_sus, "unit": "TFLOP/s",
+                    "frac": achieved / peak_sus, "traffic": load_traffic(dom),
+                    "kernel": dom, "peak_kind": f"bf16 sustained ({peaks_src})"}
+        cpu = None
+        if world == 1 and not args.no_cpu:
+            r = oracle_sample(wl, args.cpu_tokens)
+            cpu = {"value": r["tokens_per_s"], "unit": "tokens/s", "cores": cores(),
+                   "kind": "oracle", "sample": sample_text(r, wl)}
+        line = {
+            "metric": METRIC, "value": tok_s, "unit": "tokens/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic (seeded; OLMo-2-7B shapes, random weights and activations)",
+            "config": workload_config(wl, args),
+            "tflops": {"algorithmic": alg_tf, "executed": exe_tf,
+                       "frac_of_bf16_peak_burst": alg_tf / peaks.get("bf16_tflops", 1900.0),
+                       "frac_of_bf16_peak_sustained": alg_tf / peak_sus,
+                       "peaks": peaks_src},
+            "roofline": roofline,
+            "kernels_ms": stage_ms,
+            "kernels_tflops": {k: per_kernel_flops[k] / (stage_ms[k] / 1e3) / 1e12
+                               for k in per_kernel_flops},
+            "cpu_baseline": cpu,
+            "e2e": e2e,
+            "gpu_launches": launches_per_step * args.steps,
+            "clocks": clk,
+            "device_status": list(status),
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def load_traffic(kernel):
+    """Per-launch DRAM bytes of `kernel` from the committed ncu summary, or None when that
+    summary is missing or was taken on different kernel sources."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(path):
+        return None
+    with open(path) as f:
+        tr = json.load(f)
+    ent = tr.get(kernel)
+    if not ent or ent.get("sources_sha256") != sources_digest():
+        return None
+    return ent.get("bytes_per_launch")
+
+
+def sources_digest():
+    import hashlib
+    csrc = os.path.join(ROOT, "paper_2608_14563_gb300", "csrc")
+    hsh = hashlib.sha256()
+    for name in sorted(os.listdir(csrc)):
+        if name.endswith((".cu", ".cuh", ".h")):
+            with open(os.path.join(csrc, name), "rb") as f:
+                hsh.update(name.encode() + f.read())
+    return hsh.hexdigest()
+
+
+def ensure_built():
+    """Compile libfpo.so in-tree when it is missing (the package refuses to load without it)."""
+    import importlib.util
+    spec = importlib.util.spec_from_file_location(
+        "_fpo_build", os.path.join(ROOT, "paper_2608_14563_gb300", "build.py"))
+    b = importlib.util.module_from_spec(spec)
+    spec.loader.exec_module(b)
+    b.build()
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=("fpo", "reference"), default="fpo")
+    ap.add_argument("--workload", default="olmo", help="olmo | qwen | falcon | diag")
+    ap.add_argument("--t-chunk", type=int, default=0, help="tokens per E chunk (0 = all)")
+    ap.add_argument("--cpu-tokens", type=int, default=16, help="oracle sample size (tokens)")
+    ap.add_argument("--no-cpu", action="store_true", help="skip the oracle CPU baseline")
+    ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end run")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+
+    ensure_built()
+    from paper_2608_14563_gb300.synth import WORKLOADS  # noqa: E402  (after the build)
+    wl = WORKLOADS[args.workload]
+    if args.impl == "reference":
+        run_reference(args, wl)
+    else:
+        run_fpo(args, wl)
+
+
+if __name__ == "__main__":
+    main()

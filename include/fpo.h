@@ -80,7 +80,20 @@ typedef struct fpo_error_signal_desc {
     float min_rms;      /* floor on rho in the 1/rho prefactor of the VJP (0.5)  */
     float loss_scale;   /* s in e = s (softmax(z) - 1_y); 1/T = mean-reduced CE */
     int64_t t_chunk;    /* tokens per error-matrix chunk; 0 = all T at once       */
+    void* const* stage_events;  /* NULL, or FPO_STAGE_EVENTS caller-created
+                                   cudaEvent_t recorded on the stream at the stage
+                                   boundaries (profiling; see below)              */
 } fpo_error_signal_desc;
+
+/*
+ * Stage boundaries of fpo_error_signal at which desc->stage_events[i] is
+ * recorded: 0 start, 1 after the RMSNorm forward, 2 after the logits pass,
+ * 3 after the log-sum-exp combine (and loss), 4 after the recompute pass of
+ * the last token chunk, 5 after the projection of the last token chunk,
+ * 6 after the final-norm VJP.  With one chunk, [4]-[3] and [5]-[4] time the
+ * recompute and projection GEMMs alone.
+ */
+#define FPO_STAGE_EVENTS 7
 
 /* Bytes of workspace fpo_error_signal needs for `desc` (0 on a bad desc). */
 size_t fpo_error_signal_workspace(const fpo_error_signal_desc* desc);

@@ -177,9 +177,15 @@ int32_t fpo_error_signal(const fpo_error_signal_desc* desc, const void* h, const
     float* g = reinterpret_cast<float*>(ws + L.g);
     void* E = ws + L.E;
 
+    auto mark = [&](int i) -> cudaError_t {
+        if (!desc->stage_events || !desc->stage_events[i]) return cudaSuccess;
+        return cudaEventRecord(static_cast<cudaEvent_t>(desc->stage_events[i]), st);
+    };
+    FPO_TRY(mark(0));
     // 1. final RMSNorm forward: rho, yhat (and the target-range check)
     FPO_TRY(launch_rmsnorm_fwd(desc->dtype, h, norm_w, T, d, desc->eps, yhat, rho, targets, V,
                                status, st));
+    FPO_TRY(mark(1));
     // 2. logits pass: per-vocabulary-tile (max, sum exp) partials -> lse
     if (bf16)
         FPO_TRY(launch_lse_partial_bf16(yhat, W_U, targets, T, d, V, part, L.n_tiles, zy, status,
@@ -188,8 +194,10 @@ int32_t fpo_error_signal(const fpo_error_signal_desc* desc, const void* h, const
         FPO_TRY(launch_lse_partial_f32(static_cast<const float*>(yhat),
                                        static_cast<const float*>(W_U), targets, T, d, V, part,
                                        L.n_tiles, zy, st));
+    FPO_TRY(mark(2));
     FPO_TRY(launch_lse_combine(part, L.n_tiles, T, zy, lse, ce, st));
     if (loss_out) FPO_TRY(launch_mean(ce, T, loss_out, st));
+    FPO_TRY(mark(3));
     // 3./4. per token chunk: recompute logits -> E, then g = E W_U
     for (int64_t c0 = 0; c0 < T; c0 += L.Tc) {
         const int tc = static_cast<int>(L.Tc < T - c0 ? L.Tc : T - c0);
@@ -197,17 +205,21 @@ int32_t fpo_error_signal(const fpo_error_signal_desc* desc, const void* h, const
         if (bf16) {
             FPO_TRY(launch_error_bf16(yh, W_U, targets + c0, lse + c0, tc, d, V,
                                       desc->loss_scale, E, status, st));
+            if (c0 + tc >= T) FPO_TRY(mark(4));
             FPO_TRY(launch_proj_bf16(E, W_U, tc, d, V, g + c0 * d, status, st));
         } else {
             FPO_TRY(launch_error_f32(static_cast<const float*>(yh), static_cast<const float*>(W_U),
                                      targets + c0, lse + c0, tc, d, V, desc->loss_scale,
                                      static_cast<float*>(E), st));
+            if (c0 + tc >= T) FPO_TRY(mark(4));
             FPO_TRY(launch_proj_f32(static_cast<const float*>(E), static_cast<const float*>(W_U),
                                     tc, d, V, g + c0 * d, st));
         }
     }
+    FPO_TRY(mark(5));
     // 5. final-norm VJP with the min-RMS clamp -> g~
     FPO_TRY(launch_rmsnorm_vjp(desc->dtype, g, h, norm_w, rho, T, d, desc->min_rms, g_out, st));
+    FPO_TRY(mark(6));
     return FPO_OK;
 }
 
