@@ -180,6 +180,34 @@ int32_t fpo_cosine(int64_t n, int32_t dtype, const void* X, const void* Y, doubl
                    void* workspace, size_t workspace_bytes, void* stream);
 
 /*
+ * fpo_cosine_noalloc -- fpo_cosine for callers that cannot allocate device
+ * memory: code running where cudaMalloc is off limits or would break the
+ * caller's own memory accounting (inside another runtime's fixed memory pool,
+ * a custom allocator, an embedded or real-time loop), which also has no
+ * workspace to hand in.  The paper has no counterpart; this is a property of
+ * the library, not of the method.
+ *
+ * Same inputs, output and result as fpo_cosine (bit-identical: the same
+ * kernels, block count and summation order), but the pass-1 partial sums live
+ * in a static device array inside libfpo of 1024 fp64 triples (24 KiB, held by
+ * every GPU that loads the library until the process exits).  A call needs
+ * cosine-blocks(n) <= 2 x SM count slots (304 on GB300, for any n); a device
+ * whose launch would need more than 1024 returns FPO_ERR_WORKSPACE and
+ * enqueues nothing.  The call allocates nothing: no cudaMalloc, no cudaFree,
+ * no allocating library routine.
+ *
+ * - The first call on each device looks up the array's device address
+ *   (cudaGetSymbolAddress) with that device current; make that first call
+ *   before any stream capture.
+ * - All calls on a device share the one array, which keeps the last call's
+ *   partials.  Every slot a call reads is written by the same call first, so
+ *   nothing needs clearing, but two calls that overlap on the GPU (different
+ *   streams, or different host threads) race on the array: serialise them.
+ */
+int32_t fpo_cosine_noalloc(int64_t n, int32_t dtype, const void* X, const void* Y, double* out,
+                           void* stream);
+
+/*
  * Synchronise `stream`, read the device status word of `workspace` (set by the
  * last call that used it), clear it, and return FPO_OK, FPO_ERR_TARGET_RANGE
  * or FPO_ERR_TIMEOUT (the first of the two when both are set).

@@ -177,3 +177,75 @@ cudaError_t launch_cosine(int dtype, int64_t n, const void* X, const void* Y, do
 }
 
 }  // namespace fpo
+
+// ---------------------------------------------------------------------------
+// fpo_cosine_noalloc: the same two-pass reduction, for callers that cannot
+// allocate device memory (no cudaMalloc, no caching allocator, no caller-side
+// workspace), with its scratch -- one fp64 triple of partial sums per block of
+// pass 1 -- in a fixed, file-scope device array instead of a workspace.
+#include <mutex>
+
+#include "../../include/fpo.h"
+
+namespace fpo {
+namespace {
+
+// Partial-sum slots the static scratch holds: pass 1 of a call uses
+// cosine_blocks(n) <= 2 x SM count of them (304 on a 152-SM GB300).
+constexpr int kNoAllocSlots = 1024;
+
+// 24 KiB of device memory, held by every GPU that loads the library until exit.
+static __device__ __align__(256) double g_cosine_noalloc_scratch[3 * kNoAllocSlots];
+
+struct NoAllocScratch {
+    std::once_flag once;
+    double* ptr = nullptr;
+    cudaError_t err = cudaSuccess;
+};
+NoAllocScratch g_noalloc_scratch[64];
+
+// Device address of the static scratch on the current device.  In host code the
+// array's name is only a host-side stand-in, so the address is looked up once per
+// device, with that device current.
+cudaError_t noalloc_scratch(double** out) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    NoAllocScratch& s = g_noalloc_scratch[dev];
+    std::call_once(s.once, [&s] {
+        void* p = nullptr;
+        s.err = cudaGetSymbolAddress(&p, g_cosine_noalloc_scratch);
+        s.ptr = static_cast<double*>(p);
+    });
+    if (s.err != cudaSuccess) return s.err;
+    *out = s.ptr;
+    return cudaSuccess;
+}
+
+}  // namespace
+}  // namespace fpo
+
+extern "C" int32_t fpo_cosine_noalloc(int64_t n, int32_t dtype, const void* X, const void* Y,
+                                      double* out, void* stream) {
+    if (dtype != FPO_F32 && dtype != FPO_BF16) return FPO_ERR_DTYPE;
+    if (n < 0) return FPO_ERR_SHAPE;
+    if (!out || (n > 0 && (!X || !Y))) return FPO_ERR_NULL;
+    if ((reinterpret_cast<uintptr_t>(X) & 15u) || (reinterpret_cast<uintptr_t>(Y) & 15u) ||
+        (reinterpret_cast<uintptr_t>(out) & 7u))
+        return FPO_ERR_ALIGN;
+    fpo::DevInfo di;
+    if (!fpo::current_device_info(&di)) return FPO_ERR_CUDA;
+    if (di.major != 10 || di.minor != 3) return FPO_ERR_ARCH;
+    const int blocks = fpo::cosine_blocks(n);
+    if (blocks > fpo::kNoAllocSlots) return FPO_ERR_WORKSPACE;  // more partials than slots
+    double* scratch = nullptr;
+    if (fpo::noalloc_scratch(&scratch) != cudaSuccess) return FPO_ERR_CUDA;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (n == 0)
+        return cudaMemsetAsync(out, 0, 4 * sizeof(double), st) == cudaSuccess ? FPO_OK
+                                                                               : FPO_ERR_CUDA;
+    return fpo::launch_cosine(dtype, n, X, Y, scratch, blocks, out, st) == cudaSuccess
+               ? FPO_OK
+               : FPO_ERR_CUDA;
+}
