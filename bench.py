@@ -425,6 +425,8 @@ def main():
     ap.add_argument("--impl", choices=("fpo", "reference"), default="fpo")
     ap.add_argument("--workload", default="olmo", help="olmo | qwen | falcon | diag")
     ap.add_argument("--t-chunk", type=int, default=0, help="tokens per E chunk (0 = all)")
+    ap.add_argument("--shape", default=None,
+                    help="T,d,d_ff,V,layers override of the workload's shape (small ncu cases)")
     ap.add_argument("--cpu-tokens", type=int, default=16, help="oracle sample size (tokens)")
     ap.add_argument("--no-cpu", action="store_true", help="skip the oracle CPU baseline")
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end run")
@@ -435,6 +437,11 @@ def main():
     ensure_built()
     from paper_2608_14563_gb300.synth import WORKLOADS  # noqa: E402  (after the build)
     wl = WORKLOADS[args.workload]
+    if args.shape:
+        import dataclasses
+        T, d, d_ff, V, L = (int(x) for x in args.shape.split(","))
+        wl = dataclasses.replace(wl, name=f"{wl.name}@{T}x{d}x{d_ff}x{V}x{L}", T=T, d=d, d_ff=d_ff,
+                                 V=V, layers=L)
     if args.impl == "reference":
         run_reference(args, wl)
     else:
