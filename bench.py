@@ -209,6 +209,8 @@ def workload_config(wl, args):
     return {"workload": wl.name, "T": wl.T, "d": wl.d, "d_ff": wl.d_ff, "V": wl.V,
             "target_layers": wl.layers, "targets": "zipf(1.1)" if wl.targets == "zipf" else wl.targets,
             "lr": wl.lr, "t_chunk": args.t_chunk or wl.T, "global_batch_tokens": wl.T * args.gpus,
+            "error_matrix": {"auto": "stored-logits (auto)", "recompute": "recompute",
+                             "stored": "stored-logits"}[args.algo],
             "l2": "inputs larger than L2 (W_U %.0f MB, A_l %.2f GB per step); no flush"
                   % (wl.V * wl.d * 2 / 1e6, wl.layers * wl.T * wl.d_ff * 2 / 1e9)}
 
@@ -238,18 +240,23 @@ def run_fpo(args, wl):
     Wo = [torch.empty(wl.d, wl.d_ff, dtype=torch.bfloat16, device=dev) for _ in range(wl.layers)]
     g = torch.empty_like(h)
     loss = torch.empty(1, dtype=torch.float32, device=dev)
+    algo = {"auto": fpo.ES_AUTO, "recompute": fpo.ES_RECOMPUTE,
+            "stored": fpo.ES_STORED_LOGITS}[args.algo]
+    stored = algo != fpo.ES_RECOMPUTE
     desc = fpo.error_signal_desc(wl.T, wl.d, wl.V, fpo.BF16, eps=wl.eps, min_rms=wl.min_rms,
-                                 t_chunk=args.t_chunk)
+                                 t_chunk=args.t_chunk, algo=algo)
     ws_es = torch.empty(fpo.error_signal_workspace(desc), dtype=torch.uint8, device=dev)
     ws_up = torch.empty(fpo.layer_update_workspace(), dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream()
 
     n_chunks = -(-wl.T // (args.t_chunk or wl.T))
-    launches_per_step = 4 + 2 * n_chunks + 1 + 1  # fwd, lse, combine, mean, chunks, vjp, update
+    # fwd, mean, vjp, update + per chunk (stored: logits, combine, E, projection;
+    # recompute: E pass, projection; plus one logits pass and one combine)
+    launches_per_step = 4 + (4 * n_chunks if stored else 2 + 2 * n_chunks)
 
     def step(stage_events=None, upd_events=None):
         fpo.error_signal(h, w, W_U, y, g, eps=wl.eps, min_rms=wl.min_rms, t_chunk=args.t_chunk,
-                         loss_out=loss, workspace=ws_es, stage_events=stage_events)
+                         loss_out=loss, workspace=ws_es, stage_events=stage_events, algo=algo)
         if upd_events:
             upd_events[0].record(stream)
         fpo.layer_update_grouped(g, A, wl.lr, W_masters=Wm, W_outs=Wo, workspace=ws_up)
@@ -285,8 +292,8 @@ def run_fpo(args, wl):
     ms = start.elapsed_time(end) / args.steps
     status = (fpo.get_device_status(ws_es), fpo.get_device_status(ws_up))
 
-    names = ["rmsnorm_fwd", "logits_lse_pass", "lse_combine", "recompute_error_pass",
-             "projection", "rmsnorm_vjp"]
+    names = ["rmsnorm_fwd", "logits_lse_pass", "lse_combine",
+             "logits_to_error" if stored else "recompute_error_pass", "projection", "rmsnorm_vjp"]
     stage_ms = {n: statistics.mean(ev[i][k].elapsed_time(ev[i][k + 1]) for i in range(args.steps))
                 for k, n in enumerate(names)}
     stage_ms["layer_update"] = statistics.mean(uev[i][0].elapsed_time(uev[i][1])
@@ -338,13 +345,14 @@ def run_fpo(args, wl):
         peaks, peaks_src = load_peaks()
         tok_s = wl.T * world / (ms / 1e3)
         alg_tf = algorithmic_flops(wl) / (ms / 1e3) / 1e12
-        exe_tf = executed_flops(wl) / (ms / 1e3) / 1e12
+        exe_tf = (executed_flops(wl) if not stored else algorithmic_flops(wl)) / (ms / 1e3) / 1e12
         per_kernel_flops = {
             "logits_lse_pass": 2.0 * wl.T * wl.V * wl.d,
-            "recompute_error_pass": 2.0 * wl.T * wl.V * wl.d,
             "projection": 2.0 * wl.T * wl.V * wl.d,
             "layer_update": 2.0 * wl.layers * wl.T * wl.d * wl.d_ff,
         }
+        if not stored:
+            per_kernel_flops["recompute_error_pass"] = 2.0 * wl.T * wl.V * wl.d
         # dominant kernel among those whose work is algorithmic (the recompute is overhead)
         dom = max(("logits_lse_pass", "projection", "layer_update"), key=lambda k: stage_ms[k])
         peak_sus = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
@@ -371,6 +379,7 @@ def run_fpo(args, wl):
             "kernels_ms": stage_ms,
             "kernels_tflops": {k: per_kernel_flops[k] / (stage_ms[k] / 1e3) / 1e12
                                for k in per_kernel_flops},
+            "algo": "stored-logits" if stored else "recompute",
             "cpu_baseline": cpu,
             "e2e": e2e,
             "gpu_launches": launches_per_step * args.steps,
@@ -425,6 +434,8 @@ def main():
     ap.add_argument("--impl", choices=("fpo", "reference"), default="fpo")
     ap.add_argument("--workload", default="olmo", help="olmo | qwen | falcon | diag")
     ap.add_argument("--t-chunk", type=int, default=0, help="tokens per E chunk (0 = all)")
+    ap.add_argument("--algo", choices=("auto", "recompute", "stored"), default="auto",
+                    help="how the error matrix is formed (fpo_es_algo)")
     ap.add_argument("--shape", default=None,
                     help="T,d,d_ff,V,layers override of the workload's shape (small ncu cases)")
     ap.add_argument("--cpu-tokens", type=int, default=16, help="oracle sample size (tokens)")

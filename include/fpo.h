@@ -70,6 +70,27 @@ typedef enum fpo_status {
     FPO_ERR_ARG = 10           /* any other invalid argument */
 } fpo_status;
 
+/*
+ * How fpo_error_signal forms the error matrix E = s (softmax(z) - 1_y) without
+ * ever holding all T x V logits:
+ *  FPO_ES_RECOMPUTE      a logits pass keeps only per-(token, vocabulary tile)
+ *                        max / sum-exp partials; a second pass recomputes the
+ *                        logits GEMM and writes E (bf16) for one token chunk.
+ *  FPO_ES_STORED_LOGITS  the logits pass also stores the chunk's fp32 logits; a
+ *                        bandwidth-bound kernel turns them into E once the
+ *                        log-sum-exp is known (one GEMM instead of two, at the
+ *                        cost of T_chunk x V x 4 bytes of workspace and ~3 passes
+ *                        over it in HBM).
+ *  FPO_ES_AUTO           the library's choice (currently FPO_ES_STORED_LOGITS).
+ * Both compute every value with the same arithmetic: their outputs are
+ * bit-identical.
+ */
+typedef enum fpo_es_algo {
+    FPO_ES_AUTO = 0,
+    FPO_ES_RECOMPUTE = 1,
+    FPO_ES_STORED_LOGITS = 2
+} fpo_es_algo;
+
 /* Error-signal problem description (Sec. 3.1 steps 2-4, App. E). */
 typedef struct fpo_error_signal_desc {
     int64_t T;          /* tokens (B x L flattened), >= 0; T = 0 enqueues nothing */
@@ -79,6 +100,7 @@ typedef struct fpo_error_signal_desc {
     float eps;          /* RMSNorm epsilon, inside the square root (App. E)      */
     float min_rms;      /* floor on rho in the 1/rho prefactor of the VJP (0.5)  */
     float loss_scale;   /* s in e = s (softmax(z) - 1_y); 1/T = mean-reduced CE */
+    int32_t algo;       /* fpo_es_algo                                            */
     int64_t t_chunk;    /* tokens per error-matrix chunk; 0 = all T at once       */
     void* const* stage_events;  /* NULL, or FPO_STAGE_EVENTS caller-created
                                    cudaEvent_t recorded on the stream at the stage
@@ -87,11 +109,13 @@ typedef struct fpo_error_signal_desc {
 
 /*
  * Stage boundaries of fpo_error_signal at which desc->stage_events[i] is
- * recorded: 0 start, 1 after the RMSNorm forward, 2 after the logits pass,
- * 3 after the log-sum-exp combine (and loss), 4 after the recompute pass of
- * the last token chunk, 5 after the projection of the last token chunk,
- * 6 after the final-norm VJP.  With one chunk, [4]-[3] and [5]-[4] time the
- * recompute and projection GEMMs alone.
+ * recorded: 0 start, 1 after the RMSNorm forward, 2 after the logits pass (of
+ * the last token chunk for FPO_ES_STORED_LOGITS), 3 after the log-sum-exp
+ * combine (and loss), 4 after the recompute pass (FPO_ES_RECOMPUTE) or the
+ * logits-to-E conversion (FPO_ES_STORED_LOGITS) of the last token chunk, 5
+ * after the projection of the last token chunk, 6 after the final-norm VJP.
+ * With one chunk, consecutive events bracket one kernel each (plus the loss
+ * mean in [2]-[3]).
  */
 #define FPO_STAGE_EVENTS 7
 

@@ -22,6 +22,7 @@ F32, BF16 = 0, 1
 OK = 0
 MAX_GROUPED_LAYERS = 64
 STAGE_EVENTS = 7
+ES_AUTO, ES_RECOMPUTE, ES_STORED_LOGITS = 0, 1, 2
 
 if not os.path.exists(LIB_PATH):
     raise ImportError(f"libfpo.so is not built ({LIB_PATH} missing); run "
@@ -35,7 +36,7 @@ _vp, _i64, _i32, _f32, _sz = (ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32, c
 class ErrorSignalDesc(ctypes.Structure):
     """Mirror of fpo_error_signal_desc."""
     _fields_ = [("T", _i64), ("d", _i64), ("V", _i64), ("dtype", _i32), ("eps", _f32),
-                ("min_rms", _f32), ("loss_scale", _f32), ("t_chunk", _i64),
+                ("min_rms", _f32), ("loss_scale", _f32), ("algo", _i32), ("t_chunk", _i64),
                 ("stage_events", ctypes.POINTER(_vp))]
 
 
@@ -118,7 +119,7 @@ def _workspace(nbytes: int, device) -> torch.Tensor:
 
 # --------------------------------------------------------------------------- error signal
 def error_signal_desc(T, d, V, dtype=BF16, *, eps=1e-6, min_rms=0.5, loss_scale=None, t_chunk=0,
-                      stage_events=None):
+                      stage_events=None, algo=ES_AUTO):
     """fpo_error_signal_desc; ``stage_events`` is None or STAGE_EVENTS torch.cuda.Event objects
     that have been recorded once (so their CUDA handles exist)."""
     s = (1.0 / T if T > 0 else 1.0) if loss_scale is None else loss_scale
@@ -128,7 +129,7 @@ def error_signal_desc(T, d, V, dtype=BF16, *, eps=1e-6, min_rms=0.5, loss_scale=
             raise ValueError(f"stage_events needs {STAGE_EVENTS} events")
         ev = (_vp * STAGE_EVENTS)(*[e.cuda_event for e in stage_events])
     d = ErrorSignalDesc(int(T), int(d), int(V), int(dtype), float(eps), float(min_rms), float(s),
-                        int(t_chunk), ev)
+                        int(algo), int(t_chunk), ev)
     d._keep = ev
     return d
 
@@ -139,7 +140,7 @@ def error_signal_workspace(desc: ErrorSignalDesc) -> int:
 
 def error_signal(h, norm_w, W_U, targets, g_out, *, eps=1e-6, min_rms=0.5, loss_scale=None,
                  t_chunk=0, lse_out=None, loss_out=None, workspace=None, stream=None,
-                 stage_events=None):
+                 stage_events=None, algo=ES_AUTO):
     """fpo_error_signal: g~ = final-RMSNorm VJP of (softmax(z) - 1_y) W_U into ``g_out``.
 
     Returns the workspace tensor (its first word holds the device status).
@@ -147,7 +148,8 @@ def error_signal(h, norm_w, W_U, targets, g_out, *, eps=1e-6, min_rms=0.5, loss_
     T, d = h.shape
     V = W_U.shape[0]
     desc = error_signal_desc(T, d, V, _dtype_code(h), eps=eps, min_rms=min_rms,
-                             loss_scale=loss_scale, t_chunk=t_chunk, stage_events=stage_events)
+                             loss_scale=loss_scale, t_chunk=t_chunk, stage_events=stage_events,
+                             algo=algo)
     need = error_signal_workspace(desc)
     if workspace is None:
         workspace = _workspace(need, h.device)

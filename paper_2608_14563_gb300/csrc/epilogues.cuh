@@ -10,36 +10,34 @@
 #include <cuda_bf16.h>
 #include <math.h>
 
+#include "error_math.cuh"
 #include "ptx.cuh"
 #include "tc_gemm.cuh"
 
 namespace fpo {
 
-constexpr float kLog2e = 1.4426950408889634f;
-
-__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
-    __nv_bfloat162 p = __floats2bfloat162_rn(lo, hi);
-    return *reinterpret_cast<uint32_t*>(&p);
-}
-
 // ---------------------------------------------------------------------------
 // Logits pass (Sec. 3.1 step 2): per (row, vocabulary tile) the running max and
 // sum of exponentials of z = yhat W_U^T over the tile's valid columns, plus the
-// target logit z_{t, y_t} when the target falls inside the tile.
-struct EpiLsePartial {
+// target logit z_{t, y_t} when the target falls inside the tile.  With kStoreZ
+// the fp32 logits are also written to z [M, ldz] (stored-logits algorithm).
+template <bool kStoreZ>
+struct EpiLsePartialT {
     struct Params {
         float2* part;      // [M, part_ld]: (max, sum exp(z - max)) per vocabulary tile
         int part_ld;
         float* zy;         // [M] target logit, or null
         const int* y;      // [M] targets
         int M, N;
+        float* z;          // [M, ldz] logits (kStoreZ only)
+        long long ldz;
     };
     float m, s, zt;
     int yoff;
     int row;
     bool valid, has_t;
 
-    __device__ __forceinline__ EpiLsePartial(const Params& p, int, int row_, int n0)
+    __device__ __forceinline__ EpiLsePartialT(const Params& p, int, int row_, int n0)
         : m(-INFINITY), s(0.f), zt(0.f), row(row_), has_t(false) {
         valid = row_ < p.M;
         yoff = valid ? __ldg(p.y + row_) - n0 : -1;
@@ -48,6 +46,15 @@ struct EpiLsePartial {
     __device__ __forceinline__ void chunk(const Params& p, const float (&v)[32], int col0, int c0) {
         const int lim = p.N - col0;  // valid columns in this chunk (may be <= 0)
         if (lim <= 0) return;
+        if constexpr (kStoreZ) {
+            if (valid) {
+                float4* dst = reinterpret_cast<float4*>(p.z + row * p.ldz + col0);
+#pragma unroll
+                for (int q = 0; q < 8; ++q)
+                    if (q * 4 < lim)
+                        dst[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+            }
+        }
         float cm = -INFINITY;
 #pragma unroll
         for (int j = 0; j < 32; ++j)
@@ -75,6 +82,8 @@ struct EpiLsePartial {
         if (has_t && p.zy) p.zy[row] = zt;
     }
 };
+using EpiLsePartial = EpiLsePartialT<false>;
+using EpiLseStoreZ = EpiLsePartialT<true>;
 
 // ---------------------------------------------------------------------------
 // Recompute pass (Sec. 3.1 step 2): e = s (exp(z - lse) - [col == y]) rounded
@@ -103,11 +112,9 @@ struct EpiError {
         if (!valid || lim <= 0) return;
         uint32_t w[16];
 #pragma unroll
-        for (int j = 0; j < 32; j += 2) {
-            float e0 = ex2_approx(fmaf(v[j], kLog2e, -lse2)) - (col0 + j == yt ? 1.f : 0.f);
-            float e1 = ex2_approx(fmaf(v[j + 1], kLog2e, -lse2)) - (col0 + j + 1 == yt ? 1.f : 0.f);
-            w[j / 2] = pack_bf16x2(p.s * e0, p.s * e1);
-        }
+        for (int j = 0; j < 32; j += 2)
+            w[j / 2] = pack_bf16x2(error_value(v[j], lse2, col0 + j == yt, p.s),
+                                   error_value(v[j + 1], lse2, col0 + j + 1 == yt, p.s));
         uint4* dst = reinterpret_cast<uint4*>(p.E + row * p.ldE + col0);
 #pragma unroll
         for (int q = 0; q < 4; ++q)

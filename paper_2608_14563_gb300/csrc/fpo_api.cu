@@ -72,10 +72,13 @@ int32_t cuda_status(cudaError_t e) { return e == cudaSuccess ? FPO_OK : FPO_ERR_
 
 // ------------------------------------------------------------------ error signal
 struct EsLayout {
-    size_t yhat, rho, lse, zy, ce, part, g, E, total;
+    size_t yhat, rho, lse, zy, ce, part, g, E, z, total;
     int n_tiles;
     int64_t Tc;
+    bool stored;  // FPO_ES_STORED_LOGITS
 };
+
+bool es_stored(const fpo_error_signal_desc* d) { return d->algo != FPO_ES_RECOMPUTE; }
 
 int32_t es_check_desc(const fpo_error_signal_desc* d) {
     if (!d) return FPO_ERR_NULL;
@@ -84,6 +87,8 @@ int32_t es_check_desc(const fpo_error_signal_desc* d) {
     if (d->T > INT_MAX || d->d > INT_MAX || d->V > INT_MAX) return FPO_ERR_SHAPE;
     if (d->dtype == FPO_BF16 && (d->d % 8 != 0 || d->V % 8 != 0)) return FPO_ERR_SHAPE;
     if (!(d->eps >= 0.f) || !(d->min_rms >= 0.f)) return FPO_ERR_ARG;
+    if (d->algo != FPO_ES_AUTO && d->algo != FPO_ES_RECOMPUTE && d->algo != FPO_ES_STORED_LOGITS)
+        return FPO_ERR_ARG;
     return FPO_OK;
 }
 
@@ -104,6 +109,8 @@ EsLayout es_layout(const fpo_error_signal_desc* d) {
     L.part = off; off = align_up(off + T * static_cast<size_t>(L.n_tiles) * 8);
     L.g = off;    off = align_up(off + T * D * 4);
     L.E = off;    off = align_up(off + static_cast<size_t>(L.Tc) * V * esz);
+    L.stored = es_stored(d);
+    L.z = off;    off = align_up(off + (L.stored ? static_cast<size_t>(L.Tc) * V * 4 : 0));
     L.total = off;
     return L;
 }
@@ -186,34 +193,66 @@ int32_t fpo_error_signal(const fpo_error_signal_desc* desc, const void* h, const
     FPO_TRY(launch_rmsnorm_fwd(desc->dtype, h, norm_w, T, d, desc->eps, yhat, rho, targets, V,
                                status, st));
     FPO_TRY(mark(1));
-    // 2. logits pass: per-vocabulary-tile (max, sum exp) partials -> lse
-    if (bf16)
-        FPO_TRY(launch_lse_partial_bf16(yhat, W_U, targets, T, d, V, part, L.n_tiles, zy, status,
-                                        st));
-    else
-        FPO_TRY(launch_lse_partial_f32(static_cast<const float*>(yhat),
-                                       static_cast<const float*>(W_U), targets, T, d, V, part,
-                                       L.n_tiles, zy, st));
-    FPO_TRY(mark(2));
-    FPO_TRY(launch_lse_combine(part, L.n_tiles, T, zy, lse, ce, st));
-    if (loss_out) FPO_TRY(launch_mean(ce, T, loss_out, st));
-    FPO_TRY(mark(3));
-    // 3./4. per token chunk: recompute logits -> E, then g = E W_U
-    for (int64_t c0 = 0; c0 < T; c0 += L.Tc) {
-        const int tc = static_cast<int>(L.Tc < T - c0 ? L.Tc : T - c0);
-        const void* yh = static_cast<const uint8_t*>(yhat) + static_cast<size_t>(c0) * d * esz;
-        if (bf16) {
-            FPO_TRY(launch_error_bf16(yh, W_U, targets + c0, lse + c0, tc, d, V,
-                                      desc->loss_scale, E, status, st));
-            if (c0 + tc >= T) FPO_TRY(mark(4));
-            FPO_TRY(launch_proj_bf16(E, W_U, tc, d, V, g + c0 * d, status, st));
-        } else {
-            FPO_TRY(launch_error_f32(static_cast<const float*>(yh), static_cast<const float*>(W_U),
-                                     targets + c0, lse + c0, tc, d, V, desc->loss_scale,
-                                     static_cast<float*>(E), st));
-            if (c0 + tc >= T) FPO_TRY(mark(4));
-            FPO_TRY(launch_proj_f32(static_cast<const float*>(E), static_cast<const float*>(W_U),
-                                    tc, d, V, g + c0 * d, st));
+    if (!L.stored) {
+        // 2. logits pass over all tokens: per-vocabulary-tile (max, sum exp) partials -> lse
+        if (bf16)
+            FPO_TRY(launch_lse_partial_bf16(yhat, W_U, targets, T, d, V, part, L.n_tiles, zy,
+                                            nullptr, status, st));
+        else
+            FPO_TRY(launch_lse_partial_f32(static_cast<const float*>(yhat),
+                                           static_cast<const float*>(W_U), targets, T, d, V, part,
+                                           L.n_tiles, zy, nullptr, st));
+        FPO_TRY(mark(2));
+        FPO_TRY(launch_lse_combine(part, L.n_tiles, T, zy, lse, ce, st));
+        if (loss_out) FPO_TRY(launch_mean(ce, T, loss_out, st));
+        FPO_TRY(mark(3));
+        // 3./4. per token chunk: recompute the logits -> E, then g = E W_U
+        for (int64_t c0 = 0; c0 < T; c0 += L.Tc) {
+            const int tc = static_cast<int>(L.Tc < T - c0 ? L.Tc : T - c0);
+            const void* yh = static_cast<const uint8_t*>(yhat) + static_cast<size_t>(c0) * d * esz;
+            if (bf16) {
+                FPO_TRY(launch_error_bf16(yh, W_U, targets + c0, lse + c0, tc, d, V,
+                                          desc->loss_scale, E, status, st));
+                if (c0 + tc >= T) FPO_TRY(mark(4));
+                FPO_TRY(launch_proj_bf16(E, W_U, tc, d, V, g + c0 * d, status, st));
+            } else {
+                FPO_TRY(launch_error_f32(static_cast<const float*>(yh),
+                                         static_cast<const float*>(W_U), targets + c0, lse + c0,
+                                         tc, d, V, desc->loss_scale, static_cast<float*>(E), st));
+                if (c0 + tc >= T) FPO_TRY(mark(4));
+                FPO_TRY(launch_proj_f32(static_cast<const float*>(E), static_cast<const float*>(W_U),
+                                        tc, d, V, g + c0 * d, st));
+            }
+        }
+    } else {
+        // 2.-4. per token chunk: logits pass storing z -> lse -> E from z -> g = E W_U
+        float* z = reinterpret_cast<float*>(ws + L.z);
+        for (int64_t c0 = 0; c0 < T; c0 += L.Tc) {
+            const int tc = static_cast<int>(L.Tc < T - c0 ? L.Tc : T - c0);
+            const bool last = c0 + tc >= T;
+            const void* yh = static_cast<const uint8_t*>(yhat) + static_cast<size_t>(c0) * d * esz;
+            float2* pc = part + static_cast<size_t>(c0) * L.n_tiles;
+            float* zyc = zy ? zy + c0 : nullptr;
+            float* cec = ce ? ce + c0 : nullptr;
+            if (bf16)
+                FPO_TRY(launch_lse_partial_bf16(yh, W_U, targets + c0, tc, d, V, pc, L.n_tiles, zyc,
+                                                z, status, st));
+            else
+                FPO_TRY(launch_lse_partial_f32(static_cast<const float*>(yh),
+                                               static_cast<const float*>(W_U), targets + c0, tc, d,
+                                               V, pc, L.n_tiles, zyc, z, st));
+            if (last) FPO_TRY(mark(2));
+            FPO_TRY(launch_lse_combine(pc, L.n_tiles, tc, zyc, lse + c0, cec, st));
+            if (last && loss_out) FPO_TRY(launch_mean(ce, T, loss_out, st));
+            if (last) FPO_TRY(mark(3));
+            FPO_TRY(launch_error_from_logits(desc->dtype, z, lse + c0, targets + c0, tc, V,
+                                             desc->loss_scale, E, st));
+            if (last) FPO_TRY(mark(4));
+            if (bf16)
+                FPO_TRY(launch_proj_bf16(E, W_U, tc, d, V, g + c0 * d, status, st));
+            else
+                FPO_TRY(launch_proj_f32(static_cast<const float*>(E), static_cast<const float*>(W_U),
+                                        tc, d, V, g + c0 * d, st));
         }
     }
     FPO_TRY(mark(5));

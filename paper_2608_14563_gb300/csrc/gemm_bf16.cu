@@ -104,14 +104,18 @@ constexpr int kLseStages = 4;
 int lse_tile_n_bf16() { return kLseBN; }
 
 cudaError_t launch_lse_partial_bf16(const void* yhat, const void* W_U, const int32_t* y, int T,
-                                    int d, int V, float2* part, int part_ld, float* zy,
+                                    int d, int V, float2* part, int part_ld, float* zy, float* z,
                                     unsigned* status, cudaStream_t st) {
     GemmMaps<1> maps;
     if (!map_kmajor(&maps.a, yhat, T, d, kBM) || !map_kmajor(&maps.b[0], W_U, V, d, kLseBN))
         return cudaErrorInvalidValue;
-    EpiLsePartial::Params ep{part, part_ld, zy, y, T, V};
-    return run_gemm<kLseBN, false, false, kLseStages, 1, EpiLsePartial>(
-        maps, ep, make_shape(T, V, d, kLseBN, 1, kBandM), status, st);
+    const GemmShape sh = make_shape(T, V, d, kLseBN, 1, kBandM);
+    if (z) {
+        EpiLseStoreZ::Params ep{part, part_ld, zy, y, T, V, z, V};
+        return run_gemm<kLseBN, false, false, kLseStages, 1, EpiLseStoreZ>(maps, ep, sh, status, st);
+    }
+    EpiLsePartial::Params ep{part, part_ld, zy, y, T, V, nullptr, 0};
+    return run_gemm<kLseBN, false, false, kLseStages, 1, EpiLsePartial>(maps, ep, sh, status, st);
 }
 
 cudaError_t launch_error_bf16(const void* yhat, const void* W_U, const int32_t* y, const float* lse,

@@ -24,9 +24,10 @@ bool current_device_info(DevInfo* out);
 uint64_t wait_limit_ns();
 
 // ------------------------------------------------------------ bf16 (tcgen05)
-// Logits pass: part[T, n_tiles] (max, sum exp) and zy[T] (target logits).
+// Logits pass: part[T, n_tiles] (max, sum exp), zy[T] (target logits) and, when z is
+// non-null, the fp32 logits z[T, V] (stored-logits algorithm).
 cudaError_t launch_lse_partial_bf16(const void* yhat, const void* W_U, const int32_t* y, int T,
-                                    int d, int V, float2* part, int part_ld, float* zy,
+                                    int d, int V, float2* part, int part_ld, float* zy, float* z,
                                     unsigned* status, cudaStream_t s);
 int lse_tile_n_bf16();
 
@@ -55,6 +56,10 @@ cudaError_t launch_rmsnorm_fwd(int dtype, const void* h, const void* w, int T, i
 cudaError_t launch_lse_combine(const float2* part, int n_tiles, int T, const float* zy,
                                float* lse, float* ce, cudaStream_t st);
 cudaError_t launch_mean(const float* x, int n, float* out, cudaStream_t st);
+// Stored-logits algorithm: E[M, V] = s (exp(z - lse) - onehot(y)) from z[M, V] fp32, in
+// dtype (bf16 through the same formula as the recompute epilogue, or fp32).
+cudaError_t launch_error_from_logits(int dtype, const float* z, const float* lse, const int32_t* y,
+                                     int M, int V, float s, void* E, cudaStream_t st);
 // dst[n] = src[n] rounded to dtype (a plain copy for fp32).
 cudaError_t launch_cast_f32(int dtype, const float* src, size_t n, void* dst, cudaStream_t st);
 cudaError_t launch_rmsnorm_vjp(int dtype, const float* g, const void* h, const void* w,
@@ -69,7 +74,7 @@ cudaError_t launch_cosine(int dtype, int64_t n, const void* X, const void* Y, do
 // ------------------------------------------------------------ fp32 SIMT path
 constexpr int kSimtTile = 64;
 cudaError_t launch_lse_partial_f32(const float* yhat, const float* W_U, const int32_t* y, int T,
-                                   int d, int V, float2* part, int part_ld, float* zy,
+                                   int d, int V, float2* part, int part_ld, float* zy, float* z,
                                    cudaStream_t st);
 cudaError_t launch_error_f32(const float* yhat, const float* W_U, const int32_t* y,
                              const float* lse, int Tc, int d, int V, float s, float* E,

@@ -13,6 +13,7 @@
 #include <cuda_runtime.h>
 #include <math.h>
 
+#include "error_math.cuh"
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -203,6 +204,59 @@ __global__ void cast_f32_kernel(const float* __restrict__ src, size_t n, __nv_bf
         dst[i] = __float2bfloat16_rn(src[i]);
 }
 
+// One block per row (grid-stride over rows): 8 logits per thread per step,
+// two 16-byte loads of z and one 16-byte (bf16) or two (fp32) stores of E.
+constexpr int kErrThreads = 256;
+
+template <bool kBf16>
+__global__ void __launch_bounds__(kErrThreads)
+    error_from_logits_kernel(const float* __restrict__ z, const float* __restrict__ lse,
+                             const int32_t* __restrict__ y, int M, int V, float s,
+                             void* __restrict__ E) {
+    for (int row = blockIdx.x; row < M; row += gridDim.x) {
+        const float l = lse[row];
+        const float l2 = l * kLog2e;
+        const int yt = y[row];
+        const float* zr = z + static_cast<size_t>(row) * V;
+        for (int c = threadIdx.x * 8; c < V; c += kErrThreads * 8) {
+            const float4 a = __ldcs(reinterpret_cast<const float4*>(zr + c));
+            const float4 b = __ldcs(reinterpret_cast<const float4*>(zr + c + 4));
+            const float v[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+            if constexpr (kBf16) {
+                uint32_t w[4];
+#pragma unroll
+                for (int k = 0; k < 8; k += 2)
+                    w[k / 2] = pack_bf16x2(error_value(v[k], l2, c + k == yt, s),
+                                           error_value(v[k + 1], l2, c + k + 1 == yt, s));
+                *reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(E) +
+                                          static_cast<size_t>(row) * V + c) =
+                    make_uint4(w[0], w[1], w[2], w[3]);
+            } else {
+                float o[8];
+#pragma unroll
+                for (int k = 0; k < 8; ++k) o[k] = error_value_f32(v[k], l, c + k == yt, s);
+                float* dst = static_cast<float*>(E) + static_cast<size_t>(row) * V + c;
+                *reinterpret_cast<float4*>(dst) = make_float4(o[0], o[1], o[2], o[3]);
+                *reinterpret_cast<float4*>(dst + 4) = make_float4(o[4], o[5], o[6], o[7]);
+            }
+        }
+    }
+}
+
+// Scalar variant for fp32 rows whose length is not a multiple of 8.
+__global__ void __launch_bounds__(kErrThreads)
+    error_from_logits_scalar_kernel(const float* __restrict__ z, const float* __restrict__ lse,
+                                    const int32_t* __restrict__ y, int M, int V, float s,
+                                    float* __restrict__ E) {
+    for (int row = blockIdx.x; row < M; row += gridDim.x) {
+        const float l = lse[row];
+        const int yt = y[row];
+        for (int c = threadIdx.x; c < V; c += kErrThreads)
+            E[static_cast<size_t>(row) * V + c] =
+                error_value_f32(z[static_cast<size_t>(row) * V + c], l, c == yt, s);
+    }
+}
+
 int row_grid(int T) {
     DevInfo di;
     const int sms = current_device_info(&di) ? di.sm_count : 148;
@@ -261,6 +315,22 @@ cudaError_t launch_cast_f32(int dtype, const float* src, size_t n, void* dst, cu
     if (dtype != 1) return cudaMemcpyAsync(dst, src, n * sizeof(float), cudaMemcpyDeviceToDevice, st);
     cast_f32_kernel<<<row_grid(static_cast<int>((n + 255) / 256 * 8)), kRowThreads, 0, st>>>(
         src, n, static_cast<__nv_bfloat16*>(dst));
+    return cudaGetLastError();
+}
+
+cudaError_t launch_error_from_logits(int dtype, const float* z, const float* lse, const int32_t* y,
+                                     int M, int V, float s, void* E, cudaStream_t st) {
+    if (M <= 0) return cudaSuccess;
+    DevInfo di;
+    const int sms = current_device_info(&di) ? di.sm_count : 148;
+    const int grid = M < sms * 8 ? M : sms * 8;
+    if (dtype == 1)
+        error_from_logits_kernel<true><<<grid, kErrThreads, 0, st>>>(z, lse, y, M, V, s, E);
+    else if (V % 8 == 0)
+        error_from_logits_kernel<false><<<grid, kErrThreads, 0, st>>>(z, lse, y, M, V, s, E);
+    else
+        error_from_logits_scalar_kernel<<<grid, kErrThreads, 0, st>>>(z, lse, y, M, V, s,
+                                                                      static_cast<float*>(E));
     return cudaGetLastError();
 }
 

@@ -11,6 +11,7 @@
 
 #include <type_traits>
 
+#include "error_math.cuh"
 #include "internal.h"
 
 namespace fpo {
@@ -35,6 +36,8 @@ struct SEpiLse {  // per (row, 64-column tile): (max, sum exp(z - max)) and z_{t
     int part_ld;
     float* zy;
     const int32_t* y;
+    float* z;       // [M, ldz] logits for the stored-logits algorithm, or null
+    long long ldz;
 };
 struct SEpiError {  // E = s (exp(z - lse) - [col == y])
     float* E;
@@ -127,6 +130,7 @@ __global__ void __launch_bounds__(kThreads)
                 if (col < ops.N) {
                     s += expf(acc[i][j] - mx);
                     if (rv && col == yt && ep.zy) ep.zy[row] = acc[i][j];
+                    if (rv && ep.z) ep.z[row * ep.ldz + col] = acc[i][j];
                 }
             }
             s = hsum16(s);
@@ -139,8 +143,7 @@ __global__ void __launch_bounds__(kThreads)
                 if (col >= ops.N) continue;
                 const float v = acc[i][j];
                 if constexpr (std::is_same_v<Epi, SEpiError>) {
-                    const float e = expf(v - ep.lse[row]) - (col == ep.y[row] ? 1.f : 0.f);
-                    ep.E[row * ep.ldE + col] = ep.s * e;
+                    ep.E[row * ep.ldE + col] = error_value_f32(v, ep.lse[row], col == ep.y[row], ep.s);
                 } else if constexpr (std::is_same_v<Epi, SEpiStore>) {
                     ep.C[row * ep.ld + col] = v;
                 } else {
@@ -183,9 +186,9 @@ SimtOps ops_of(const float* A, long long sam, long long sak, const float* B, lon
 }  // namespace
 
 cudaError_t launch_lse_partial_f32(const float* yhat, const float* W_U, const int32_t* y, int T,
-                                   int d, int V, float2* part, int part_ld, float* zy,
+                                   int d, int V, float2* part, int part_ld, float* zy, float* z,
                                    cudaStream_t st) {
-    SEpiLse ep{part, part_ld, zy, y};
+    SEpiLse ep{part, part_ld, zy, y, z, V};
     return run(ops_of(yhat, d, 1, W_U, d, 1, T, V, d), ep, 1, st);
 }
 

@@ -61,13 +61,14 @@ def L():
 def test_error_signal_workspace_query(L):
     fpo = L.fpo
     small = fpo.error_signal_desc(128, 64, 512, fpo.F32)
-    chunked = fpo.error_signal_desc(4096, 4096, 151936, fpo.BF16, t_chunk=1024)
-    full = fpo.error_signal_desc(4096, 4096, 151936, fpo.BF16)
     assert fpo.error_signal_workspace(small) > 0
-    assert fpo.error_signal_workspace(chunked) < fpo.error_signal_workspace(full)
-    # E chunk is Tc x V bf16: the difference is exactly (4096 - 1024) * V * 2 bytes (256-aligned)
-    diff = fpo.error_signal_workspace(full) - fpo.error_signal_workspace(chunked)
-    assert abs(diff - 3072 * 151936 * 2) < 512
+    # recompute: the E chunk is Tc x V bf16; stored logits add Tc x V fp32 of logits
+    for algo, per in ((fpo.ES_RECOMPUTE, 2), (fpo.ES_STORED_LOGITS, 6), (fpo.ES_AUTO, 6)):
+        chunked = fpo.error_signal_desc(4096, 4096, 151936, fpo.BF16, t_chunk=1024, algo=algo)
+        full = fpo.error_signal_desc(4096, 4096, 151936, fpo.BF16, algo=algo)
+        diff = fpo.error_signal_workspace(full) - fpo.error_signal_workspace(chunked)
+        assert abs(diff - 3072 * 151936 * per) < 1024
+    assert fpo.error_signal_workspace(fpo.error_signal_desc(64, 64, 256, fpo.BF16, algo=7)) == 0
     bad = fpo.error_signal_desc(16, 12, 512, fpo.BF16)  # d not a multiple of 8
     assert fpo.error_signal_workspace(bad) == 0
     assert L.lib.fpo_error_signal_workspace(None) == 0

@@ -23,7 +23,7 @@ BF16_COS = 0.9995
 F32_TOL = 1e-5
 
 
-def gpu_step(fpo, wl, inp, *, t_chunk=0, lr=None, grouped=True):
+def gpu_step(fpo, wl, inp, *, t_chunk=0, lr=None, grouped=True, algo=0):
     """One FPO step on the GPU: error signal, then the update of every layer."""
     lr = wl.lr if lr is None else lr
     h, w, W_U, y = (inp[k].cuda() for k in ("h", "w", "W_U", "y"))
@@ -32,7 +32,8 @@ def gpu_step(fpo, wl, inp, *, t_chunk=0, lr=None, grouped=True):
     lse = torch.empty(T, dtype=torch.float32, device="cuda")
     loss = torch.empty(1, dtype=torch.float32, device="cuda")
     ws = fpo.error_signal(h, w, W_U, y, g, eps=wl.eps, min_rms=wl.min_rms,
-                          loss_scale=wl.loss_scale, t_chunk=t_chunk, lse_out=lse, loss_out=loss)
+                          loss_scale=wl.loss_scale, t_chunk=t_chunk, lse_out=lse, loss_out=loss,
+                          algo=algo)
     assert fpo.get_device_status(ws) == fpo.OK
     A = [a.cuda() for a in inp["A"]]
     Wm = [W.cuda().clone() for W in inp["W"]]
@@ -105,13 +106,23 @@ def test_bf16_ragged_matches_oracle(fpo, ragged):
     check(gpu, ref, inp, RAGGED.lr, BF16_TOL, BF16_COS)
 
 
-def test_bf16_token_chunking_is_bitwise_identical(fpo, ragged):
-    inp, _ = ragged
-    a = gpu_step(fpo, RAGGED, inp, t_chunk=0)
-    b = gpu_step(fpo, RAGGED, inp, t_chunk=128)
-    c = gpu_step(fpo, RAGGED, inp, t_chunk=37)
-    assert torch.equal(a["g"], b["g"]) and torch.equal(a["g"], c["g"])
-    assert torch.equal(a["lse"], b["lse"])
+@pytest.mark.parametrize("algo", [1, 2])  # FPO_ES_RECOMPUTE, FPO_ES_STORED_LOGITS
+def test_bf16_both_algorithms_match_oracle(fpo, ragged, algo):
+    inp, ref = ragged
+    gpu = gpu_step(fpo, RAGGED, inp, algo=algo)
+    check(gpu, ref, inp, RAGGED.lr, BF16_TOL, BF16_COS)
+
+
+@pytest.mark.parametrize("wl_name", ["tiny", "ragged"])
+def test_algorithms_and_chunkings_are_bitwise_identical(fpo, ragged, wl_name):
+    wl, inp = (RAGGED, ragged[0]) if wl_name == "ragged" else (
+        synth.WORKLOADS["tiny"], synth.make_all(synth.WORKLOADS["tiny"]))
+    runs = [gpu_step(fpo, wl, inp, algo=a, t_chunk=c)
+            for a in (1, 2) for c in (0, 128, 37)]
+    for r in runs[1:]:
+        assert torch.equal(runs[0]["g"], r["g"])
+        assert torch.equal(runs[0]["lse"], r["lse"])
+        assert torch.equal(runs[0]["loss"], r["loss"])
 
 
 def test_grouped_update_equals_per_layer_calls(fpo, ragged):
