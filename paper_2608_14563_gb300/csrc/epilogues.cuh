@@ -2,9 +2,11 @@
 //
 // Each epilogue thread owns one output row of a 128 x BN tile and receives its
 // fp32 accumulator 32 columns at a time: Epi(params, group, row, n0), then
-// chunk(params, v[32], col_of_v0, col_offset_in_tile) for each 32-column chunk
-// in order, then finish(params, n_block).  Rows >= M and columns >= N belong
-// to the zero-filled tile overhang and are never written.
+// chunk(params, v[32], col_of_v0, col_offset_in_tile, io) for each 32-column
+// chunk in order, then finish(params, n_block).  Rows >= M and columns >= N
+// belong to the zero-filled tile overhang and are never written.  Dense
+// outputs go through the warp's swizzled staging buffers and TMA stores
+// (one 32-row x 128-byte box per store; the TMA engine clips the overhang).
 #pragma once
 
 #include <cuda_bf16.h>
@@ -24,13 +26,12 @@ namespace fpo {
 template <bool kStoreZ>
 struct EpiLsePartialT {
     struct Params {
+        CUtensorMap zmap;  // fp32 logits [M, N], box 32 x 32 (kStoreZ only)
         float2* part;      // [M, part_ld]: (max, sum exp(z - max)) per vocabulary tile
         int part_ld;
         float* zy;         // [M] target logit, or null
         const int* y;      // [M] targets
         int M, N;
-        float* z;          // [M, ldz] logits (kStoreZ only)
-        long long ldz;
     };
     float m, s, zt;
     int yoff;
@@ -43,16 +44,18 @@ struct EpiLsePartialT {
         yoff = valid ? __ldg(p.y + row_) - n0 : -1;
     }
 
-    __device__ __forceinline__ void chunk(const Params& p, const float (&v)[32], int col0, int c0) {
+    __device__ __forceinline__ void chunk(const Params& p, const float (&v)[32], int col0, int c0,
+                                          EpiIO& io) {
         const int lim = p.N - col0;  // valid columns in this chunk (may be <= 0)
         if (lim <= 0) return;
         if constexpr (kStoreZ) {
-            if (valid) {
-                float4* dst = reinterpret_cast<float4*>(p.z + row * p.ldz + col0);
+            if (io.row0 < p.M) {
+                const uint32_t buf = out_acquire(io);
+                uint32_t w[32];
 #pragma unroll
-                for (int q = 0; q < 8; ++q)
-                    if (q * 4 < lim)
-                        dst[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+                for (int j = 0; j < 32; ++j) w[j] = __float_as_uint(v[j]);
+                out_stage_row(buf, io.lane, w);
+                out_commit(io, &p.zmap, buf, col0, io.row0);
             }
         }
         float cm = -INFINITY;
@@ -87,11 +90,11 @@ using EpiLseStoreZ = EpiLsePartialT<true>;
 
 // ---------------------------------------------------------------------------
 // Recompute pass (Sec. 3.1 step 2): e = s (exp(z - lse) - [col == y]) rounded
-// to bf16 into the error matrix E [M, N] (row stride ldE).
+// to bf16 into the error matrix E [M, N]; two 32-column chunks fill one
+// 64-column bf16 staging row before each TMA store.
 struct EpiError {
     struct Params {
-        __nv_bfloat16* E;
-        long long ldE;
+        CUtensorMap Emap;  // bf16 E [M, N], box 64 x 32
         const float* lse;  // [M]
         const int* y;      // [M]
         int M, N;
@@ -99,53 +102,59 @@ struct EpiError {
     };
     int row, yt;
     float lse2;
-    bool valid;
+    bool pair_out;  // the current 64-column pair lies beyond N
+    uint32_t w[32];
 
     __device__ __forceinline__ EpiError(const Params& p, int, int row_, int) : row(row_) {
-        valid = row_ < p.M;
+        const bool valid = row_ < p.M;
         yt = valid ? __ldg(p.y + row_) : -1;
         lse2 = valid ? __ldg(p.lse + row_) * kLog2e : 0.f;
+        pair_out = false;
     }
 
-    __device__ __forceinline__ void chunk(const Params& p, const float (&v)[32], int col0, int) {
-        const int lim = p.N - col0;
-        if (!valid || lim <= 0) return;
-        uint32_t w[16];
+    __device__ __forceinline__ void chunk(const Params& p, const float (&v)[32], int col0, int c0,
+                                          EpiIO& io) {
+        const bool second = (c0 & 32) != 0;
+        if (!second) pair_out = col0 >= p.N || io.row0 >= p.M;
+        if (pair_out) return;
+        if (!second) {
 #pragma unroll
-        for (int j = 0; j < 32; j += 2)
-            w[j / 2] = pack_bf16x2(error_value(v[j], lse2, col0 + j == yt, p.s),
-                                   error_value(v[j + 1], lse2, col0 + j + 1 == yt, p.s));
-        uint4* dst = reinterpret_cast<uint4*>(p.E + row * p.ldE + col0);
+            for (int j = 0; j < 32; j += 2)
+                w[j / 2] = pack_bf16x2(error_value(v[j], lse2, col0 + j == yt, p.s),
+                                       error_value(v[j + 1], lse2, col0 + j + 1 == yt, p.s));
+        } else {
 #pragma unroll
-        for (int q = 0; q < 4; ++q)
-            if (q * 8 < lim) dst[q] = make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
+            for (int j = 0; j < 32; j += 2)
+                w[16 + j / 2] = pack_bf16x2(error_value(v[j], lse2, col0 + j == yt, p.s),
+                                            error_value(v[j + 1], lse2, col0 + j + 1 == yt, p.s));
+            const uint32_t buf = out_acquire(io);
+            out_stage_row(buf, io.lane, w);
+            out_commit(io, &p.Emap, buf, col0 - 32, io.row0);
+        }
     }
 
     __device__ __forceinline__ void finish(const Params&, int) {}
 };
 
 // ---------------------------------------------------------------------------
-// Plain fp32 store of C [M, N] (row stride ld): the projection g = E W_U (Eq. gproj).
+// Plain fp32 store of C [M, N]: the projection g = E W_U (Eq. gproj).
 struct EpiStoreF32 {
     struct Params {
-        float* C;
-        long long ld;
+        CUtensorMap Cmap;  // fp32 C [M, N], box 32 x 32
         int M, N;
     };
-    int row;
-    bool valid;
 
-    __device__ __forceinline__ EpiStoreF32(const Params& p, int, int row_, int) : row(row_) {
-        valid = row_ < p.M;
-    }
+    __device__ __forceinline__ EpiStoreF32(const Params&, int, int, int) {}
 
-    __device__ __forceinline__ void chunk(const Params& p, const float (&v)[32], int col0, int) {
-        const int lim = p.N - col0;
-        if (!valid || lim <= 0) return;
-        float4* dst = reinterpret_cast<float4*>(p.C + row * p.ld + col0);
+    __device__ __forceinline__ void chunk(const Params& p, const float (&v)[32], int col0, int,
+                                          EpiIO& io) {
+        if (col0 >= p.N || io.row0 >= p.M) return;
+        const uint32_t buf = out_acquire(io);
+        uint32_t w[32];
 #pragma unroll
-        for (int q = 0; q < 8; ++q)
-            if (q * 4 < lim) dst[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+        for (int j = 0; j < 32; ++j) w[j] = __float_as_uint(v[j]);
+        out_stage_row(buf, io.lane, w);
+        out_commit(io, &p.Cmap, buf, col0, io.row0);
     }
 
     __device__ __forceinline__ void finish(const Params&, int) {}
@@ -171,7 +180,8 @@ struct EpiUpdate {
         valid = row_ < p.M;
     }
 
-    __device__ __forceinline__ void chunk(const Params& p, const float (&v)[32], int col0, int) {
+    __device__ __forceinline__ void chunk(const Params& p, const float (&v)[32], int col0, int,
+                                          EpiIO&) {
         const int lim = p.N - col0;
         if (!valid || lim <= 0) return;
         const long long off = row * p.ld + col0;

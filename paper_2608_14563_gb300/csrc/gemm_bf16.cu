@@ -40,19 +40,30 @@ EncodeTiledFn encode_fn() {
     return fn;
 }
 
-// 2-D bf16 tensor [outer, inner] with row stride `ld` elements, box
-// {box_inner, box_outer}, 128-byte swizzle, zero fill outside the tensor.
+// 2-D tensor [outer, inner] of bf16 (esz 2) or fp32 (esz 4) with row stride
+// `ld` elements, box {box_inner, box_outer}, 128-byte swizzle, zero fill
+// outside the tensor on loads (and clipping on stores).
 bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, uint64_t ld,
-              uint32_t box_inner, uint32_t box_outer) {
+              uint32_t box_inner, uint32_t box_outer, int esz = 2) {
     EncodeTiledFn fn = encode_fn();
     if (!fn) return false;
     cuuint64_t dims[2] = {inner, outer};
-    cuuint64_t strides[1] = {ld * 2};
+    cuuint64_t strides[1] = {ld * static_cast<uint64_t>(esz)};
     cuuint32_t box[2] = {box_inner, box_outer};
     cuuint32_t es[2] = {1, 1};
-    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
-              es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+    const CUtensorMapDataType dt =
+        esz == 4 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+    return fn(m, dt, 2, const_cast<void*>(base), dims, strides, box, es,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Output maps of the epilogues: 32 rows x 128 bytes per store.
+bool map_out_f32(CUtensorMap* m, void* base, int rows, int cols) {
+    return make_map(m, base, cols, rows, cols, 32, 32, 4);
+}
+bool map_out_bf16(CUtensorMap* m, void* base, int rows, int cols) {
+    return make_map(m, base, cols, rows, cols, 64, 32, 2);
 }
 
 // K-major operand [rows, K]: box {64 (K), rows_per_tile}
@@ -111,10 +122,24 @@ cudaError_t launch_lse_partial_bf16(const void* yhat, const void* W_U, const int
         return cudaErrorInvalidValue;
     const GemmShape sh = make_shape(T, V, d, kLseBN, 1, kBandM);
     if (z) {
-        EpiLseStoreZ::Params ep{part, part_ld, zy, y, T, V, z, V};
+        EpiLseStoreZ::Params ep;
+        if (!map_out_f32(&ep.zmap, z, T, V)) return cudaErrorInvalidValue;
+        ep.part = part;
+        ep.part_ld = part_ld;
+        ep.zy = zy;
+        ep.y = y;
+        ep.M = T;
+        ep.N = V;
         return run_gemm<kLseBN, false, false, kLseStages, 1, EpiLseStoreZ>(maps, ep, sh, status, st);
     }
-    EpiLsePartial::Params ep{part, part_ld, zy, y, T, V, nullptr, 0};
+    EpiLsePartial::Params ep;
+    ep.zmap = maps.a;  // unused
+    ep.part = part;
+    ep.part_ld = part_ld;
+    ep.zy = zy;
+    ep.y = y;
+    ep.M = T;
+    ep.N = V;
     return run_gemm<kLseBN, false, false, kLseStages, 1, EpiLsePartial>(maps, ep, sh, status, st);
 }
 
@@ -124,7 +149,13 @@ cudaError_t launch_error_bf16(const void* yhat, const void* W_U, const int32_t* 
     GemmMaps<1> maps;
     if (!map_kmajor(&maps.a, yhat, Tc, d, kBM) || !map_kmajor(&maps.b[0], W_U, V, d, kLseBN))
         return cudaErrorInvalidValue;
-    EpiError::Params ep{static_cast<__nv_bfloat16*>(E), V, lse, y, Tc, V, s};
+    EpiError::Params ep;
+    if (!map_out_bf16(&ep.Emap, E, Tc, V)) return cudaErrorInvalidValue;
+    ep.lse = lse;
+    ep.y = y;
+    ep.M = Tc;
+    ep.N = V;
+    ep.s = s;
     return run_gemm<kLseBN, false, false, kLseStages, 1, EpiError>(
         maps, ep, make_shape(Tc, V, d, kLseBN, 1, kBandM), status, st);
 }
@@ -137,7 +168,10 @@ cudaError_t launch_proj_bf16(const void* E, const void* W_U, int Tc, int d, int 
     GemmMaps<1> maps;
     if (!map_kmajor(&maps.a, E, Tc, V, kBM) || !map_mnmajor(&maps.b[0], W_U, V, d))
         return cudaErrorInvalidValue;
-    EpiStoreF32::Params ep{g, d, Tc, d};
+    EpiStoreF32::Params ep;
+    if (!map_out_f32(&ep.Cmap, g, Tc, d)) return cudaErrorInvalidValue;
+    ep.M = Tc;
+    ep.N = d;
     return run_gemm<kProjBN, false, true, kProjStages, 1, EpiStoreF32>(
         maps, ep, make_shape(Tc, d, V, kProjBN, 1, kBandM), status, st);
 }
@@ -180,7 +214,10 @@ cudaError_t launch_test_gemm_bf16(int M, int N, int K, bool a_mn, bool b_mn, con
     bool ok = a_mn ? map_mnmajor(&maps.a, A, K, M) : map_kmajor(&maps.a, A, M, K, kBM);
     ok = ok && (b_mn ? map_mnmajor(&maps.b[0], B, K, N) : map_kmajor(&maps.b[0], B, N, K, 256));
     if (!ok) return cudaErrorInvalidValue;
-    EpiStoreF32::Params ep{C, N, M, N};
+    EpiStoreF32::Params ep;
+    if (!map_out_f32(&ep.Cmap, C, M, N)) return cudaErrorInvalidValue;
+    ep.M = M;
+    ep.N = N;
     const GemmShape sh = make_shape(M, N, K, 256, 1, kBandM);
     if (!a_mn && !b_mn) return run_gemm<256, false, false, 4, 1, EpiStoreF32>(maps, ep, sh, status, st);
     if (!a_mn && b_mn) return run_gemm<256, false, true, 4, 1, EpiStoreF32>(maps, ep, sh, status, st);

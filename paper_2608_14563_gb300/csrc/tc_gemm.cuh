@@ -44,12 +44,18 @@ struct GemmMaps {
     CUtensorMap b[MAXG];    // one per group
 };
 
+// Output staging for TMA stores: per epilogue warp two 4 KB buffers, each a
+// 32-row x 128-byte tile in the 128-byte-swizzled layout (1024-byte aligned).
+constexpr int kOutBufBytes = 4096;
+constexpr int kOutBytesPerWarp = 2 * kOutBufBytes;
+
 template <int BN, int STAGES>
 struct GemmSmem {
     static constexpr int kABytes = kBM * kBK * 2;
     static constexpr int kBBytes = BN * kBK * 2;
     static constexpr int kStageBytes = kABytes + kBBytes;
-    static constexpr int kBarOffset = STAGES * kStageBytes;
+    static constexpr int kOutOffset = STAGES * kStageBytes;
+    static constexpr int kBarOffset = kOutOffset + 4 * kOutBytesPerWarp;
     // full[S], empty[S], tmem_full[2], tmem_empty[2], drain[1]
     static constexpr int kNumBars = 2 * STAGES + 5;
     static constexpr int kMiscOffset = kBarOffset + kNumBars * 8;
@@ -95,6 +101,47 @@ __device__ __forceinline__ uint64_t operand_desc(uint32_t base, int kk) {
         return smem_desc_sw128(base + kk * (kUmmaK * 2), 16, 1024);
     else
         return smem_desc_sw128(base + kk * (kUmmaK * 128), 64 * kBK * 2, 1024);
+}
+
+// Per-warp output context of the epilogue: the warp's staging buffers and the
+// count of TMA stores it issued (which buffer is next).  All decisions that
+// touch it are warp-uniform.
+struct EpiIO {
+    uint32_t out;     // shared address of this warp's two staging buffers
+    int lane;
+    int row0;         // absolute output row of lane 0 of this warp
+    uint32_t count;   // stores issued so far
+};
+
+// Next staging buffer, once the store that last used it has read it.
+__device__ __forceinline__ uint32_t out_acquire(const EpiIO& io) {
+    if (io.lane == 0) bulk_wait_group_read<1>();
+    __syncwarp();
+    return io.out + (io.count & 1u) * kOutBufBytes;
+}
+
+// Each thread writes its 128-byte row r (32 words) of a staging buffer: 16-byte
+// piece c goes to position c ^ (r mod 8), the 128-byte swizzle the TMA store
+// undoes; 8 consecutive rows hit 8 different bank groups.
+__device__ __forceinline__ void out_stage_row(uint32_t buf, int r, const uint32_t (&w)[32]) {
+    const uint32_t row = buf + static_cast<uint32_t>(r) * 128u;
+#pragma unroll
+    for (int c = 0; c < 8; ++c)
+        st_shared_v4(row + ((static_cast<uint32_t>(c) ^ (static_cast<uint32_t>(r) & 7u)) << 4),
+                     w[4 * c], w[4 * c + 1], w[4 * c + 2], w[4 * c + 3]);
+}
+
+// Store a filled staging buffer to (x, y) of `map` (rows/columns outside the
+// tensor are clipped by the TMA engine).
+__device__ __forceinline__ void out_commit(EpiIO& io, const CUtensorMap* map, uint32_t buf, int x,
+                                           int y) {
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (io.lane == 0) {
+        tma_store_2d(map, buf, x, y);
+        bulk_commit_group();
+    }
+    ++io.count;
 }
 
 template <int BN, bool A_MN, bool B_MN, int STAGES, int MAXG, class Epi>
@@ -222,6 +269,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         // ------------------------------------------------------- epilogue
         const int q = warp & 3;  // TMEM lane quarter this warp may access
         const int r_in_tile = q * 32 + lane;
+        EpiIO io{sbase + L::kOutOffset + static_cast<uint32_t>((warp - 2) * kOutBytesPerWarp), lane,
+                 0, 0u};
         int acc = 0;
         uint32_t acc_phase = 0;
         for (long long t = blockIdx.x; t < sh.tiles; t += gridDim.x) {
@@ -231,6 +280,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             tc_fence_after();
             const int row = mb * kBM + r_in_tile;
             const int n0 = nb * BN;
+            io.row0 = mb * kBM + q * 32;
             Epi epi(ep, g, row, n0);
             const uint32_t t_row = tmem_base + (static_cast<uint32_t>(q * 32) << 16) +
                                    static_cast<uint32_t>(acc * BN);
@@ -238,7 +288,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             for (int c = 0; c < BN / 32; ++c) {
                 float v[32];
                 tmem_ld_32x32b_x32(t_row + c * 32, v);
-                epi.chunk(ep, v, n0 + c * 32, c * 32);
+                epi.chunk(ep, v, n0 + c * 32, c * 32, io);
             }
             epi.finish(ep, nb);
             tc_fence_before();
@@ -246,6 +296,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             if (lane == 0) mbar_arrive(tempty_bar(acc));
             if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
         }
+        if (lane == 0) bulk_wait_group_all();  // stores done before shared memory goes away
+        __syncwarp();
     }
 
     tc_fence_before();
