@@ -307,12 +307,24 @@ def run_fpo(args, wl):
         A_host = [a.cpu().pin_memory() for a in A]
         loss_host = torch.empty(1, dtype=torch.float32).pin_memory()
 
+        copy_stream = torch.cuda.Stream(device=dev)
+        a_ready = torch.cuda.Event()
+
         def e2e_step():
+            # h and targets feed the first kernel: copy them on the compute stream.
             h.copy_(h_host, non_blocking=True)
             y.copy_(y_host, non_blocking=True)
-            for a_d, a_h in zip(A, A_host):
-                a_d.copy_(a_h, non_blocking=True)
-            step()
+            # A_l is first read by the layer update: copy it on a side stream while the
+            # error signal runs (after the previous step's update has finished reading it).
+            copy_stream.wait_stream(stream)
+            with torch.cuda.stream(copy_stream):
+                for a_d, a_h in zip(A, A_host):
+                    a_d.copy_(a_h, non_blocking=True)
+                a_ready.record(copy_stream)
+            fpo.error_signal(h, w, W_U, y, g, eps=wl.eps, min_rms=wl.min_rms,
+                             t_chunk=args.t_chunk, loss_out=loss, workspace=ws_es, algo=algo)
+            stream.wait_event(a_ready)
+            fpo.layer_update_grouped(g, A, wl.lr, W_masters=Wm, W_outs=Wo, workspace=ws_up)
             loss_host.copy_(loss, non_blocking=True)
 
         for _ in range(max(1, args.warmup)):
@@ -334,7 +346,9 @@ def run_fpo(args, wl):
         h2d = (h.numel() * h.element_size() + y.numel() * 4
                + sum(a.numel() * a.element_size() for a in A))
         e2e = {"value": wl.T * world / (e2e_ms / 1e3), "unit": "tokens/s",
-               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": 4, "ms_per_step": e2e_ms}
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": 4, "ms_per_step": e2e_ms,
+               "pipeline": "h, targets H2D on the compute stream; A_l H2D on a copy stream "
+                           "overlapping the error signal; loss D2H"}
 
     if world > 1:
         t = torch.tensor([ms], device=dev)
