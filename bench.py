@@ -228,6 +228,10 @@ def run_fpo(args, wl):
     import paper_2608_14563_gb300 as fpo
     from paper_2608_14563_gb300 import synth
 
+    if args.gemm_variant >= 0:
+        fpo.set_gemm_variant(args.gemm_variant)
+    variant = fpo.set_gemm_variant(-1)  # read back (a negative value changes nothing)
+
     wl_r = synth.Workload(wl.name, T=wl.T, d=wl.d, d_ff=wl.d_ff, V=wl.V, layers=wl.layers,
                           dtype=wl.dtype, targets=wl.targets, lr=wl.lr, seed=rank)
     dev = torch.device("cuda", local)
@@ -394,6 +398,8 @@ def run_fpo(args, wl):
             "kernels_tflops": {k: per_kernel_flops[k] / (stage_ms[k] / 1e3) / 1e12
                                for k in per_kernel_flops},
             "algo": "stored-logits" if stored else "recompute",
+            "gemm_kernel": "cta-pair 256x256 (tcgen05 cta_group::2)" if variant == 1
+                           else "single-cta 128x256 (tcgen05 cta_group::1)",
             "cpu_baseline": cpu,
             "e2e": e2e,
             "gpu_launches": launches_per_step * args.steps,
@@ -450,6 +456,9 @@ def main():
     ap.add_argument("--t-chunk", type=int, default=0, help="tokens per E chunk (0 = all)")
     ap.add_argument("--algo", choices=("auto", "recompute", "stored"), default="auto",
                     help="how the error matrix is formed (fpo_es_algo)")
+    ap.add_argument("--gemm-variant", type=int, choices=(-1, 0, 1), default=-1,
+                    help="tensor-core GEMM kernel: 0 single-CTA tiles, 1 CTA-pair tiles, "
+                         "-1 library default")
     ap.add_argument("--shape", default=None,
                     help="T,d,d_ff,V,layers override of the workload's shape (small ncu cases)")
     ap.add_argument("--cpu-tokens", type=int, default=16, help="oracle sample size (tokens)")

@@ -27,6 +27,21 @@ int32_t fpo_testing_gemm_bf16(int64_t M, int64_t N, int64_t K, int32_t a_mn, int
                               const void* A, const void* B, float* C, void* workspace,
                               size_t workspace_bytes, void* stream);
 
+/*
+ * Select the tensor-core GEMM kernel every later call uses (process-wide):
+ * 0 = one CTA per 128 x 256 output tile, 1 = a CTA pair (tcgen05 cta_group::2)
+ * per 256 x 256 tile (the default).  Returns the previous setting.  Both compute the same
+ * sums in the same order per output element.
+ */
+int32_t fpo_testing_set_gemm_variant(int32_t variant);
+
+/*
+ * Override the height, in output tiles, of the bands in which GEMM tiles are
+ * rasterised for L2 reuse (0 restores the default: bands of 2048 output rows).
+ * Tuning hook; results do not depend on it.
+ */
+void fpo_testing_set_band(int32_t band);
+
 #ifdef __cplusplus
 }
 #endif

@@ -65,6 +65,8 @@ _lib.fpo_cosine.argtypes = [_i64, _i32, _vp, _vp, _vp, _vp, _sz, _vp]
 _lib.fpo_cosine.restype = _i32
 _lib.fpo_get_device_status.argtypes = [_vp, _vp]
 _lib.fpo_get_device_status.restype = _i32
+_lib.fpo_testing_set_gemm_variant.argtypes = [_i32]
+_lib.fpo_testing_set_gemm_variant.restype = _i32
 
 
 class FpoError(RuntimeError):
@@ -83,6 +85,16 @@ def abi_version() -> int:
 
 def set_wait_limit_ns(ns: int) -> None:
     _lib.fpo_set_wait_limit_ns(int(ns))
+
+
+def set_gemm_variant(variant: int) -> int:
+    """fpo_testing_set_gemm_variant: 0 single-CTA, 1 CTA-pair tiles; a negative value only
+    reads the current setting.  Returns the setting in force before the call."""
+    if variant < 0:
+        cur = _lib.fpo_testing_set_gemm_variant(0)
+        _lib.fpo_testing_set_gemm_variant(cur)
+        return cur
+    return _lib.fpo_testing_set_gemm_variant(int(variant))
 
 
 def _check(code: int, where: str) -> None:

@@ -374,6 +374,14 @@ int32_t fpo_testing_gemm_bf16(int64_t M, int64_t N, int64_t K, int32_t a_mn, int
                                              status, st));
 }
 
+int32_t fpo_testing_set_gemm_variant(int32_t variant) {
+    const int32_t prev = gemm_variant();
+    set_gemm_variant(variant);
+    return prev;
+}
+
+void fpo_testing_set_band(int32_t band) { set_band_override(band); }
+
 int32_t fpo_get_device_status(void* workspace, void* stream) {
     if (!workspace) return FPO_ERR_WORKSPACE;
     cudaStream_t st = static_cast<cudaStream_t>(stream);

@@ -14,9 +14,12 @@
 
 #include <mutex>
 
+#include <atomic>
+
 #include "epilogues.cuh"
 #include "internal.h"
 #include "tc_gemm.cuh"
+#include "tc_gemm_pair.cuh"
 
 namespace fpo {
 namespace {
@@ -75,12 +78,12 @@ bool map_mnmajor(CUtensorMap* m, const void* base, int K, int mn) {
     return make_map(m, base, mn, K, mn, 64, kBK);
 }
 
-GemmShape make_shape(int M, int N, int K, int BN, int groups, int band) {
+GemmShape make_shape(int M, int N, int K, int BN, int groups, int band, int BM = kBM) {
     GemmShape sh;
     sh.M = M;
     sh.N = N;
     sh.K = K;
-    sh.m_blocks = (M + kBM - 1) / kBM;
+    sh.m_blocks = (M + BM - 1) / BM;
     sh.n_blocks = (N + BN - 1) / BN;
     sh.k_blocks = (K + kBK - 1) / kBK;
     sh.groups = groups;
@@ -106,9 +109,61 @@ cudaError_t run_gemm(const GemmMaps<MAXG>& maps, const typename Epi::Params& ep,
     return cudaGetLastError();
 }
 
-constexpr int kBandM = 16;
+// Clusters of two CTAs that can be resident at once for a pair-kernel instantiation.
+template <class Kern>
+int pair_clusters(Kern kern, int smem_bytes, int sm_count) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(sm_count & ~1), 1, 1);
+    cfg.blockDim = dim3(kGemmThreads, 1, 1);
+    cfg.dynamicSmemBytes = static_cast<size_t>(smem_bytes);
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess || n < 1) {
+        cudaGetLastError();
+        n = sm_count / 2;
+    }
+    return n;
+}
+
+template <int BN, bool A_MN, bool B_MN, int STAGES, int MAXG, class Epi>
+cudaError_t run_gemm_pair(const GemmMaps<MAXG>& maps, const typename Epi::Params& ep,
+                          const GemmShape& sh, unsigned* status, cudaStream_t st) {
+    if (sh.tiles <= 0 || sh.k_blocks <= 0) return cudaSuccess;
+    using L = GemmPairSmem<BN, STAGES>;
+    auto kern = tc_gemm_pair_kernel<BN, A_MN, B_MN, STAGES, MAXG, Epi>;
+    static cudaError_t attr_err =
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::kBytes);
+    if (attr_err != cudaSuccess) return attr_err;
+    DevInfo di;
+    if (!current_device_info(&di)) return cudaErrorUnknown;
+    static int max_clusters = pair_clusters(kern, L::kBytes, di.sm_count);
+    const long long clusters = sh.tiles < max_clusters ? sh.tiles : max_clusters;
+    kern<<<static_cast<unsigned>(2 * clusters), kGemmThreads, L::kBytes, st>>>(maps, ep, sh, status,
+                                                                              wait_limit_ns());
+    return cudaGetLastError();
+}
+
+constexpr int kPairStages = 6;
+
+std::atomic<int> g_gemm_variant{1};  // 0 = single-CTA tiles, 1 = CTA-pair tiles (default)
+std::atomic<int> g_band_override{0};  // > 0: rasterisation band height (tests / tuning)
+
+bool use_pair() { return g_gemm_variant.load(std::memory_order_relaxed) == 1; }
+
+// Rasterisation band in tile rows: a band spans kBandRows output rows (16 single-CTA
+// tiles, 8 pair tiles), unless overridden.
+constexpr int kBandRows = 2048;
+int band_for(bool pair) {
+    const int o = g_band_override.load(std::memory_order_relaxed);
+    if (o > 0) return o;
+    return kBandRows / (pair ? kPairBM : kBM);
+}
 
 }  // namespace
+
+void set_band_override(int b) { g_band_override.store(b > 0 ? b : 0, std::memory_order_relaxed); }
+
+void set_gemm_variant(int v) { g_gemm_variant.store(v == 1 ? 1 : 0, std::memory_order_relaxed); }
+int gemm_variant() { return g_gemm_variant.load(std::memory_order_relaxed); }
 
 constexpr int kLseBN = 256;
 constexpr int kLseStages = 4;
@@ -117,10 +172,12 @@ int lse_tile_n_bf16() { return kLseBN; }
 cudaError_t launch_lse_partial_bf16(const void* yhat, const void* W_U, const int32_t* y, int T,
                                     int d, int V, float2* part, int part_ld, float* zy, float* z,
                                     unsigned* status, cudaStream_t st) {
+    const bool pair = use_pair();
     GemmMaps<1> maps;
-    if (!map_kmajor(&maps.a, yhat, T, d, kBM) || !map_kmajor(&maps.b[0], W_U, V, d, kLseBN))
+    if (!map_kmajor(&maps.a, yhat, T, d, kBM) ||
+        !map_kmajor(&maps.b[0], W_U, V, d, pair ? kLseBN / 2 : kLseBN))
         return cudaErrorInvalidValue;
-    const GemmShape sh = make_shape(T, V, d, kLseBN, 1, kBandM);
+    const GemmShape sh = make_shape(T, V, d, kLseBN, 1, band_for(pair), pair ? kPairBM : kBM);
     if (z) {
         EpiLseStoreZ::Params ep;
         if (!map_out_f32(&ep.zmap, z, T, V)) return cudaErrorInvalidValue;
@@ -130,6 +187,9 @@ cudaError_t launch_lse_partial_bf16(const void* yhat, const void* W_U, const int
         ep.y = y;
         ep.M = T;
         ep.N = V;
+        if (pair)
+            return run_gemm_pair<kLseBN, false, false, kPairStages, 1, EpiLseStoreZ>(maps, ep, sh,
+                                                                                     status, st);
         return run_gemm<kLseBN, false, false, kLseStages, 1, EpiLseStoreZ>(maps, ep, sh, status, st);
     }
     EpiLsePartial::Params ep;
@@ -140,14 +200,19 @@ cudaError_t launch_lse_partial_bf16(const void* yhat, const void* W_U, const int
     ep.y = y;
     ep.M = T;
     ep.N = V;
+    if (pair)
+        return run_gemm_pair<kLseBN, false, false, kPairStages, 1, EpiLsePartial>(maps, ep, sh,
+                                                                                  status, st);
     return run_gemm<kLseBN, false, false, kLseStages, 1, EpiLsePartial>(maps, ep, sh, status, st);
 }
 
 cudaError_t launch_error_bf16(const void* yhat, const void* W_U, const int32_t* y, const float* lse,
                               int Tc, int d, int V, float s, void* E, unsigned* status,
                               cudaStream_t st) {
+    const bool pair = use_pair();
     GemmMaps<1> maps;
-    if (!map_kmajor(&maps.a, yhat, Tc, d, kBM) || !map_kmajor(&maps.b[0], W_U, V, d, kLseBN))
+    if (!map_kmajor(&maps.a, yhat, Tc, d, kBM) ||
+        !map_kmajor(&maps.b[0], W_U, V, d, pair ? kLseBN / 2 : kLseBN))
         return cudaErrorInvalidValue;
     EpiError::Params ep;
     if (!map_out_bf16(&ep.Emap, E, Tc, V)) return cudaErrorInvalidValue;
@@ -156,8 +221,11 @@ cudaError_t launch_error_bf16(const void* yhat, const void* W_U, const int32_t* 
     ep.M = Tc;
     ep.N = V;
     ep.s = s;
-    return run_gemm<kLseBN, false, false, kLseStages, 1, EpiError>(
-        maps, ep, make_shape(Tc, V, d, kLseBN, 1, kBandM), status, st);
+    const GemmShape sh = make_shape(Tc, V, d, kLseBN, 1, band_for(pair), pair ? kPairBM : kBM);
+    if (pair)
+        return run_gemm_pair<kLseBN, false, false, kPairStages, 1, EpiError>(maps, ep, sh, status,
+                                                                             st);
+    return run_gemm<kLseBN, false, false, kLseStages, 1, EpiError>(maps, ep, sh, status, st);
 }
 
 constexpr int kProjBN = 256;
@@ -172,8 +240,11 @@ cudaError_t launch_proj_bf16(const void* E, const void* W_U, int Tc, int d, int 
     if (!map_out_f32(&ep.Cmap, g, Tc, d)) return cudaErrorInvalidValue;
     ep.M = Tc;
     ep.N = d;
+    if (use_pair())
+        return run_gemm_pair<kProjBN, false, true, kPairStages, 1, EpiStoreF32>(
+            maps, ep, make_shape(Tc, d, V, kProjBN, 1, band_for(true), kPairBM), status, st);
     return run_gemm<kProjBN, false, true, kProjStages, 1, EpiStoreF32>(
-        maps, ep, make_shape(Tc, d, V, kProjBN, 1, kBandM), status, st);
+        maps, ep, make_shape(Tc, d, V, kProjBN, 1, band_for(false)), status, st);
 }
 
 constexpr int kUpdBN = 256;
@@ -204,21 +275,36 @@ cudaError_t launch_update_bf16(int n, int T, int d, int d_ff, const void* g, con
     ep.M = d;
     ep.N = d_ff;
     ep.neg_lr = -lr;
+    if (use_pair())
+        return run_gemm_pair<kUpdBN, true, true, kPairStages, kMaxGroups, EpiUpdate>(
+            maps, ep, make_shape(d, d_ff, T, kUpdBN, n, band_for(true), kPairBM), status, st);
     return run_gemm<kUpdBN, true, true, kUpdStages, kMaxGroups, EpiUpdate>(
-        maps, ep, make_shape(d, d_ff, T, kUpdBN, n, kBandM), status, st);
+        maps, ep, make_shape(d, d_ff, T, kUpdBN, n, band_for(false)), status, st);
 }
 
 cudaError_t launch_test_gemm_bf16(int M, int N, int K, bool a_mn, bool b_mn, const void* A,
                                   const void* B, float* C, unsigned* status, cudaStream_t st) {
+    const bool pair = use_pair();
     GemmMaps<1> maps;
     bool ok = a_mn ? map_mnmajor(&maps.a, A, K, M) : map_kmajor(&maps.a, A, M, K, kBM);
-    ok = ok && (b_mn ? map_mnmajor(&maps.b[0], B, K, N) : map_kmajor(&maps.b[0], B, N, K, 256));
+    ok = ok && (b_mn ? map_mnmajor(&maps.b[0], B, K, N)
+                     : map_kmajor(&maps.b[0], B, N, K, pair ? 128 : 256));
     if (!ok) return cudaErrorInvalidValue;
     EpiStoreF32::Params ep;
     if (!map_out_f32(&ep.Cmap, C, M, N)) return cudaErrorInvalidValue;
     ep.M = M;
     ep.N = N;
-    const GemmShape sh = make_shape(M, N, K, 256, 1, kBandM);
+    if (pair) {
+        const GemmShape sh = make_shape(M, N, K, 256, 1, band_for(true), kPairBM);
+        if (!a_mn && !b_mn)
+            return run_gemm_pair<256, false, false, kPairStages, 1, EpiStoreF32>(maps, ep, sh, status, st);
+        if (!a_mn && b_mn)
+            return run_gemm_pair<256, false, true, kPairStages, 1, EpiStoreF32>(maps, ep, sh, status, st);
+        if (a_mn && b_mn)
+            return run_gemm_pair<256, true, true, kPairStages, 1, EpiStoreF32>(maps, ep, sh, status, st);
+        return cudaErrorInvalidValue;
+    }
+    const GemmShape sh = make_shape(M, N, K, 256, 1, band_for(false));
     if (!a_mn && !b_mn) return run_gemm<256, false, false, 4, 1, EpiStoreF32>(maps, ep, sh, status, st);
     if (!a_mn && b_mn) return run_gemm<256, false, true, 4, 1, EpiStoreF32>(maps, ep, sh, status, st);
     if (a_mn && b_mn) return run_gemm<256, true, true, 4, 1, EpiStoreF32>(maps, ep, sh, status, st);

@@ -45,6 +45,13 @@ cudaError_t launch_update_bf16(int n, int T, int d, int d_ff, const void* g, con
                                float lr, float* const* W_master, void* const* W_out,
                                void* const* G_out, unsigned* status, cudaStream_t st);
 
+// Which tcgen05 GEMM kernel the launchers use: 0 = single-CTA 128 x 256 tiles,
+// 1 = CTA-pair 256 x 256 tiles.
+void set_gemm_variant(int v);
+int gemm_variant();
+// Override of the L2 rasterisation band height in tiles (0 = default).
+void set_band_override(int b);
+
 // Plain GEMM with an fp32 store epilogue (test entry point).
 cudaError_t launch_test_gemm_bf16(int M, int N, int K, bool a_mn, bool b_mn, const void* A,
                                   const void* B, float* C, unsigned* status, cudaStream_t st);

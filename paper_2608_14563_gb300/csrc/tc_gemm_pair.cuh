@@ -1,0 +1,268 @@
+// tc_gemm_pair.cuh -- CTA-pair variant of the persistent tcgen05 GEMM.
+//
+// A cluster of two CTAs (on two SMs) computes one 256 x BN output tile with
+// tcgen05.mma.cta_group::2: CTA r holds rows [128 r, 128 r + 128) of the A
+// tile and columns [BN/2 r, BN/2 (r + 1)) of the B tile in its own shared
+// memory, and its TMEM receives output rows [128 r, 128 r + 128).  Per SM a
+// k-block stage is A 16 KB + B 16 KB (instead of A 16 KB + B 32 KB), so six
+// stages fit and each SM streams a third less operand data per FLOP.
+//
+//   both CTAs, warp 0   TMA loads of the CTA's halves; completion is counted
+//                       on the LEADER's (rank 0) full barrier
+//   leader, warp 1      issues the pair MMAs and commits to the empty /
+//                       accumulator-ready barriers of BOTH CTAs (multicast)
+//   both CTAs, warps 2-5  epilogue on the CTA's 128 rows; arrive on the
+//                       leader's accumulator-empty barrier (8 arrivals)
+// TMEM (2 x BN columns) is allocated collectively by warp 1 of both CTAs.
+// All waits are bounded as in the single-CTA kernel; the pair meets at a
+// cluster barrier before TMEM is freed and before either CTA exits.
+#pragma once
+
+#include "tc_gemm.cuh"
+
+namespace fpo {
+
+constexpr int kPairBM = 256;  // output rows of one pair tile
+
+template <int BN, int STAGES>
+struct GemmPairSmem {
+    static constexpr int kABytes = 128 * kBK * 2;
+    static constexpr int kBBytes = (BN / 2) * kBK * 2;
+    static constexpr int kStageBytes = kABytes + kBBytes;
+    static constexpr int kOutOffset = STAGES * kStageBytes;
+    static constexpr int kBarOffset = kOutOffset + 4 * kOutBytesPerWarp;
+    static constexpr int kNumBars = 2 * STAGES + 5;
+    static constexpr int kMiscOffset = kBarOffset + kNumBars * 8;
+    static constexpr int kBytes = kMiscOffset + 16 + 1024;
+};
+
+__device__ __forceinline__ bool mbar_try_wait_cluster(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// mbar_wait with cluster-scope acquire (the barriers of the pair kernel are
+// arrived on by the other CTA too).
+__device__ __forceinline__ bool mbar_wait_cl(uint32_t bar, uint32_t parity, const WaitGuard& g) {
+    if (mbar_try_wait_cluster(bar, parity)) return true;
+    const uint64_t t0 = global_timer_ns();
+    while (true) {
+#pragma unroll 1
+        for (int i = 0; i < 32; ++i)
+            if (mbar_try_wait_cluster(bar, parity)) return true;
+        if (*g.abort_flag) return false;
+        if (global_timer_ns() - t0 > g.limit_ns) {
+            *g.abort_flag = 1;
+            if (g.status) atomicOr(g.status, kDevTimeout);
+            return false;
+        }
+    }
+}
+
+__device__ __forceinline__ bool mbar_wait_cl_drain(uint32_t bar, uint32_t parity, uint64_t limit_ns) {
+    const uint64_t t0 = global_timer_ns();
+    while (!mbar_try_wait_cluster(bar, parity))
+        if (global_timer_ns() - t0 > limit_ns) return false;
+    return true;
+}
+
+// One CTA's half of an operand k-block, counted on the leader's barrier.
+template <bool MN, int ROWS>
+__device__ __forceinline__ void load_operand_pair(const CUtensorMap* map, uint32_t dst,
+                                                  uint32_t bar_leader, int row0, int k0) {
+    if constexpr (!MN) {
+        tma_load_2d_pair(map, dst, bar_leader, k0, row0);
+    } else {
+#pragma unroll
+        for (int i = 0; i < ROWS / 64; ++i)
+            tma_load_2d_pair(map, dst + i * (64 * kBK * 2), bar_leader, row0 + 64 * i, k0);
+    }
+}
+
+template <int BN, bool A_MN, bool B_MN, int STAGES, int MAXG, class Epi>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
+    tc_gemm_pair_kernel(const __grid_constant__ GemmMaps<MAXG> maps,
+                        const __grid_constant__ typename Epi::Params ep, const GemmShape sh,
+                        unsigned int* status, unsigned long long wait_limit_ns) {
+    using L = GemmPairSmem<BN, STAGES>;
+    constexpr int kBHalf = BN / 2;
+    constexpr uint32_t kIdesc = idesc_bf16_f32(kPairBM, BN, A_MN, B_MN);
+    constexpr int kTmemCols = 2 * BN;
+    constexpr uint16_t kBoth = 0x3;
+
+    extern __shared__ uint8_t smem_raw[];
+    const uint32_t raw = smem_u32(smem_raw);
+    const uint32_t pad = (1024u - (raw & 1023u)) & 1023u;
+    uint8_t* smem = smem_raw + pad;
+    const uint32_t sbase = raw + pad;
+
+    const uint32_t rank = cluster_ctarank();
+    const bool leader = rank == 0;
+    const long long cluster = blockIdx.x >> 1;
+    const long long n_clusters = gridDim.x >> 1;
+
+    const uint32_t bar0 = sbase + L::kBarOffset;
+    auto full_bar = [&](int s) { return bar0 + 8u * s; };
+    auto empty_bar = [&](int s) { return bar0 + 8u * (STAGES + s); };
+    auto tfull_bar = [&](int a) { return bar0 + 8u * (2 * STAGES + a); };
+    auto tempty_bar = [&](int a) { return bar0 + 8u * (2 * STAGES + 2 + a); };
+    const uint32_t drain_bar = bar0 + 8u * (2 * STAGES + 4);
+    uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(smem + L::kMiscOffset);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::kMiscOffset + 4);
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            mbar_init(full_bar(s), 1);   // leader's: one expect_tx arrival, both CTAs' bytes
+            mbar_init(empty_bar(s), 1);  // one multicast commit from the leader
+        }
+        for (int a = 0; a < 2; ++a) {
+            mbar_init(tfull_bar(a), 1);
+            mbar_init(tempty_bar(a), 8);  // leader's: 4 epilogue warps x 2 CTAs
+        }
+        mbar_init(drain_bar, 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+        tma_prefetch_desc(&maps.a);
+    }
+    if (warp == 1) {
+        tmem_alloc_pair<kTmemCols>(smem_u32(tmem_holder));
+        tmem_relinquish_pair();
+    }
+    tc_fence_before();
+    __syncthreads();
+    cluster_sync();  // barrier initialisation and TMEM allocation visible to the pair
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_holder;
+
+    const WaitGuard guard{abort_flag, status, wait_limit_ns};
+
+    if (warp == 0) {
+        // ------------------------------------------------------- TMA producer (both CTAs)
+        if (lane == 0) {
+            int stage = 0;
+            uint32_t phase = 0;
+            uint32_t issued_mask = 0, issued_parity = 0;
+            bool ok = true;
+            for (long long t = cluster; t < sh.tiles && ok; t += n_clusters) {
+                int g, mp, nb;
+                tile_coords(t, sh, g, mp, nb);
+                const CUtensorMap* bmap = &maps.b[MAXG == 1 ? 0 : g];
+                const int a_row = mp * kPairBM + 128 * static_cast<int>(rank);
+                const int b_row = nb * BN + kBHalf * static_cast<int>(rank);
+                for (int kb = 0; kb < sh.k_blocks; ++kb) {
+                    if (!mbar_wait_cl(empty_bar(stage), phase ^ 1u, guard)) { ok = false; break; }
+                    const uint32_t sa = sbase + stage * L::kStageBytes;
+                    const uint32_t sb = sa + L::kABytes;
+                    const uint32_t fb = mapa_shared(full_bar(stage), 0);
+                    if (leader) mbar_arrive_expect_tx(full_bar(stage), 2 * L::kStageBytes);
+                    load_operand_pair<A_MN, 128>(&maps.a, sa, fb, a_row, kb * kBK);
+                    load_operand_pair<B_MN, kBHalf>(bmap, sb, fb, b_row, kb * kBK);
+                    issued_mask |= 1u << stage;
+                    issued_parity = (issued_parity & ~(1u << stage)) | (phase << stage);
+                    if (++stage == STAGES) { stage = 0; phase ^= 1u; }
+                }
+            }
+            if (!ok && leader) {
+                // The leader's full barriers count both CTAs' bytes: wait for the
+                // copies in flight before the pair meets at the final barrier.
+                for (int s = 0; s < STAGES; ++s)
+                    if (issued_mask & (1u << s))
+                        mbar_wait_cl_drain(full_bar(s), (issued_parity >> s) & 1u, wait_limit_ns);
+            }
+        }
+        __syncwarp();
+    } else if (warp == 1) {
+        // ------------------------------------------------------- pair MMA (leader only)
+        if (leader && lane == 0) {
+            int stage = 0;
+            uint32_t phase = 0;
+            int acc = 0;
+            uint32_t acc_phase = 0;
+            bool ok = true, issued_any = false;
+            for (long long t = cluster; t < sh.tiles && ok; t += n_clusters) {
+                if (!mbar_wait_cl(tempty_bar(acc), acc_phase ^ 1u, guard)) { ok = false; break; }
+                tc_fence_after();
+                const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * BN);
+                for (int kb = 0; kb < sh.k_blocks; ++kb) {
+                    if (!mbar_wait_cl(full_bar(stage), phase, guard)) { ok = false; break; }
+                    tc_fence_after();
+                    const uint32_t sa = sbase + stage * L::kStageBytes;
+                    const uint32_t sb = sa + L::kABytes;
+#pragma unroll
+                    for (int kk = 0; kk < kBK / kUmmaK; ++kk)
+                        tc_mma_bf16_pair(d_tmem, operand_desc<A_MN>(sa, kk),
+                                         operand_desc<B_MN>(sb, kk), kIdesc, (kb | kk) != 0 ? 1u : 0u);
+                    issued_any = true;
+                    tc_commit_pair_multicast(empty_bar(stage), kBoth);
+                    if (++stage == STAGES) { stage = 0; phase ^= 1u; }
+                }
+                if (!ok) break;
+                tc_commit_pair_multicast(tfull_bar(acc), kBoth);
+                if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
+            }
+            if (!ok && issued_any) {
+                tc_commit_pair_multicast(drain_bar, 0x1);
+                mbar_wait_cl_drain(drain_bar, 0, wait_limit_ns);
+            }
+        }
+        __syncwarp();
+    } else {
+        // ------------------------------------------------------- epilogue (both CTAs)
+        const int q = warp & 3;
+        const int r_in_tile = 128 * static_cast<int>(rank) + q * 32 + lane;
+        EpiIO io{sbase + L::kOutOffset + static_cast<uint32_t>((warp - 2) * kOutBytesPerWarp), lane,
+                 0, 0u};
+        int acc = 0;
+        uint32_t acc_phase = 0;
+        for (long long t = cluster; t < sh.tiles; t += n_clusters) {
+            int g, mp, nb;
+            tile_coords(t, sh, g, mp, nb);
+            if (!mbar_wait_cl(tfull_bar(acc), acc_phase, guard)) break;
+            tc_fence_after();
+            const int row = mp * kPairBM + r_in_tile;
+            const int n0 = nb * BN;
+            io.row0 = mp * kPairBM + 128 * static_cast<int>(rank) + q * 32;
+            Epi epi(ep, g, row, n0);
+            const uint32_t t_row = tmem_base + (static_cast<uint32_t>(q * 32) << 16) +
+                                   static_cast<uint32_t>(acc * BN);
+#pragma unroll 1
+            for (int c = 0; c < BN / 32; ++c) {
+                float v[32];
+                tmem_ld_32x32b_x32(t_row + c * 32, v);
+                epi.chunk(ep, v, n0 + c * 32, c * 32, io);
+            }
+            epi.finish(ep, nb);
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) {
+                if (leader)
+                    mbar_arrive(tempty_bar(acc));
+                else
+                    mbar_arrive_cluster(mapa_shared(tempty_bar(acc), 0));
+            }
+            if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
+        }
+        if (lane == 0) bulk_wait_group_all();
+        __syncwarp();
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    cluster_sync();  // neither CTA frees TMEM or exits while the pair may still touch it
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc_pair<kTmemCols>(tmem_base);
+    }
+}
+
+}  // namespace fpo

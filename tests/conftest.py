@@ -31,9 +31,14 @@ _ensure_built()
 
 @pytest.fixture(scope="session")
 def fpo():
-    """The CUDA library through its Python binding; skips when no GPU is present."""
+    """The CUDA library through its Python binding; skips when no GPU is present.
+    FPO_TEST_GEMM_VARIANT=0|1 runs the suite on the single-CTA or the CTA-pair GEMM
+    kernel instead of the library default."""
     import torch
     if not torch.cuda.is_available():
         pytest.skip("no CUDA device")
     import paper_2608_14563_gb300 as lib
+    v = os.environ.get("FPO_TEST_GEMM_VARIANT")
+    if v is not None:
+        lib.set_gemm_variant(int(v))
     return lib

@@ -16,14 +16,19 @@ pytestmark = pytest.mark.gpu
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 
-@pytest.fixture(scope="module")
-def tlib(fpo):
+@pytest.fixture(scope="module", params=[0, 1], ids=["cta", "cta_pair"])
+def tlib(fpo, request):
+    """The test entry points, with the GEMM kernel variant selected (single CTA / CTA pair)."""
     lib = ctypes.CDLL(os.path.join(ROOT, "paper_2608_14563_gb300", "libfpo.so"))
     vp = ctypes.c_void_p
     lib.fpo_testing_gemm_bf16.argtypes = [ctypes.c_int64] * 3 + [ctypes.c_int32] * 2 + [vp] * 4 + [
         ctypes.c_size_t, vp]
     lib.fpo_testing_gemm_bf16.restype = ctypes.c_int32
-    return lib
+    lib.fpo_testing_set_gemm_variant.argtypes = [ctypes.c_int32]
+    lib.fpo_testing_set_gemm_variant.restype = ctypes.c_int32
+    prev = lib.fpo_testing_set_gemm_variant(request.param)
+    yield lib
+    lib.fpo_testing_set_gemm_variant(prev)
 
 
 def gemm(tlib, fpo, M, N, K, a_mn, b_mn, seed=0):
@@ -61,6 +66,13 @@ def test_many_tiles_ragged(tlib, fpo, a_mn, b_mn):
 def test_persistent_many_tiles_long_k(tlib, fpo, a_mn, b_mn):
     # more tiles than SMs (persistent loop, both TMEM buffers) and a long K ring
     got, ref = gemm(tlib, fpo, 1536, 2816, 1040, a_mn, b_mn, seed=2)
+    assert rel_frob(got, ref) < 1e-5
+
+
+@pytest.mark.parametrize("M", [256, 384, 136])
+def test_pair_row_halves(tlib, fpo, M):
+    # a tile pair whose second half is partly or wholly outside M
+    got, ref = gemm(tlib, fpo, M, 512, 192, 0, 0, seed=4)
     assert rel_frob(got, ref) < 1e-5
 
 
