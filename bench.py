@@ -110,6 +110,22 @@ class ClockSampler:
                 "power_w_max": max(power) if power else None}
 
 
+def max_over_ranks(x, device="cpu"):
+    """Max of a per-rank scalar over all ranks (the slowest replica sets the time)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return float(x)
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return t.item()
+
+
+def whole_job_tokens_per_s(tokens_per_rank, world, max_ms):
+    """Whole-job throughput: the tokens every replica processed over the slowest time."""
+    return tokens_per_rank * world / (max_ms / 1e3)
+
+
 def dist_setup():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -342,26 +358,19 @@ def run_fpo(args, wl):
             e2e_step()
         e2.record(stream)
         torch.cuda.synchronize()
-        e2e_ms = s2.elapsed_time(e2) / args.steps
-        if world > 1:
-            t = torch.tensor([e2e_ms], device=dev)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            e2e_ms = t.item()
+        e2e_ms = max_over_ranks(s2.elapsed_time(e2) / args.steps, dev)
         h2d = (h.numel() * h.element_size() + y.numel() * 4
                + sum(a.numel() * a.element_size() for a in A))
-        e2e = {"value": wl.T * world / (e2e_ms / 1e3), "unit": "tokens/s",
+        e2e = {"value": whole_job_tokens_per_s(wl.T, world, e2e_ms), "unit": "tokens/s",
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": 4, "ms_per_step": e2e_ms,
                "pipeline": "h, targets H2D on the compute stream; A_l H2D on a copy stream "
                            "overlapping the error signal; loss D2H"}
 
-    if world > 1:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = t.item()
+    ms = max_over_ranks(ms, dev)
 
     if rank == 0:
         peaks, peaks_src = load_peaks()
-        tok_s = wl.T * world / (ms / 1e3)
+        tok_s = whole_job_tokens_per_s(wl.T, world, ms)
         alg_tf = algorithmic_flops(wl) / (ms / 1e3) / 1e12
         exe_tf = (executed_flops(wl) if not stored else algorithmic_flops(wl)) / (ms / 1e3) / 1e12
         per_kernel_flops = {
@@ -411,28 +420,38 @@ def run_fpo(args, wl):
         dist.destroy_process_group()
 
 
+# Files that define each kernel whose DRAM traffic profiles/traffic.json records.
+GEMM_SOURCES = ("tc_gemm.cuh", "tc_gemm_pair.cuh", "epilogues.cuh", "error_math.cuh", "ptx.cuh",
+                "gemm_bf16.cu")
+KERNEL_SOURCES = {
+    "logits_lse_pass": GEMM_SOURCES,
+    "projection": GEMM_SOURCES,
+    "layer_update": GEMM_SOURCES,
+    "logits_to_error": ("rowwise.cu", "error_math.cuh"),
+}
+
+
 def load_traffic(kernel):
     """Per-launch DRAM bytes of `kernel` from the committed ncu summary, or None when that
-    summary is missing or was taken on different kernel sources."""
+    summary is missing or was taken on different sources of that kernel."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
-    if not os.path.exists(path):
+    if not os.path.exists(path) or kernel not in KERNEL_SOURCES:
         return None
     with open(path) as f:
         tr = json.load(f)
     ent = tr.get(kernel)
-    if not ent or ent.get("sources_sha256") != sources_digest():
+    if not ent or ent.get("sources_sha256") != sources_digest(KERNEL_SOURCES[kernel]):
         return None
     return ent.get("bytes_per_launch")
 
 
-def sources_digest():
+def sources_digest(files):
     import hashlib
     csrc = os.path.join(ROOT, "paper_2608_14563_gb300", "csrc")
     hsh = hashlib.sha256()
-    for name in sorted(os.listdir(csrc)):
-        if name.endswith((".cu", ".cuh", ".h")):
-            with open(os.path.join(csrc, name), "rb") as f:
-                hsh.update(name.encode() + f.read())
+    for name in sorted(files):
+        with open(os.path.join(csrc, name), "rb") as f:
+            hsh.update(name.encode() + f.read())
     return hsh.hexdigest()
 
 

@@ -42,6 +42,16 @@ int32_t fpo_testing_set_gemm_variant(int32_t variant);
  */
 void fpo_testing_set_band(int32_t band);
 
+/*
+ * Failure-detection check of the bounded waits every kernel uses: launches one
+ * block that waits on a shared-memory mbarrier nothing ever arrives on, with
+ * a limit of `limit_ns` nanoseconds.  The wait gives up, the kernel records
+ * FPO_ERR_TIMEOUT in the workspace status word and returns, leaving the CUDA
+ * context usable; fpo_get_device_status(workspace, stream) then reports it.
+ */
+int32_t fpo_testing_wait_timeout(uint64_t limit_ns, void* workspace, size_t workspace_bytes,
+                                 void* stream);
+
 #ifdef __cplusplus
 }
 #endif

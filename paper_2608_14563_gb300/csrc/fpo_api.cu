@@ -382,6 +382,17 @@ int32_t fpo_testing_set_gemm_variant(int32_t variant) {
 
 void fpo_testing_set_band(int32_t band) { set_band_override(band); }
 
+int32_t fpo_testing_wait_timeout(uint64_t limit_ns, void* workspace, size_t workspace_bytes,
+                                 void* stream) {
+    if (!workspace || workspace_bytes < kStatusBytes) return FPO_ERR_WORKSPACE;
+    if (limit_ns == 0 || limit_ns > 10000000000ull) return FPO_ERR_ARG;  // at most 10 s
+    int32_t rc = check_arch();
+    if (rc != FPO_OK) return rc;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    FPO_TRY(cudaMemsetAsync(workspace, 0, sizeof(unsigned), st));
+    return cuda_status(launch_wait_timeout(static_cast<unsigned*>(workspace), limit_ns, st));
+}
+
 int32_t fpo_get_device_status(void* workspace, void* stream) {
     if (!workspace) return FPO_ERR_WORKSPACE;
     cudaStream_t st = static_cast<cudaStream_t>(stream);

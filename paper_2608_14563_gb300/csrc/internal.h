@@ -73,6 +73,9 @@ cudaError_t launch_rmsnorm_vjp(int dtype, const float* g, const void* h, const v
                                const float* rho, int T, int d, float min_rms, void* out,
                                cudaStream_t st);
 
+// One block waiting on an mbarrier nothing arrives on, bounded by limit_ns.
+cudaError_t launch_wait_timeout(unsigned* status, uint64_t limit_ns, cudaStream_t st);
+
 // ------------------------------------------------------------ cosine
 int cosine_blocks(int64_t n);
 cudaError_t launch_cosine(int dtype, int64_t n, const void* X, const void* Y, double* partial,

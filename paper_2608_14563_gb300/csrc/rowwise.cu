@@ -257,6 +257,22 @@ __global__ void __launch_bounds__(kErrThreads)
     }
 }
 
+// A wait on an mbarrier that no thread arrives on: ends by its time limit.
+__global__ void wait_timeout_kernel(unsigned* status, unsigned long long limit_ns) {
+    __shared__ __align__(8) uint64_t bar;
+    __shared__ int abort_flag;
+    if (threadIdx.x == 0) {
+        mbar_init(smem_u32(&bar), 1);
+        abort_flag = 0;
+        fence_mbar_init();
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        const WaitGuard g{&abort_flag, status, limit_ns};
+        mbar_wait(smem_u32(&bar), 0, g);
+    }
+}
+
 int row_grid(int T) {
     DevInfo di;
     const int sms = current_device_info(&di) ? di.sm_count : 148;
@@ -331,6 +347,11 @@ cudaError_t launch_error_from_logits(int dtype, const float* z, const float* lse
     else
         error_from_logits_scalar_kernel<<<grid, kErrThreads, 0, st>>>(z, lse, y, M, V, s,
                                                                       static_cast<float*>(E));
+    return cudaGetLastError();
+}
+
+cudaError_t launch_wait_timeout(unsigned* status, uint64_t limit_ns, cudaStream_t st) {
+    wait_timeout_kernel<<<1, 32, 0, st>>>(status, limit_ns);
     return cudaGetLastError();
 }
 

@@ -1,0 +1,71 @@
+"""The N>1 replica path of bench.py on CPU: two gloo ranks (127.0.0.1), each with its
+own step time; the reported time is the max over ranks and the throughput counts the
+tokens of every replica.  The reference arm runs on rank 0 only."""
+import importlib.util
+import io
+import os
+import socket
+import contextlib
+
+import pytest
+import torch.multiprocessing as mp
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _bench():
+    spec = importlib.util.spec_from_file_location("bench", os.path.join(ROOT, "bench.py"))
+    b = importlib.util.module_from_spec(spec)
+    spec.loader.exec_module(b)
+    return b
+
+
+def _free_port():
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _worker(rank, world, port, q):
+    import torch.distributed as dist
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank),
+                      WORLD_SIZE=str(world), LOCAL_RANK=str(rank))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        b = _bench()
+        ms = 10.0 + 5.0 * rank  # rank 1 is the slow replica
+        dist.barrier()
+        m = b.max_over_ranks(ms)
+        tok = b.whole_job_tokens_per_s(16384, world, m)
+        # the reference arm prints only on rank 0
+        args = type("A", (), {"cpu_tokens": 1, "warmup": 0, "steps": 0, "gpus": world})()
+        buf = io.StringIO()
+        if rank != 0:
+            with contextlib.redirect_stdout(buf):
+                b.run_reference(args, None)
+        q.put((rank, m, tok, buf.getvalue()))
+    finally:
+        dist.destroy_process_group()
+
+
+def test_two_gloo_ranks_take_max_time_and_sum_tokens():
+    world, port = 2, _free_port()
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    procs = [ctx.Process(target=_worker, args=(r, world, port, q)) for r in range(world)]
+    for p in procs:
+        p.start()
+    res = sorted(q.get(timeout=120) for _ in range(world))
+    for p in procs:
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    for rank, m, tok, out in res:
+        assert m == 15.0
+        assert abs(tok - 16384 * 2 / 0.015) < 1e-6
+        assert out == ""
+
+
+def test_single_rank_needs_no_process_group():
+    b = _bench()
+    assert b.max_over_ranks(12.5) == 12.5
+    assert b.whole_job_tokens_per_s(100, 1, 10.0) == 10000.0
