@@ -227,6 +227,7 @@ def workload_config(wl, args):
             "lr": wl.lr, "t_chunk": args.t_chunk or wl.T, "global_batch_tokens": wl.T * args.gpus,
             "error_matrix": {"auto": "stored-logits (auto)", "recompute": "recompute",
                              "stored": "stored-logits"}[args.algo],
+            "norms_composed": "final + post-FFN per layer" if args.post_ffn_norm else "final",
             "l2": "inputs larger than L2 (W_U %.0f MB, A_l %.2f GB per step); no flush"
                   % (wl.V * wl.d * 2 / 1e6, wl.layers * wl.T * wl.d_ff * 2 / 1e9)}
 
@@ -260,6 +261,11 @@ def run_fpo(args, wl):
     Wo = [torch.empty(wl.d, wl.d_ff, dtype=torch.bfloat16, device=dev) for _ in range(wl.layers)]
     g = torch.empty_like(h)
     loss = torch.empty(1, dtype=torch.float32, device=dev)
+    post = args.post_ffn_norm
+    if post:  # per-layer MLP outputs, post-FFN norm weights and layer-specific signals
+        m_out = [synth.make_mlp_out(wl_r, l, dev) for l in range(wl.layers)]
+        gp = [synth.make_post_norm_w(wl_r, l, dev) for l in range(wl.layers)]
+        g_l = [torch.empty_like(h) for _ in range(wl.layers)]
     algo = {"auto": fpo.ES_AUTO, "recompute": fpo.ES_RECOMPUTE,
             "stored": fpo.ES_STORED_LOGITS}[args.algo]
     stored = algo != fpo.ES_RECOMPUTE
@@ -273,13 +279,24 @@ def run_fpo(args, wl):
     # fwd, mean, vjp, update + per chunk (stored: logits, combine, E, projection;
     # recompute: E pass, projection; plus one logits pass and one combine)
     launches_per_step = 4 + (4 * n_chunks if stored else 2 + 2 * n_chunks)
+    if post:
+        launches_per_step += wl.layers
 
     def step(stage_events=None, upd_events=None):
         fpo.error_signal(h, w, W_U, y, g, eps=wl.eps, min_rms=wl.min_rms, t_chunk=args.t_chunk,
                          loss_out=loss, workspace=ws_es, stage_events=stage_events, algo=algo)
+        if post:
+            if upd_events:
+                upd_events[2].record(stream)
+            for l in range(wl.layers):
+                fpo.rmsnorm_vjp(g, m_out[l], gp[l], g_l[l], eps=wl.eps, min_rms=wl.min_rms)
         if upd_events:
             upd_events[0].record(stream)
-        fpo.layer_update_grouped(g, A, wl.lr, W_masters=Wm, W_outs=Wo, workspace=ws_up)
+        if post:
+            fpo.layer_update_grouped_signals(g_l, A, wl.lr, W_masters=Wm, W_outs=Wo,
+                                             workspace=ws_up)
+        else:
+            fpo.layer_update_grouped(g, A, wl.lr, W_masters=Wm, W_outs=Wo, workspace=ws_up)
         if upd_events:
             upd_events[1].record(stream)
 
@@ -291,7 +308,7 @@ def run_fpo(args, wl):
     # per-stage events for every timed step (recorded once so their handles exist)
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(fpo.STAGE_EVENTS)]
           for _ in range(args.steps)]
-    uev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(args.steps)]
+    uev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
     for e in [x for row in ev + uev for x in row]:
         e.record(stream)
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -318,6 +335,9 @@ def run_fpo(args, wl):
                 for k, n in enumerate(names)}
     stage_ms["layer_update"] = statistics.mean(uev[i][0].elapsed_time(uev[i][1])
                                                for i in range(args.steps))
+    if post:
+        stage_ms["post_ffn_vjp"] = statistics.mean(uev[i][2].elapsed_time(uev[i][0])
+                                                   for i in range(args.steps))
 
     # ------------------------------------------------ end to end through the public API
     e2e = None
@@ -325,6 +345,7 @@ def run_fpo(args, wl):
         h_host = h.cpu().pin_memory()
         y_host = y.cpu().pin_memory()
         A_host = [a.cpu().pin_memory() for a in A]
+        m_host = [x.cpu().pin_memory() for x in m_out] if post else []
         loss_host = torch.empty(1, dtype=torch.float32).pin_memory()
 
         copy_stream = torch.cuda.Stream(device=dev)
@@ -340,11 +361,20 @@ def run_fpo(args, wl):
             with torch.cuda.stream(copy_stream):
                 for a_d, a_h in zip(A, A_host):
                     a_d.copy_(a_h, non_blocking=True)
+                for m_d, m_h in zip(m_out if post else [], m_host):
+                    m_d.copy_(m_h, non_blocking=True)
                 a_ready.record(copy_stream)
             fpo.error_signal(h, w, W_U, y, g, eps=wl.eps, min_rms=wl.min_rms,
                              t_chunk=args.t_chunk, loss_out=loss, workspace=ws_es, algo=algo)
             stream.wait_event(a_ready)
-            fpo.layer_update_grouped(g, A, wl.lr, W_masters=Wm, W_outs=Wo, workspace=ws_up)
+            if post:
+                for l in range(wl.layers):
+                    fpo.rmsnorm_vjp(g, m_out[l], gp[l], g_l[l], eps=wl.eps, min_rms=wl.min_rms)
+            if post:
+                fpo.layer_update_grouped_signals(g_l, A, wl.lr, W_masters=Wm, W_outs=Wo,
+                                                 workspace=ws_up)
+            else:
+                fpo.layer_update_grouped(g, A, wl.lr, W_masters=Wm, W_outs=Wo, workspace=ws_up)
             loss_host.copy_(loss, non_blocking=True)
 
         for _ in range(max(1, args.warmup)):
@@ -361,6 +391,8 @@ def run_fpo(args, wl):
         e2e_ms = max_over_ranks(s2.elapsed_time(e2) / args.steps, dev)
         h2d = (h.numel() * h.element_size() + y.numel() * 4
                + sum(a.numel() * a.element_size() for a in A))
+        if post:
+            h2d += sum(x.numel() * x.element_size() for x in m_out)
         e2e = {"value": whole_job_tokens_per_s(wl.T, world, e2e_ms), "unit": "tokens/s",
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": 4, "ms_per_step": e2e_ms,
                "pipeline": "h, targets H2D on the compute stream; A_l H2D on a copy stream "
@@ -473,6 +505,8 @@ def main():
     ap.add_argument("--impl", choices=("fpo", "reference"), default="fpo")
     ap.add_argument("--workload", default="olmo", help="olmo | qwen | falcon | diag")
     ap.add_argument("--t-chunk", type=int, default=0, help="tokens per E chunk (0 = all)")
+    ap.add_argument("--post-ffn-norm", action="store_true",
+                    help="compose each layer's post-FFN RMSNorm VJP (OLMo-2 layout) in the step")
     ap.add_argument("--algo", choices=("auto", "recompute", "stored"), default="auto",
                     help="how the error matrix is formed (fpo_es_algo)")
     ap.add_argument("--gemm-variant", type=int, choices=(-1, 0, 1), default=-1,

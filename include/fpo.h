@@ -188,6 +188,34 @@ int32_t fpo_layer_update_grouped(int32_t n_layers, int64_t T, int64_t d, int64_t
                                  void* const* G_out, void* workspace, size_t workspace_bytes,
                                  void* stream);
 
+/*
+ * fpo_layer_update_grouped_signals -- fpo_layer_update_grouped where layer l
+ * has its own signal g[l] (HOST array of n_layers device pointers, [T, d]
+ * each): the layer-specific g~^(l) of Sec. 3.1 step 4 for architectures with a
+ * per-layer post-feedforward RMSNorm (OLMo-2, Gemma 3), obtained from g~ with
+ * fpo_rmsnorm_vjp at that layer's cached MLP output.  Entries may repeat.
+ */
+int32_t fpo_layer_update_grouped_signals(int32_t n_layers, int64_t T, int64_t d, int64_t d_ff,
+                                         int32_t dtype, const void* const* g,
+                                         const void* const* A, float lr, float* const* W_master,
+                                         void* const* W_out, void* const* G_out, void* workspace,
+                                         size_t workspace_bytes, void* stream);
+
+/*
+ * fpo_rmsnorm_vjp -- the closed-form RMSNorm Jacobian applied to an upstream
+ * gradient (App. E Eq. (rmsnorm-vjp) with the min-RMS clamp), at any norm the
+ * method corrects for; for the post-feedforward norm of OLMo-2 / Gemma 3
+ * (Sec. 3.2) x is the layer's cached MLP output and gamma its post-FFN weight:
+ *
+ *   rho = sqrt(mean_j x_j^2 + eps),  xhat = x / rho
+ *   g_out = (gamma (.) g - xhat <xhat, gamma (.) g> / d) / max(rho, min_rms)
+ *
+ * g, x, g_out [T, d] and gamma [d] in dtype; g_out may not alias g or x.
+ * fp32 accumulation; no workspace; asynchronous on `stream`.
+ */
+int32_t fpo_rmsnorm_vjp(int64_t T, int64_t d, int32_t dtype, const void* g, const void* x,
+                        const void* gamma, float eps, float min_rms, void* g_out, void* stream);
+
 /* Bytes of workspace fpo_cosine needs for n elements. */
 size_t fpo_cosine_workspace(int64_t n);
 

@@ -9,6 +9,8 @@ Each function follows one passage of the paper:
 
 * :func:`error_signal`  Sec. 3.1 steps 2-4, Eq. (gproj), App. E Eq. (rmsnorm-vjp)
   with the min-RMS clamp.
+* :func:`rmsnorm_vjp`   App. E Eq. (rmsnorm-vjp) at any norm (the per-layer post-FFN
+  norm of OLMo-2 / Gemma 3, Sec. 3.2).
 * :func:`pseudograd`    Sec. 3.1 step 5, Eq. (w3update).
 * :func:`sgd_update`    App. A, fp32 master weights cast to bf16.
 * :func:`cosine`        Sec. 2.2, Eq. (cosine).
@@ -53,6 +55,8 @@ def _load():
     lib.oracle_error_signal.argtypes = [i64, i64, i64, i32, vp, vp, vp, vp, dbl, dbl, dbl,
                                         vp, i64, vp, vp, vp, vp, vp, vp]
     lib.oracle_error_signal.restype = i32
+    lib.oracle_rmsnorm_vjp.argtypes = [i64, i64, i32, vp, i32, vp, vp, dbl, dbl, vp]
+    lib.oracle_rmsnorm_vjp.restype = i32
     lib.oracle_pseudograd.argtypes = [i64, i64, i64, i32, vp, i32, vp, vp, vp, i64, vp]
     lib.oracle_pseudograd.restype = i32
     lib.oracle_sgd_update.argtypes = [i64, vp, vp, dbl, vp, vp]
@@ -119,6 +123,27 @@ def error_signal(h, w, W_U, y, *, eps=1e-6, min_rms=0.5, s=1.0, rows=None, want_
         raise ValueError(f"oracle_error_signal failed ({rc})")
     if want_e:
         out["e"] = e
+    return out
+
+
+def rmsnorm_vjp(g, x, gamma, *, eps=1e-6, min_rms=0.5):
+    """App. E Eq. (rmsnorm-vjp) with the min-RMS clamp at norm input x, weight gamma.
+
+    g, x: [T, d]; gamma: [d] (same dtype as x).  Returns fp64 [T, d].
+    """
+    dtg, g = _typed(g)
+    dtx, x = _typed(x)
+    dtw, gamma = _typed(gamma)
+    if dtw != dtx:
+        raise TypeError("x and gamma must share one dtype")
+    T, d = x.shape
+    if g.shape != x.shape or gamma.shape != (d,):
+        raise ValueError("g and x must be [T, d] and gamma [d]")
+    out = np.zeros((T, d))
+    rc = _load().oracle_rmsnorm_vjp(T, d, dtg, _ptr(g), dtx, _ptr(x), _ptr(gamma), eps, min_rms,
+                                    _ptr(out))
+    if rc != 0:
+        raise ValueError(f"oracle_rmsnorm_vjp failed ({rc})")
     return out
 
 

@@ -12,6 +12,7 @@
  *
  *   oracle_error_signal  Sec. 3.1 steps 2-4, Eq. (gproj), App. E Eq. (rmsnorm-vjp)
  *                        and the min-RMS clamp (Sec. 3.2 / App. E)
+ *   oracle_rmsnorm_vjp   App. E Eq. (rmsnorm-vjp) at any norm (post-FFN, Sec. 3.2)
  *   oracle_pseudograd    Sec. 3.1 step 5, Eq. (w3update): G = g~^T h_mid
  *   oracle_sgd_update    App. A (fp32 master weights, cast to bf16)
  *   oracle_cosine        Sec. 2.2, Eq. (cosine)
@@ -141,6 +142,39 @@ int oracle_error_signal(int64_t T, int64_t d, int64_t V, int dt,
         free(gt);
     }
     return bad_target ? -2 : 0;
+}
+
+/*
+ * App. E Eq. (rmsnorm-vjp), the closed-form RMSNorm Jacobian applied to an
+ * upstream gradient g at a cached norm input x with weight gamma (the same
+ * expression the paper composes at every norm it corrects for: the final norm,
+ * and per layer the post-feedforward norm of OLMo-2 / Gemma 3, Sec. 3.2):
+ *   rho  = sqrt(mean_j x_j^2 + eps),  xhat = x / rho
+ *   c    = <xhat, gamma (.) g>
+ *   out  = (gamma (.) g - xhat c / d) / max(rho, rho_min)
+ * g, x: [T, d] (dtypes dt_g, dt_x); gamma: [d] (dt_x); out: [T, d] fp64.
+ */
+int oracle_rmsnorm_vjp(int64_t T, int64_t d, int dt_g, const void* g, int dt_x, const void* x,
+                       const void* gamma, double eps, double min_rms, double* out) {
+    if (T < 0 || d <= 0 || !out || (T > 0 && (!g || !x || !gamma))) return -1;
+#pragma omp parallel for schedule(static)
+    for (int64_t t = 0; t < T; ++t) {
+        double ss = 0.0;
+        for (int64_t j = 0; j < d; ++j) {
+            double v = orc_load(dt_x, x, t * d + j);
+            ss += v * v;
+        }
+        double rh = sqrt(ss / (double)d + eps);
+        double c = 0.0;
+        for (int64_t j = 0; j < d; ++j)
+            c += (orc_load(dt_x, x, t * d + j) / rh) * orc_load(dt_x, gamma, j) *
+                 orc_load(dt_g, g, t * d + j);
+        double denom = rh > min_rms ? rh : min_rms;
+        for (int64_t j = 0; j < d; ++j)
+            out[t * d + j] = (orc_load(dt_x, gamma, j) * orc_load(dt_g, g, t * d + j) -
+                              (orc_load(dt_x, x, t * d + j) / rh) * c / (double)d) / denom;
+    }
+    return 0;
 }
 
 /*

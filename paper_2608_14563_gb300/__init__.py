@@ -59,6 +59,13 @@ _lib.fpo_layer_update_grouped.argtypes = [_i32, _i64, _i64, _i64, _i32, _vp,
                                           ctypes.POINTER(_vp), _f32, ctypes.POINTER(_vp),
                                           ctypes.POINTER(_vp), ctypes.POINTER(_vp), _vp, _sz, _vp]
 _lib.fpo_layer_update_grouped.restype = _i32
+_lib.fpo_layer_update_grouped_signals.argtypes = [_i32, _i64, _i64, _i64, _i32,
+                                                  ctypes.POINTER(_vp), ctypes.POINTER(_vp), _f32,
+                                                  ctypes.POINTER(_vp), ctypes.POINTER(_vp),
+                                                  ctypes.POINTER(_vp), _vp, _sz, _vp]
+_lib.fpo_layer_update_grouped_signals.restype = _i32
+_lib.fpo_rmsnorm_vjp.argtypes = [_i64, _i64, _i32, _vp, _vp, _vp, _f32, _f32, _vp, _vp]
+_lib.fpo_rmsnorm_vjp.restype = _i32
 _lib.fpo_cosine_workspace.argtypes = [_i64]
 _lib.fpo_cosine_workspace.restype = _sz
 _lib.fpo_cosine.argtypes = [_i64, _i32, _vp, _vp, _vp, _vp, _sz, _vp]
@@ -213,6 +220,31 @@ def layer_update_grouped(g, As, lr, *, W_masters=None, W_outs=None, G_outs=None,
                                        _stream(stream))
     _check(rc, "fpo_layer_update_grouped")
     return workspace
+
+
+def layer_update_grouped_signals(gs, As, lr, *, W_masters=None, W_outs=None, G_outs=None,
+                                 workspace=None, stream=None):
+    """fpo_layer_update_grouped_signals: layer l uses its own signal gs[l]."""
+    n = len(As)
+    T, d = gs[0].shape
+    d_ff = As[0].shape[1]
+    if workspace is None:
+        workspace = _workspace(layer_update_workspace(), gs[0].device)
+    rc = _lib.fpo_layer_update_grouped_signals(
+        n, T, d, d_ff, _dtype_code(gs[0]), _ptr_array(gs, n), _ptr_array(As, n), float(lr),
+        _ptr_array(W_masters, n), _ptr_array(W_outs, n), _ptr_array(G_outs, n), _ptr(workspace),
+        workspace.numel(), _stream(stream))
+    _check(rc, "fpo_layer_update_grouped_signals")
+    return workspace
+
+
+def rmsnorm_vjp(g, x, gamma, g_out, *, eps=1e-6, min_rms=0.5, stream=None):
+    """fpo_rmsnorm_vjp: the RMSNorm Jacobian (with the min-RMS clamp) applied to g at x."""
+    T, d = x.shape
+    rc = _lib.fpo_rmsnorm_vjp(T, d, _dtype_code(x), _ptr(g), _ptr(x), _ptr(gamma), float(eps),
+                              float(min_rms), _ptr(g_out), _stream(stream))
+    _check(rc, "fpo_rmsnorm_vjp")
+    return g_out
 
 
 # --------------------------------------------------------------------------- cosine

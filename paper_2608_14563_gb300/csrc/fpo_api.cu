@@ -264,10 +264,11 @@ int32_t fpo_error_signal(const fpo_error_signal_desc* desc, const void* h, const
 
 size_t fpo_layer_update_workspace(void) { return kStatusBytes; }
 
-int32_t fpo_layer_update_grouped(int32_t n_layers, int64_t T, int64_t d, int64_t d_ff,
-                                 int32_t dtype, const void* g, const void* const* A, float lr,
-                                 float* const* W_master, void* const* W_out, void* const* G_out,
-                                 void* workspace, size_t workspace_bytes, void* stream) {
+int32_t fpo_layer_update_grouped_signals(int32_t n_layers, int64_t T, int64_t d, int64_t d_ff,
+                                         int32_t dtype, const void* const* g,
+                                         const void* const* A, float lr, float* const* W_master,
+                                         void* const* W_out, void* const* G_out, void* workspace,
+                                         size_t workspace_bytes, void* stream) {
     if (dtype != FPO_F32 && dtype != FPO_BF16) return FPO_ERR_DTYPE;
     if (n_layers < 1 || n_layers > FPO_MAX_GROUPED_LAYERS) return FPO_ERR_SHAPE;
     if (T < 0 || d <= 0 || d_ff <= 0 || T > INT_MAX || d > INT_MAX || d_ff > INT_MAX)
@@ -276,16 +277,16 @@ int32_t fpo_layer_update_grouped(int32_t n_layers, int64_t T, int64_t d, int64_t
     if (!(lr == lr)) return FPO_ERR_ARG;
     if (!workspace || workspace_bytes < kStatusBytes) return FPO_ERR_WORKSPACE;
     if ((reinterpret_cast<uintptr_t>(workspace) % kAlign) != 0) return FPO_ERR_ALIGN;
-    if (!A || (T > 0 && !g)) return FPO_ERR_NULL;
-    if (!aligned16(g)) return FPO_ERR_ALIGN;
+    if (!A || !g) return FPO_ERR_NULL;
     for (int l = 0; l < n_layers; ++l) {
         float* wm = W_master ? W_master[l] : nullptr;
         void* wo = W_out ? W_out[l] : nullptr;
         void* go = G_out ? G_out[l] : nullptr;
-        if (T > 0 && !A[l]) return FPO_ERR_NULL;
+        if (T > 0 && (!A[l] || !g[l])) return FPO_ERR_NULL;
         if (!wm && !go) return FPO_ERR_NULL;
         if (wo && !wm) return FPO_ERR_NULL;
-        if (!aligned16(A[l]) || !aligned16(wm) || !aligned16(wo) || !aligned16(go))
+        if (!aligned16(g[l]) || !aligned16(A[l]) || !aligned16(wm) || !aligned16(wo) ||
+            !aligned16(go))
             return FPO_ERR_ALIGN;
     }
     int32_t rc = check_arch();
@@ -310,9 +311,38 @@ int32_t fpo_layer_update_grouped(int32_t n_layers, int64_t T, int64_t d, int64_t
         return cuda_status(launch_update_bf16(n_layers, Ti, di, fi, g, A, lr, W_master, W_out,
                                               G_out, status, st));
     return cuda_status(launch_update_f32(
-        n_layers, Ti, di, fi, static_cast<const float*>(g), reinterpret_cast<const float* const*>(A),
-        lr, W_master, reinterpret_cast<float* const*>(W_out), reinterpret_cast<float* const*>(G_out),
-        st));
+        n_layers, Ti, di, fi, reinterpret_cast<const float* const*>(g),
+        reinterpret_cast<const float* const*>(A), lr, W_master,
+        reinterpret_cast<float* const*>(W_out), reinterpret_cast<float* const*>(G_out), st));
+}
+
+int32_t fpo_layer_update_grouped(int32_t n_layers, int64_t T, int64_t d, int64_t d_ff,
+                                 int32_t dtype, const void* g, const void* const* A, float lr,
+                                 float* const* W_master, void* const* W_out, void* const* G_out,
+                                 void* workspace, size_t workspace_bytes, void* stream) {
+    if (n_layers < 1 || n_layers > FPO_MAX_GROUPED_LAYERS) return FPO_ERR_SHAPE;
+    if (T > 0 && !g) return FPO_ERR_NULL;
+    const void* gs[FPO_MAX_GROUPED_LAYERS];
+    for (int l = 0; l < n_layers; ++l) gs[l] = g;
+    return fpo_layer_update_grouped_signals(n_layers, T, d, d_ff, dtype, gs, A, lr, W_master,
+                                            W_out, G_out, workspace, workspace_bytes, stream);
+}
+
+int32_t fpo_rmsnorm_vjp(int64_t T, int64_t d, int32_t dtype, const void* g, const void* x,
+                        const void* gamma, float eps, float min_rms, void* g_out, void* stream) {
+    if (dtype != FPO_F32 && dtype != FPO_BF16) return FPO_ERR_DTYPE;
+    if (T < 0 || d <= 0 || T > INT_MAX || d > INT_MAX) return FPO_ERR_SHAPE;
+    if (dtype == FPO_BF16 && d % 8 != 0) return FPO_ERR_SHAPE;
+    if (!(eps >= 0.f) || !(min_rms >= 0.f)) return FPO_ERR_ARG;
+    if (T > 0 && (!g || !x || !gamma || !g_out)) return FPO_ERR_NULL;
+    if (!aligned16(g) || !aligned16(x) || !aligned16(gamma) || !aligned16(g_out))
+        return FPO_ERR_ALIGN;
+    int32_t rc = check_arch();
+    if (rc != FPO_OK) return rc;
+    if (T == 0) return FPO_OK;
+    return cuda_status(launch_rmsnorm_vjp_at(dtype, g, x, gamma, static_cast<int>(T),
+                                             static_cast<int>(d), eps, min_rms, g_out,
+                                             static_cast<cudaStream_t>(stream)));
 }
 
 int32_t fpo_layer_update(int64_t T, int64_t d, int64_t d_ff, int32_t dtype, const void* g,

@@ -174,7 +174,7 @@ cudaError_t launch_lse_partial_bf16(const void* yhat, const void* W_U, const int
                                     unsigned* status, cudaStream_t st) {
     const bool pair = use_pair();
     GemmMaps<1> maps;
-    if (!map_kmajor(&maps.a, yhat, T, d, kBM) ||
+    if (!map_kmajor(&maps.a[0], yhat, T, d, kBM) ||
         !map_kmajor(&maps.b[0], W_U, V, d, pair ? kLseBN / 2 : kLseBN))
         return cudaErrorInvalidValue;
     const GemmShape sh = make_shape(T, V, d, kLseBN, 1, band_for(pair), pair ? kPairBM : kBM);
@@ -193,7 +193,7 @@ cudaError_t launch_lse_partial_bf16(const void* yhat, const void* W_U, const int
         return run_gemm<kLseBN, false, false, kLseStages, 1, EpiLseStoreZ>(maps, ep, sh, status, st);
     }
     EpiLsePartial::Params ep;
-    ep.zmap = maps.a;  // unused
+    ep.zmap = maps.a[0];  // unused
     ep.part = part;
     ep.part_ld = part_ld;
     ep.zy = zy;
@@ -211,7 +211,7 @@ cudaError_t launch_error_bf16(const void* yhat, const void* W_U, const int32_t* 
                               cudaStream_t st) {
     const bool pair = use_pair();
     GemmMaps<1> maps;
-    if (!map_kmajor(&maps.a, yhat, Tc, d, kBM) ||
+    if (!map_kmajor(&maps.a[0], yhat, Tc, d, kBM) ||
         !map_kmajor(&maps.b[0], W_U, V, d, pair ? kLseBN / 2 : kLseBN))
         return cudaErrorInvalidValue;
     EpiError::Params ep;
@@ -234,7 +234,7 @@ constexpr int kProjStages = 4;
 cudaError_t launch_proj_bf16(const void* E, const void* W_U, int Tc, int d, int V, float* g,
                              unsigned* status, cudaStream_t st) {
     GemmMaps<1> maps;
-    if (!map_kmajor(&maps.a, E, Tc, V, kBM) || !map_mnmajor(&maps.b[0], W_U, V, d))
+    if (!map_kmajor(&maps.a[0], E, Tc, V, kBM) || !map_mnmajor(&maps.b[0], W_U, V, d))
         return cudaErrorInvalidValue;
     EpiStoreF32::Params ep;
     if (!map_out_f32(&ep.Cmap, g, Tc, d)) return cudaErrorInvalidValue;
@@ -250,22 +250,27 @@ cudaError_t launch_proj_bf16(const void* E, const void* W_U, int Tc, int d, int 
 constexpr int kUpdBN = 256;
 constexpr int kUpdStages = 4;
 
-cudaError_t launch_update_bf16(int n, int T, int d, int d_ff, const void* g, const void* const* A,
-                               float lr, float* const* W_master, void* const* W_out,
-                               void* const* G_out, unsigned* status, cudaStream_t st) {
+cudaError_t launch_update_bf16(int n, int T, int d, int d_ff, const void* const* g,
+                               const void* const* A, float lr, float* const* W_master,
+                               void* const* W_out, void* const* G_out, unsigned* status,
+                               cudaStream_t st) {
     if (n < 1 || n > kMaxGroups) return cudaErrorInvalidValue;
     static GemmMaps<kMaxGroups> maps;  // host staging; copied into the launch parameters
     static EpiUpdate::Params ep;
     static std::mutex mu;
     std::lock_guard<std::mutex> lock(mu);
-    if (!map_mnmajor(&maps.a, g, T, d)) return cudaErrorInvalidValue;
     for (int l = 0; l < n; ++l) {
+        if (l > 0 && g[l] == g[0])
+            maps.a[l] = maps.a[0];
+        else if (!map_mnmajor(&maps.a[l], g[l], T, d))
+            return cudaErrorInvalidValue;
         if (!map_mnmajor(&maps.b[l], A[l], T, d_ff)) return cudaErrorInvalidValue;
         ep.W_master[l] = W_master ? W_master[l] : nullptr;
         ep.W_out[l] = W_out ? static_cast<__nv_bfloat16*>(W_out[l]) : nullptr;
         ep.G_out[l] = G_out ? static_cast<__nv_bfloat16*>(G_out[l]) : nullptr;
     }
     for (int l = n; l < kMaxGroups; ++l) {
+        maps.a[l] = maps.a[0];
         maps.b[l] = maps.b[0];
         ep.W_master[l] = nullptr;
         ep.W_out[l] = nullptr;
@@ -286,7 +291,7 @@ cudaError_t launch_test_gemm_bf16(int M, int N, int K, bool a_mn, bool b_mn, con
                                   const void* B, float* C, unsigned* status, cudaStream_t st) {
     const bool pair = use_pair();
     GemmMaps<1> maps;
-    bool ok = a_mn ? map_mnmajor(&maps.a, A, K, M) : map_kmajor(&maps.a, A, M, K, kBM);
+    bool ok = a_mn ? map_mnmajor(&maps.a[0], A, K, M) : map_kmajor(&maps.a[0], A, M, K, kBM);
     ok = ok && (b_mn ? map_mnmajor(&maps.b[0], B, K, N)
                      : map_kmajor(&maps.b[0], B, N, K, pair ? 128 : 256));
     if (!ok) return cudaErrorInvalidValue;

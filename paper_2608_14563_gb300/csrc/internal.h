@@ -40,10 +40,11 @@ cudaError_t launch_error_bf16(const void* yhat, const void* W_U, const int32_t* 
 cudaError_t launch_proj_bf16(const void* E, const void* W_U, int Tc, int d, int V, float* g,
                              unsigned* status, cudaStream_t st);
 
-// Grouped pseudogradient update over n layers.
-cudaError_t launch_update_bf16(int n, int T, int d, int d_ff, const void* g, const void* const* A,
-                               float lr, float* const* W_master, void* const* W_out,
-                               void* const* G_out, unsigned* status, cudaStream_t st);
+// Grouped pseudogradient update over n layers, layer l with signal g[l] (host array).
+cudaError_t launch_update_bf16(int n, int T, int d, int d_ff, const void* const* g,
+                               const void* const* A, float lr, float* const* W_master,
+                               void* const* W_out, void* const* G_out, unsigned* status,
+                               cudaStream_t st);
 
 // Which tcgen05 GEMM kernel the launchers use: 0 = single-CTA 128 x 256 tiles,
 // 1 = CTA-pair 256 x 256 tiles.
@@ -72,6 +73,10 @@ cudaError_t launch_cast_f32(int dtype, const float* src, size_t n, void* dst, cu
 cudaError_t launch_rmsnorm_vjp(int dtype, const float* g, const void* h, const void* w,
                                const float* rho, int T, int d, float min_rms, void* out,
                                cudaStream_t st);
+// RMSNorm VJP at a norm input x (rho from x itself): out = vjp(g, x, gamma), all in dtype.
+cudaError_t launch_rmsnorm_vjp_at(int dtype, const void* g, const void* x, const void* gamma,
+                                  int T, int d, float eps, float min_rms, void* out,
+                                  cudaStream_t st);
 
 // One block waiting on an mbarrier nothing arrives on, bounded by limit_ns.
 cudaError_t launch_wait_timeout(unsigned* status, uint64_t limit_ns, cudaStream_t st);
@@ -91,7 +96,7 @@ cudaError_t launch_error_f32(const float* yhat, const float* W_U, const int32_t*
                              cudaStream_t st);
 cudaError_t launch_proj_f32(const float* E, const float* W_U, int Tc, int d, int V, float* g,
                             cudaStream_t st);
-cudaError_t launch_update_f32(int n, int T, int d, int d_ff, const float* g,
+cudaError_t launch_update_f32(int n, int T, int d, int d_ff, const float* const* g,
                               const float* const* A, float lr, float* const* W_master,
                               float* const* W_out, float* const* G_out, cudaStream_t st);
 

@@ -158,6 +158,49 @@ __global__ void __launch_bounds__(kRowThreads)
     }
 }
 
+// RMSNorm VJP at a norm input x whose rho is recomputed from x: one pass for
+// sum x^2 and sum x gamma g, then the output pass (App. E Eq. rmsnorm-vjp).
+template <typename TT, int VEC>
+__global__ void __launch_bounds__(kRowThreads)
+    rmsnorm_vjp_at_kernel(const TT* __restrict__ g, const TT* __restrict__ x,
+                          const TT* __restrict__ gamma, int T, int d, float eps, float min_rms,
+                          TT* __restrict__ out) {
+    const int lane = threadIdx.x & 31;
+    const int wpb = blockDim.x >> 5;
+    for (int row = blockIdx.x * wpb + (threadIdx.x >> 5); row < T; row += gridDim.x * wpb) {
+        const TT* gr = g + static_cast<size_t>(row) * d;
+        const TT* xr = x + static_cast<size_t>(row) * d;
+        float ss = 0.f, xg = 0.f;
+        for (int j = lane * VEC; j < d; j += 32 * VEC) {
+            float gv[VEC], xv[VEC], wv[VEC];
+            ld_vec<VEC>(gr + j, gv);
+            ld_vec<VEC>(xr + j, xv);
+            ld_vec<VEC>(gamma + j, wv);
+#pragma unroll
+            for (int k = 0; k < VEC; ++k) {
+                ss = fmaf(xv[k], xv[k], ss);
+                xg = fmaf(xv[k], wv[k] * gv[k], xg);
+            }
+        }
+        ss = warp_sum(ss);
+        xg = warp_sum(xg);
+        const float r = sqrtf(ss / static_cast<float>(d) + eps);
+        const float inv_r = 1.0f / r;
+        const float kd = (xg * inv_r) / static_cast<float>(d);
+        const float pref = 1.0f / fmaxf(r, min_rms);
+        TT* orow = out + static_cast<size_t>(row) * d;
+        for (int j = lane * VEC; j < d; j += 32 * VEC) {
+            float gv[VEC], xv[VEC], wv[VEC], o[VEC];
+            ld_vec<VEC>(gr + j, gv);
+            ld_vec<VEC>(xr + j, xv);
+            ld_vec<VEC>(gamma + j, wv);
+#pragma unroll
+            for (int k = 0; k < VEC; ++k) o[k] = (wv[k] * gv[k] - (xv[k] * inv_r) * kd) * pref;
+            st_vec<VEC>(orow + j, o);
+        }
+    }
+}
+
 __global__ void __launch_bounds__(kRowThreads)
     lse_combine_kernel(const float2* __restrict__ part, int n_tiles, int T,
                        const float* __restrict__ zy, float* __restrict__ lse, float* __restrict__ ce) {
@@ -352,6 +395,28 @@ cudaError_t launch_error_from_logits(int dtype, const float* z, const float* lse
 
 cudaError_t launch_wait_timeout(unsigned* status, uint64_t limit_ns, cudaStream_t st) {
     wait_timeout_kernel<<<1, 32, 0, st>>>(status, limit_ns);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_rmsnorm_vjp_at(int dtype, const void* g, const void* x, const void* gamma,
+                                  int T, int d, float eps, float min_rms, void* out,
+                                  cudaStream_t st) {
+    if (T <= 0) return cudaSuccess;
+    const int grid = row_grid(T);
+    if (dtype == 1) {
+        rmsnorm_vjp_at_kernel<__nv_bfloat16, 8><<<grid, kRowThreads, 0, st>>>(
+            static_cast<const __nv_bfloat16*>(g), static_cast<const __nv_bfloat16*>(x),
+            static_cast<const __nv_bfloat16*>(gamma), T, d, eps, min_rms,
+            static_cast<__nv_bfloat16*>(out));
+    } else if (d % 4 == 0) {
+        rmsnorm_vjp_at_kernel<float, 4><<<grid, kRowThreads, 0, st>>>(
+            static_cast<const float*>(g), static_cast<const float*>(x),
+            static_cast<const float*>(gamma), T, d, eps, min_rms, static_cast<float*>(out));
+    } else {
+        rmsnorm_vjp_at_kernel<float, 1><<<grid, kRowThreads, 0, st>>>(
+            static_cast<const float*>(g), static_cast<const float*>(x),
+            static_cast<const float*>(gamma), T, d, eps, min_rms, static_cast<float*>(out));
+    }
     return cudaGetLastError();
 }
 

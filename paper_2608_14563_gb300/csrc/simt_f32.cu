@@ -23,7 +23,7 @@ constexpr int kThreads = 256;
 constexpr int kMaxG = 64;
 
 struct SimtOps {
-    const float* A;
+    const float* A[kMaxG];
     long long sam, sak;
     const float* B[kMaxG];
     long long sbn, sbk;
@@ -78,7 +78,7 @@ __global__ void __launch_bounds__(kThreads)
     const int m0 = blockIdx.y * kT, n0 = blockIdx.x * kT;
     const int tid = threadIdx.x;
     const int tx = tid & 15, ty = tid >> 4;
-    const float* A = ops.A;
+    const float* A = ops.A[g];
     const float* B = ops.B[g];
     float acc[4][4] = {};
 
@@ -171,7 +171,7 @@ cudaError_t run(const SimtOps& ops, const Epi& ep, int groups, cudaStream_t st) 
 SimtOps ops_of(const float* A, long long sam, long long sak, const float* B, long long sbn,
                long long sbk, int M, int N, int K) {
     SimtOps o;
-    o.A = A;
+    for (int i = 0; i < kMaxG; ++i) o.A[i] = A;
     o.sam = sam;
     o.sak = sak;
     for (int i = 0; i < kMaxG; ++i) o.B[i] = B;
@@ -206,15 +206,16 @@ cudaError_t launch_proj_f32(const float* E, const float* W_U, int Tc, int d, int
     return run(ops_of(E, V, 1, W_U, 1, d, Tc, d, V), ep, 1, st);
 }
 
-cudaError_t launch_update_f32(int n, int T, int d, int d_ff, const float* g,
+cudaError_t launch_update_f32(int n, int T, int d, int d_ff, const float* const* g,
                               const float* const* A, float lr, float* const* W_master,
                               float* const* W_out, float* const* G_out, cudaStream_t st) {
     if (n < 1 || n > kMaxG) return cudaErrorInvalidValue;
     // G[i, j] = sum_t g[t, i] A[t, j]: A-operand(m=i, k=t) = g[t*d + i], B(n=j, k=t) = A[t*d_ff + j]
-    SimtOps ops = ops_of(g, 1, d, A[0], 1, d_ff, d, d_ff, T);
+    SimtOps ops = ops_of(g[0], 1, d, A[0], 1, d_ff, d, d_ff, T);
     SEpiUpdate ep;
     for (int l = 0; l < kMaxG; ++l) {
         const bool in = l < n;
+        ops.A[l] = in ? g[l] : g[0];
         ops.B[l] = in ? A[l] : A[0];
         ep.W_master[l] = in && W_master ? W_master[l] : nullptr;
         ep.W_out[l] = in && W_out ? W_out[l] : nullptr;

@@ -40,7 +40,7 @@ struct GemmShape {
 
 template <int MAXG>
 struct GemmMaps {
-    CUtensorMap a;          // shared by all groups
+    CUtensorMap a[MAXG];    // one per group (copies of one map when the groups share A)
     CUtensorMap b[MAXG];    // one per group
 };
 
@@ -183,7 +183,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         mbar_init(drain_bar, 1);
         *abort_flag = 0;
         fence_mbar_init();
-        tma_prefetch_desc(&maps.a);
+        tma_prefetch_desc(&maps.a[0]);
     }
     if (warp == 1) {
         tmem_alloc<kTmemCols>(smem_u32(tmem_holder));
@@ -207,13 +207,14 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             for (long long t = blockIdx.x; t < sh.tiles && ok; t += gridDim.x) {
                 int g, mb, nb;
                 tile_coords(t, sh, g, mb, nb);
+                const CUtensorMap* amap = &maps.a[MAXG == 1 ? 0 : g];
                 const CUtensorMap* bmap = &maps.b[MAXG == 1 ? 0 : g];
                 for (int kb = 0; kb < sh.k_blocks; ++kb) {
                     if (!mbar_wait(empty_bar(stage), phase ^ 1u, guard)) { ok = false; break; }
                     const uint32_t sa = sbase + stage * L::kStageBytes;
                     const uint32_t sb = sa + L::kABytes;
                     mbar_arrive_expect_tx(full_bar(stage), L::kStageBytes);
-                    load_operand<A_MN, kBM>(&maps.a, sa, full_bar(stage), mb * kBM, kb * kBK);
+                    load_operand<A_MN, kBM>(amap, sa, full_bar(stage), mb * kBM, kb * kBK);
                     load_operand<B_MN, BN>(bmap, sb, full_bar(stage), nb * BN, kb * kBK);
                     issued_mask |= 1u << stage;
                     issued_parity = (issued_parity & ~(1u << stage)) | (phase << stage);

@@ -132,7 +132,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
         mbar_init(drain_bar, 1);
         *abort_flag = 0;
         fence_mbar_init();
-        tma_prefetch_desc(&maps.a);
+        tma_prefetch_desc(&maps.a[0]);
     }
     if (warp == 1) {
         tmem_alloc_pair<kTmemCols>(smem_u32(tmem_holder));
@@ -156,6 +156,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
             for (long long t = cluster; t < sh.tiles && ok; t += n_clusters) {
                 int g, mp, nb;
                 tile_coords(t, sh, g, mp, nb);
+                const CUtensorMap* amap = &maps.a[MAXG == 1 ? 0 : g];
                 const CUtensorMap* bmap = &maps.b[MAXG == 1 ? 0 : g];
                 const int a_row = mp * kPairBM + 128 * static_cast<int>(rank);
                 const int b_row = nb * BN + kBHalf * static_cast<int>(rank);
@@ -165,7 +166,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
                     const uint32_t sb = sa + L::kABytes;
                     const uint32_t fb = mapa_shared(full_bar(stage), 0);
                     if (leader) mbar_arrive_expect_tx(full_bar(stage), 2 * L::kStageBytes);
-                    load_operand_pair<A_MN, 128>(&maps.a, sa, fb, a_row, kb * kBK);
+                    load_operand_pair<A_MN, 128>(amap, sa, fb, a_row, kb * kBK);
                     load_operand_pair<B_MN, kBHalf>(bmap, sb, fb, b_row, kb * kBK);
                     issued_mask |= 1u << stage;
                     issued_parity = (issued_parity & ~(1u << stage)) | (phase << stage);

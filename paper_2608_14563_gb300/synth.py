@@ -16,6 +16,10 @@ Recipe (every tensor has its own generator seeded from (seed, tensor, layer)):
 * W_l    ~ N(0, 0.02^2), fp32 master    down-projection weight      [d, d_ff] per layer
 * y      uniform on [0, V), or Zipf(1.1) over token ranks (P(r) ~ r^-1.1,
          token id = r - 1, inverse-CDF on an fp64 CDF table)         [T] int32
+* m_l    = N(0, 1) * exp(0.5 N(0, 1)) per token, every 64th token x 0.1
+         (the per-layer MLP output feeding a post-FFN norm: per-token RMS
+         varies widely and a few outlier tokens sit near 0.1)      [T, d] per layer
+* gp_l   = 0.3 + 0.05 N(0, 1)         post-FFN RMSNorm weight      [d] per layer
 
 Tensors are generated in fp32 and rounded to the storage dtype by torch.
 """
@@ -25,7 +29,7 @@ from dataclasses import dataclass, field
 
 import torch
 
-_TENSOR_IDS = {"h": 1, "w": 2, "W_U": 3, "A": 4, "W": 5, "y": 6, "noise": 7}
+_TENSOR_IDS = {"h": 1, "w": 2, "W_U": 3, "A": 4, "W": 5, "y": 6, "noise": 7, "m": 8, "gp": 9}
 
 
 @dataclass(frozen=True)
@@ -128,6 +132,20 @@ def make_targets(wl: Workload, device="cpu"):
         idx = torch.searchsorted(cdf, u, right=True).clamp_(max=wl.V - 1)
         return idx.to(torch.int32)
     raise ValueError(f"unknown target distribution {wl.targets!r}")
+
+
+def make_mlp_out(wl: Workload, layer: int, device="cpu"):
+    g = _gen(wl.seed, "m", layer, device)
+    m = torch.randn((wl.T, wl.d), generator=g, device=device, dtype=torch.float32)
+    scale = torch.exp(0.5 * torch.randn((wl.T, 1), generator=g, device=device,
+                                        dtype=torch.float32))
+    scale[::64] = 0.1
+    return (m * scale).to(wl.torch_dtype)
+
+
+def make_post_norm_w(wl: Workload, layer: int, device="cpu"):
+    return normal((wl.d,), std=0.05, mean=0.3, seed=wl.seed, tensor="gp", layer=layer,
+                  device=device, dtype=wl.torch_dtype)
 
 
 def make_noise(n: int, *, seed=0, layer=0, device="cpu"):

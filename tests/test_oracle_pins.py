@@ -306,3 +306,71 @@ def test_cosine_noise_expectation():
         Y = G + sigma * np.linalg.norm(G) / math.sqrt(n) * Z
         c = oracle.cosine(G, Y)[3]
         assert abs(c - 1.0 / math.sqrt(1.0 + sigma * sigma)) < 3e-3
+
+
+# ---------------------------------------------------------------------------
+# Post-feedforward RMSNorm (OLMo-2 / Gemma 3, Sec. 3.2 and App. E)
+# ---------------------------------------------------------------------------
+def _post_ffn_toy(seed, T=5, d=6, d_ff=7, V=10, small_rms_token=None, w_scale=0.3):
+    rng = np.random.default_rng(seed)
+    h0 = rng.standard_normal((T, d))
+    A = rng.standard_normal((T, d_ff))
+    W = w_scale * rng.standard_normal((d, d_ff))
+    gam = 0.3 + 0.05 * rng.standard_normal(d)      # post-FFN norm weight
+    w = 1.0 + 0.1 * rng.standard_normal(d)         # final norm weight
+    W_U = 0.5 * rng.standard_normal((V, d))
+    y = rng.integers(0, V, T).astype(np.int32)
+    if small_rms_token is not None:
+        A[small_rms_token] *= 0.02                 # MLP output RMS far below 0.5
+    return h0, A, W, gam, w, W_U, y
+
+
+def _post_ffn_loss(h0, A, Wx, gam, w, W_U, y, eps, s):
+    m = A @ Wx.T                                   # MLP (down-projection) output
+    rho = np.sqrt(np.mean(m * m, axis=1, keepdims=True) + eps)
+    return forward_loss(h0 + gam * m / rho, w, W_U, y, eps, s)
+
+
+def test_post_ffn_vjp_is_gradient_through_the_norm():
+    """With a post-FFN norm and nothing above the layer, the composed signal gives
+    the exact down-projection gradient: dL/dW = rmsnorm_vjp(g~, m, gamma)^T A."""
+    h0, A, W, gam, w, W_U, y = _post_ffn_toy(20)
+    s, eps = 1.0 / len(y), 1e-6
+    m = A @ W.T
+    h = h0 + gam * m / np.sqrt(np.mean(m * m, axis=1, keepdims=True) + eps)
+    gt = oracle.error_signal(h, w, W_U, y, eps=eps, min_rms=0.0, s=s)["g_tilde"]
+    gl = oracle.rmsnorm_vjp(gt, m, gam, eps=eps, min_rms=0.0)
+    G = oracle.pseudograd(gl, A)
+    fd = fd_grad(lambda Wx: _post_ffn_loss(h0, A, Wx, gam, w, W_U, y, eps, s), W.copy())
+    assert rel_err(G, fd) < 1e-7
+
+
+def test_post_ffn_clamp_caps_small_rms_tokens():
+    """A token whose MLP output RMS is below rho_min gets (rho/rho_min) x its exact
+    gradient (clamp on the 1/rho prefactor only), the others the exact one."""
+    h0, A, W, gam, w, W_U, y = _post_ffn_toy(21, small_rms_token=2, w_scale=1.0)
+    s, eps = 1.0, 1e-6
+    m = A @ W.T
+    rho = np.sqrt(np.mean(m * m, axis=1) + eps)
+    assert rho[2] < 0.5 and np.all(np.delete(rho, 2) > 0.5)
+    h = h0 + gam * m / rho[:, None]
+    gt = oracle.error_signal(h, w, W_U, y, eps=eps, min_rms=0.5, s=s)["g_tilde"]
+    exact = oracle.rmsnorm_vjp(gt, m, gam, eps=eps, min_rms=0.0)
+    clamped = oracle.rmsnorm_vjp(gt, m, gam, eps=eps, min_rms=0.5)
+    expect = exact.copy()
+    expect[2] *= rho[2] / 0.5
+    assert rel_err(clamped, expect) < 1e-14
+    # the unclamped composition is the finite-difference gradient w.r.t. m
+    def loss_of_m(mx):
+        r = np.sqrt(np.mean(mx * mx, axis=1, keepdims=True) + eps)
+        return forward_loss(h0 + gam * mx / r, w, W_U, y, eps, s)
+    assert rel_err(exact, fd_grad(loss_of_m, m.copy())) < 1e-7
+
+
+def test_rmsnorm_vjp_matches_error_signal_final_norm_step():
+    """Applied at the final norm with the pre-VJP signal g, the standalone VJP
+    reproduces the error signal's own step 5."""
+    h, w, W_U, y = _toy(T=6, seed=22)
+    out = oracle.error_signal(h, w, W_U, y, eps=1e-6, min_rms=0.5, s=0.3)
+    again = oracle.rmsnorm_vjp(out["g"], h, w, eps=1e-6, min_rms=0.5)
+    assert rel_err(again, out["g_tilde"]) < 1e-14
