@@ -228,6 +228,8 @@ def workload_config(wl, args):
             "error_matrix": {"auto": "stored-logits (auto)", "recompute": "recompute",
                              "stored": "stored-logits"}[args.algo],
             "norms_composed": "final + post-FFN per layer" if args.post_ffn_norm else "final",
+            "optimizer": ("plain SGD fused in the update GEMM epilogue" if args.optimizer == "fused-sgd"
+                          else f"{args.optimizer} on fp32 masters, clip={args.clip} (1% of ||W||_F)"),
             "l2": "inputs larger than L2 (W_U %.0f MB, A_l %.2f GB per step); no flush"
                   % (wl.V * wl.d * 2 / 1e6, wl.layers * wl.T * wl.d_ff * 2 / 1e9)}
 
@@ -273,6 +275,18 @@ def run_fpo(args, wl):
                                  t_chunk=args.t_chunk, algo=algo)
     ws_es = torch.empty(fpo.error_signal_workspace(desc), dtype=torch.uint8, device=dev)
     ws_up = torch.empty(fpo.layer_update_workspace(), dtype=torch.uint8, device=dev)
+    optimize = args.optimizer != "fused-sgd"
+    if optimize:
+        kind = {"sgd": fpo.OPT_SGD, "sgdm": fpo.OPT_SGD_MOMENTUM, "adamw": fpo.OPT_ADAMW}[
+            args.optimizer]
+        clip = {"none": fpo.CLIP_NONE, "step": fpo.CLIP_STEP, "grad": fpo.CLIP_GRADIENT}[args.clip]
+        opt = fpo.optimizer_desc(kind, lr=wl.lr, clip=clip, step=10)
+        st1 = ([torch.zeros(wl.d, wl.d_ff, device=dev) for _ in range(wl.layers)]
+               if kind != fpo.OPT_SGD else None)
+        st2 = ([torch.zeros(wl.d, wl.d_ff, device=dev) for _ in range(wl.layers)]
+               if kind == fpo.OPT_ADAMW else None)
+        ws_up = torch.empty(fpo.layer_optimize_workspace(wl.layers, wl.d, wl.d_ff),
+                            dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream()
 
     n_chunks = -(-wl.T // (args.t_chunk or wl.T))
@@ -281,6 +295,19 @@ def run_fpo(args, wl):
     launches_per_step = 4 + (4 * n_chunks if stored else 2 + 2 * n_chunks)
     if post:
         launches_per_step += wl.layers
+    if args.optimizer != "fused-sgd":  # G GEMM + optimizer (norms, scale, apply with a clip)
+        launches_per_step += 3 if args.clip != "none" else 1
+
+    def update():
+        signals = g_l if post else [g] * wl.layers
+        if optimize:
+            fpo.layer_optimize_grouped(signals, A, opt, Wm, W_outs=Wo, states1=st1, states2=st2,
+                                       workspace=ws_up)
+        elif post:
+            fpo.layer_update_grouped_signals(g_l, A, wl.lr, W_masters=Wm, W_outs=Wo,
+                                             workspace=ws_up)
+        else:
+            fpo.layer_update_grouped(g, A, wl.lr, W_masters=Wm, W_outs=Wo, workspace=ws_up)
 
     def step(stage_events=None, upd_events=None):
         fpo.error_signal(h, w, W_U, y, g, eps=wl.eps, min_rms=wl.min_rms, t_chunk=args.t_chunk,
@@ -292,11 +319,7 @@ def run_fpo(args, wl):
                 fpo.rmsnorm_vjp(g, m_out[l], gp[l], g_l[l], eps=wl.eps, min_rms=wl.min_rms)
         if upd_events:
             upd_events[0].record(stream)
-        if post:
-            fpo.layer_update_grouped_signals(g_l, A, wl.lr, W_masters=Wm, W_outs=Wo,
-                                             workspace=ws_up)
-        else:
-            fpo.layer_update_grouped(g, A, wl.lr, W_masters=Wm, W_outs=Wo, workspace=ws_up)
+        update()
         if upd_events:
             upd_events[1].record(stream)
 
@@ -370,11 +393,7 @@ def run_fpo(args, wl):
             if post:
                 for l in range(wl.layers):
                     fpo.rmsnorm_vjp(g, m_out[l], gp[l], g_l[l], eps=wl.eps, min_rms=wl.min_rms)
-            if post:
-                fpo.layer_update_grouped_signals(g_l, A, wl.lr, W_masters=Wm, W_outs=Wo,
-                                                 workspace=ws_up)
-            else:
-                fpo.layer_update_grouped(g, A, wl.lr, W_masters=Wm, W_outs=Wo, workspace=ws_up)
+            update()
             loss_host.copy_(loss, non_blocking=True)
 
         for _ in range(max(1, args.warmup)):
@@ -505,6 +524,12 @@ def main():
     ap.add_argument("--impl", choices=("fpo", "reference"), default="fpo")
     ap.add_argument("--workload", default="olmo", help="olmo | qwen | falcon | diag")
     ap.add_argument("--t-chunk", type=int, default=0, help="tokens per E chunk (0 = all)")
+    ap.add_argument("--optimizer", choices=("fused-sgd", "sgd", "sgdm", "adamw"),
+                    default="fused-sgd",
+                    help="fused-sgd: W -= lr G in the GEMM epilogue; otherwise G, the relative "
+                         "clip and the optimizer step on the fp32 masters (fpo_layer_optimize_grouped)")
+    ap.add_argument("--clip", choices=("none", "step", "grad"), default="step",
+                    help="relative clip to 1%% of ||W||_F for --optimizer sgd/sgdm/adamw")
     ap.add_argument("--post-ffn-norm", action="store_true",
                     help="compose each layer's post-FFN RMSNorm VJP (OLMo-2 layout) in the step")
     ap.add_argument("--algo", choices=("auto", "recompute", "stored"), default="auto",

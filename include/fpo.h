@@ -216,6 +216,56 @@ int32_t fpo_layer_update_grouped_signals(int32_t n_layers, int64_t T, int64_t d,
 int32_t fpo_rmsnorm_vjp(int64_t T, int64_t d, int32_t dtype, const void* g, const void* x,
                         const void* gamma, float eps, float min_rms, void* g_out, void* stream);
 
+/* Optimizers of Sec. 3.1 on the fp32 master copies. */
+typedef enum fpo_optimizer_kind {
+    FPO_OPT_SGD = 0,           /* step = -lr G                                           */
+    FPO_OPT_SGD_MOMENTUM = 1,  /* buf = mu buf + G; step = -lr buf                       */
+    FPO_OPT_ADAMW = 2          /* m, v moments; step = -lr (mhat/(sqrt(vhat)+eps) + wd W) */
+} fpo_optimizer_kind;
+
+/* The relative clip of App. A, ||.||_F <= clip_frac ||W||_F (W before the step). */
+typedef enum fpo_clip_mode {
+    FPO_CLIP_NONE = 0,
+    FPO_CLIP_STEP = 1,      /* scale the optimizer's step (the update Delta W) */
+    FPO_CLIP_GRADIENT = 2   /* scale G before the optimizer sees it            */
+} fpo_clip_mode;
+
+typedef struct fpo_optimizer_desc {
+    int32_t kind;          /* fpo_optimizer_kind                                  */
+    int32_t clip;          /* fpo_clip_mode                                       */
+    float lr;
+    float momentum;        /* SGD with momentum: mu (0.9)                         */
+    float beta1, beta2;    /* AdamW moment decays (0.9, 0.999)                    */
+    float adam_eps;        /* AdamW epsilon (1e-8)                                */
+    float weight_decay;    /* AdamW decoupled weight decay (0.01)                 */
+    float clip_frac;       /* relative clip bound (0.01)                          */
+    int64_t step;          /* AdamW step index t >= 1, for the bias corrections   */
+} fpo_optimizer_desc;
+
+/* Bytes of workspace fpo_layer_optimize_grouped needs. */
+size_t fpo_layer_optimize_workspace(int32_t n_layers, int64_t d, int64_t d_ff);
+
+/*
+ * fpo_layer_optimize_grouped -- the pseudogradient of every target layer
+ * (Eq. (w3update), as in fpo_layer_update_grouped_signals) followed by an
+ * optimizer step on its fp32 master (Sec. 3.1: SGD with momentum 0.9 or AdamW
+ * with weight decay 0.01) with the relative clip of App. A:
+ *   G_l = g[l]^T A[l]                 fp32, in the workspace
+ *   c   = clip factor from ||G_l||, ||step_l|| and ||W_l|| (see fpo_clip_mode)
+ *   state_l, W_master,l updated; W_out,l = W_master,l rounded to dtype.
+ * state1[l] is the momentum buffer (SGD_MOMENTUM) or the first moment (ADAMW),
+ * state2[l] the second moment (ADAMW); fp32 [d, d_ff], updated in place (NULL
+ * arrays when the optimizer has no such state).  W_out may be NULL.  The clip
+ * needs all of G_l before any element steps, so G lives in the workspace
+ * (n_layers x d x d_ff x 4 bytes).  g, A, W_out: as fpo_layer_update_grouped_signals.
+ */
+int32_t fpo_layer_optimize_grouped(int32_t n_layers, int64_t T, int64_t d, int64_t d_ff,
+                                   int32_t dtype, const void* const* g, const void* const* A,
+                                   const fpo_optimizer_desc* opt, float* const* W_master,
+                                   void* const* W_out, float* const* state1,
+                                   float* const* state2, void* workspace, size_t workspace_bytes,
+                                   void* stream);
+
 /* Bytes of workspace fpo_cosine needs for n elements. */
 size_t fpo_cosine_workspace(int64_t n);
 

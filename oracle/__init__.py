@@ -13,6 +13,7 @@ Each function follows one passage of the paper:
   norm of OLMo-2 / Gemma 3, Sec. 3.2).
 * :func:`pseudograd`    Sec. 3.1 step 5, Eq. (w3update).
 * :func:`sgd_update`    App. A, fp32 master weights cast to bf16.
+* :func:`optimizer_step`  Sec. 3.1 AdamW / SGD with momentum, App. A relative clip.
 * :func:`cosine`        Sec. 2.2, Eq. (cosine).
 """
 from __future__ import annotations
@@ -61,6 +62,9 @@ def _load():
     lib.oracle_pseudograd.restype = i32
     lib.oracle_sgd_update.argtypes = [i64, vp, vp, dbl, vp, vp]
     lib.oracle_sgd_update.restype = None
+    lib.oracle_optimizer_step.argtypes = [i64, i32, dbl, dbl, dbl, dbl, dbl, dbl, i64, i32, dbl,
+                                          vp, vp, vp, vp, vp, vp, vp, vp]
+    lib.oracle_optimizer_step.restype = dbl
     lib.oracle_f32_to_bf16.argtypes = [i64, vp, vp]
     lib.oracle_f32_to_bf16.restype = None
     lib.oracle_cosine.argtypes = [i64, i32, vp, vp, vp]
@@ -180,6 +184,32 @@ def sgd_update(W_master, G, lr):
     W_b = np.empty(W.shape, dtype=np.uint16)
     _load().oracle_sgd_update(W.size, _ptr(W), _ptr(G), float(lr), _ptr(W_new), _ptr(W_b))
     return W_new, W_b
+
+
+SGD, SGD_MOMENTUM, ADAMW = 0, 1, 2
+CLIP_NONE, CLIP_UPDATE, CLIP_GRADIENT = 0, 1, 2
+
+
+def optimizer_step(W_master, G, *, kind, lr, momentum=0.9, beta1=0.9, beta2=0.999, eps=1e-8,
+                   weight_decay=0.01, t=1, clip=CLIP_NONE, frac=0.01, s1=None, s2=None):
+    """Sec. 3.1 optimizers on the fp32 master with the App. A relative clip.
+
+    Returns dict(W fp32, W_bf16 uint16, s1 fp32 or None, s2 fp32 or None, scale)."""
+    W = np.ascontiguousarray(W_master, dtype=np.float32)
+    G = np.ascontiguousarray(G, dtype=np.float64)
+    if W.shape != G.shape:
+        raise ValueError("W_master and G must have the same shape")
+    z = np.zeros(W.shape, dtype=np.float32)
+    s1 = z if s1 is None else np.ascontiguousarray(s1, dtype=np.float32)
+    s2 = z if s2 is None else np.ascontiguousarray(s2, dtype=np.float32)
+    W_new = np.empty_like(W)
+    W_b = np.empty(W.shape, dtype=np.uint16)
+    s1n = np.empty_like(W) if kind in (SGD_MOMENTUM, ADAMW) else None
+    s2n = np.empty_like(W) if kind == ADAMW else None
+    scale = _load().oracle_optimizer_step(W.size, kind, lr, momentum, beta1, beta2, eps,
+                                          weight_decay, t, clip, frac, _ptr(W), _ptr(G), _ptr(s1),
+                                          _ptr(s2), _ptr(W_new), _ptr(W_b), _ptr(s1n), _ptr(s2n))
+    return {"W": W_new, "W_bf16": W_b, "s1": s1n, "s2": s2n, "scale": scale}
 
 
 def f32_to_bf16_bits(x):

@@ -15,6 +15,7 @@
  *   oracle_rmsnorm_vjp   App. E Eq. (rmsnorm-vjp) at any norm (post-FFN, Sec. 3.2)
  *   oracle_pseudograd    Sec. 3.1 step 5, Eq. (w3update): G = g~^T h_mid
  *   oracle_sgd_update    App. A (fp32 master weights, cast to bf16)
+ *   oracle_optimizer_step  Sec. 3.1 (AdamW / SGD with momentum) + App. A relative clip
  *   oracle_cosine        Sec. 2.2, Eq. (cosine)
  *
  * Inputs are the exact stored values (fp32, bf16 or fp64) upcast to fp64 as
@@ -241,6 +242,66 @@ void oracle_sgd_update(int64_t n, const float* W, const double* G, double lr,
         if (W_new) W_new[k] = wn;
         if (W_bf16) W_bf16[k] = orc_f32_to_bf16(wn);
     }
+}
+
+/*
+ * One optimizer step on the fp32 master copy of one layer (Sec. 3.1: AdamW with
+ * weight decay 0.01 or SGD with momentum 0.9; App. A: fp32 master weights, and
+ * a relative clip of each step to frac * ||W||_F).  kind: 0 SGD, 1 SGD with
+ * momentum (buf = mu buf + G, step = -lr buf), 2 AdamW (m = b1 m + (1-b1) G,
+ * v = b2 v + (1-b2) G^2, step = -lr (mhat / (sqrt(vhat) + eps) + wd W) with
+ * mhat = m / (1 - b1^t), vhat = v / (1 - b2^t)).
+ * clip: 0 none; 1 the step itself is scaled so ||step||_F <= frac ||W||_F (the
+ * optimizer state is updated with the unscaled gradient); 2 the gradient is
+ * scaled so ||G||_F <= frac ||W||_F before the optimizer sees it.
+ * Norms are of the fp32 master W before the step.  Everything is evaluated in
+ * fp64 from the stored fp32 values; outputs (W, state) are rounded to fp32 and
+ * W_bf16 = RNE16(W_new).  s1 (momentum buffer / m) and s2 (v) may be NULL when
+ * the kind has no such state.  Returns the clip factor applied (1 if none).
+ */
+double oracle_optimizer_step(int64_t n, int kind, double lr, double mu, double b1, double b2,
+                             double eps, double wd, int64_t t, int clip, double frac,
+                             const float* W, const double* G, const float* s1, const float* s2,
+                             float* W_new, uint16_t* W_bf16, float* s1_new, float* s2_new) {
+    double ww = 0.0, gg = 0.0;
+    for (int64_t k = 0; k < n; ++k) {
+        ww += (double)W[k] * (double)W[k];
+        gg += G[k] * G[k];
+    }
+    const double wnorm = sqrt(ww);
+    double gscale = 1.0;
+    if (clip == 2 && sqrt(gg) > frac * wnorm) gscale = frac * wnorm / sqrt(gg);
+    const double bc1 = 1.0 - pow(b1, (double)t), bc2 = 1.0 - pow(b2, (double)t);
+    double* step = (double*)malloc(sizeof(double) * (size_t)(n > 0 ? n : 1));
+    double dd = 0.0;
+    for (int64_t k = 0; k < n; ++k) {
+        const double g = gscale * G[k];
+        double st;
+        if (kind == 0) {
+            st = -lr * g;
+        } else if (kind == 1) {
+            const double buf = mu * (double)s1[k] + g;
+            if (s1_new) s1_new[k] = (float)buf;
+            st = -lr * buf;
+        } else {
+            const double m = b1 * (double)s1[k] + (1.0 - b1) * g;
+            const double v = b2 * (double)s2[k] + (1.0 - b2) * g * g;
+            if (s1_new) s1_new[k] = (float)m;
+            if (s2_new) s2_new[k] = (float)v;
+            st = -lr * ((m / bc1) / (sqrt(v / bc2) + eps) + wd * (double)W[k]);
+        }
+        step[k] = st;
+        dd += st * st;
+    }
+    double sscale = 1.0;
+    if (clip == 1 && sqrt(dd) > frac * wnorm) sscale = frac * wnorm / sqrt(dd);
+    for (int64_t k = 0; k < n; ++k) {
+        const float wn = (float)((double)W[k] + sscale * step[k]);
+        if (W_new) W_new[k] = wn;
+        if (W_bf16) W_bf16[k] = orc_f32_to_bf16(wn);
+    }
+    free(step);
+    return clip == 2 ? gscale : sscale;
 }
 
 /* Plain RNE conversion of an fp32 array to bf16 bits (test helper for the

@@ -66,6 +66,22 @@ _lib.fpo_layer_update_grouped_signals.argtypes = [_i32, _i64, _i64, _i64, _i32,
 _lib.fpo_layer_update_grouped_signals.restype = _i32
 _lib.fpo_rmsnorm_vjp.argtypes = [_i64, _i64, _i32, _vp, _vp, _vp, _f32, _f32, _vp, _vp]
 _lib.fpo_rmsnorm_vjp.restype = _i32
+class OptimizerDesc(ctypes.Structure):
+    """Mirror of fpo_optimizer_desc."""
+    _fields_ = [("kind", _i32), ("clip", _i32), ("lr", _f32), ("momentum", _f32),
+                ("beta1", _f32), ("beta2", _f32), ("adam_eps", _f32), ("weight_decay", _f32),
+                ("clip_frac", _f32), ("step", _i64)]
+
+
+OPT_SGD, OPT_SGD_MOMENTUM, OPT_ADAMW = 0, 1, 2
+CLIP_NONE, CLIP_STEP, CLIP_GRADIENT = 0, 1, 2
+_lib.fpo_layer_optimize_workspace.argtypes = [_i32, _i64, _i64]
+_lib.fpo_layer_optimize_workspace.restype = _sz
+_lib.fpo_layer_optimize_grouped.argtypes = [_i32, _i64, _i64, _i64, _i32, ctypes.POINTER(_vp),
+                                            ctypes.POINTER(_vp), ctypes.POINTER(OptimizerDesc),
+                                            ctypes.POINTER(_vp), ctypes.POINTER(_vp),
+                                            ctypes.POINTER(_vp), ctypes.POINTER(_vp), _vp, _sz, _vp]
+_lib.fpo_layer_optimize_grouped.restype = _i32
 _lib.fpo_cosine_workspace.argtypes = [_i64]
 _lib.fpo_cosine_workspace.restype = _sz
 _lib.fpo_cosine.argtypes = [_i64, _i32, _vp, _vp, _vp, _vp, _sz, _vp]
@@ -235,6 +251,32 @@ def layer_update_grouped_signals(gs, As, lr, *, W_masters=None, W_outs=None, G_o
         _ptr_array(W_masters, n), _ptr_array(W_outs, n), _ptr_array(G_outs, n), _ptr(workspace),
         workspace.numel(), _stream(stream))
     _check(rc, "fpo_layer_update_grouped_signals")
+    return workspace
+
+
+def optimizer_desc(kind=OPT_ADAMW, *, lr=1e-4, momentum=0.9, beta1=0.9, beta2=0.999, eps=1e-8,
+                   weight_decay=0.01, clip=CLIP_STEP, clip_frac=0.01, step=1):
+    return OptimizerDesc(int(kind), int(clip), float(lr), float(momentum), float(beta1),
+                         float(beta2), float(eps), float(weight_decay), float(clip_frac), int(step))
+
+
+def layer_optimize_workspace(n_layers, d, d_ff) -> int:
+    return int(_lib.fpo_layer_optimize_workspace(int(n_layers), int(d), int(d_ff)))
+
+
+def layer_optimize_grouped(gs, As, opt, W_masters, *, W_outs=None, states1=None, states2=None,
+                           workspace=None, stream=None):
+    """fpo_layer_optimize_grouped: G_l = g_l^T A_l, relative clip, optimizer step."""
+    n = len(As)
+    T, d = gs[0].shape
+    d_ff = As[0].shape[1]
+    if workspace is None:
+        workspace = _workspace(layer_optimize_workspace(n, d, d_ff), gs[0].device)
+    rc = _lib.fpo_layer_optimize_grouped(
+        n, T, d, d_ff, _dtype_code(gs[0]), _ptr_array(gs, n), _ptr_array(As, n), ctypes.byref(opt),
+        _ptr_array(W_masters, n), _ptr_array(W_outs, n), _ptr_array(states1, n),
+        _ptr_array(states2, n), _ptr(workspace), workspace.numel(), _stream(stream))
+    _check(rc, "fpo_layer_optimize_grouped")
     return workspace
 
 

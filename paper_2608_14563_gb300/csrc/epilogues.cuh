@@ -225,4 +225,34 @@ struct EpiUpdate {
     __device__ __forceinline__ void finish(const Params&, int) {}
 };
 
+// ---------------------------------------------------------------------------
+// Pseudogradient only, fp32, one output per group (layer): G[g] = g~^T A_l, for
+// the optimizers that need the whole G (and its norm) before they step.
+struct EpiStoreGroupF32 {
+    struct Params {
+        float* G[kMaxGroups];
+        long long ld;
+        int M, N;
+    };
+    int row, g;
+    bool valid;
+
+    __device__ __forceinline__ EpiStoreGroupF32(const Params& p, int g_, int row_, int)
+        : row(row_), g(g_) {
+        valid = row_ < p.M;
+    }
+
+    __device__ __forceinline__ void chunk(const Params& p, const float (&v)[32], int col0, int,
+                                          EpiIO&) {
+        const int lim = p.N - col0;
+        if (!valid || lim <= 0) return;
+        float4* dst = reinterpret_cast<float4*>(p.G[g] + row * p.ld + col0);
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+            if (q * 4 < lim) dst[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+    }
+
+    __device__ __forceinline__ void finish(const Params&, int) {}
+};
+
 }  // namespace fpo

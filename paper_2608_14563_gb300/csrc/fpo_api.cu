@@ -6,6 +6,7 @@
 
 #include <atomic>
 #include <climits>
+#include <cmath>
 #include <mutex>
 
 #include "../../include/fpo.h"
@@ -326,6 +327,93 @@ int32_t fpo_layer_update_grouped(int32_t n_layers, int64_t T, int64_t d, int64_t
     for (int l = 0; l < n_layers; ++l) gs[l] = g;
     return fpo_layer_update_grouped_signals(n_layers, T, d, d_ff, dtype, gs, A, lr, W_master,
                                             W_out, G_out, workspace, workspace_bytes, stream);
+}
+
+size_t fpo_layer_optimize_workspace(int32_t n_layers, int64_t d, int64_t d_ff) {
+    if (n_layers < 1 || n_layers > FPO_MAX_GROUPED_LAYERS || d <= 0 || d_ff <= 0) return 0;
+    return kStatusBytes + align_up(static_cast<size_t>(n_layers) * static_cast<size_t>(d) *
+                                   static_cast<size_t>(d_ff) * 4) +
+           align_up(optim_partials_bytes(n_layers)) + align_up(static_cast<size_t>(n_layers) * 4);
+}
+
+int32_t fpo_layer_optimize_grouped(int32_t n_layers, int64_t T, int64_t d, int64_t d_ff,
+                                   int32_t dtype, const void* const* g, const void* const* A,
+                                   const fpo_optimizer_desc* opt, float* const* W_master,
+                                   void* const* W_out, float* const* state1,
+                                   float* const* state2, void* workspace, size_t workspace_bytes,
+                                   void* stream) {
+    if (!opt) return FPO_ERR_NULL;
+    if (dtype != FPO_F32 && dtype != FPO_BF16) return FPO_ERR_DTYPE;
+    if (n_layers < 1 || n_layers > FPO_MAX_GROUPED_LAYERS) return FPO_ERR_SHAPE;
+    if (T < 0 || d <= 0 || d_ff <= 0 || T > INT_MAX || d > INT_MAX || d_ff > INT_MAX)
+        return FPO_ERR_SHAPE;
+    if (dtype == FPO_BF16 && (d % 8 != 0 || d_ff % 8 != 0)) return FPO_ERR_SHAPE;
+    if (opt->kind < FPO_OPT_SGD || opt->kind > FPO_OPT_ADAMW || opt->clip < FPO_CLIP_NONE ||
+        opt->clip > FPO_CLIP_GRADIENT || !(opt->lr == opt->lr) || !(opt->clip_frac >= 0.f) ||
+        (opt->kind == FPO_OPT_ADAMW && (opt->step < 1 || !(opt->beta1 >= 0.f && opt->beta1 < 1.f) ||
+                                       !(opt->beta2 >= 0.f && opt->beta2 < 1.f))))
+        return FPO_ERR_ARG;
+    if (!A || !g || !W_master) return FPO_ERR_NULL;
+    if ((opt->kind != FPO_OPT_SGD && !state1) || (opt->kind == FPO_OPT_ADAMW && !state2))
+        return FPO_ERR_NULL;
+    const size_t need = fpo_layer_optimize_workspace(n_layers, d, d_ff);
+    if (!workspace || workspace_bytes < need) return FPO_ERR_WORKSPACE;
+    if ((reinterpret_cast<uintptr_t>(workspace) % kAlign) != 0) return FPO_ERR_ALIGN;
+    for (int l = 0; l < n_layers; ++l) {
+        if ((T > 0 && (!A[l] || !g[l])) || !W_master[l]) return FPO_ERR_NULL;
+        if (opt->kind != FPO_OPT_SGD && !state1[l]) return FPO_ERR_NULL;
+        if (opt->kind == FPO_OPT_ADAMW && !state2[l]) return FPO_ERR_NULL;
+        if (!aligned16(g[l]) || !aligned16(A[l]) || !aligned16(W_master[l]) ||
+            !aligned16(W_out ? W_out[l] : nullptr) || !aligned16(state1 ? state1[l] : nullptr) ||
+            !aligned16(state2 ? state2[l] : nullptr))
+            return FPO_ERR_ALIGN;
+    }
+    int32_t rc = check_arch();
+    if (rc != FPO_OK) return rc;
+
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    uint8_t* ws = static_cast<uint8_t*>(workspace);
+    unsigned* status = reinterpret_cast<unsigned*>(ws);
+    FPO_TRY(cudaMemsetAsync(status, 0, sizeof(unsigned), st));
+    const size_t n = static_cast<size_t>(d) * static_cast<size_t>(d_ff);
+    float* Gbuf = reinterpret_cast<float*>(ws + kStatusBytes);
+    double* partials = reinterpret_cast<double*>(ws + kStatusBytes + align_up(n_layers * n * 4));
+    float* scales = reinterpret_cast<float*>(ws + kStatusBytes + align_up(n_layers * n * 4) +
+                                             align_up(optim_partials_bytes(n_layers)));
+    float* G[FPO_MAX_GROUPED_LAYERS];
+    for (int l = 0; l < n_layers; ++l) G[l] = Gbuf + static_cast<size_t>(l) * n;
+
+    // 1. G_l = g_l^T A_l (fp32)
+    if (T == 0) {
+        FPO_TRY(cudaMemsetAsync(Gbuf, 0, n_layers * n * 4, st));
+    } else if (dtype == FPO_BF16) {
+        FPO_TRY(launch_grad_bf16(n_layers, static_cast<int>(T), static_cast<int>(d),
+                                 static_cast<int>(d_ff), g, A, G, status, st));
+    } else {
+        FPO_TRY(launch_update_f32(n_layers, static_cast<int>(T), static_cast<int>(d),
+                                  static_cast<int>(d_ff), reinterpret_cast<const float* const*>(g),
+                                  reinterpret_cast<const float* const*>(A), 0.f, nullptr, nullptr,
+                                  G, st));
+    }
+    // 2. clip factor and optimizer step on the fp32 masters
+    OptimParams op;
+    op.kind = opt->kind;
+    op.clip = opt->clip;
+    op.lr = opt->lr;
+    op.momentum = opt->momentum;
+    op.beta1 = opt->beta1;
+    op.beta2 = opt->beta2;
+    op.eps = opt->adam_eps;
+    op.weight_decay = opt->weight_decay;
+    op.clip_frac = opt->clip_frac;
+    const double t = static_cast<double>(opt->step < 1 ? 1 : opt->step);
+    op.inv_bc1 = static_cast<float>(1.0 / (1.0 - pow(static_cast<double>(opt->beta1), t)));
+    op.inv_sqrt_bc2 = static_cast<float>(1.0 / sqrt(1.0 - pow(static_cast<double>(opt->beta2), t)));
+    if (opt->kind != FPO_OPT_ADAMW) op.inv_bc1 = op.inv_sqrt_bc2 = 1.f;
+    return cuda_status(launch_optimizer(dtype, n_layers, n, op, G, W_master, W_out,
+                                        opt->kind != FPO_OPT_SGD ? state1 : nullptr,
+                                        opt->kind == FPO_OPT_ADAMW ? state2 : nullptr, partials,
+                                        scales, st));
 }
 
 int32_t fpo_rmsnorm_vjp(int64_t T, int64_t d, int32_t dtype, const void* g, const void* x,

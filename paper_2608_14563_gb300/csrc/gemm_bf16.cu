@@ -287,6 +287,37 @@ cudaError_t launch_update_bf16(int n, int T, int d, int d_ff, const void* const*
         maps, ep, make_shape(d, d_ff, T, kUpdBN, n, band_for(false)), status, st);
 }
 
+cudaError_t launch_grad_bf16(int n, int T, int d, int d_ff, const void* const* g,
+                             const void* const* A, float* const* G_out, unsigned* status,
+                             cudaStream_t st) {
+    if (n < 1 || n > kMaxGroups) return cudaErrorInvalidValue;
+    static GemmMaps<kMaxGroups> maps;
+    static EpiStoreGroupF32::Params ep;
+    static std::mutex mu;
+    std::lock_guard<std::mutex> lock(mu);
+    for (int l = 0; l < n; ++l) {
+        if (l > 0 && g[l] == g[0])
+            maps.a[l] = maps.a[0];
+        else if (!map_mnmajor(&maps.a[l], g[l], T, d))
+            return cudaErrorInvalidValue;
+        if (!map_mnmajor(&maps.b[l], A[l], T, d_ff)) return cudaErrorInvalidValue;
+        ep.G[l] = G_out[l];
+    }
+    for (int l = n; l < kMaxGroups; ++l) {
+        maps.a[l] = maps.a[0];
+        maps.b[l] = maps.b[0];
+        ep.G[l] = G_out[0];
+    }
+    ep.ld = d_ff;
+    ep.M = d;
+    ep.N = d_ff;
+    if (use_pair())
+        return run_gemm_pair<kUpdBN, true, true, kPairStages, kMaxGroups, EpiStoreGroupF32>(
+            maps, ep, make_shape(d, d_ff, T, kUpdBN, n, band_for(true), kPairBM), status, st);
+    return run_gemm<kUpdBN, true, true, kUpdStages, kMaxGroups, EpiStoreGroupF32>(
+        maps, ep, make_shape(d, d_ff, T, kUpdBN, n, band_for(false)), status, st);
+}
+
 cudaError_t launch_test_gemm_bf16(int M, int N, int K, bool a_mn, bool b_mn, const void* A,
                                   const void* B, float* C, unsigned* status, cudaStream_t st) {
     const bool pair = use_pair();

@@ -46,6 +46,24 @@ cudaError_t launch_update_bf16(int n, int T, int d, int d_ff, const void* const*
                                void* const* W_out, void* const* G_out, unsigned* status,
                                cudaStream_t st);
 
+// Grouped pseudogradients only: G_out[l] (fp32 [d, d_ff]) = g[l]^T A[l].
+cudaError_t launch_grad_bf16(int n, int T, int d, int d_ff, const void* const* g,
+                             const void* const* A, float* const* G_out, unsigned* status,
+                             cudaStream_t st);
+
+// Optimizer step of n layers of n_elem elements from fp32 G (optimizer.cu).
+struct OptimParams {
+    int kind;          // 0 SGD, 1 SGD with momentum, 2 AdamW
+    int clip;          // 0 none, 1 the step, 2 the gradient
+    float lr, momentum, beta1, beta2, eps, weight_decay, clip_frac;
+    float inv_bc1, inv_sqrt_bc2;  // AdamW bias corrections 1/(1-b1^t), 1/sqrt(1-b2^t)
+};
+size_t optim_partials_bytes(int n_layers);
+cudaError_t launch_optimizer(int dtype, int n_layers, size_t n_elem, const OptimParams& op,
+                             float* const* G, float* const* W_master, void* const* W_out,
+                             float* const* s1, float* const* s2, double* partials, float* scales,
+                             cudaStream_t st);
+
 // Which tcgen05 GEMM kernel the launchers use: 0 = single-CTA 128 x 256 tiles,
 // 1 = CTA-pair 256 x 256 tiles.
 void set_gemm_variant(int v);

@@ -1,0 +1,92 @@
+"""Optimizer row (Sec. 3.1 AdamW / SGD with momentum, App. A relative clip) through
+fpo_layer_optimize_grouped against the oracle's optimizer step on the oracle's G."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from helpers import f64, rel_frob
+from paper_2608_14563_gb300 import synth
+from paper_2608_14563_gb300.synth import Workload
+
+pytestmark = pytest.mark.gpu
+
+KINDS = {"sgd": 0, "sgdm": 1, "adamw": 2}
+CLIPS = {"none": 0, "step": 1, "grad": 2}
+
+
+def _case(dtype, seed):
+    if dtype == "bf16":
+        wl = Workload("opt-bf16", T=300, d=136, d_ff=264, V=8, layers=2, seed=seed)
+    else:
+        wl = Workload("opt-f32", T=70, d=33, d_ff=65, V=8, layers=2, dtype="f32", seed=seed)
+    gs = [synth.normal((wl.T, wl.d), std=1e-2, seed=seed, tensor="h", layer=l).to(wl.torch_dtype)
+          for l in range(wl.layers)]
+    A = [synth.make_A(wl, l) for l in range(wl.layers)]
+    W = [synth.make_W_master(wl, l) for l in range(wl.layers)]
+    return wl, gs, A, W
+
+
+def _states(wl, Gs, kind, t):
+    """Optimizer state before step t (zero at t = 1, synthetic and consistent otherwise)."""
+    s1, s2 = [], []
+    for l, G in enumerate(Gs):
+        sc = float(np.sqrt(np.mean(G * G)))
+        if t == 1:
+            s1.append(np.zeros(G.shape, np.float32))
+            s2.append(np.zeros(G.shape, np.float32))
+        else:
+            a = synth.normal(G.shape, std=sc, seed=wl.seed, tensor="noise", layer=10 + l).numpy()
+            b = synth.normal(G.shape, std=1.0, seed=wl.seed, tensor="noise", layer=20 + l).numpy()
+            s1.append(a.astype(np.float32))
+            s2.append((sc * sc * (0.5 + np.abs(b))).astype(np.float32))
+    return s1, s2
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("kind", list(KINDS))
+@pytest.mark.parametrize("clip", list(CLIPS))
+def test_optimizer_step_matches_oracle(fpo, dtype, kind, clip):
+    wl, gs, A, W = _case(dtype, seed=40 + 3 * KINDS[kind] + CLIPS[clip])
+    Gs = [oracle.pseudograd(synth.to_numpy_exact(g), synth.to_numpy_exact(a)) for g, a in zip(gs, A)]
+    t = 1 if kind == "sgdm" else 3
+    s1, s2 = _states(wl, Gs, kind, t)
+    lr = {"sgd": 0.5, "sgdm": 0.05, "adamw": 2e-3}[kind]
+    opt = fpo.optimizer_desc(KINDS[kind], lr=lr, clip=CLIPS[clip], step=t)
+    Wm = [w.cuda() for w in W]
+    Wo = [torch.empty(w.shape, dtype=wl.torch_dtype, device="cuda") for w in W]
+    S1 = [torch.from_numpy(x).cuda() for x in s1] if kind != "sgd" else None
+    S2 = [torch.from_numpy(x).cuda() for x in s2] if kind == "adamw" else None
+    ws = fpo.layer_optimize_grouped([g.cuda() for g in gs], [a.cuda() for a in A], opt, Wm,
+                                    W_outs=Wo, states1=S1, states2=S2)
+    assert fpo.get_device_status(ws) == fpo.OK
+    tol = 2e-2 if dtype == "bf16" else 1e-5
+    for l in range(wl.layers):
+        ref = oracle.optimizer_step(W[l].numpy(), Gs[l], kind=KINDS[kind], lr=lr, t=t,
+                                    clip=CLIPS[clip], s1=s1[l], s2=s2[l])
+        W0 = W[l].double().numpy()
+        d_ref = ref["W"].astype(np.float64) - W0
+        ulp = np.spacing(np.abs(ref["W"]).astype(np.float32)).astype(np.float64)
+        q = np.linalg.norm(ulp) / np.linalg.norm(d_ref)
+        d_got = f64(Wm[l]) - W0
+        assert rel_frob(d_got, d_ref) < tol + q, f"layer {l}"
+        if clip != "none" and ref["scale"] < 1.0:
+            # an active clip pins the step (or the gradient) at 1% of ||W||
+            if clip == "step":
+                assert abs(np.linalg.norm(d_got) / (0.01 * np.linalg.norm(W0)) - 1) < 1e-3
+        if kind != "sgd":
+            assert rel_frob(f64(S1[l]), ref["s1"]) < tol
+        if kind == "adamw":
+            assert rel_frob(f64(S2[l]), ref["s2"]) < tol
+        assert rel_frob(f64(Wo[l]), ref["W"]) < max(tol, 4e-3 if dtype == "bf16" else 0)
+
+
+def test_clip_is_active_in_the_step_cases(fpo):
+    # guard: the parametrised cases above do exercise an active clip
+    wl, gs, A, W = _case("bf16", seed=40 + 3 * 2 + 1)
+    G = oracle.pseudograd(synth.to_numpy_exact(gs[0]), synth.to_numpy_exact(A[0]))
+    s1, s2 = _states(wl, [G], "adamw", 3)
+    r = oracle.optimizer_step(W[0].numpy(), G, kind=2, lr=2e-3, t=3, clip=1, s1=s1[0], s2=s2[0])
+    assert r["scale"] < 1.0
+    r = oracle.optimizer_step(W[0].numpy(), G, kind=0, lr=0.5, clip=2)
+    assert r["scale"] < 1.0

@@ -374,3 +374,76 @@ def test_rmsnorm_vjp_matches_error_signal_final_norm_step():
     out = oracle.error_signal(h, w, W_U, y, eps=1e-6, min_rms=0.5, s=0.3)
     again = oracle.rmsnorm_vjp(out["g"], h, w, eps=1e-6, min_rms=0.5)
     assert rel_err(again, out["g_tilde"]) < 1e-14
+
+
+# ---------------------------------------------------------------------------
+# Optimizers on the fp32 master and the relative clip (Sec. 3.1, App. A)
+# ---------------------------------------------------------------------------
+def _opt_case(seed, n=(6, 9)):
+    rng = np.random.default_rng(seed)
+    W = (0.02 * rng.standard_normal(n)).astype(np.float32)
+    G = 1e-3 * rng.standard_normal(n)
+    return W, G
+
+
+def test_sgd_momentum_and_adamw_match_torch_optim():
+    """Three steps against torch.optim.SGD(momentum=0.9) / AdamW(wd=0.01) in fp64."""
+    torch = pytest.importorskip("torch")
+    rng = np.random.default_rng(30)
+    W0 = (0.02 * rng.standard_normal((5, 7))).astype(np.float32)
+    grads = [1e-3 * rng.standard_normal((5, 7)) for _ in range(3)]
+    for kind in (oracle.SGD_MOMENTUM, oracle.ADAMW):
+        p = torch.nn.Parameter(torch.tensor(W0, dtype=torch.float64))
+        opt = (torch.optim.SGD([p], lr=0.1, momentum=0.9) if kind == oracle.SGD_MOMENTUM else
+               torch.optim.AdamW([p], lr=1e-3, betas=(0.9, 0.999), eps=1e-8, weight_decay=0.01))
+        W, s1, s2 = W0.copy(), None, None
+        for t, G in enumerate(grads, start=1):
+            p.grad = torch.tensor(G)
+            opt.step()
+            r = oracle.optimizer_step(W, G, kind=kind, lr=0.1 if kind == oracle.SGD_MOMENTUM
+                                      else 1e-3, t=t, s1=s1, s2=s2)
+            # the oracle stores W and state in fp32, torch in fp64: compare to fp32 resolution
+            assert np.allclose(r["W"], p.detach().numpy(), rtol=0, atol=2e-8)
+            W, s1, s2 = r["W"], r["s1"], r["s2"]
+            # keep torch on the same fp32-rounded trajectory
+            with torch.no_grad():
+                p.copy_(torch.tensor(W.astype(np.float64)))
+            st = opt.state[p]
+            if kind == oracle.SGD_MOMENTUM:
+                assert np.allclose(s1, st["momentum_buffer"].numpy(), rtol=1e-6, atol=1e-12)
+                st["momentum_buffer"].copy_(torch.tensor(s1.astype(np.float64)))
+            else:
+                assert np.allclose(s1, st["exp_avg"].numpy(), rtol=1e-6, atol=1e-14)
+                assert np.allclose(s2, st["exp_avg_sq"].numpy(), rtol=1e-6, atol=1e-20)
+                st["exp_avg"].copy_(torch.tensor(s1.astype(np.float64)))
+                st["exp_avg_sq"].copy_(torch.tensor(s2.astype(np.float64)))
+
+
+def test_momentum_with_zero_buffer_first_step_is_sgd():
+    W, G = _opt_case(31)
+    a = oracle.optimizer_step(W, G, kind=oracle.SGD_MOMENTUM, lr=0.05)
+    b = oracle.optimizer_step(W, G, kind=oracle.SGD, lr=0.05)
+    sg, _ = oracle.sgd_update(W, G, 0.05)
+    assert np.array_equal(a["W"], b["W"]) and np.array_equal(b["W"], sg)
+    assert np.array_equal(a["s1"], G.astype(np.float32))
+
+
+def test_relative_clip_bounds_the_step_or_the_gradient():
+    W, G = _opt_case(32)
+    wn = np.linalg.norm(W.astype(np.float64))
+    # update clip, active: ||W' - W|| == 0.01 ||W|| (to fp32 rounding of W')
+    r = oracle.optimizer_step(W, G, kind=oracle.SGD, lr=50.0, clip=oracle.CLIP_UPDATE)
+    step = r["W"].astype(np.float64) - W
+    assert r["scale"] < 1 and abs(np.linalg.norm(step) - 0.01 * wn) < 1e-6 * wn
+    assert rel_err(step / np.linalg.norm(step), -G / np.linalg.norm(G)) < 1e-5
+    # inactive: identical to no clip
+    q = oracle.optimizer_step(W, G, kind=oracle.SGD, lr=1e-3, clip=oracle.CLIP_UPDATE)
+    assert q["scale"] == 1.0
+    assert np.array_equal(q["W"], oracle.optimizer_step(W, G, kind=oracle.SGD, lr=1e-3)["W"])
+    # gradient clip: the optimizer sees G scaled to 0.01 ||W||
+    big = 10.0 * G / np.linalg.norm(G) * wn
+    c = oracle.optimizer_step(W, big, kind=oracle.SGD_MOMENTUM, lr=0.1, clip=oracle.CLIP_GRADIENT)
+    assert abs(np.linalg.norm(c["s1"].astype(np.float64)) - 0.01 * wn) < 1e-6 * wn
+    # AdamW at t=1 with the update clip: the direction is -sign(G) - wd W / ... unchanged
+    a = oracle.optimizer_step(W, G, kind=oracle.ADAMW, lr=1.0, clip=oracle.CLIP_UPDATE)
+    assert abs(np.linalg.norm(a["W"].astype(np.float64) - W) - 0.01 * wn) < 1e-6 * wn
