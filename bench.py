@@ -228,6 +228,7 @@ def workload_config(wl, args):
             "error_matrix": {"auto": "stored-logits (auto)", "recompute": "recompute",
                              "stored": "stored-logits"}[args.algo],
             "norms_composed": "final + post-FFN per layer" if args.post_ffn_norm else "final",
+            "weights_updated": "W3, W1, W2 (W1/W2 via W3_init feedback)" if args.gate_up else "W3",
             "optimizer": ("plain SGD fused in the update GEMM epilogue" if args.optimizer == "fused-sgd"
                           else f"{args.optimizer} on fp32 masters, clip={args.clip} (1% of ||W||_F)"),
             "l2": "inputs larger than L2 (W_U %.0f MB, A_l %.2f GB per step); no flush"
@@ -264,6 +265,17 @@ def run_fpo(args, wl):
     g = torch.empty_like(h)
     loss = torch.empty(1, dtype=torch.float32, device=dev)
     post = args.post_ffn_norm
+    gate_up = args.gate_up
+    if gate_up:  # SwiGLU caches, W3_init feedback, gate/up masters and signal buffers
+        gu_ab = [synth.make_gate_up(wl_r, l, dev) for l in range(wl.layers)]
+        gu_x = [synth.make_mlp_in(wl_r, l, dev) for l in range(wl.layers)]
+        gu_W3 = [synth.make_W_master(wl_r, l, dev).to(torch.bfloat16) for l in range(wl.layers)]
+        gu_W12 = [m for l in range(wl.layers) for m in synth.make_gate_up_master(wl_r, l, dev)]
+        gu_out = [torch.empty(wl.d_ff, wl.d, dtype=torch.bfloat16, device=dev) for _ in gu_W12]
+        gu_sig = [torch.empty(wl.T, wl.d_ff, dtype=torch.bfloat16, device=dev)
+                  for _ in range(2 * wl.layers)]
+        gu_act = [x for x in gu_x for _ in range(2)]
+        ws_gu = torch.empty(fpo.layer_update_workspace(), dtype=torch.uint8, device=dev)
     if post:  # per-layer MLP outputs, post-FFN norm weights and layer-specific signals
         m_out = [synth.make_mlp_out(wl_r, l, dev) for l in range(wl.layers)]
         gp = [synth.make_post_norm_w(wl_r, l, dev) for l in range(wl.layers)]
@@ -297,6 +309,8 @@ def run_fpo(args, wl):
         launches_per_step += wl.layers
     if args.optimizer != "fused-sgd":  # G GEMM + optimizer (norms, scale, apply with a clip)
         launches_per_step += 3 if args.clip != "none" else 1
+    if args.gate_up:  # one error_h GEMM per layer + one grouped W1/W2 update
+        launches_per_step += wl.layers + 1
 
     def update():
         signals = g_l if post else [g] * wl.layers
@@ -308,6 +322,13 @@ def run_fpo(args, wl):
                                              workspace=ws_up)
         else:
             fpo.layer_update_grouped(g, A, wl.lr, W_masters=Wm, W_outs=Wo, workspace=ws_up)
+
+    def gate_up_update():
+        for l in range(wl.layers):
+            fpo.gate_up_signals(g_l[l] if post else g, gu_W3[l], gu_ab[l][0], gu_ab[l][1],
+                                gu_sig[2 * l], gu_sig[2 * l + 1], workspace=ws_gu)
+        fpo.layer_update_grouped_signals(gu_sig, gu_act, wl.lr, W_masters=gu_W12, W_outs=gu_out,
+                                         workspace=ws_gu)
 
     def step(stage_events=None, upd_events=None):
         fpo.error_signal(h, w, W_U, y, g, eps=wl.eps, min_rms=wl.min_rms, t_chunk=args.t_chunk,
@@ -322,6 +343,10 @@ def run_fpo(args, wl):
         update()
         if upd_events:
             upd_events[1].record(stream)
+        if gate_up:
+            gate_up_update()
+            if upd_events:
+                upd_events[3].record(stream)
 
     for _ in range(args.warmup):
         step()
@@ -331,7 +356,7 @@ def run_fpo(args, wl):
     # per-stage events for every timed step (recorded once so their handles exist)
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(fpo.STAGE_EVENTS)]
           for _ in range(args.steps)]
-    uev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    uev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
     for e in [x for row in ev + uev for x in row]:
         e.record(stream)
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -361,6 +386,9 @@ def run_fpo(args, wl):
     if post:
         stage_ms["post_ffn_vjp"] = statistics.mean(uev[i][2].elapsed_time(uev[i][0])
                                                    for i in range(args.steps))
+    if gate_up:
+        stage_ms["gate_up"] = statistics.mean(uev[i][1].elapsed_time(uev[i][3])
+                                              for i in range(args.steps))
 
     # ------------------------------------------------ end to end through the public API
     e2e = None
@@ -394,6 +422,8 @@ def run_fpo(args, wl):
                 for l in range(wl.layers):
                     fpo.rmsnorm_vjp(g, m_out[l], gp[l], g_l[l], eps=wl.eps, min_rms=wl.min_rms)
             update()
+            if gate_up:
+                gate_up_update()
             loss_host.copy_(loss, non_blocking=True)
 
         for _ in range(max(1, args.warmup)):
@@ -422,8 +452,11 @@ def run_fpo(args, wl):
     if rank == 0:
         peaks, peaks_src = load_peaks()
         tok_s = whole_job_tokens_per_s(wl.T, world, ms)
-        alg_tf = algorithmic_flops(wl) / (ms / 1e3) / 1e12
-        exe_tf = (executed_flops(wl) if not stored else algorithmic_flops(wl)) / (ms / 1e3) / 1e12
+        # the W1/W2 path adds error_h = g W3_init and the two gradient GEMMs per layer
+        gu_flops = 6.0 * wl.layers * wl.T * wl.d * wl.d_ff if gate_up else 0.0
+        alg_tf = (algorithmic_flops(wl) + gu_flops) / (ms / 1e3) / 1e12
+        exe_tf = ((executed_flops(wl) if not stored else algorithmic_flops(wl)) + gu_flops) / (
+            ms / 1e3) / 1e12
         per_kernel_flops = {
             "logits_lse_pass": 2.0 * wl.T * wl.V * wl.d,
             "projection": 2.0 * wl.T * wl.V * wl.d,
@@ -431,6 +464,8 @@ def run_fpo(args, wl):
         }
         if not stored:
             per_kernel_flops["recompute_error_pass"] = 2.0 * wl.T * wl.V * wl.d
+        if gate_up:
+            per_kernel_flops["gate_up"] = gu_flops
         # dominant kernel among those whose work is algorithmic (the recompute is overhead)
         dom = max(("logits_lse_pass", "projection", "layer_update"), key=lambda k: stage_ms[k])
         peak_sus = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
@@ -530,6 +565,8 @@ def main():
                          "clip and the optimizer step on the fp32 masters (fpo_layer_optimize_grouped)")
     ap.add_argument("--clip", choices=("none", "step", "grad"), default="step",
                     help="relative clip to 1%% of ||W||_F for --optimizer sgd/sgdm/adamw")
+    ap.add_argument("--gate-up", action="store_true",
+                    help="also update W1/W2 of every layer through the cached W3_init feedback")
     ap.add_argument("--post-ffn-norm", action="store_true",
                     help="compose each layer's post-FFN RMSNorm VJP (OLMo-2 layout) in the step")
     ap.add_argument("--algo", choices=("auto", "recompute", "stored"), default="auto",

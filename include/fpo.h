@@ -266,6 +266,28 @@ int32_t fpo_layer_optimize_grouped(int32_t n_layers, int64_t T, int64_t d, int64
                                    float* const* state2, void* workspace, size_t workspace_bytes,
                                    void* stream);
 
+/*
+ * fpo_gate_up_signals -- the hidden-space signals for the gate (W1) and up (W2)
+ * projections of one SwiGLU target layer (Sec. 3.1 step 5, Eq. (errh)), with the
+ * cached W3_init as the fixed feedback matrix:
+ *
+ *   error_h = g W3_init                                   [T, d_ff]
+ *   dA = error_h (.) b (.) silu'(a),  dB = error_h (.) silu(a)
+ *
+ * where a = x W1^T and b = x W2^T are the layer's cached gate and up
+ * pre-activations (h_mid = silu(a) (.) b) and silu'(a) = sigma(a)(1 + a(1 - sigma(a))).
+ * The W1 / W2 pseudogradients are then G1 = dA^T x, G2 = dB^T x ([d_ff, d], the
+ * nn.Linear layout of W1, W2), i.e. fpo_layer_update_grouped_signals with
+ * signals {dA, dB} and "activations" {x, x} (x: the MLP input [T, d]).
+ * The paper leaves the activation derivative to the MLP; these are SwiGLU's.
+ *
+ * g [T, d], W3_init [d, d_ff], a, b, dA, dB [T, d_ff], all in dtype.
+ * workspace: fpo_layer_update_workspace() bytes (device status word).
+ */
+int32_t fpo_gate_up_signals(int64_t T, int64_t d, int64_t d_ff, int32_t dtype, const void* g,
+                            const void* W3_init, const void* a, const void* b, void* dA, void* dB,
+                            void* workspace, size_t workspace_bytes, void* stream);
+
 /* Bytes of workspace fpo_cosine needs for n elements. */
 size_t fpo_cosine_workspace(int64_t n);
 

@@ -11,6 +11,7 @@ Each function follows one passage of the paper:
   with the min-RMS clamp.
 * :func:`rmsnorm_vjp`   App. E Eq. (rmsnorm-vjp) at any norm (the per-layer post-FFN
   norm of OLMo-2 / Gemma 3, Sec. 3.2).
+* :func:`gate_up_signals`  Sec. 3.1 step 5, Eq. (errh): W1/W2 signals of a SwiGLU MLP.
 * :func:`pseudograd`    Sec. 3.1 step 5, Eq. (w3update).
 * :func:`sgd_update`    App. A, fp32 master weights cast to bf16.
 * :func:`optimizer_step`  Sec. 3.1 AdamW / SGD with momentum, App. A relative clip.
@@ -58,6 +59,8 @@ def _load():
     lib.oracle_error_signal.restype = i32
     lib.oracle_rmsnorm_vjp.argtypes = [i64, i64, i32, vp, i32, vp, vp, dbl, dbl, vp]
     lib.oracle_rmsnorm_vjp.restype = i32
+    lib.oracle_gate_up_signals.argtypes = [i64, i64, i64, i32, vp, vp, vp, vp, vp, vp]
+    lib.oracle_gate_up_signals.restype = i32
     lib.oracle_pseudograd.argtypes = [i64, i64, i64, i32, vp, i32, vp, vp, vp, i64, vp]
     lib.oracle_pseudograd.restype = i32
     lib.oracle_sgd_update.argtypes = [i64, vp, vp, dbl, vp, vp]
@@ -149,6 +152,28 @@ def rmsnorm_vjp(g, x, gamma, *, eps=1e-6, min_rms=0.5):
     if rc != 0:
         raise ValueError(f"oracle_rmsnorm_vjp failed ({rc})")
     return out
+
+
+def gate_up_signals(g, W3_init, a, b):
+    """Sec. 3.1 step 5, Eq. (errh), SwiGLU: returns (dA, dB) fp64 [T, d_ff] with
+    error_h = g W3_init, dA = error_h * b * silu'(a), dB = error_h * silu(a)."""
+    dt, g = _typed(g)
+    d2, W3_init = _typed(W3_init)
+    d3, a = _typed(a)
+    d4, b = _typed(b)
+    if not (dt == d2 == d3 == d4):
+        raise TypeError("g, W3_init, a and b must share one dtype")
+    T, d = g.shape
+    d_ff = W3_init.shape[1]
+    if W3_init.shape[0] != d or a.shape != (T, d_ff) or b.shape != (T, d_ff):
+        raise ValueError("shapes: g [T,d], W3_init [d,d_ff], a and b [T,d_ff]")
+    dA = np.zeros((T, d_ff))
+    dB = np.zeros((T, d_ff))
+    rc = _load().oracle_gate_up_signals(T, d, d_ff, dt, _ptr(g), _ptr(W3_init), _ptr(a), _ptr(b),
+                                        _ptr(dA), _ptr(dB))
+    if rc != 0:
+        raise ValueError(f"oracle_gate_up_signals failed ({rc})")
+    return dA, dB
 
 
 def pseudograd(g_tilde, A, pairs=None):

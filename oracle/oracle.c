@@ -13,6 +13,7 @@
  *   oracle_error_signal  Sec. 3.1 steps 2-4, Eq. (gproj), App. E Eq. (rmsnorm-vjp)
  *                        and the min-RMS clamp (Sec. 3.2 / App. E)
  *   oracle_rmsnorm_vjp   App. E Eq. (rmsnorm-vjp) at any norm (post-FFN, Sec. 3.2)
+ *   oracle_gate_up_signals  Sec. 3.1 step 5, Eq. (errh): W1/W2 signals of a SwiGLU MLP
  *   oracle_pseudograd    Sec. 3.1 step 5, Eq. (w3update): G = g~^T h_mid
  *   oracle_sgd_update    App. A (fp32 master weights, cast to bf16)
  *   oracle_optimizer_step  Sec. 3.1 (AdamW / SGD with momentum) + App. A relative clip
@@ -174,6 +175,33 @@ int oracle_rmsnorm_vjp(int64_t T, int64_t d, int dt_g, const void* g, int dt_x, 
         for (int64_t j = 0; j < d; ++j)
             out[t * d + j] = (orc_load(dt_x, gamma, j) * orc_load(dt_g, g, t * d + j) -
                               (orc_load(dt_x, x, t * d + j) / rh) * c / (double)d) / denom;
+    }
+    return 0;
+}
+
+/*
+ * Gate / up signals of a SwiGLU MLP (Sec. 3.1 step 5, Eq. (errh)):
+ *   error_h = g W3_init                        [T, d_ff]   (g [T, d], W3_init [d, d_ff])
+ * and, with the cached gate and up pre-activations a, b ([T, d_ff];
+ * h_mid = silu(a) (.) b, silu(a) = a sigma(a)):
+ *   dA = error_h (.) b (.) silu'(a),  silu'(a) = sigma(a) (1 + a (1 - sigma(a)))
+ *   dB = error_h (.) silu(a)
+ * so that G1 = dA^T x and G2 = dB^T x (x the MLP input) are the W1 / W2
+ * pseudogradients.  Outputs fp64 [T, d_ff].
+ */
+int oracle_gate_up_signals(int64_t T, int64_t d, int64_t d_ff, int dt, const void* g,
+                           const void* W3, const void* a, const void* b, double* dA, double* dB) {
+    if (T < 0 || d <= 0 || d_ff <= 0 || !dA || !dB || (T > 0 && (!g || !W3 || !a || !b))) return -1;
+#pragma omp parallel for schedule(static)
+    for (int64_t t = 0; t < T; ++t) {
+        for (int64_t f = 0; f < d_ff; ++f) {
+            double e = 0.0;
+            for (int64_t j = 0; j < d; ++j) e += orc_load(dt, g, t * d + j) * orc_load(dt, W3, j * d_ff + f);
+            const double av = orc_load(dt, a, t * d_ff + f), bv = orc_load(dt, b, t * d_ff + f);
+            const double sg = 1.0 / (1.0 + exp(-av));
+            dA[t * d_ff + f] = e * bv * sg * (1.0 + av * (1.0 - sg));
+            dB[t * d_ff + f] = e * av * sg;
+        }
     }
     return 0;
 }

@@ -82,6 +82,9 @@ _lib.fpo_layer_optimize_grouped.argtypes = [_i32, _i64, _i64, _i64, _i32, ctypes
                                             ctypes.POINTER(_vp), ctypes.POINTER(_vp),
                                             ctypes.POINTER(_vp), ctypes.POINTER(_vp), _vp, _sz, _vp]
 _lib.fpo_layer_optimize_grouped.restype = _i32
+_lib.fpo_gate_up_signals.argtypes = [_i64, _i64, _i64, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
+                                     _sz, _vp]
+_lib.fpo_gate_up_signals.restype = _i32
 _lib.fpo_cosine_workspace.argtypes = [_i64]
 _lib.fpo_cosine_workspace.restype = _sz
 _lib.fpo_cosine.argtypes = [_i64, _i32, _vp, _vp, _vp, _vp, _sz, _vp]
@@ -277,6 +280,19 @@ def layer_optimize_grouped(gs, As, opt, W_masters, *, W_outs=None, states1=None,
         _ptr_array(W_masters, n), _ptr_array(W_outs, n), _ptr_array(states1, n),
         _ptr_array(states2, n), _ptr(workspace), workspace.numel(), _stream(stream))
     _check(rc, "fpo_layer_optimize_grouped")
+    return workspace
+
+
+def gate_up_signals(g, W3_init, a, b, dA, dB, *, workspace=None, stream=None):
+    """fpo_gate_up_signals: SwiGLU W1/W2 signals through the cached W3_init feedback."""
+    T, d = g.shape
+    d_ff = W3_init.shape[1]
+    if workspace is None:
+        workspace = _workspace(layer_update_workspace(), g.device)
+    rc = _lib.fpo_gate_up_signals(T, d, d_ff, _dtype_code(g), _ptr(g), _ptr(W3_init), _ptr(a),
+                                  _ptr(b), _ptr(dA), _ptr(dB), _ptr(workspace), workspace.numel(),
+                                  _stream(stream))
+    _check(rc, "fpo_gate_up_signals")
     return workspace
 
 

@@ -255,4 +255,90 @@ struct EpiStoreGroupF32 {
     __device__ __forceinline__ void finish(const Params&, int) {}
 };
 
+// ---------------------------------------------------------------------------
+// Gate / up signals of a SwiGLU MLP (Sec. 3.1 step 5, Eq. errh): the GEMM gives
+// error_h = g W3_init; with the cached pre-activations a (gate) and b (up),
+//   dA = error_h (.) b (.) silu'(a),  dB = error_h (.) silu(a)   (bf16 out)
+// Each 64-column pair of chunks fills one dA and one dB staging buffer (the
+// warp's two buffers), stored by two TMA stores in one bulk group.
+struct EpiSwiglu {
+    struct Params {
+        CUtensorMap dAmap;  // bf16 [M, N], box 64 x 32
+        CUtensorMap dBmap;
+        const __nv_bfloat16* a;  // [M, N]
+        const __nv_bfloat16* b;
+        long long ld;
+        int M, N;
+    };
+    int row;
+    bool valid, pair_out;
+
+    __device__ __forceinline__ EpiSwiglu(const Params& p, int, int row_, int) : row(row_) {
+        valid = row_ < p.M;
+        pair_out = false;
+    }
+
+    __device__ __forceinline__ void chunk(const Params& p, const float (&v)[32], int col0, int c0,
+                                          EpiIO& io) {
+        const bool second = (c0 & 32) != 0;
+        if (!second) {
+            pair_out = col0 >= p.N || io.row0 >= p.M;
+            if (pair_out) return;
+            if (io.lane == 0) bulk_wait_group_read<0>();  // both buffers free again
+            __syncwarp();
+        }
+        if (pair_out) return;
+        const int lim = p.N - col0;
+        float av[32], bv[32];
+        const uint4* pa = reinterpret_cast<const uint4*>(p.a + row * p.ld + col0);
+        const uint4* pb = reinterpret_cast<const uint4*>(p.b + row * p.ld + col0);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            uint4 ua = make_uint4(0, 0, 0, 0), ub = make_uint4(0, 0, 0, 0);
+            if (valid && q * 8 < lim) {
+                ua = pa[q];
+                ub = pb[q];
+            }
+            const __nv_bfloat162* ha = reinterpret_cast<const __nv_bfloat162*>(&ua);
+            const __nv_bfloat162* hb = reinterpret_cast<const __nv_bfloat162*>(&ub);
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const float2 fa = __bfloat1622float2(ha[k]), fb = __bfloat1622float2(hb[k]);
+                av[8 * q + 2 * k] = fa.x;
+                av[8 * q + 2 * k + 1] = fa.y;
+                bv[8 * q + 2 * k] = fb.x;
+                bv[8 * q + 2 * k + 1] = fb.y;
+            }
+        }
+        uint32_t wa[16], wb[16];
+#pragma unroll
+        for (int j = 0; j < 32; j += 2) {
+            float da[2], db[2];
+#pragma unroll
+            for (int k = 0; k < 2; ++k) {
+                const float x = av[j + k];
+                const float sg = 1.f / (1.f + __expf(-x));
+                da[k] = v[j + k] * bv[j + k] * sg * fmaf(x, 1.f - sg, 1.f);
+                db[k] = v[j + k] * x * sg;
+            }
+            wa[j / 2] = pack_bf16x2(da[0], da[1]);
+            wb[j / 2] = pack_bf16x2(db[0], db[1]);
+        }
+        const uint32_t bufA = io.out, bufB = io.out + kOutBufBytes;
+        out_stage_half(bufA, io.lane, second ? 1 : 0, wa);
+        out_stage_half(bufB, io.lane, second ? 1 : 0, wb);
+        if (second) {
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (io.lane == 0) {
+                tma_store_2d(&p.dAmap, bufA, col0 - 32, io.row0);
+                tma_store_2d(&p.dBmap, bufB, col0 - 32, io.row0);
+                bulk_commit_group();
+            }
+        }
+    }
+
+    __device__ __forceinline__ void finish(const Params&, int) {}
+};
+
 }  // namespace fpo

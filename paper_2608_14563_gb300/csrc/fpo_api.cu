@@ -416,6 +416,34 @@ int32_t fpo_layer_optimize_grouped(int32_t n_layers, int64_t T, int64_t d, int64
                                         scales, st));
 }
 
+int32_t fpo_gate_up_signals(int64_t T, int64_t d, int64_t d_ff, int32_t dtype, const void* g,
+                            const void* W3_init, const void* a, const void* b, void* dA, void* dB,
+                            void* workspace, size_t workspace_bytes, void* stream) {
+    if (dtype != FPO_F32 && dtype != FPO_BF16) return FPO_ERR_DTYPE;
+    if (T < 0 || d <= 0 || d_ff <= 0 || T > INT_MAX || d > INT_MAX || d_ff > INT_MAX)
+        return FPO_ERR_SHAPE;
+    if (dtype == FPO_BF16 && (d % 8 != 0 || d_ff % 8 != 0)) return FPO_ERR_SHAPE;
+    if (T > 0 && (!g || !W3_init || !a || !b || !dA || !dB)) return FPO_ERR_NULL;
+    if (!aligned16(g) || !aligned16(W3_init) || !aligned16(a) || !aligned16(b) || !aligned16(dA) ||
+        !aligned16(dB))
+        return FPO_ERR_ALIGN;
+    if (!workspace || workspace_bytes < kStatusBytes) return FPO_ERR_WORKSPACE;
+    if ((reinterpret_cast<uintptr_t>(workspace) % kAlign) != 0) return FPO_ERR_ALIGN;
+    int32_t rc = check_arch();
+    if (rc != FPO_OK) return rc;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    unsigned* status = static_cast<unsigned*>(workspace);
+    FPO_TRY(cudaMemsetAsync(status, 0, sizeof(unsigned), st));
+    if (T == 0) return FPO_OK;
+    const int Ti = static_cast<int>(T), di = static_cast<int>(d), fi = static_cast<int>(d_ff);
+    if (dtype == FPO_BF16)
+        return cuda_status(launch_swiglu_bf16(Ti, di, fi, g, W3_init, a, b, dA, dB, status, st));
+    return cuda_status(launch_swiglu_f32(Ti, di, fi, static_cast<const float*>(g),
+                                         static_cast<const float*>(W3_init),
+                                         static_cast<const float*>(a), static_cast<const float*>(b),
+                                         static_cast<float*>(dA), static_cast<float*>(dB), st));
+}
+
 int32_t fpo_rmsnorm_vjp(int64_t T, int64_t d, int32_t dtype, const void* g, const void* x,
                         const void* gamma, float eps, float min_rms, void* g_out, void* stream) {
     if (dtype != FPO_F32 && dtype != FPO_BF16) return FPO_ERR_DTYPE;

@@ -318,6 +318,27 @@ cudaError_t launch_grad_bf16(int n, int T, int d, int d_ff, const void* const* g
         maps, ep, make_shape(d, d_ff, T, kUpdBN, n, band_for(false)), status, st);
 }
 
+cudaError_t launch_swiglu_bf16(int T, int d, int d_ff, const void* g, const void* W3,
+                               const void* a, const void* b, void* dA, void* dB, unsigned* status,
+                               cudaStream_t st) {
+    GemmMaps<1> maps;
+    if (!map_kmajor(&maps.a[0], g, T, d, kBM) || !map_mnmajor(&maps.b[0], W3, d, d_ff))
+        return cudaErrorInvalidValue;
+    EpiSwiglu::Params ep;
+    if (!map_out_bf16(&ep.dAmap, dA, T, d_ff) || !map_out_bf16(&ep.dBmap, dB, T, d_ff))
+        return cudaErrorInvalidValue;
+    ep.a = static_cast<const __nv_bfloat16*>(a);
+    ep.b = static_cast<const __nv_bfloat16*>(b);
+    ep.ld = d_ff;
+    ep.M = T;
+    ep.N = d_ff;
+    if (use_pair())
+        return run_gemm_pair<256, false, true, kPairStages, 1, EpiSwiglu>(
+            maps, ep, make_shape(T, d_ff, d, 256, 1, band_for(true), kPairBM), status, st);
+    return run_gemm<256, false, true, 4, 1, EpiSwiglu>(
+        maps, ep, make_shape(T, d_ff, d, 256, 1, band_for(false)), status, st);
+}
+
 cudaError_t launch_test_gemm_bf16(int M, int N, int K, bool a_mn, bool b_mn, const void* A,
                                   const void* B, float* C, unsigned* status, cudaStream_t st) {
     const bool pair = use_pair();

@@ -51,6 +51,15 @@ cudaError_t launch_grad_bf16(int n, int T, int d, int d_ff, const void* const* g
                              const void* const* A, float* const* G_out, unsigned* status,
                              cudaStream_t st);
 
+// SwiGLU gate / up signals: dA, dB [T, d_ff] from error_h = g W3 (W3 [d, d_ff]) and the
+// cached pre-activations a, b [T, d_ff].
+cudaError_t launch_swiglu_bf16(int T, int d, int d_ff, const void* g, const void* W3,
+                               const void* a, const void* b, void* dA, void* dB, unsigned* status,
+                               cudaStream_t st);
+cudaError_t launch_swiglu_f32(int T, int d, int d_ff, const float* g, const float* W3,
+                              const float* a, const float* b, float* dA, float* dB,
+                              cudaStream_t st);
+
 // Optimizer step of n layers of n_elem elements from fp32 G (optimizer.cu).
 struct OptimParams {
     int kind;          // 0 SGD, 1 SGD with momentum, 2 AdamW

@@ -50,6 +50,13 @@ struct SEpiStore {
     float* C;
     long long ld;
 };
+struct SEpiSwiglu {  // dA = e b silu'(a), dB = e silu(a) from e = g W3 and cached a, b
+    float* dA;
+    float* dB;
+    const float* a;
+    const float* b;
+    long long ld;
+};
 struct SEpiUpdate {
     float* W_master[kMaxG];
     float* W_out[kMaxG];
@@ -146,6 +153,12 @@ __global__ void __launch_bounds__(kThreads)
                     ep.E[row * ep.ldE + col] = error_value_f32(v, ep.lse[row], col == ep.y[row], ep.s);
                 } else if constexpr (std::is_same_v<Epi, SEpiStore>) {
                     ep.C[row * ep.ld + col] = v;
+                } else if constexpr (std::is_same_v<Epi, SEpiSwiglu>) {
+                    const long long off = row * ep.ld + col;
+                    const float x = ep.a[off];
+                    const float sg = 1.f / (1.f + expf(-x));
+                    ep.dA[off] = v * ep.b[off] * sg * fmaf(x, 1.f - sg, 1.f);
+                    ep.dB[off] = v * x * sg;
                 } else {
                     const long long off = row * ep.ld + col;
                     if (float* wm = ep.W_master[g]) {
@@ -204,6 +217,14 @@ cudaError_t launch_proj_f32(const float* E, const float* W_U, int Tc, int d, int
     // g[t, j] = sum_v E[t, v] W_U[v, j]: B(n=j, k=v) = W_U[v*d + j]
     SEpiStore ep{g, d};
     return run(ops_of(E, V, 1, W_U, 1, d, Tc, d, V), ep, 1, st);
+}
+
+cudaError_t launch_swiglu_f32(int T, int d, int d_ff, const float* g, const float* W3,
+                              const float* a, const float* b, float* dA, float* dB,
+                              cudaStream_t st) {
+    // e[t, f] = sum_j g[t, j] W3[j, f]: A(m=t, k=j) = g[t*d + j], B(n=f, k=j) = W3[j*d_ff + f]
+    SEpiSwiglu ep{dA, dB, a, b, d_ff};
+    return run(ops_of(g, d, 1, W3, 1, d_ff, T, d_ff, d), ep, 1, st);
 }
 
 cudaError_t launch_update_f32(int n, int T, int d, int d_ff, const float* const* g,

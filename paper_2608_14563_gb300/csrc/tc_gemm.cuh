@@ -131,6 +131,16 @@ __device__ __forceinline__ void out_stage_row(uint32_t buf, int r, const uint32_
                      w[4 * c], w[4 * c + 1], w[4 * c + 2], w[4 * c + 3]);
 }
 
+// Write 16 words (64 bytes) of row r into half `h` (pieces 4h..4h+3) of a
+// staging buffer, same swizzle as out_stage_row.
+__device__ __forceinline__ void out_stage_half(uint32_t buf, int r, int h, const uint32_t (&w)[16]) {
+    const uint32_t row = buf + static_cast<uint32_t>(r) * 128u;
+#pragma unroll
+    for (int c = 0; c < 4; ++c)
+        st_shared_v4(row + (((static_cast<uint32_t>(4 * h + c)) ^ (static_cast<uint32_t>(r) & 7u)) << 4),
+                     w[4 * c], w[4 * c + 1], w[4 * c + 2], w[4 * c + 3]);
+}
+
 // Store a filled staging buffer to (x, y) of `map` (rows/columns outside the
 // tensor are clipped by the TMA engine).
 __device__ __forceinline__ void out_commit(EpiIO& io, const CUtensorMap* map, uint32_t buf, int x,

@@ -20,6 +20,10 @@ Recipe (every tensor has its own generator seeded from (seed, tensor, layer)):
          (the per-layer MLP output feeding a post-FFN norm: per-token RMS
          varies widely and a few outlier tokens sit near 0.1)      [T, d] per layer
 * gp_l   = 0.3 + 0.05 N(0, 1)         post-FFN RMSNorm weight      [d] per layer
+* a_l, b_l  the two N(0, 1) draws behind A_l (gate and up pre-activations of
+         the SwiGLU MLP, A_l = SiLU(a_l) b_l)                         [T, d_ff] per layer
+* x_l    ~ N(0, 1)                      MLP input (after its norm)  [T, d] per layer
+* W1_l, W2_l ~ N(0, 0.02^2), fp32 master  gate / up weights          [d_ff, d] per layer
 
 Tensors are generated in fp32 and rounded to the storage dtype by torch.
 """
@@ -29,7 +33,8 @@ from dataclasses import dataclass, field
 
 import torch
 
-_TENSOR_IDS = {"h": 1, "w": 2, "W_U": 3, "A": 4, "W": 5, "y": 6, "noise": 7, "m": 8, "gp": 9}
+_TENSOR_IDS = {"h": 1, "w": 2, "W_U": 3, "A": 4, "W": 5, "y": 6, "noise": 7, "m": 8, "gp": 9,
+               "x": 10, "W1": 11, "W2": 12}
 
 
 @dataclass(frozen=True)
@@ -113,6 +118,26 @@ def make_A(wl: Workload, layer: int, device="cpu"):
     b = torch.randn((wl.T, wl.d_ff), generator=g, device=device, dtype=torch.float32)
     a = torch.nn.functional.silu(a).mul_(b)
     return a.to(wl.torch_dtype)
+
+
+def make_gate_up(wl: Workload, layer: int, device="cpu"):
+    """(a_l, b_l): the gate and up pre-activations whose SwiGLU product is make_A's A_l."""
+    g = _gen(wl.seed, "A", layer, device)
+    a = torch.randn((wl.T, wl.d_ff), generator=g, device=device, dtype=torch.float32)
+    b = torch.randn((wl.T, wl.d_ff), generator=g, device=device, dtype=torch.float32)
+    return a.to(wl.torch_dtype), b.to(wl.torch_dtype)
+
+
+def make_mlp_in(wl: Workload, layer: int, device="cpu"):
+    return normal((wl.T, wl.d), seed=wl.seed, tensor="x", layer=layer, device=device,
+                  dtype=wl.torch_dtype)
+
+
+def make_gate_up_master(wl: Workload, layer: int, device="cpu"):
+    return (normal((wl.d_ff, wl.d), std=0.02, seed=wl.seed, tensor="W1", layer=layer,
+                   device=device),
+            normal((wl.d_ff, wl.d), std=0.02, seed=wl.seed, tensor="W2", layer=layer,
+                   device=device))
 
 
 def make_W_master(wl: Workload, layer: int, device="cpu"):

@@ -447,3 +447,59 @@ def test_relative_clip_bounds_the_step_or_the_gradient():
     # AdamW at t=1 with the update clip: the direction is -sign(G) - wd W / ... unchanged
     a = oracle.optimizer_step(W, G, kind=oracle.ADAMW, lr=1.0, clip=oracle.CLIP_UPDATE)
     assert abs(np.linalg.norm(a["W"].astype(np.float64) - W) - 0.01 * wn) < 1e-6 * wn
+
+
+# ---------------------------------------------------------------------------
+# Gate / up updates through the cached W3_init feedback (Sec. 3.1 step 5, Eq. errh)
+# ---------------------------------------------------------------------------
+def _silu(a):
+    return a / (1.0 + np.exp(-a))
+
+
+def test_gate_up_signals_are_exact_gradients_at_step_zero():
+    """Nothing above the layer and W3_init = W3 (step 0, where the paper notes the
+    feedback is exact): dA^T x and dB^T x are dL/dW1 and dL/dW2 of the SwiGLU MLP."""
+    rng = np.random.default_rng(50)
+    T, d, d_ff, V = 5, 6, 7, 9
+    h0 = rng.standard_normal((T, d))
+    x = rng.standard_normal((T, d))
+    W1 = 0.4 * rng.standard_normal((d_ff, d))
+    W2 = 0.4 * rng.standard_normal((d_ff, d))
+    W3 = 0.4 * rng.standard_normal((d, d_ff))
+    w = 1.0 + 0.1 * rng.standard_normal(d)
+    W_U = 0.5 * rng.standard_normal((V, d))
+    y = rng.integers(0, V, T).astype(np.int32)
+    s, eps = 1.0 / T, 1e-6
+
+    def loss(W1x, W2x):
+        return forward_loss(h0 + (_silu(x @ W1x.T) * (x @ W2x.T)) @ W3.T, w, W_U, y, eps, s)
+
+    a, b = x @ W1.T, x @ W2.T
+    h = h0 + (_silu(a) * b) @ W3.T
+    gt = oracle.error_signal(h, w, W_U, y, eps=eps, min_rms=0.0, s=s)["g_tilde"]
+    dA, dB = oracle.gate_up_signals(gt, W3, a, b)
+    G1 = oracle.pseudograd(dA, x)   # [d_ff, d] = dA^T x
+    G2 = oracle.pseudograd(dB, x)
+    fd1 = fd_grad(lambda W1x: loss(W1x, W2), W1.copy())
+    fd2 = fd_grad(lambda W2x: loss(W1, W2x), W2.copy())
+    assert rel_err(G1, fd1) < 1e-7
+    assert rel_err(G2, fd2) < 1e-7
+    # and the down-projection signal of the same layer stays g~^T h_mid
+    fd3 = fd_grad(lambda W3x: forward_loss(h0 + (_silu(a) * b) @ W3x.T, w, W_U, y, eps, s),
+                  W3.copy())
+    assert rel_err(oracle.pseudograd(gt, _silu(a) * b), fd3) < 1e-7
+
+
+def test_silu_derivative_against_autograd():
+    torch = pytest.importorskip("torch")
+    a = np.linspace(-8, 8, 101)
+    at = torch.tensor(a, requires_grad=True)
+    torch.nn.functional.silu(at).sum().backward()
+    # dB / error_h = silu(a) and dA / (error_h b) = silu'(a) with error_h = b = 1
+    T = 1
+    g = np.ones((T, 1))
+    W3 = np.ones((1, a.size))
+    dA, dB = oracle.gate_up_signals(g, W3, a[None, :], np.ones((T, a.size)))
+    assert np.allclose(dA[0], at.grad.numpy(), rtol=1e-12, atol=1e-14)
+    assert np.allclose(dB[0], torch.nn.functional.silu(torch.tensor(a)).numpy(), rtol=1e-12,
+                       atol=1e-14)
