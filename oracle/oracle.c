@@ -53,6 +53,9 @@ int oracle_abi_version(void) { return 1; }
  *   z_v   = <yhat, W_U[v,:]>                                logits (Sec. 3.1 step 2)
  *   lse   = m + log sum_v exp(z_v - m),  m = max_v z_v
  *   e_v   = s * (exp(z_v - lse) - [v == y_t])              softmax(z) - 1_y, loss scale s
+ *           (the target entry as -s sum_{v != y_t} exp(z_v - lse): the softmax
+ *           sums to one, so this is the same number, and it keeps its digits
+ *           when 1 - p_y is below the fp64 ulp of lse, where p_y - 1 has none)
  *   g_j   = sum_v e_v W_U[v,j]                              Eq. (gproj)
  *   c     = <xhat, w (.) g>
  *   g~_j  = (w_j g_j - xhat_j c / d) / max(rho, rho_min)    Eq. (rmsnorm-vjp) + min-RMS clamp
@@ -109,15 +112,17 @@ int oracle_error_signal(int64_t T, int64_t d, int64_t V, int dt,
         for (int64_t v = 0; v < V; ++v) se += exp(z[v] - m);
         double l = m + log(se);
 
-        /* e overwrites z in place: e_v = s (p_v - [v == y]). */
+        /* e overwrites z in place: e_v = s p_v off the target, and
+         * e_y = -s sum_{v != y} p_v (summed in index order). */
+        if (zy) zy[r] = z[yt];
+        double rest = 0.0;
         for (int64_t v = 0; v < V; ++v) {
+            if (v == yt) continue;
             double p = exp(z[v] - l);
-            if (v == yt) {
-                if (zy) zy[r] = z[v];
-                p -= 1.0;
-            }
+            rest += p;
             z[v] = s * p;
         }
+        z[yt] = -s * rest;
         if (e) memcpy(e + r * V, z, sizeof(double) * (size_t)V);
 
         for (int64_t j = 0; j < d; ++j) gt[j] = 0.0;

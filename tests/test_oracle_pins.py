@@ -115,6 +115,19 @@ def test_rows_of_error_sum_to_zero():
     assert np.all(out["e"][np.arange(6), y] < 0)
 
 
+def test_confident_token_target_entry_closed_form():
+    """Two-word vocabulary, logits (40, 0), target 0: p_1 = 1 / (1 + e^40) ~ 4.2e-18, so
+    e_0 = -p_1, e_1 = p_1 and g = e W_U = -40 p_1 (Sec. 3.1 step 2), values that p_0 - 1
+    cannot carry in fp64 (1 / (1 + 4.2e-18) rounds to 1)."""
+    h, w = np.array([[1.0]]), np.array([1.0])  # eps = 0: rho = 1, yhat = 1
+    W_U = np.array([[40.0], [0.0]])
+    out = oracle.error_signal(h, w, W_U, np.array([0]), eps=0.0, min_rms=0.0, s=1.0, want_e=True)
+    p1 = 1.0 / (1.0 + math.exp(40.0))
+    assert abs(out["e"][0, 1] - p1) <= 1e-14 * p1
+    assert abs(out["e"][0, 0] + p1) <= 1e-14 * p1
+    assert abs(out["g"][0, 0] + 40.0 * p1) <= 1e-14 * 40.0 * p1
+
+
 def test_eps0_vjp_orthogonal_to_h():
     """At eps = 0 the RMSNorm VJP is orthogonal to h, clamped tokens included."""
     h, w, W_U, y = _toy(T=5, seed=5)
