@@ -225,8 +225,8 @@ def workload_config(wl, args):
     return {"workload": wl.name, "T": wl.T, "d": wl.d, "d_ff": wl.d_ff, "V": wl.V,
             "target_layers": wl.layers, "targets": "zipf(1.1)" if wl.targets == "zipf" else wl.targets,
             "lr": wl.lr, "t_chunk": args.t_chunk or wl.T, "global_batch_tokens": wl.T * args.gpus,
-            "error_matrix": {"auto": "stored-logits (auto)", "recompute": "recompute",
-                             "stored": "stored-logits"}[args.algo],
+            "error_matrix": {"auto": "direct (auto)", "recompute": "recompute",
+                             "stored": "stored-logits", "direct": "direct"}[args.algo],
             "norms_composed": "final + post-FFN per layer" if args.post_ffn_norm else "final",
             "weights_updated": "W3, W1, W2 (W1/W2 via W3_init feedback)" if args.gate_up else "W3",
             "optimizer": ("plain SGD fused in the update GEMM epilogue" if args.optimizer == "fused-sgd"
@@ -251,6 +251,8 @@ def run_fpo(args, wl):
     if args.gemm_variant >= 0:
         fpo.set_gemm_variant(args.gemm_variant)
     variant = fpo.set_gemm_variant(-1)  # read back (a negative value changes nothing)
+    if args.band:
+        fpo._lib.fpo_testing_set_band(args.band)
 
     wl_r = synth.Workload(wl.name, T=wl.T, d=wl.d, d_ff=wl.d_ff, V=wl.V, layers=wl.layers,
                           dtype=wl.dtype, targets=wl.targets, lr=wl.lr, seed=rank)
@@ -281,8 +283,10 @@ def run_fpo(args, wl):
         gp = [synth.make_post_norm_w(wl_r, l, dev) for l in range(wl.layers)]
         g_l = [torch.empty_like(h) for _ in range(wl.layers)]
     algo = {"auto": fpo.ES_AUTO, "recompute": fpo.ES_RECOMPUTE,
-            "stored": fpo.ES_STORED_LOGITS}[args.algo]
-    stored = algo != fpo.ES_RECOMPUTE
+            "stored": fpo.ES_STORED_LOGITS, "direct": fpo.ES_DIRECT}[args.algo]
+    # the algorithm that runs (bf16: AUTO is the direct algorithm)
+    algo_name = {fpo.ES_RECOMPUTE: "recompute", fpo.ES_STORED_LOGITS: "stored-logits"}.get(
+        algo, "direct")
     desc = fpo.error_signal_desc(wl.T, wl.d, wl.V, fpo.BF16, eps=wl.eps, min_rms=wl.min_rms,
                                  t_chunk=args.t_chunk, algo=algo)
     ws_es = torch.empty(fpo.error_signal_workspace(desc), dtype=torch.uint8, device=dev)
@@ -302,9 +306,11 @@ def run_fpo(args, wl):
     stream = torch.cuda.current_stream()
 
     n_chunks = -(-wl.T // (args.t_chunk or wl.T))
-    # fwd, mean, vjp, update + per chunk (stored: logits, combine, E, projection;
-    # recompute: E pass, projection; plus one logits pass and one combine)
-    launches_per_step = 4 + (4 * n_chunks if stored else 2 + 2 * n_chunks)
+    # fwd, mean, vjp, update + per chunk (direct: logits, combine, fixup, fixup factors,
+    # projection; stored: logits, combine, E, projection; recompute: E pass, projection,
+    # plus one logits pass and one combine)
+    launches_per_step = 4 + {"direct": 5 * n_chunks, "stored-logits": 4 * n_chunks,
+                             "recompute": 2 + 2 * n_chunks}[algo_name]
     if post:
         launches_per_step += wl.layers
     if args.optimizer != "fused-sgd":  # G GEMM + optimizer (norms, scale, apply with a clip)
@@ -378,7 +384,8 @@ def run_fpo(args, wl):
     status = (fpo.get_device_status(ws_es), fpo.get_device_status(ws_up))
 
     names = ["rmsnorm_fwd", "logits_lse_pass", "lse_combine",
-             "logits_to_error" if stored else "recompute_error_pass", "projection", "rmsnorm_vjp"]
+             {"direct": "direct_fixup", "stored-logits": "logits_to_error",
+              "recompute": "recompute_error_pass"}[algo_name], "projection", "rmsnorm_vjp"]
     stage_ms = {n: statistics.mean(ev[i][k].elapsed_time(ev[i][k + 1]) for i in range(args.steps))
                 for k, n in enumerate(names)}
     stage_ms["layer_update"] = statistics.mean(uev[i][0].elapsed_time(uev[i][1])
@@ -455,14 +462,15 @@ def run_fpo(args, wl):
         # the W1/W2 path adds error_h = g W3_init and the two gradient GEMMs per layer
         gu_flops = 6.0 * wl.layers * wl.T * wl.d * wl.d_ff if gate_up else 0.0
         alg_tf = (algorithmic_flops(wl) + gu_flops) / (ms / 1e3) / 1e12
-        exe_tf = ((executed_flops(wl) if not stored else algorithmic_flops(wl)) + gu_flops) / (
+        exe_tf = ((executed_flops(wl) if algo_name == "recompute" else algorithmic_flops(wl))
+                  + gu_flops) / (
             ms / 1e3) / 1e12
         per_kernel_flops = {
             "logits_lse_pass": 2.0 * wl.T * wl.V * wl.d,
             "projection": 2.0 * wl.T * wl.V * wl.d,
             "layer_update": 2.0 * wl.layers * wl.T * wl.d * wl.d_ff,
         }
-        if not stored:
+        if algo_name == "recompute":
             per_kernel_flops["recompute_error_pass"] = 2.0 * wl.T * wl.V * wl.d
         if gate_up:
             per_kernel_flops["gate_up"] = gu_flops
@@ -492,7 +500,7 @@ def run_fpo(args, wl):
             "kernels_ms": stage_ms,
             "kernels_tflops": {k: per_kernel_flops[k] / (stage_ms[k] / 1e3) / 1e12
                                for k in per_kernel_flops},
-            "algo": "stored-logits" if stored else "recompute",
+            "algo": algo_name,
             "gemm_kernel": "cta-pair 256x256 (tcgen05 cta_group::2)" if variant == 1
                            else "single-cta 128x256 (tcgen05 cta_group::1)",
             "cpu_baseline": cpu,
@@ -569,8 +577,10 @@ def main():
                     help="also update W1/W2 of every layer through the cached W3_init feedback")
     ap.add_argument("--post-ffn-norm", action="store_true",
                     help="compose each layer's post-FFN RMSNorm VJP (OLMo-2 layout) in the step")
-    ap.add_argument("--algo", choices=("auto", "recompute", "stored"), default="auto",
+    ap.add_argument("--algo", choices=("auto", "recompute", "stored", "direct"), default="auto",
                     help="how the error matrix is formed (fpo_es_algo)")
+    ap.add_argument("--band", type=int, default=0,
+                    help="GEMM rasterisation band height in tiles (0: library default; tuning)")
     ap.add_argument("--gemm-variant", type=int, choices=(-1, 0, 1), default=-1,
                     help="tensor-core GEMM kernel: 0 single-CTA tiles, 1 CTA-pair tiles, "
                          "-1 library default")

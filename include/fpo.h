@@ -81,14 +81,32 @@ typedef enum fpo_status {
  *                        log-sum-exp is known (one GEMM instead of two, at the
  *                        cost of T_chunk x V x 4 bytes of workspace and ~3 passes
  *                        over it in HBM).
- *  FPO_ES_AUTO           the library's choice (currently FPO_ES_STORED_LOGITS).
- * Both compute every value with the same arithmetic: their outputs are
- * bit-identical.
+ *  FPO_ES_DIRECT         (bf16 only) no E at all.  With the anchor c_t =
+ *                        <xhat_t (.) norm_w, W_U[y_t]> (the target logit, from the
+ *                        RMSNorm forward), the logits pass writes
+ *                        P_tj = exp(z_tj - c_t) in bf16 with the target column 0,
+ *                        and the projection forms
+ *                          g_t = s e^{c_t - lse_t} (P_t W_U - S'_t W_U[y_t]),
+ *                        S'_t the sum of row t of the rounded P.  This equals
+ *                        e_t W_U exactly in real arithmetic (the target entry of
+ *                        e_t is -sum of the others), rounds each probability to
+ *                        bf16 once like E, and saves the E pass: T_chunk x V x 2
+ *                        bytes of workspace.  Rows with S'_t outside
+ *                        [2^-80, 2^80] (token cross-entropy beyond ~55 nats, or
+ *                        1 - p_target below ~1e-24) are recomputed by an fp32
+ *                        SIMT kernel anchored at lse_t before the projection.
+ *  FPO_ES_AUTO           the library's choice: FPO_ES_DIRECT for bf16,
+ *                        FPO_ES_STORED_LOGITS for fp32 (where DIRECT also runs
+ *                        the stored-logits algorithm).
+ * RECOMPUTE and STORED_LOGITS compute every value with the same arithmetic:
+ * their outputs are bit-identical.  DIRECT agrees with them to the bf16
+ * rounding of the probabilities, and is bit-identical across t_chunk values.
  */
 typedef enum fpo_es_algo {
     FPO_ES_AUTO = 0,
     FPO_ES_RECOMPUTE = 1,
-    FPO_ES_STORED_LOGITS = 2
+    FPO_ES_STORED_LOGITS = 2,
+    FPO_ES_DIRECT = 3
 } fpo_es_algo;
 
 /* Error-signal problem description (Sec. 3.1 steps 2-4, App. E). */
@@ -111,8 +129,9 @@ typedef struct fpo_error_signal_desc {
  * Stage boundaries of fpo_error_signal at which desc->stage_events[i] is
  * recorded: 0 start, 1 after the RMSNorm forward, 2 after the logits pass (of
  * the last token chunk for FPO_ES_STORED_LOGITS), 3 after the log-sum-exp
- * combine (and loss), 4 after the recompute pass (FPO_ES_RECOMPUTE) or the
- * logits-to-E conversion (FPO_ES_STORED_LOGITS) of the last token chunk, 5
+ * combine (and loss), 4 after the recompute pass (FPO_ES_RECOMPUTE), the
+ * logits-to-E conversion (FPO_ES_STORED_LOGITS) or the anchor-window fixup
+ * (FPO_ES_DIRECT) of the last token chunk, 5
  * after the projection of the last token chunk, 6 after the final-norm VJP.
  * With one chunk, consecutive events bracket one kernel each (plus the loss
  * mean in [2]-[3]).

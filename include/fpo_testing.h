@@ -8,6 +8,8 @@
 #include <stddef.h>
 #include <stdint.h>
 
+#include "fpo.h"
+
 #ifdef __cplusplus
 extern "C" {
 #endif
@@ -37,10 +39,20 @@ int32_t fpo_testing_set_gemm_variant(int32_t variant);
 
 /*
  * Override the height, in output tiles, of the bands in which GEMM tiles are
- * rasterised for L2 reuse (0 restores the default: bands of 2048 output rows).
+ * rasterised for L2 reuse (0 restores the default: bands of 16 tile rows).
  * Tuning hook; results do not depend on it.
  */
 void fpo_testing_set_band(int32_t band);
+
+/*
+ * Rows of the last token chunk of the most recent fpo_error_signal call on
+ * `workspace` (with this `desc`) that the direct algorithm recomputed because
+ * S'_t fell outside its anchor window (see FPO_ES_DIRECT).  Synchronizes
+ * `stream`.  Returns -1 when desc does not select the direct algorithm, or on
+ * a CUDA error.
+ */
+int64_t fpo_testing_direct_fixup_rows(const fpo_error_signal_desc* desc,
+                                      const void* workspace, void* stream);
 
 /*
  * Failure-detection check of the bounded waits every kernel uses: launches one

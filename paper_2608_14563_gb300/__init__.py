@@ -22,7 +22,7 @@ F32, BF16 = 0, 1
 OK = 0
 MAX_GROUPED_LAYERS = 64
 STAGE_EVENTS = 7
-ES_AUTO, ES_RECOMPUTE, ES_STORED_LOGITS = 0, 1, 2
+ES_AUTO, ES_RECOMPUTE, ES_STORED_LOGITS, ES_DIRECT = 0, 1, 2, 3
 
 if not os.path.exists(LIB_PATH):
     raise ImportError(f"libfpo.so is not built ({LIB_PATH} missing); run "
@@ -91,6 +91,8 @@ _lib.fpo_cosine.argtypes = [_i64, _i32, _vp, _vp, _vp, _vp, _sz, _vp]
 _lib.fpo_cosine.restype = _i32
 _lib.fpo_get_device_status.argtypes = [_vp, _vp]
 _lib.fpo_get_device_status.restype = _i32
+_lib.fpo_testing_direct_fixup_rows.argtypes = [ctypes.POINTER(ErrorSignalDesc), _vp, _vp]
+_lib.fpo_testing_direct_fixup_rows.restype = _i64
 _lib.fpo_testing_set_gemm_variant.argtypes = [_i32]
 _lib.fpo_testing_set_gemm_variant.restype = _i32
 
@@ -196,6 +198,15 @@ def error_signal(h, norm_w, W_U, targets, g_out, *, eps=1e-6, min_rms=0.5, loss_
                                workspace.numel() * workspace.element_size(), _stream(stream))
     _check(rc, "fpo_error_signal")
     return workspace
+
+
+def direct_fixup_rows(h, W_U, workspace, *, t_chunk=0, algo=ES_AUTO, stream=None) -> int:
+    """fpo_testing_direct_fixup_rows: rows of the last token chunk of the latest error_signal
+    call on ``workspace`` that the direct algorithm recomputed (-1: not the direct algorithm)."""
+    T, d = h.shape
+    desc = error_signal_desc(T, d, W_U.shape[0], _dtype_code(h), t_chunk=t_chunk, algo=algo)
+    return int(_lib.fpo_testing_direct_fixup_rows(ctypes.byref(desc), _ptr(workspace),
+                                                  _stream(stream)))
 
 
 # --------------------------------------------------------------------------- layer update

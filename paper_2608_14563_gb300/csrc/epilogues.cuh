@@ -89,6 +89,96 @@ using EpiLsePartial = EpiLsePartialT<false>;
 using EpiLseStoreZ = EpiLsePartialT<true>;
 
 // ---------------------------------------------------------------------------
+// Logits pass of the direct algorithm (Sec. 3.1 step 2 rewritten around a
+// per-token anchor c_t): besides the (max, sum exp) partial and the target
+// logit of EpiLsePartial, every valid non-target logit leaves
+//   p~_tj = exp(z_tj - c_t)              rounded to bf16 into P [M, N]
+// (the target column and the overhang are written as 0), and the tile's sum of
+// those rounded values, S'_t partial, goes to sx [M, part_ld].  Two 32-column
+// chunks fill one 64-column bf16 staging row before each TMA store.
+struct EpiLseProb {
+    struct Params {
+        CUtensorMap pmap;     // bf16 P [M, N], box 64 x 32
+        float2* part;         // [M, part_ld] (max, sum exp(z - max))
+        float* sx;            // [M, part_ld] sum of the rounded p~ of the tile
+        int part_ld;
+        float* zy;            // [M] target logit, or null
+        const int* y;         // [M] targets
+        const float* anchor;  // [M] c_t
+        int M, N;
+    };
+    float m, s, zt, sxs, c2;
+    int yoff;
+    int row;
+    bool valid, has_t, pair_out;
+    uint32_t w[32];
+
+    __device__ __forceinline__ EpiLseProb(const Params& p, int, int row_, int n0)
+        : m(-INFINITY), s(0.f), zt(0.f), sxs(0.f), row(row_), has_t(false), pair_out(false) {
+        valid = row_ < p.M;
+        yoff = valid ? __ldg(p.y + row_) - n0 : -1;
+        c2 = valid ? __ldg(p.anchor + row_) * kLog2e : 0.f;
+    }
+
+    // p~ of logits j, j+1 of the chunk (0 for the target and for columns >= lim),
+    // packed to bf16; the rounded values are added to the tile sum.
+    __device__ __forceinline__ uint32_t prob_pair(const float (&v)[32], int j, int lim, int r) {
+        const float a = (j < lim && j != r) ? ex2_approx(fmaf(v[j], kLog2e, -c2)) : 0.f;
+        const float b = (j + 1 < lim && j + 1 != r) ? ex2_approx(fmaf(v[j + 1], kLog2e, -c2)) : 0.f;
+        const uint32_t pk = pack_bf16x2(a, b);
+        sxs += __uint_as_float(pk << 16) + __uint_as_float(pk & 0xffff0000u);
+        return pk;
+    }
+
+    __device__ __forceinline__ void chunk(const Params& p, const float (&v)[32], int col0, int c0,
+                                          EpiIO& io) {
+        const bool second = (c0 & 32) != 0;
+        if (!second) pair_out = col0 >= p.N || io.row0 >= p.M;
+        const int lim = p.N - col0;  // valid columns in this chunk (may be <= 0)
+        const int r = yoff - c0;     // target position in this chunk, if in [0, 32)
+        if (lim > 0) {
+            float cm = -INFINITY;
+#pragma unroll
+            for (int j = 0; j < 32; ++j)
+                if (j < lim) cm = fmaxf(cm, v[j]);
+            const float nm = fmaxf(m, cm);
+            const float nml = nm * kLog2e;
+            float acc = (m == -INFINITY) ? 0.f : s * ex2_approx(m * kLog2e - nml);
+#pragma unroll
+            for (int j = 0; j < 32; ++j)
+                if (j < lim) acc += ex2_approx(fmaf(v[j], kLog2e, -nml));
+            s = acc;
+            m = nm;
+            if (static_cast<unsigned>(r) < 32u) {
+#pragma unroll
+                for (int j = 0; j < 32; ++j)
+                    if (j == r) zt = v[j];
+                has_t = true;
+            }
+        }
+        if (pair_out) return;
+        if (!second) {
+#pragma unroll
+            for (int j = 0; j < 32; j += 2) w[j / 2] = prob_pair(v, j, lim, r);
+        } else {
+#pragma unroll
+            for (int j = 0; j < 32; j += 2) w[16 + j / 2] = prob_pair(v, j, lim, r);
+            const uint32_t buf = out_acquire(io);
+            out_stage_row(buf, io.lane, w);
+            out_commit(io, &p.pmap, buf, col0 - 32, io.row0);
+        }
+    }
+
+    __device__ __forceinline__ void finish(const Params& p, int nb) {
+        if (!valid) return;
+        const long long o = static_cast<long long>(row) * p.part_ld + nb;
+        p.part[o] = make_float2(m, s);
+        p.sx[o] = sxs;
+        if (has_t && p.zy) p.zy[row] = zt;
+    }
+};
+
+// ---------------------------------------------------------------------------
 // Recompute pass (Sec. 3.1 step 2): e = s (exp(z - lse) - [col == y]) rounded
 // to bf16 into the error matrix E [M, N]; two 32-column chunks fill one
 // 64-column bf16 staging row before each TMA store.
@@ -154,6 +244,68 @@ struct EpiStoreF32 {
 #pragma unroll
         for (int j = 0; j < 32; ++j) w[j] = __float_as_uint(v[j]);
         out_stage_row(buf, io.lane, w);
+        out_commit(io, &p.Cmap, buf, col0, io.row0);
+    }
+
+    __device__ __forceinline__ void finish(const Params&, int) {}
+};
+
+// ---------------------------------------------------------------------------
+// Projection of the direct algorithm: with acc = P W_U (target column of P
+// zero), the unnormalised error signal of token t is
+//   g_t = alpha_t acc_t + beta_t W_U[y_t],   alpha_t = s exp(c_t - lse_t),
+//   beta_t = -alpha_t S'_t,
+// which is s (softmax(z_t) - 1_{y_t}) W_U written with the anchor c_t.  A row
+// with alpha_t == 0 is written as zeros (rows the fixup kernel recomputes, or
+// s == 0); beta_t == 0 skips the read of the target's W_U row.
+struct EpiProjDirect {
+    struct Params {
+        CUtensorMap Cmap;  // fp32 g [M, N], box 32 x 32
+        const float* alpha;
+        const float* beta;
+        const int* y;
+        const __nv_bfloat16* W_U;  // [V, N]
+        int M, N;
+    };
+    float a, b;
+    const __nv_bfloat16* wy;
+
+    __device__ __forceinline__ EpiProjDirect(const Params& p, int, int row, int) {
+        const bool valid = row < p.M;
+        a = valid ? __ldg(p.alpha + row) : 0.f;
+        b = valid ? __ldg(p.beta + row) : 0.f;
+        wy = (a != 0.f && b != 0.f) ? p.W_U + static_cast<long long>(__ldg(p.y + row)) * p.N
+                                    : nullptr;
+    }
+
+    __device__ __forceinline__ void chunk(const Params& p, const float (&v)[32], int col0, int,
+                                          EpiIO& io) {
+        if (col0 >= p.N || io.row0 >= p.M) return;
+        const int lim = p.N - col0;  // a multiple of 8: N % 8 == 0 and col0 % 32 == 0
+        uint32_t o[32];
+        if (a == 0.f) {
+#pragma unroll
+            for (int j = 0; j < 32; ++j) o[j] = 0u;
+        } else if (wy) {
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                uint4 u = make_uint4(0, 0, 0, 0);
+                if (q * 8 < lim) u = __ldg(reinterpret_cast<const uint4*>(wy + col0) + q);
+                const uint32_t h[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    const int j = 8 * q + 2 * k;
+                    o[j] = __float_as_uint(fmaf(a, v[j], b * __uint_as_float(h[k] << 16)));
+                    o[j + 1] =
+                        __float_as_uint(fmaf(a, v[j + 1], b * __uint_as_float(h[k] & 0xffff0000u)));
+                }
+            }
+        } else {
+#pragma unroll
+            for (int j = 0; j < 32; ++j) o[j] = __float_as_uint(a * v[j]);
+        }
+        const uint32_t buf = out_acquire(io);
+        out_stage_row(buf, io.lane, o);
         out_commit(io, &p.Cmap, buf, col0, io.row0);
     }
 

@@ -73,13 +73,20 @@ int32_t cuda_status(cudaError_t e) { return e == cudaSuccess ? FPO_OK : FPO_ERR_
 
 // ------------------------------------------------------------------ error signal
 struct EsLayout {
-    size_t yhat, rho, lse, zy, ce, part, g, E, z, total;
+    size_t yhat, rho, lse, zy, ce, part, g, E, z, anchor, sx, alpha, beta, fix, fix_count, total;
     int n_tiles;
     int64_t Tc;
-    bool stored;  // FPO_ES_STORED_LOGITS
+    int algo;  // the algorithm that runs: FPO_ES_RECOMPUTE, _STORED_LOGITS or _DIRECT
 };
 
-bool es_stored(const fpo_error_signal_desc* d) { return d->algo != FPO_ES_RECOMPUTE; }
+// The algorithm a descriptor selects: AUTO is the direct algorithm for bf16; the
+// fp32 path has no direct form and runs the stored-logits algorithm for it.
+int es_algo(const fpo_error_signal_desc* d) {
+    if (d->algo == FPO_ES_RECOMPUTE) return FPO_ES_RECOMPUTE;
+    if (d->dtype == FPO_BF16 && (d->algo == FPO_ES_AUTO || d->algo == FPO_ES_DIRECT))
+        return FPO_ES_DIRECT;
+    return FPO_ES_STORED_LOGITS;
+}
 
 int32_t es_check_desc(const fpo_error_signal_desc* d) {
     if (!d) return FPO_ERR_NULL;
@@ -88,7 +95,8 @@ int32_t es_check_desc(const fpo_error_signal_desc* d) {
     if (d->T > INT_MAX || d->d > INT_MAX || d->V > INT_MAX) return FPO_ERR_SHAPE;
     if (d->dtype == FPO_BF16 && (d->d % 8 != 0 || d->V % 8 != 0)) return FPO_ERR_SHAPE;
     if (!(d->eps >= 0.f) || !(d->min_rms >= 0.f)) return FPO_ERR_ARG;
-    if (d->algo != FPO_ES_AUTO && d->algo != FPO_ES_RECOMPUTE && d->algo != FPO_ES_STORED_LOGITS)
+    if (d->algo != FPO_ES_AUTO && d->algo != FPO_ES_RECOMPUTE && d->algo != FPO_ES_STORED_LOGITS &&
+        d->algo != FPO_ES_DIRECT)
         return FPO_ERR_ARG;
     return FPO_OK;
 }
@@ -110,8 +118,16 @@ EsLayout es_layout(const fpo_error_signal_desc* d) {
     L.part = off; off = align_up(off + T * static_cast<size_t>(L.n_tiles) * 8);
     L.g = off;    off = align_up(off + T * D * 4);
     L.E = off;    off = align_up(off + static_cast<size_t>(L.Tc) * V * esz);
-    L.stored = es_stored(d);
-    L.z = off;    off = align_up(off + (L.stored ? static_cast<size_t>(L.Tc) * V * 4 : 0));
+    L.algo = es_algo(d);
+    const bool stored = L.algo == FPO_ES_STORED_LOGITS, direct = L.algo == FPO_ES_DIRECT;
+    L.z = off;    off = align_up(off + (stored ? static_cast<size_t>(L.Tc) * V * 4 : 0));
+    const size_t Tdir = direct ? T : 0, Tcdir = direct ? static_cast<size_t>(L.Tc) : 0;
+    L.anchor = off;    off = align_up(off + Tdir * 4);
+    L.sx = off;        off = align_up(off + Tdir * static_cast<size_t>(L.n_tiles) * 4);
+    L.alpha = off;     off = align_up(off + Tdir * 4);
+    L.beta = off;      off = align_up(off + Tdir * 4);
+    L.fix = off;       off = align_up(off + Tcdir * 4);
+    L.fix_count = off; off = align_up(off + (direct ? 4 : 0));
     L.total = off;
     return L;
 }
@@ -189,12 +205,47 @@ int32_t fpo_error_signal(const fpo_error_signal_desc* desc, const void* h, const
         if (!desc->stage_events || !desc->stage_events[i]) return cudaSuccess;
         return cudaEventRecord(static_cast<cudaEvent_t>(desc->stage_events[i]), st);
     };
+    const bool direct = L.algo == FPO_ES_DIRECT;
+    float* anchor = reinterpret_cast<float*>(ws + L.anchor);
     FPO_TRY(mark(0));
-    // 1. final RMSNorm forward: rho, yhat (and the target-range check)
+    // 1. final RMSNorm forward: rho, yhat (and the target-range check; the anchor
+    //    c_t = <yhat_t, W_U[y_t]> for the direct algorithm)
     FPO_TRY(launch_rmsnorm_fwd(desc->dtype, h, norm_w, T, d, desc->eps, yhat, rho, targets, V,
-                               status, st));
+                               status, st, direct ? W_U : nullptr, direct ? anchor : nullptr));
     FPO_TRY(mark(1));
-    if (!L.stored) {
+    if (direct) {
+        // 2.-4. per token chunk: logits pass writing P = exp(z - c) -> lse and row
+        //       factors -> fixup of rows outside the anchor window -> g = alpha P W_U + beta W_U[y]
+        float* sx = reinterpret_cast<float*>(ws + L.sx);
+        float* alpha = reinterpret_cast<float*>(ws + L.alpha);
+        float* beta = reinterpret_cast<float*>(ws + L.beta);
+        int* fix = reinterpret_cast<int*>(ws + L.fix);
+        int* fix_count = reinterpret_cast<int*>(ws + L.fix_count);
+        float* zyd = reinterpret_cast<float*>(ws + L.zy);
+        for (int64_t c0 = 0; c0 < T; c0 += L.Tc) {
+            const int tc = static_cast<int>(L.Tc < T - c0 ? L.Tc : T - c0);
+            const bool last = c0 + tc >= T;
+            const void* yh = static_cast<const uint8_t*>(yhat) + static_cast<size_t>(c0) * d * esz;
+            float2* pc = part + static_cast<size_t>(c0) * L.n_tiles;
+            float* sxc = sx + static_cast<size_t>(c0) * L.n_tiles;
+            float* cec = ce ? ce + c0 : nullptr;
+            FPO_TRY(cudaMemsetAsync(fix_count, 0, sizeof(int), st));
+            FPO_TRY(launch_lse_prob_bf16(yh, W_U, targets + c0, anchor + c0, tc, d, V, pc, sxc,
+                                         L.n_tiles, zyd + c0, E, status, st));
+            if (last) FPO_TRY(mark(2));
+            FPO_TRY(launch_direct_combine(pc, sxc, L.n_tiles, tc, V, targets + c0, anchor + c0,
+                                          zyd + c0, desc->loss_scale, lse + c0, cec, alpha + c0,
+                                          beta + c0, fix, fix_count, st));
+            if (last && loss_out) FPO_TRY(launch_mean(ce, T, loss_out, st));
+            if (last) FPO_TRY(mark(3));
+            FPO_TRY(launch_direct_fixup(yh, W_U, targets + c0, lse + c0, fix, fix_count, d, V,
+                                        L.n_tiles, desc->loss_scale, E, sxc, alpha + c0, beta + c0,
+                                        st));
+            if (last) FPO_TRY(mark(4));
+            FPO_TRY(launch_proj_direct_bf16(E, W_U, targets + c0, alpha + c0, beta + c0, tc, d, V,
+                                            g + c0 * d, status, st));
+        }
+    } else if (L.algo == FPO_ES_RECOMPUTE) {
         // 2. logits pass over all tokens: per-vocabulary-tile (max, sum exp) partials -> lse
         if (bf16)
             FPO_TRY(launch_lse_partial_bf16(yhat, W_U, targets, T, d, V, part, L.n_tiles, zy,
@@ -527,6 +578,19 @@ int32_t fpo_testing_set_gemm_variant(int32_t variant) {
 }
 
 void fpo_testing_set_band(int32_t band) { set_band_override(band); }
+
+int64_t fpo_testing_direct_fixup_rows(const fpo_error_signal_desc* desc, const void* workspace,
+                                      void* stream) {
+    if (es_check_desc(desc) != FPO_OK || !workspace || desc->T == 0) return -1;
+    const EsLayout L = es_layout(desc);
+    if (L.algo != FPO_ES_DIRECT) return -1;
+    if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return -1;
+    int n = 0;
+    if (cudaMemcpy(&n, static_cast<const uint8_t*>(workspace) + L.fix_count, sizeof n,
+                   cudaMemcpyDeviceToHost) != cudaSuccess)
+        return -1;
+    return n;
+}
 
 int32_t fpo_testing_wait_timeout(uint64_t limit_ns, void* workspace, size_t workspace_bytes,
                                  void* stream) {

@@ -2,7 +2,9 @@
 //
 //   logits pass      z = yhat W_U^T      M=T  N=V    K=d   A K-major, B K-major
 //   recompute pass   same GEMM, epilogue writes E = s (softmax - onehot)
+//   direct logits    same GEMM, epilogue writes P = exp(z - c) (target zero)
 //   projection       g = E W_U           M=T  N=d    K=V   A K-major, B MN-major
+//                    (or g = alpha P W_U + beta W_U[y] in the direct algorithm)
 //   update           G = g~^T A_l        M=d  N=d_ff K=T   A MN-major, B MN-major
 //
 // Tensor maps are encoded per call (a few microseconds of host work) through
@@ -149,13 +151,14 @@ std::atomic<int> g_band_override{0};  // > 0: rasterisation band height (tests /
 
 bool use_pair() { return g_gemm_variant.load(std::memory_order_relaxed) == 1; }
 
-// Rasterisation band in tile rows: a band spans kBandRows output rows (16 single-CTA
-// tiles, 8 pair tiles), unless overridden.
-constexpr int kBandRows = 2048;
-int band_for(bool pair) {
+// Rasterisation band in tile rows, unless overridden: 16 tile rows, i.e. 2048
+// output rows of single-CTA tiles and 4096 of pair tiles.  With pair tiles the
+// 4096-row band gave the lowest DRAM traffic of the three GEMMs of the OLMo-2-7B
+// shape (band heights 2 to 32 measured).
+constexpr int kBandTiles = 16;
+int band_for(bool) {
     const int o = g_band_override.load(std::memory_order_relaxed);
-    if (o > 0) return o;
-    return kBandRows / (pair ? kPairBM : kBM);
+    return o > 0 ? o : kBandTiles;
 }
 
 }  // namespace
@@ -228,8 +231,55 @@ cudaError_t launch_error_bf16(const void* yhat, const void* W_U, const int32_t* 
     return run_gemm<kLseBN, false, false, kLseStages, 1, EpiError>(maps, ep, sh, status, st);
 }
 
+cudaError_t launch_lse_prob_bf16(const void* yhat, const void* W_U, const int32_t* y,
+                                 const float* anchor, int T, int d, int V, float2* part, float* sx,
+                                 int part_ld, float* zy, void* P, unsigned* status,
+                                 cudaStream_t st) {
+    const bool pair = use_pair();
+    GemmMaps<1> maps;
+    if (!map_kmajor(&maps.a[0], yhat, T, d, kBM) ||
+        !map_kmajor(&maps.b[0], W_U, V, d, pair ? kLseBN / 2 : kLseBN))
+        return cudaErrorInvalidValue;
+    EpiLseProb::Params ep;
+    if (!map_out_bf16(&ep.pmap, P, T, V)) return cudaErrorInvalidValue;
+    ep.part = part;
+    ep.sx = sx;
+    ep.part_ld = part_ld;
+    ep.zy = zy;
+    ep.y = y;
+    ep.anchor = anchor;
+    ep.M = T;
+    ep.N = V;
+    const GemmShape sh = make_shape(T, V, d, kLseBN, 1, band_for(pair), pair ? kPairBM : kBM);
+    if (pair)
+        return run_gemm_pair<kLseBN, false, false, kPairStages, 1, EpiLseProb>(maps, ep, sh, status,
+                                                                               st);
+    return run_gemm<kLseBN, false, false, kLseStages, 1, EpiLseProb>(maps, ep, sh, status, st);
+}
+
 constexpr int kProjBN = 256;
 constexpr int kProjStages = 4;
+
+cudaError_t launch_proj_direct_bf16(const void* P, const void* W_U, const int32_t* y,
+                                    const float* alpha, const float* beta, int Tc, int d, int V,
+                                    float* g, unsigned* status, cudaStream_t st) {
+    GemmMaps<1> maps;
+    if (!map_kmajor(&maps.a[0], P, Tc, V, kBM) || !map_mnmajor(&maps.b[0], W_U, V, d))
+        return cudaErrorInvalidValue;
+    EpiProjDirect::Params ep;
+    if (!map_out_f32(&ep.Cmap, g, Tc, d)) return cudaErrorInvalidValue;
+    ep.alpha = alpha;
+    ep.beta = beta;
+    ep.y = y;
+    ep.W_U = static_cast<const __nv_bfloat16*>(W_U);
+    ep.M = Tc;
+    ep.N = d;
+    if (use_pair())
+        return run_gemm_pair<kProjBN, false, true, kPairStages, 1, EpiProjDirect>(
+            maps, ep, make_shape(Tc, d, V, kProjBN, 1, band_for(true), kPairBM), status, st);
+    return run_gemm<kProjBN, false, true, kProjStages, 1, EpiProjDirect>(
+        maps, ep, make_shape(Tc, d, V, kProjBN, 1, band_for(false)), status, st);
+}
 
 cudaError_t launch_proj_bf16(const void* E, const void* W_U, int Tc, int d, int V, float* g,
                              unsigned* status, cudaStream_t st) {

@@ -40,6 +40,18 @@ cudaError_t launch_error_bf16(const void* yhat, const void* W_U, const int32_t* 
 cudaError_t launch_proj_bf16(const void* E, const void* W_U, int Tc, int d, int V, float* g,
                              unsigned* status, cudaStream_t st);
 
+// Direct algorithm, logits pass: as launch_lse_partial_bf16 (z never stored), plus
+// P[T, V] = exp(z - anchor) in bf16 with the target column zero, and sx[T, part_ld]
+// the per-tile sums of the rounded P.
+cudaError_t launch_lse_prob_bf16(const void* yhat, const void* W_U, const int32_t* y,
+                                 const float* anchor, int T, int d, int V, float2* part, float* sx,
+                                 int part_ld, float* zy, void* P, unsigned* status,
+                                 cudaStream_t st);
+// Direct algorithm, projection: g[Tc, d] = alpha (.) (P W_U) + beta (.) W_U[y] (row-wise).
+cudaError_t launch_proj_direct_bf16(const void* P, const void* W_U, const int32_t* y,
+                                    const float* alpha, const float* beta, int Tc, int d, int V,
+                                    float* g, unsigned* status, cudaStream_t st);
+
 // Grouped pseudogradient update over n layers, layer l with signal g[l] (host array).
 cudaError_t launch_update_bf16(int n, int T, int d, int d_ff, const void* const* g,
                                const void* const* A, float lr, float* const* W_master,
@@ -85,9 +97,22 @@ cudaError_t launch_test_gemm_bf16(int M, int N, int K, bool a_mn, bool b_mn, con
                                   const void* B, float* C, unsigned* status, cudaStream_t st);
 
 // ------------------------------------------------------------ row-wise kernels
+// With anchor non-null (direct algorithm) also anchor[t] = <yhat_t, W_U[y_t]>.
 cudaError_t launch_rmsnorm_fwd(int dtype, const void* h, const void* w, int T, int d, float eps,
                                void* yhat, float* rho, const int32_t* y, int V, unsigned* status,
-                               cudaStream_t st);
+                               cudaStream_t st, const void* W_U = nullptr,
+                               float* anchor = nullptr);
+// Direct algorithm (bf16): lse, ce, the projection's row factors alpha, beta, and the
+// rows outside the anchor window (fix[0 .. *fix_count), appended atomically).
+cudaError_t launch_direct_combine(const float2* part, const float* sx, int n_tiles, int T, int V,
+                                  const int32_t* y, const float* anchor, const float* zy, float s,
+                                  float* lse, float* ce, float* alpha, float* beta, int* fix,
+                                  int* fix_count, cudaStream_t st);
+// Recompute the P rows, sx partials and row factors of the listed rows, anchored at lse.
+cudaError_t launch_direct_fixup(const void* yhat, const void* W_U, const int32_t* y,
+                                const float* lse, const int* fix, const int* fix_count, int d,
+                                int V, int n_tiles, float s, void* P, float* sx, float* alpha,
+                                float* beta, cudaStream_t st);
 cudaError_t launch_lse_combine(const float2* part, int n_tiles, int T, const float* zy,
                                float* lse, float* ce, cudaStream_t st);
 cudaError_t launch_mean(const float* x, int n, float* out, cudaStream_t st);

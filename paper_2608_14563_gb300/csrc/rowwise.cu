@@ -2,8 +2,12 @@
 //
 //   rmsnorm_fwd   rho_t = sqrt(mean_j h_tj^2 + eps), yhat_t = w (.) h_t / rho_t
 //                 (the final RMSNorm forward of App. E), plus the target-range
-//                 check of every token
+//                 check of every token and, for the direct algorithm, the
+//                 anchor c_t = <yhat_t, W_U[y_t]> (the target logit)
 //   lse_combine   lse_t from the per-vocabulary-tile (max, sum exp) partials
+//   direct_combine  the same, plus the direct algorithm's row factors
+//                 alpha_t, beta_t and the list of rows outside the anchor window
+//   direct_fixup  recomputes the P rows of those rows, anchored at lse_t
 //   mean          mean of a vector in a fixed order (the mean cross-entropy)
 //   rmsnorm_vjp   App. E Eq. (rmsnorm-vjp) with the min-RMS clamp:
 //                 g~ = (w (.) g - xhat <xhat, w (.) g> / d) / max(rho, rho_min)
@@ -83,17 +87,31 @@ __device__ __forceinline__ void st_vec(__nv_bfloat16* p, const float (&v)[VEC]) 
     *reinterpret_cast<uint4*>(p) = a;
 }
 
+// x rounded to the storage type TT and back.
+template <typename TT>
+__device__ __forceinline__ float round_to(float x) {
+    if constexpr (sizeof(TT) == 2)
+        return __bfloat162float(__float2bfloat16_rn(x));
+    else
+        return x;
+}
+
 constexpr int kRowThreads = 256;  // 8 warps, one row each
 
 template <typename TT, int VEC>
 __global__ void __launch_bounds__(kRowThreads)
     rmsnorm_fwd_kernel(const TT* __restrict__ h, const TT* __restrict__ w, int T, int d, float eps,
                        TT* __restrict__ yhat, float* __restrict__ rho, const int32_t* __restrict__ y,
-                       int V, unsigned* status) {
+                       int V, unsigned* status, const TT* __restrict__ W_U,
+                       float* __restrict__ anchor) {
     const int lane = threadIdx.x & 31;
     const int wpb = blockDim.x >> 5;
     for (int row = blockIdx.x * wpb + (threadIdx.x >> 5); row < T; row += gridDim.x * wpb) {
         const TT* hr = h + static_cast<size_t>(row) * d;
+        const int t = y[row];
+        const bool t_ok = t >= 0 && t < V;
+        // the target's unembedding row, read only for an in-range target
+        const TT* ur = (anchor && t_ok) ? W_U + static_cast<size_t>(t) * d : nullptr;
         float ss = 0.f;
         for (int j = lane * VEC; j < d; j += 32 * VEC) {
             float x[VEC];
@@ -105,6 +123,7 @@ __global__ void __launch_bounds__(kRowThreads)
         const float r = sqrtf(ss / static_cast<float>(d) + eps);
         const float inv = 1.0f / r;
         TT* yr = yhat + static_cast<size_t>(row) * d;
+        float zt = 0.f;
         for (int j = lane * VEC; j < d; j += 32 * VEC) {
             float x[VEC], wv[VEC], o[VEC];
             ld_vec<VEC>(hr + j, x);
@@ -112,11 +131,18 @@ __global__ void __launch_bounds__(kRowThreads)
 #pragma unroll
             for (int k = 0; k < VEC; ++k) o[k] = wv[k] * (x[k] * inv);
             st_vec<VEC>(yr + j, o);
+            if (ur) {
+                float u[VEC];
+                ld_vec<VEC>(ur + j, u);
+#pragma unroll
+                for (int k = 0; k < VEC; ++k) zt = fmaf(round_to<TT>(o[k]), u[k], zt);
+            }
         }
+        if (anchor) zt = warp_sum(zt);
         if (lane == 0) {
             rho[row] = r;
-            const int t = y[row];
-            if (t < 0 || t >= V) atomicOr(status, kDevTargetRange);
+            if (!t_ok) atomicOr(status, kDevTargetRange);
+            if (anchor) anchor[row] = zt;
         }
     }
 }
@@ -225,6 +251,137 @@ __global__ void __launch_bounds__(kRowThreads)
     }
 }
 
+// Direct algorithm, per token: lse_t and ce_t as lse_combine, S'_t = sum of the
+// tiles' rounded p~ (fixed order), and the row factors of the projection
+//   alpha_t = s exp(c_t - lse_t),  beta_t = -alpha_t S'_t.
+// The anchor window: with c_t the target logit, p~ = exp(z - c_t) holds every
+// probability that matters as a normal bf16 number, and the projection's fp32
+// sums stay finite, while 2^-80 <= S'_t <= 2^80.  A row outside it (or with a
+// non-finite S'_t) gets alpha_t = beta_t = 0 here and is appended to `fix` for
+// direct_fixup; a row with an out-of-range target gets zeros and no fixup.
+constexpr float kWindowHi = 1.2089258196146292e24f;   // 2^80
+constexpr float kWindowLo = 8.271806125530277e-25f;  // 2^-80
+
+__global__ void __launch_bounds__(kRowThreads)
+    direct_combine_kernel(const float2* __restrict__ part, const float* __restrict__ sx,
+                          int n_tiles, int T, int V, const int32_t* __restrict__ y,
+                          const float* __restrict__ anchor, const float* __restrict__ zy, float s,
+                          float* __restrict__ lse, float* __restrict__ ce,
+                          float* __restrict__ alpha, float* __restrict__ beta,
+                          int* __restrict__ fix, int* __restrict__ fix_count) {
+    const int lane = threadIdx.x & 31;
+    const int wpb = blockDim.x >> 5;
+    for (int row = blockIdx.x * wpb + (threadIdx.x >> 5); row < T; row += gridDim.x * wpb) {
+        const float2* pr = part + static_cast<size_t>(row) * n_tiles;
+        const float* xr = sx + static_cast<size_t>(row) * n_tiles;
+        float m = -INFINITY;
+        for (int i = lane; i < n_tiles; i += 32) m = fmaxf(m, pr[i].x);
+        m = warp_max(m);
+        float e = 0.f, S = 0.f;
+        for (int i = lane; i < n_tiles; i += 32) {
+            const float2 p = pr[i];
+            if (p.y > 0.f) e += p.y * expf(p.x - m);
+            S += xr[i];
+        }
+        e = warp_sum(e);
+        S = warp_sum(S);
+        const float l = m + logf(e);
+        if (lane == 0) {
+            lse[row] = l;
+            if (ce) ce[row] = l - zy[row];
+            const int t = y[row];
+            float a = 0.f, b = 0.f;
+            if (t >= 0 && t < V) {
+                const bool inside = S <= kWindowHi && (S >= kWindowLo || V == 1);
+                if (inside) {
+                    a = s * expf(anchor[row] - l);
+                    b = -a * S;
+                } else {
+                    fix[atomicAdd(fix_count, 1)] = row;
+                }
+            }
+            alpha[row] = a;
+            beta[row] = b;
+        }
+    }
+}
+
+// Rows outside the anchor window, one (row, vocabulary tile) per work item:
+// z_tj = <yhat_t, W_U[j]> in fp32 (one warp per column), then the tile of P is
+// rewritten as p_tj = exp(z_tj - lse_t) in bf16 (target zero) and sx[t, tile]
+// as the sum of the rounded values.  The row count is read on the device, so
+// the launch is the same whether or not any row needs it.
+constexpr int kFixTile = 256;  // vocabulary columns per work item (the logits tile width)
+
+template <int VEC>
+__global__ void __launch_bounds__(kRowThreads)
+    direct_fixup_kernel(const __nv_bfloat16* __restrict__ yhat,
+                        const __nv_bfloat16* __restrict__ W_U, const int32_t* __restrict__ y,
+                        const float* __restrict__ lse, const int* __restrict__ fix,
+                        const int* __restrict__ fix_count, int d, int V, int n_tiles,
+                        __nv_bfloat16* __restrict__ P, float* __restrict__ sx) {
+    __shared__ float part_sum[kRowThreads / 32];
+    const int lane = threadIdx.x & 31;
+    const int warp = threadIdx.x >> 5;
+    const long long items = static_cast<long long>(*fix_count) * n_tiles;
+    for (long long it = blockIdx.x; it < items; it += gridDim.x) {
+        const int row = fix[it / n_tiles];
+        const int tile = static_cast<int>(it % n_tiles);
+        const int t = y[row];
+        const float l = lse[row];
+        const __nv_bfloat16* xr = yhat + static_cast<size_t>(row) * d;
+        float acc = 0.f;
+        for (int c = warp; c < kFixTile; c += kRowThreads / 32) {
+            const int j = tile * kFixTile + c;
+            if (j >= V) break;
+            const __nv_bfloat16* ur = W_U + static_cast<size_t>(j) * d;
+            float z = 0.f;
+            for (int k = lane * VEC; k < d; k += 32 * VEC) {
+                float a[VEC], b[VEC];
+                ld_vec<VEC>(xr + k, a);
+                ld_vec<VEC>(ur + k, b);
+#pragma unroll
+                for (int q = 0; q < VEC; ++q) z = fmaf(a[q], b[q], z);
+            }
+            z = warp_sum(z);
+            if (lane == 0) {
+                const __nv_bfloat16 p = __float2bfloat16_rn(j == t ? 0.f : expf(z - l));
+                P[static_cast<size_t>(row) * V + j] = p;
+                acc += __bfloat162float(p);
+            }
+        }
+        if (lane == 0) part_sum[warp] = acc;
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            float S = 0.f;
+            for (int i = 0; i < kRowThreads / 32; ++i) S += part_sum[i];
+            sx[static_cast<size_t>(row) * n_tiles + tile] = S;
+        }
+        __syncthreads();
+    }
+}
+
+// Row factors of the fixed rows (anchored at lse: alpha = s, beta = -s S').
+__global__ void __launch_bounds__(kRowThreads)
+    direct_fixup_factors_kernel(const float* __restrict__ sx, const int* __restrict__ fix,
+                                const int* __restrict__ fix_count, int n_tiles, float s,
+                                float* __restrict__ alpha, float* __restrict__ beta) {
+    const int lane = threadIdx.x & 31;
+    const int wpb = blockDim.x >> 5;
+    const int n = *fix_count;
+    for (int i = blockIdx.x * wpb + (threadIdx.x >> 5); i < n; i += gridDim.x * wpb) {
+        const int row = fix[i];
+        const float* xr = sx + static_cast<size_t>(row) * n_tiles;
+        float S = 0.f;
+        for (int k = lane; k < n_tiles; k += 32) S += xr[k];
+        S = warp_sum(S);
+        if (lane == 0) {
+            alpha[row] = s;
+            beta[row] = -s * S;
+        }
+    }
+}
+
 constexpr int kMeanThreads = 1024;
 
 __global__ void __launch_bounds__(kMeanThreads) mean_kernel(const float* __restrict__ x, int n,
@@ -329,22 +486,49 @@ int row_grid(int T) {
 
 cudaError_t launch_rmsnorm_fwd(int dtype, const void* h, const void* w, int T, int d, float eps,
                                void* yhat, float* rho, const int32_t* y, int V, unsigned* status,
-                               cudaStream_t st) {
+                               cudaStream_t st, const void* W_U, float* anchor) {
     if (T <= 0) return cudaSuccess;
     const int grid = row_grid(T);
     if (dtype == 1) {
         rmsnorm_fwd_kernel<__nv_bfloat16, 8><<<grid, kRowThreads, 0, st>>>(
             static_cast<const __nv_bfloat16*>(h), static_cast<const __nv_bfloat16*>(w), T, d, eps,
-            static_cast<__nv_bfloat16*>(yhat), rho, y, V, status);
+            static_cast<__nv_bfloat16*>(yhat), rho, y, V, status,
+            static_cast<const __nv_bfloat16*>(W_U), anchor);
     } else if (d % 4 == 0) {
         rmsnorm_fwd_kernel<float, 4><<<grid, kRowThreads, 0, st>>>(
             static_cast<const float*>(h), static_cast<const float*>(w), T, d, eps,
-            static_cast<float*>(yhat), rho, y, V, status);
+            static_cast<float*>(yhat), rho, y, V, status, static_cast<const float*>(W_U), anchor);
     } else {
         rmsnorm_fwd_kernel<float, 1><<<grid, kRowThreads, 0, st>>>(
             static_cast<const float*>(h), static_cast<const float*>(w), T, d, eps,
-            static_cast<float*>(yhat), rho, y, V, status);
+            static_cast<float*>(yhat), rho, y, V, status, static_cast<const float*>(W_U), anchor);
     }
+    return cudaGetLastError();
+}
+
+cudaError_t launch_direct_combine(const float2* part, const float* sx, int n_tiles, int T, int V,
+                                  const int32_t* y, const float* anchor, const float* zy, float s,
+                                  float* lse, float* ce, float* alpha, float* beta, int* fix,
+                                  int* fix_count, cudaStream_t st) {
+    if (T <= 0) return cudaSuccess;
+    direct_combine_kernel<<<row_grid(T), kRowThreads, 0, st>>>(
+        part, sx, n_tiles, T, V, y, anchor, zy, s, lse, ce, alpha, beta, fix, fix_count);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_direct_fixup(const void* yhat, const void* W_U, const int32_t* y,
+                                const float* lse, const int* fix, const int* fix_count, int d,
+                                int V, int n_tiles, float s, void* P, float* sx, float* alpha,
+                                float* beta, cudaStream_t st) {
+    DevInfo di;
+    const int sms = current_device_info(&di) ? di.sm_count : 148;
+    direct_fixup_kernel<8><<<sms * 4, kRowThreads, 0, st>>>(
+        static_cast<const __nv_bfloat16*>(yhat), static_cast<const __nv_bfloat16*>(W_U), y, lse,
+        fix, fix_count, d, V, n_tiles, static_cast<__nv_bfloat16*>(P), sx);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    direct_fixup_factors_kernel<<<sms, kRowThreads, 0, st>>>(sx, fix, fix_count, n_tiles, s, alpha,
+                                                            beta);
     return cudaGetLastError();
 }
 

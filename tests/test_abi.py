@@ -9,11 +9,12 @@ import pytest
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 HEADER = os.path.join(ROOT, "include", "fpo.h")
+TESTING_HEADER = os.path.join(ROOT, "include", "fpo_testing.h")
 LIB = os.path.join(ROOT, "paper_2608_14563_gb300", "libfpo.so")
 
 
-def declared_functions():
-    text = open(HEADER).read()
+def declared_functions(header=HEADER):
+    text = open(header).read()
     text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
     return sorted(set(re.findall(r"\b(fpo_[a-z0-9_]+)\s*\(", text)))
 
@@ -31,10 +32,12 @@ def test_library_exports_every_declared_symbol():
     out = subprocess.run(["nm", "-D", "--defined-only", LIB], capture_output=True, text=True,
                          check=True).stdout
     exported = set(re.findall(r"\sT\s+(fpo_\w+)$", out, flags=re.M))
-    missing = [n for n in declared_functions() if n not in exported]
+    names = declared_functions() + declared_functions(TESTING_HEADER)
+    assert "fpo_testing_direct_fixup_rows" in names
+    missing = [n for n in names if n not in exported]
     assert not missing, missing
     lib = ctypes.CDLL(LIB)
-    for n in declared_functions():
+    for n in names:
         assert hasattr(lib, n)
 
 
@@ -62,12 +65,19 @@ def test_error_signal_workspace_query(L):
     fpo = L.fpo
     small = fpo.error_signal_desc(128, 64, 512, fpo.F32)
     assert fpo.error_signal_workspace(small) > 0
-    # recompute: the E chunk is Tc x V bf16; stored logits add Tc x V fp32 of logits
-    for algo, per in ((fpo.ES_RECOMPUTE, 2), (fpo.ES_STORED_LOGITS, 6), (fpo.ES_AUTO, 6)):
-        chunked = fpo.error_signal_desc(4096, 4096, 151936, fpo.BF16, t_chunk=1024, algo=algo)
-        full = fpo.error_signal_desc(4096, 4096, 151936, fpo.BF16, algo=algo)
+    # per token of the chunk: recompute holds a bf16 row of E; stored logits add an fp32
+    # row of logits; direct (the bf16 default) holds a bf16 row of P and one fixup-list entry
+    V = 151936
+    for algo, per in ((fpo.ES_RECOMPUTE, 2 * V), (fpo.ES_STORED_LOGITS, 6 * V),
+                      (fpo.ES_DIRECT, 2 * V + 4), (fpo.ES_AUTO, 2 * V + 4)):
+        chunked = fpo.error_signal_desc(4096, 4096, V, fpo.BF16, t_chunk=1024, algo=algo)
+        full = fpo.error_signal_desc(4096, 4096, V, fpo.BF16, algo=algo)
         diff = fpo.error_signal_workspace(full) - fpo.error_signal_workspace(chunked)
-        assert abs(diff - 3072 * 151936 * per) < 1024
+        assert abs(diff - 3072 * per) < 1024
+    # fp32 has no direct form: AUTO and DIRECT take the stored-logits layout
+    f32 = [fpo.error_signal_workspace(fpo.error_signal_desc(512, 64, 1000, fpo.F32, algo=a))
+           for a in (fpo.ES_AUTO, fpo.ES_DIRECT, fpo.ES_STORED_LOGITS)]
+    assert f32[0] == f32[1] == f32[2]
     assert fpo.error_signal_workspace(fpo.error_signal_desc(64, 64, 256, fpo.BF16, algo=7)) == 0
     bad = fpo.error_signal_desc(16, 12, 512, fpo.BF16)  # d not a multiple of 8
     assert fpo.error_signal_workspace(bad) == 0

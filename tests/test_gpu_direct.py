@@ -1,0 +1,158 @@
+"""The direct error-matrix algorithm (FPO_ES_DIRECT, the bf16 default) against
+the fp64 oracle, including the rows it hands to its fp32 fixup kernel.
+
+The direct algorithm never forms E = s (softmax(z) - 1_y) (Sec. 3.1 step 2):
+with the anchor c_t = z_{t, y_t} it stores p~ = exp(z - c_t) (target column 0)
+and projects g_t = s e^{c_t - lse_t} (p~_t W_U - S'_t W_U[y_t]), S'_t = sum of
+row t of p~.  Rows whose S'_t leaves [2^-80, 2^80] are recomputed, anchored at
+lse_t, before the projection.
+
+The fixup input is built so that every normalised hidden state is exact in bf16
+(h = +-1, eps = 0: rho = 1 and yhat = norm_w (.) h), so the oracle's logits and
+the GPU's differ only by fp32 accumulation, even at logit scales of ~100:
+  * rows 0-49    anti-aligned with W_U[y=0]: cross-entropy ~160 nats (S' overflows)
+  * rows 50-99   aligned with W_U[y=0]: 1 - p_target ~ e^-110 (S' underflows)
+  * rows 100-149 partly aligned, y = 0: confident, 1 - p_target ~ e^-17 (inside)
+  * rows 150-    random signs, random targets (inside)
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from helpers import cos, f64, rel_frob
+from paper_2608_14563_gb300 import synth
+from paper_2608_14563_gb300.synth import Workload
+
+pytestmark = pytest.mark.gpu
+
+TOL = 2e-2
+COS_MIN = 0.9995
+
+RAGGED = Workload("ragged-bf16", T=300, d=520, d_ff=600, V=1000, layers=1, targets="zipf")
+
+
+def run(fpo, h, w, W_U, y, *, eps, algo, t_chunk=0, loss_scale=None):
+    h, w, W_U, y = h.cuda(), w.cuda(), W_U.cuda(), y.cuda()
+    g = torch.empty_like(h)
+    lse = torch.empty(h.shape[0], dtype=torch.float32, device="cuda")
+    loss = torch.empty(1, dtype=torch.float32, device="cuda")
+    ws = fpo.error_signal(h, w, W_U, y, g, eps=eps, min_rms=0.5, loss_scale=loss_scale,
+                          t_chunk=t_chunk, lse_out=lse, loss_out=loss, algo=algo)
+    assert fpo.get_device_status(ws) == fpo.OK
+    fixed = fpo.direct_fixup_rows(h, W_U, ws, t_chunk=t_chunk, algo=algo)
+    return {"g": g, "lse": lse, "loss": loss, "fixed": fixed}
+
+
+def reference(h, w, W_U, y, *, eps, s):
+    return oracle.error_signal(synth.to_numpy_exact(h), synth.to_numpy_exact(w),
+                               synth.to_numpy_exact(W_U), y.numpy(), eps=eps, min_rms=0.5, s=s)
+
+
+@pytest.fixture(scope="module")
+def ragged():
+    inp = synth.make_all(RAGGED)
+    ref = reference(inp["h"], inp["w"], inp["W_U"], inp["y"], eps=RAGGED.eps,
+                    s=RAGGED.loss_scale)
+    return inp, ref
+
+
+def test_direct_matches_oracle(fpo, ragged):
+    inp, ref = ragged
+    out = run(fpo, inp["h"], inp["w"], inp["W_U"], inp["y"], eps=RAGGED.eps, algo=fpo.ES_DIRECT)
+    g = f64(out["g"])
+    assert rel_frob(g, ref["g_tilde"]) < TOL and cos(g, ref["g_tilde"]) >= COS_MIN
+    assert np.max(np.abs(f64(out["lse"]) - ref["lse"])) < 1e-2
+    ce = oracle.mean_ce(ref["lse"], ref["zy"])
+    assert abs(out["loss"].item() - ce) < 1e-3 * ce
+    assert out["fixed"] == 0
+
+
+def test_auto_is_direct_for_bf16(fpo, ragged):
+    inp, _ = ragged
+    a = run(fpo, inp["h"], inp["w"], inp["W_U"], inp["y"], eps=RAGGED.eps, algo=fpo.ES_AUTO)
+    b = run(fpo, inp["h"], inp["w"], inp["W_U"], inp["y"], eps=RAGGED.eps, algo=fpo.ES_DIRECT)
+    assert torch.equal(a["g"], b["g"]) and torch.equal(a["loss"], b["loss"])
+
+
+def test_direct_is_bitwise_identical_across_token_chunks(fpo, ragged):
+    inp, _ = ragged
+    runs = [run(fpo, inp["h"], inp["w"], inp["W_U"], inp["y"], eps=RAGGED.eps,
+                algo=fpo.ES_DIRECT, t_chunk=c) for c in (0, 128, 37)]
+    for r in runs[1:]:
+        assert torch.equal(runs[0]["g"], r["g"])
+        assert torch.equal(runs[0]["lse"], r["lse"])
+        assert torch.equal(runs[0]["loss"], r["loss"])
+
+
+def test_direct_is_bitwise_identical_across_gemm_kernels(fpo, ragged):
+    inp, _ = ragged
+    prev = fpo.set_gemm_variant(0)
+    try:
+        a = run(fpo, inp["h"], inp["w"], inp["W_U"], inp["y"], eps=RAGGED.eps, algo=fpo.ES_DIRECT)
+        fpo.set_gemm_variant(1)
+        b = run(fpo, inp["h"], inp["w"], inp["W_U"], inp["y"], eps=RAGGED.eps, algo=fpo.ES_DIRECT)
+    finally:
+        fpo.set_gemm_variant(prev)
+    assert torch.equal(a["g"], b["g"]) and torch.equal(a["lse"], b["lse"])
+
+
+def test_direct_agrees_with_stored_logits(fpo, ragged):
+    inp, _ = ragged
+    a = run(fpo, inp["h"], inp["w"], inp["W_U"], inp["y"], eps=RAGGED.eps, algo=fpo.ES_DIRECT)
+    b = run(fpo, inp["h"], inp["w"], inp["W_U"], inp["y"], eps=RAGGED.eps,
+            algo=fpo.ES_STORED_LOGITS)
+    assert torch.equal(a["lse"], b["lse"])  # same logits pass partials
+    assert rel_frob(f64(a["g"]), f64(b["g"])) < 1e-2
+
+
+def _window_input():
+    """h = +-1 rows of four kinds (module docstring), W_U x 16 (exact in bf16)."""
+    T, d, V = 300, 520, 1000
+    wl = Workload("window", T=T, d=d, d_ff=8, V=V, layers=1, targets="uniform", eps=0.0)
+    w = synth.make_norm_w(wl)
+    W_U = synth.make_W_U(wl) * 16
+    align = torch.sign(W_U[0].float() * w.float())
+    align[align == 0] = 1.0
+    rnd = torch.sign(synth.normal((T, d), seed=3, tensor="h"))
+    rnd[rnd == 0] = 1.0
+    h = rnd.clone()
+    h[0:50] = -align
+    h[50:100] = align
+    part = torch.arange(d) < int(0.3 * d)
+    h[100:150] = torch.where(part, align, rnd[100:150])
+    y = synth.make_targets(wl)
+    y[0:150] = 0
+    return h.to(torch.bfloat16), w, W_U, y
+
+
+def test_rows_outside_the_anchor_window_are_fixed(fpo):
+    h, w, W_U, y = _window_input()
+    T = h.shape[0]
+    ref = reference(h, w, W_U, y, eps=0.0, s=1.0 / T)
+    ce = ref["lse"] - ref["zy"]
+    # the input is as intended: log2 S'_t from fp64 logits of the exact yhat = w (.) h
+    z = (f64(h) * f64(w)[None, :]) @ f64(W_U).T
+    zy = z[np.arange(T), y.numpy()]
+    zo = z.copy()
+    zo[np.arange(T), y.numpy()] = -np.inf
+    mo = zo.max(axis=1)
+    log2_S = (mo - zy + np.log(np.exp(zo - mo[:, None]).sum(axis=1))) / np.log(2.0)
+    assert np.all(log2_S[0:50] > 100) and np.all(log2_S[50:100] < -100)
+    assert np.all(np.abs(log2_S[100:]) < 70)
+    outs = [run(fpo, h, w, W_U, y, eps=0.0, algo=fpo.ES_DIRECT, t_chunk=c) for c in (0, 64)]
+    assert outs[0]["fixed"] == 100
+    assert torch.equal(outs[0]["g"], outs[1]["g"]) and torch.equal(outs[0]["loss"], outs[1]["loss"])
+    g = f64(outs[0]["g"])
+    G = ref["g_tilde"]
+    for lo, hi in ((0, 50), (100, 150), (150, T)):
+        assert rel_frob(g[lo:hi], G[lo:hi]) < TOL, (lo, hi)
+        assert cos(g[lo:hi], G[lo:hi]) >= COS_MIN, (lo, hi)
+    # confident rows: the error signal itself is ~1e-8 of a typical row and still exact
+    # to bf16 rounding (no 1 - p cancellation), row by row
+    for t in range(100, 150):
+        assert rel_frob(g[t], G[t]) < TOL, t
+    # rows with 1 - p_target ~ e^-110: the signal is below fp32 range
+    assert np.max(np.abs(g[50:100] - G[50:100])) < 1e-30
+    assert np.max(np.abs(f64(outs[0]["lse"]) - ref["lse"]) / np.maximum(1, np.abs(ref["lse"]))) < 1e-5
+    assert abs(outs[0]["loss"].item() - oracle.mean_ce(ref["lse"], ref["zy"])) < 1e-4 * np.mean(ce)
