@@ -276,7 +276,6 @@ def run_fpo(args, wl):
         gu_out = [torch.empty(wl.d_ff, wl.d, dtype=torch.bfloat16, device=dev) for _ in gu_W12]
         gu_sig = [torch.empty(wl.T, wl.d_ff, dtype=torch.bfloat16, device=dev)
                   for _ in range(2 * wl.layers)]
-        gu_act = [x for x in gu_x for _ in range(2)]
         ws_gu = torch.empty(fpo.layer_update_workspace(), dtype=torch.uint8, device=dev)
     if post:  # per-layer MLP outputs, post-FFN norm weights and layer-specific signals
         m_out = [synth.make_mlp_out(wl_r, l, dev) for l in range(wl.layers)]
@@ -318,44 +317,53 @@ def run_fpo(args, wl):
     if args.gate_up:  # one error_h GEMM per layer + one grouped W1/W2 update
         launches_per_step += wl.layers + 1
 
-    def update():
+    # The tensors one step reads that come from the forward pass / the data: the
+    # end-to-end loop below copies them from host memory every step.
+    X0 = {"h": h, "y": y, "A": A, "m": m_out if post else [],
+          "ab": [t for pair in gu_ab for t in pair] if gate_up else [],
+          "x": gu_x if gate_up else []}
+
+    def update(X):
         signals = g_l if post else [g] * wl.layers
         if optimize:
-            fpo.layer_optimize_grouped(signals, A, opt, Wm, W_outs=Wo, states1=st1, states2=st2,
-                                       workspace=ws_up)
+            fpo.layer_optimize_grouped(signals, X["A"], opt, Wm, W_outs=Wo, states1=st1,
+                                       states2=st2, workspace=ws_up)
         elif post:
-            fpo.layer_update_grouped_signals(g_l, A, wl.lr, W_masters=Wm, W_outs=Wo,
+            fpo.layer_update_grouped_signals(g_l, X["A"], wl.lr, W_masters=Wm, W_outs=Wo,
                                              workspace=ws_up)
         else:
-            fpo.layer_update_grouped(g, A, wl.lr, W_masters=Wm, W_outs=Wo, workspace=ws_up)
+            fpo.layer_update_grouped(g, X["A"], wl.lr, W_masters=Wm, W_outs=Wo, workspace=ws_up)
 
-    def gate_up_update():
+    def gate_up_update(X):
         for l in range(wl.layers):
-            fpo.gate_up_signals(g_l[l] if post else g, gu_W3[l], gu_ab[l][0], gu_ab[l][1],
-                                gu_sig[2 * l], gu_sig[2 * l + 1], workspace=ws_gu)
+            fpo.gate_up_signals(g_l[l] if post else g, gu_W3[l], X["ab"][2 * l],
+                                X["ab"][2 * l + 1], gu_sig[2 * l], gu_sig[2 * l + 1],
+                                workspace=ws_gu)
+        gu_act = [x for x in X["x"] for _ in range(2)]
         fpo.layer_update_grouped_signals(gu_sig, gu_act, wl.lr, W_masters=gu_W12, W_outs=gu_out,
                                          workspace=ws_gu)
 
-    def step(stage_events=None, upd_events=None):
-        fpo.error_signal(h, w, W_U, y, g, eps=wl.eps, min_rms=wl.min_rms, t_chunk=args.t_chunk,
-                         loss_out=loss, workspace=ws_es, stage_events=stage_events, algo=algo)
+    def step(X, stage_events=None, upd_events=None):
+        fpo.error_signal(X["h"], w, W_U, X["y"], g, eps=wl.eps, min_rms=wl.min_rms,
+                         t_chunk=args.t_chunk, loss_out=loss, workspace=ws_es,
+                         stage_events=stage_events, algo=algo)
         if post:
             if upd_events:
                 upd_events[2].record(stream)
             for l in range(wl.layers):
-                fpo.rmsnorm_vjp(g, m_out[l], gp[l], g_l[l], eps=wl.eps, min_rms=wl.min_rms)
+                fpo.rmsnorm_vjp(g, X["m"][l], gp[l], g_l[l], eps=wl.eps, min_rms=wl.min_rms)
         if upd_events:
             upd_events[0].record(stream)
-        update()
+        update(X)
         if upd_events:
             upd_events[1].record(stream)
         if gate_up:
-            gate_up_update()
+            gate_up_update(X)
             if upd_events:
                 upd_events[3].record(stream)
 
     for _ in range(args.warmup):
-        step()
+        step(X0)
     torch.cuda.synchronize()
     assert fpo.get_device_status(ws_es) == fpo.OK and fpo.get_device_status(ws_up) == fpo.OK
 
@@ -374,7 +382,7 @@ def run_fpo(args, wl):
     time.sleep(0.3)
     start.record(stream)
     for i in range(args.steps):
-        step(ev[i], uev[i])
+        step(X0, ev[i], uev[i])
     end.record(stream)
     torch.cuda.synchronize()
     clk = clocks.stop()
@@ -398,61 +406,68 @@ def run_fpo(args, wl):
                                               for i in range(args.steps))
 
     # ------------------------------------------------ end to end through the public API
+    # Every step copies its inputs (h, targets, every A_l, and the per-layer caches of the
+    # optional rows) from pinned host memory and reads the loss back.  The inputs rotate
+    # through `depth` device sets: while step i computes on one set, the inputs of step
+    # i + depth - 1 are copied into the set step i - 1 has finished reading, on a copy
+    # stream, so copies may run up to depth - 1 steps ahead (slack for a host link whose
+    # throughput stalls now and then).  Inside the timed region each step issues exactly
+    # one step's copies, and the region ends only after the copy stream has drained.
     e2e = None
     if not args.no_e2e:
-        h_host = h.cpu().pin_memory()
-        y_host = y.cpu().pin_memory()
-        A_host = [a.cpu().pin_memory() for a in A]
-        m_host = [x.cpu().pin_memory() for x in m_out] if post else []
+        def clone_set(X):
+            return {k: (v.clone() if torch.is_tensor(v) else [t.clone() for t in v])
+                    for k, v in X.items()}
+
+        def flat(X):
+            return [X["h"], X["y"]] + [t for k in ("A", "m", "ab", "x") for t in X[k]]
+
+        depth = max(2, args.e2e_depth)
+        sets = [X0] + [clone_set(X0) for _ in range(depth - 1)]
+        host = [t.cpu().pin_memory() for t in flat(X0)]
         loss_host = torch.empty(1, dtype=torch.float32).pin_memory()
-
         copy_stream = torch.cuda.Stream(device=dev)
-        a_ready = torch.cuda.Event()
+        ready = [torch.cuda.Event() for _ in range(depth)]
+        freed = [torch.cuda.Event() for _ in range(depth)]
+        for e in freed:
+            e.record(stream)
 
-        def e2e_step():
-            # h and targets feed the first kernel: copy them on the compute stream.
-            h.copy_(h_host, non_blocking=True)
-            y.copy_(y_host, non_blocking=True)
-            # A_l is first read by the layer update: copy it on a side stream while the
-            # error signal runs (after the previous step's update has finished reading it).
-            copy_stream.wait_stream(stream)
+        def prefetch(b):
+            copy_stream.wait_event(freed[b])
             with torch.cuda.stream(copy_stream):
-                for a_d, a_h in zip(A, A_host):
-                    a_d.copy_(a_h, non_blocking=True)
-                for m_d, m_h in zip(m_out if post else [], m_host):
-                    m_d.copy_(m_h, non_blocking=True)
-                a_ready.record(copy_stream)
-            fpo.error_signal(h, w, W_U, y, g, eps=wl.eps, min_rms=wl.min_rms,
-                             t_chunk=args.t_chunk, loss_out=loss, workspace=ws_es, algo=algo)
-            stream.wait_event(a_ready)
-            if post:
-                for l in range(wl.layers):
-                    fpo.rmsnorm_vjp(g, m_out[l], gp[l], g_l[l], eps=wl.eps, min_rms=wl.min_rms)
-            update()
-            if gate_up:
-                gate_up_update()
+                for d_t, h_t in zip(flat(sets[b]), host):
+                    d_t.copy_(h_t, non_blocking=True)
+                ready[b].record(copy_stream)
+
+        def e2e_step(i):
+            b = i % depth
+            prefetch((i + depth - 1) % depth)  # the inputs of step i + depth - 1
+            stream.wait_event(ready[b])
+            step(sets[b])
+            freed[b].record(stream)
             loss_host.copy_(loss, non_blocking=True)
 
-        for _ in range(max(1, args.warmup)):
-            e2e_step()
+        for b in range(depth - 1):
+            prefetch(b)
+        for i in range(max(1, args.warmup)):
+            e2e_step(i)
         torch.cuda.synchronize()
         if world > 1:
             dist.barrier()
         s2, e2 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         s2.record(stream)
-        for _ in range(args.steps):
-            e2e_step()
+        for i in range(max(1, args.warmup), max(1, args.warmup) + args.steps):
+            e2e_step(i)
+        stream.wait_stream(copy_stream)
         e2.record(stream)
         torch.cuda.synchronize()
         e2e_ms = max_over_ranks(s2.elapsed_time(e2) / args.steps, dev)
-        h2d = (h.numel() * h.element_size() + y.numel() * 4
-               + sum(a.numel() * a.element_size() for a in A))
-        if post:
-            h2d += sum(x.numel() * x.element_size() for x in m_out)
+        h2d = sum(t.numel() * t.element_size() for t in host)
         e2e = {"value": whole_job_tokens_per_s(wl.T, world, e2e_ms), "unit": "tokens/s",
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": 4, "ms_per_step": e2e_ms,
-               "pipeline": "h, targets H2D on the compute stream; A_l H2D on a copy stream "
-                           "overlapping the error signal; loss D2H"}
+               "pipeline": f"all step inputs H2D from pinned memory each step, {depth} device "
+                           "sets: copies run on a copy stream up to "
+                           f"{depth - 1} steps ahead of compute; loss D2H"}
 
     ms = max_over_ranks(ms, dev)
 
@@ -579,6 +594,8 @@ def main():
                     help="compose each layer's post-FFN RMSNorm VJP (OLMo-2 layout) in the step")
     ap.add_argument("--algo", choices=("auto", "recompute", "stored", "direct"), default="auto",
                     help="how the error matrix is formed (fpo_es_algo)")
+    ap.add_argument("--e2e-depth", type=int, default=3,
+                    help="device input sets of the end-to-end loop (copies run depth-1 steps ahead)")
     ap.add_argument("--band", type=int, default=0,
                     help="GEMM rasterisation band height in tiles (0: library default; tuning)")
     ap.add_argument("--gemm-variant", type=int, choices=(-1, 0, 1), default=-1,
