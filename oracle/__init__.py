@@ -16,6 +16,7 @@ Each function follows one passage of the paper:
 * :func:`sgd_update`    App. A, fp32 master weights cast to bf16.
 * :func:`optimizer_step`  Sec. 3.1 AdamW / SGD with momentum, App. A relative clip.
 * :func:`cosine`        Sec. 2.2, Eq. (cosine).
+* :func:`norm_ratio`    App. C update-magnitude ratios, Sec. C.2 implied SGD rate.
 """
 from __future__ import annotations
 
@@ -73,6 +74,8 @@ def _load():
     lib.oracle_cosine.argtypes = [i64, i32, vp, vp, vp]
     lib.oracle_cosine.restype = None
     lib.oracle_mean_ce.argtypes = [i64, vp, vp]
+    lib.oracle_norm_ratio.argtypes = [i64, i64, i32, vp, i32, vp, dbl, vp]
+    lib.oracle_norm_ratio.restype = None
     lib.oracle_mean_ce.restype = dbl
     _lib = lib
     return lib
@@ -260,6 +263,26 @@ def cosine(X, Y):
     out = np.zeros(4)
     _load().oracle_cosine(X.size, dtx, _ptr(X.reshape(-1)), _ptr(Y.reshape(-1)), _ptr(out))
     return tuple(out)
+
+
+def norm_ratio(G, W, rel=0.01):
+    """App. C: per layer (||G_l||^2, ||W_l||^2, ||G_l||/||W_l||, rel/(||G_l||/||W_l||)) in fp64,
+    for lists of same-size arrays G (one dtype) and W (one dtype); returns [L, 4]."""
+    if len(G) != len(W):
+        raise ValueError("G and W need one array per layer")
+    typed_g = [_typed(x) for x in G]
+    typed_w = [_typed(x) for x in W]
+    n = typed_g[0][1].size if G else 0
+    if any(a.size != n for _, a in typed_g + typed_w):
+        raise ValueError("every G_l and W_l must have the same size")
+    if len({t for t, _ in typed_g}) > 1 or len({t for t, _ in typed_w}) > 1:
+        raise TypeError("the G_l share one dtype and the W_l share one dtype")
+    g_arr = (ctypes.c_void_p * max(1, len(G)))(*[_ptr(a.reshape(-1)).value for _, a in typed_g])
+    w_arr = (ctypes.c_void_p * max(1, len(W)))(*[_ptr(a.reshape(-1)).value for _, a in typed_w])
+    out = np.zeros((len(G), 4))
+    _load().oracle_norm_ratio(len(G), n, typed_g[0][0] if G else 0, g_arr,
+                              typed_w[0][0] if W else 0, w_arr, float(rel), _ptr(out))
+    return out
 
 
 def mean_ce(lse, zy):

@@ -18,6 +18,8 @@
  *   oracle_sgd_update    App. A (fp32 master weights, cast to bf16)
  *   oracle_optimizer_step  Sec. 3.1 (AdamW / SGD with momentum) + App. A relative clip
  *   oracle_cosine        Sec. 2.2, Eq. (cosine)
+ *   oracle_norm_ratio    App. C (update-magnitude ratios) and Sec. C.2: ||G||/||W||
+ *                        and the SGD learning rate of a relative step
  *
  * Inputs are the exact stored values (fp32, bf16 or fp64) upcast to fp64 as
  * they are read.  OpenMP parallelises only over independent tokens / output
@@ -367,4 +369,29 @@ double oracle_mean_ce(int64_t n, const double* lse, const double* zy) {
     double acc = 0.0;
     for (int64_t k = 0; k < n; ++k) acc += lse[k] - zy[k];
     return n > 0 ? acc / (double)n : 0.0;
+}
+
+/*
+ * Update-magnitude ratio of App. C: for layer l, the fractional weight change
+ * per unit learning rate ||g~ (x) h||_F / ||W||_F with g~ (x) h = G_l, and the
+ * plain-SGD learning rate whose step -lr G_l has norm rel * ||W_l||_F (rel =
+ * 0.01: the table's "1% step" column).  out[4 l + {0,1,2,3}] =
+ * { ||G_l||^2, ||W_l||^2, ||G_l|| / ||W_l||, rel / (||G_l|| / ||W_l||) },
+ * fp64 sums in index order (IEEE division: x/0 = inf, 0/0 = NaN).
+ */
+void oracle_norm_ratio(int64_t n_layers, int64_t n, int g_dt, const void* const* G, int w_dt,
+                       const void* const* W, double rel, double* out) {
+    for (int64_t l = 0; l < n_layers; ++l) {
+        double gg = 0.0, ww = 0.0;
+        for (int64_t k = 0; k < n; ++k) {
+            double g = orc_load(g_dt, G[l], k), w = orc_load(w_dt, W[l], k);
+            gg += g * g;
+            ww += w * w;
+        }
+        double r = sqrt(gg) / sqrt(ww);
+        out[4 * l + 0] = gg;
+        out[4 * l + 1] = ww;
+        out[4 * l + 2] = r;
+        out[4 * l + 3] = rel / r;
+    }
 }

@@ -516,3 +516,37 @@ def test_silu_derivative_against_autograd():
     assert np.allclose(dA[0], at.grad.numpy(), rtol=1e-12, atol=1e-14)
     assert np.allclose(dB[0], torch.nn.functional.silu(torch.tensor(a)).numpy(), rtol=1e-12,
                        atol=1e-14)
+
+
+def test_norm_ratio_closed_forms_and_library_norms():
+    """App. C update-magnitude ratio ||G||_F / ||W||_F: G = c W gives |c|; random arrays
+    (bf16 bits and fp32) against numpy's Frobenius norms; the rate is rel / ratio."""
+    rng = np.random.default_rng(11)
+    W = rng.standard_normal(1000).astype(np.float32)
+    out = oracle.norm_ratio([(-0.37 * W.astype(np.float64)).astype(np.float32)], [W], rel=0.01)
+    assert abs(out[0, 2] - 0.37) < 1e-6 and abs(out[0, 3] - 0.01 / 0.37) < 1e-6
+    Gs = [rng.standard_normal(777).astype(np.float32) * s for s in (1e-3, 2.0, 5.0)]
+    Ws = [rng.standard_normal(777).astype(np.float32) for _ in range(3)]
+    Gb = [oracle.f32_to_bf16_bits(g) for g in Gs]
+    out = oracle.norm_ratio(Gb, Ws, rel=0.05)
+    for l in range(3):
+        gv = oracle.bf16_bits_to_f64(Gb[l])
+        wv = Ws[l].astype(np.float64)
+        assert abs(out[l, 0] - np.linalg.norm(gv) ** 2) <= 1e-12 * out[l, 0]
+        assert abs(out[l, 1] - np.linalg.norm(wv) ** 2) <= 1e-12 * out[l, 1]
+        r = np.linalg.norm(gv) / np.linalg.norm(wv)
+        assert abs(out[l, 2] - r) <= 1e-12 * r and abs(out[l, 3] - 0.05 / r) <= 1e-12 / r
+    z = oracle.norm_ratio([np.zeros(4, np.float32)], [np.ones(4, np.float32)], rel=0.01)
+    assert z[0, 2] == 0.0 and math.isinf(z[0, 3])
+
+
+def test_norm_ratio_reproduces_the_papers_implied_learning_rates():
+    """The App. C table's implied-SGD-LR column is the 1% relative step over the ratio."""
+    with open(os.path.join(GOLDEN, "update_ratio_olmo2_table.json")) as f:
+        tab = json.load(f)
+    for row in tab["rows"]:
+        r = row["ratio_post_ffn"]
+        out = oracle.norm_ratio([np.array([r, 0.0])], [np.array([0.0, 1.0])],
+                                rel=tab["relative_step"])
+        assert abs(out[0, 2] - r) < 1e-15
+        assert round(out[0, 3], 4) == row["implied_sgd_lr"], row["layer"]
