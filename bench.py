@@ -316,6 +316,8 @@ def run_fpo(args, wl):
         launches_per_step += 3 if args.clip != "none" else 1
     if args.gate_up:  # one error_h GEMM per layer + one grouped W1/W2 update
         launches_per_step += wl.layers + 1
+    if args.norm_ratio:  # partial sums over all layers + the per-layer final
+        launches_per_step += 2
 
     # The tensors one step reads that come from the forward pass / the data: the
     # end-to-end loop below copies them from host memory every step.
@@ -323,16 +325,28 @@ def run_fpo(args, wl):
           "ab": [t for pair in gu_ab for t in pair] if gate_up else [],
           "x": gu_x if gate_up else []}
 
+    ratio = args.norm_ratio
+    if ratio:  # App. C update-magnitude ratio on each step's G_l (bf16) and fp32 masters
+        if optimize:
+            raise SystemExit("--norm-ratio reads G_l from the fused update (--optimizer fused-sgd)")
+        Go = [torch.empty(wl.d, wl.d_ff, dtype=torch.bfloat16, device=dev)
+              for _ in range(wl.layers)]
+        ratio_out = torch.empty(wl.layers, 4, dtype=torch.float64, device=dev)
+        ws_nr = torch.empty(fpo.norm_ratio_workspace(wl.layers, wl.d * wl.d_ff),
+                            dtype=torch.uint8, device=dev)
+
     def update(X):
         signals = g_l if post else [g] * wl.layers
+        G_outs = Go if ratio else None
         if optimize:
             fpo.layer_optimize_grouped(signals, X["A"], opt, Wm, W_outs=Wo, states1=st1,
                                        states2=st2, workspace=ws_up)
         elif post:
             fpo.layer_update_grouped_signals(g_l, X["A"], wl.lr, W_masters=Wm, W_outs=Wo,
-                                             workspace=ws_up)
+                                             G_outs=G_outs, workspace=ws_up)
         else:
-            fpo.layer_update_grouped(g, X["A"], wl.lr, W_masters=Wm, W_outs=Wo, workspace=ws_up)
+            fpo.layer_update_grouped(g, X["A"], wl.lr, W_masters=Wm, W_outs=Wo, G_outs=G_outs,
+                                     workspace=ws_up)
 
     def gate_up_update(X):
         for l in range(wl.layers):
@@ -361,6 +375,12 @@ def run_fpo(args, wl):
             gate_up_update(X)
             if upd_events:
                 upd_events[3].record(stream)
+        if ratio:
+            if upd_events:
+                upd_events[4].record(stream)
+            fpo.norm_ratio(Go, Wm, rel_step=0.01, out=ratio_out, workspace=ws_nr)
+            if upd_events:
+                upd_events[5].record(stream)
 
     for _ in range(args.warmup):
         step(X0)
@@ -370,7 +390,7 @@ def run_fpo(args, wl):
     # per-stage events for every timed step (recorded once so their handles exist)
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(fpo.STAGE_EVENTS)]
           for _ in range(args.steps)]
-    uev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    uev = [[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(args.steps)]
     for e in [x for row in ev + uev for x in row]:
         e.record(stream)
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -404,6 +424,9 @@ def run_fpo(args, wl):
     if gate_up:
         stage_ms["gate_up"] = statistics.mean(uev[i][1].elapsed_time(uev[i][3])
                                               for i in range(args.steps))
+    if ratio:
+        stage_ms["norm_ratio"] = statistics.mean(uev[i][4].elapsed_time(uev[i][5])
+                                                 for i in range(args.steps))
 
     # ------------------------------------------------ end to end through the public API
     # Every step copies its inputs (h, targets, every A_l, and the per-layer caches of the
@@ -515,6 +538,10 @@ def run_fpo(args, wl):
             "kernels_ms": stage_ms,
             "kernels_tflops": {k: per_kernel_flops[k] / (stage_ms[k] / 1e3) / 1e12
                                for k in per_kernel_flops},
+            "kernels_gbs": ({"norm_ratio": wl.layers * wl.d * wl.d_ff * (2 + 4)
+                             / (stage_ms["norm_ratio"] / 1e3) / 1e9} if ratio else {}),
+            "norm_ratio": ({"ratio": ratio_out[:, 2].tolist(),
+                            "implied_sgd_lr_1pct": ratio_out[:, 3].tolist()} if ratio else None),
             "algo": algo_name,
             "gemm_kernel": "cta-pair 256x256 (tcgen05 cta_group::2)" if variant == 1
                            else "single-cta 128x256 (tcgen05 cta_group::1)",
@@ -594,6 +621,8 @@ def main():
                     help="compose each layer's post-FFN RMSNorm VJP (OLMo-2 layout) in the step")
     ap.add_argument("--algo", choices=("auto", "recompute", "stored", "direct"), default="auto",
                     help="how the error matrix is formed (fpo_es_algo)")
+    ap.add_argument("--norm-ratio", action="store_true",
+                    help="add the App. C update-magnitude ratio ||G_l||/||W_l|| to every step")
     ap.add_argument("--e2e-depth", type=int, default=3,
                     help="device input sets of the end-to-end loop (copies run depth-1 steps ahead)")
     ap.add_argument("--band", type=int, default=0,

@@ -350,6 +350,33 @@ int32_t fpo_cosine(int64_t n, int32_t dtype, const void* X, const void* Y, doubl
 int32_t fpo_cosine_noalloc(int64_t n, int32_t dtype, const void* X, const void* Y, double* out,
                            void* stream);
 
+/* Bytes of workspace fpo_norm_ratio needs (0 for an invalid n_layers or n). */
+size_t fpo_norm_ratio_workspace(int32_t n_layers, int64_t n);
+
+/*
+ * fpo_norm_ratio -- the update-magnitude ratio of App. C ("Update-magnitude
+ * ratios": the fractional weight change per unit learning rate,
+ * ||g~ (x) h|| / ||W_3||) and the learning rate it implies (Sec. C.2), for
+ * n_layers target layers in one call:
+ *   out[4 l + 0] = ||G_l||_F^2        out[4 l + 1] = ||W_l||_F^2
+ *   out[4 l + 2] = r_l = ||G_l||_F / ||W_l||_F
+ *   out[4 l + 3] = rel_step / r_l     (the plain-SGD rate whose step -lr G_l has
+ *                                      norm rel_step ||W_l||_F; 0.01 = the
+ *                                      paper's "1% step")
+ * IEEE division (x / 0 = inf, 0 / 0 = NaN), so r_l = NaN for n = 0.
+ *
+ * G, W     host arrays of n_layers device pointers, each to n elements: G_l in
+ *          g_dtype (a pseudogradient, e.g. G_out of fpo_layer_update_grouped),
+ *          W_l in w_dtype (the fp32 master, or the bf16 weight); 16-byte aligned
+ * out      device, 4 x n_layers fp64, 8-byte aligned
+ * 1 <= n_layers <= FPO_MAX_GROUPED_LAYERS.  Squares are summed in fp32 over
+ * runs of at most 128 elements and in fp64 after that, in a fixed order (repeat
+ * calls give identical bits).  workspace: fpo_norm_ratio_workspace(n_layers, n) bytes.
+ */
+int32_t fpo_norm_ratio(int32_t n_layers, int64_t n, int32_t g_dtype, const void* const* G,
+                       int32_t w_dtype, const void* const* W, double rel_step, double* out,
+                       void* workspace, size_t workspace_bytes, void* stream);
+
 /*
  * Synchronise `stream`, read the device status word of `workspace` (set by the
  * last call that used it), clear it, and return FPO_OK, FPO_ERR_TARGET_RANGE

@@ -91,6 +91,11 @@ _lib.fpo_cosine.argtypes = [_i64, _i32, _vp, _vp, _vp, _vp, _sz, _vp]
 _lib.fpo_cosine.restype = _i32
 _lib.fpo_get_device_status.argtypes = [_vp, _vp]
 _lib.fpo_get_device_status.restype = _i32
+_lib.fpo_norm_ratio_workspace.argtypes = [_i32, _i64]
+_lib.fpo_norm_ratio_workspace.restype = _sz
+_lib.fpo_norm_ratio.argtypes = [_i32, _i64, _i32, ctypes.POINTER(_vp), _i32, ctypes.POINTER(_vp),
+                                ctypes.c_double, _vp, _vp, _sz, _vp]
+_lib.fpo_norm_ratio.restype = _i32
 _lib.fpo_testing_direct_fixup_rows.argtypes = [ctypes.POINTER(ErrorSignalDesc), _vp, _vp]
 _lib.fpo_testing_direct_fixup_rows.restype = _i64
 _lib.fpo_testing_set_gemm_variant.argtypes = [_i32]
@@ -331,6 +336,34 @@ def cosine(X, Y, out=None, *, workspace=None, stream=None):
     rc = _lib.fpo_cosine(n, _dtype_code(X), _ptr(X), _ptr(Y), _ptr(out), _ptr(workspace),
                          workspace.numel(), _stream(stream))
     _check(rc, "fpo_cosine")
+    return out
+
+
+def norm_ratio_workspace(n_layers: int, n: int) -> int:
+    return int(_lib.fpo_norm_ratio_workspace(int(n_layers), int(n)))
+
+
+def norm_ratio(G, W, rel_step=0.01, out=None, *, workspace=None, stream=None):
+    """fpo_norm_ratio: per layer [||G_l||^2, ||W_l||^2, ||G_l||/||W_l||, rel_step/ratio] as a
+    device fp64 tensor [len(G), 4]; G and W are lists of same-size tensors."""
+    n_layers = len(G)
+    if n_layers != len(W) or n_layers == 0:
+        raise ValueError("G and W need one tensor per layer")
+    n = G[0].numel()
+    if any(t.numel() != n for t in list(G) + list(W)):
+        raise ValueError("every G_l and W_l must have the same number of elements")
+    if any(t.dtype != G[0].dtype for t in G) or any(t.dtype != W[0].dtype for t in W):
+        raise TypeError("the G_l share one dtype and the W_l share one dtype")
+    if out is None:
+        out = torch.empty(n_layers, 4, dtype=torch.float64, device=G[0].device)
+    if workspace is None:
+        workspace = _workspace(norm_ratio_workspace(n_layers, n), G[0].device)
+    garr = (_vp * n_layers)(*[_ptr(t) for t in G])
+    warr = (_vp * n_layers)(*[_ptr(t) for t in W])
+    rc = _lib.fpo_norm_ratio(n_layers, n, _dtype_code(G[0]), garr, _dtype_code(W[0]), warr,
+                             float(rel_step), _ptr(out), _ptr(workspace), workspace.numel(),
+                             _stream(stream))
+    _check(rc, "fpo_norm_ratio")
     return out
 
 

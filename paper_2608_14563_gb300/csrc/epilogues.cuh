@@ -92,10 +92,11 @@ using EpiLseStoreZ = EpiLsePartialT<true>;
 // Logits pass of the direct algorithm (Sec. 3.1 step 2 rewritten around a
 // per-token anchor c_t): besides the (max, sum exp) partial and the target
 // logit of EpiLsePartial, every valid non-target logit leaves
-//   p~_tj = exp(z_tj - c_t)              rounded to bf16 into P [M, N]
-// (the target column and the overhang are written as 0), and the tile's sum of
-// those rounded values, S'_t partial, goes to sx [M, part_ld].  Two 32-column
-// chunks fill one 64-column bf16 staging row before each TMA store.
+//   p~_tj = exp(z_tj - c_t) = exp(z_tj - m) exp(m - c_t)   (m: the running max)
+// rounded to bf16 into P [M, N] (the target column and the overhang are written
+// as 0), and the tile's sum of those rounded values, S'_t partial, goes to
+// sx [M, part_ld].  Two 32-column chunks fill one 64-column bf16 staging row
+// before each TMA store.
 struct EpiLseProb {
     struct Params {
         CUtensorMap pmap;     // bf16 P [M, N], box 64 x 32
@@ -120,11 +121,12 @@ struct EpiLseProb {
         c2 = valid ? __ldg(p.anchor + row_) * kLog2e : 0.f;
     }
 
-    // p~ of logits j, j+1 of the chunk (0 for the target and for columns >= lim),
-    // packed to bf16; the rounded values are added to the tile sum.
-    __device__ __forceinline__ uint32_t prob_pair(const float (&v)[32], int j, int lim, int r) {
-        const float a = (j < lim && j != r) ? ex2_approx(fmaf(v[j], kLog2e, -c2)) : 0.f;
-        const float b = (j + 1 < lim && j + 1 != r) ? ex2_approx(fmaf(v[j + 1], kLog2e, -c2)) : 0.f;
+    // p~ of logits j, j+1 of the chunk from their exponentials e relative to the running
+    // max (0 for the target and for columns >= lim, where e is 0), scaled by
+    // f = exp(max - c); packed to bf16, the rounded values added to the tile sum.
+    __device__ __forceinline__ uint32_t prob_pair(const float (&e)[32], float f, int j, int r) {
+        const float a = j != r ? e[j] * f : 0.f;
+        const float b = j + 1 != r ? e[j + 1] * f : 0.f;
         const uint32_t pk = pack_bf16x2(a, b);
         sxs += __uint_as_float(pk << 16) + __uint_as_float(pk & 0xffff0000u);
         return pk;
@@ -136,6 +138,8 @@ struct EpiLseProb {
         if (!second) pair_out = col0 >= p.N || io.row0 >= p.M;
         const int lim = p.N - col0;  // valid columns in this chunk (may be <= 0)
         const int r = yoff - c0;     // target position in this chunk, if in [0, 32)
+        float e[32];
+        float f = 0.f;
         if (lim > 0) {
             float cm = -INFINITY;
 #pragma unroll
@@ -145,24 +149,30 @@ struct EpiLseProb {
             const float nml = nm * kLog2e;
             float acc = (m == -INFINITY) ? 0.f : s * ex2_approx(m * kLog2e - nml);
 #pragma unroll
-            for (int j = 0; j < 32; ++j)
-                if (j < lim) acc += ex2_approx(fmaf(v[j], kLog2e, -nml));
+            for (int j = 0; j < 32; ++j) {
+                e[j] = j < lim ? ex2_approx(fmaf(v[j], kLog2e, -nml)) : 0.f;
+                acc += e[j];
+            }
             s = acc;
             m = nm;
+            f = ex2_approx(nml - c2);
             if (static_cast<unsigned>(r) < 32u) {
 #pragma unroll
                 for (int j = 0; j < 32; ++j)
                     if (j == r) zt = v[j];
                 has_t = true;
             }
+        } else {
+#pragma unroll
+            for (int j = 0; j < 32; ++j) e[j] = 0.f;
         }
         if (pair_out) return;
         if (!second) {
 #pragma unroll
-            for (int j = 0; j < 32; j += 2) w[j / 2] = prob_pair(v, j, lim, r);
+            for (int j = 0; j < 32; j += 2) w[j / 2] = prob_pair(e, f, j, r);
         } else {
 #pragma unroll
-            for (int j = 0; j < 32; j += 2) w[16 + j / 2] = prob_pair(v, j, lim, r);
+            for (int j = 0; j < 32; j += 2) w[16 + j / 2] = prob_pair(e, f, j, r);
             const uint32_t buf = out_acquire(io);
             out_stage_row(buf, io.lane, w);
             out_commit(io, &p.pmap, buf, col0 - 32, io.row0);

@@ -552,6 +552,38 @@ int32_t fpo_cosine(int64_t n, int32_t dtype, const void* X, const void* Y, doubl
                                      blocks, out, st));
 }
 
+size_t fpo_norm_ratio_workspace(int32_t n_layers, int64_t n) {
+    if (n_layers < 1 || n_layers > FPO_MAX_GROUPED_LAYERS || n < 0) return 0;
+    return kStatusBytes +
+           align_up(static_cast<size_t>(n_layers) * norm_ratio_blocks(n_layers, n) * 2 *
+                    sizeof(double));
+}
+
+int32_t fpo_norm_ratio(int32_t n_layers, int64_t n, int32_t g_dtype, const void* const* G,
+                       int32_t w_dtype, const void* const* W, double rel_step, double* out,
+                       void* workspace, size_t workspace_bytes, void* stream) {
+    if ((g_dtype != FPO_F32 && g_dtype != FPO_BF16) || (w_dtype != FPO_F32 && w_dtype != FPO_BF16))
+        return FPO_ERR_DTYPE;
+    if (n_layers < 1 || n_layers > FPO_MAX_GROUPED_LAYERS || n < 0) return FPO_ERR_SHAPE;
+    if (!G || !W || !out) return FPO_ERR_NULL;
+    for (int l = 0; l < n_layers; ++l) {
+        if (n > 0 && (!G[l] || !W[l])) return FPO_ERR_NULL;
+        if (!aligned16(G[l]) || !aligned16(W[l])) return FPO_ERR_ALIGN;
+    }
+    if (reinterpret_cast<uintptr_t>(out) & 7u) return FPO_ERR_ALIGN;
+    if (!workspace) return FPO_ERR_WORKSPACE;
+    if ((reinterpret_cast<uintptr_t>(workspace) % kAlign) != 0) return FPO_ERR_ALIGN;
+    if (workspace_bytes < fpo_norm_ratio_workspace(n_layers, n)) return FPO_ERR_WORKSPACE;
+    int32_t rc = check_arch();
+    if (rc != FPO_OK) return rc;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    uint8_t* ws = static_cast<uint8_t*>(workspace);
+    FPO_TRY(cudaMemsetAsync(ws, 0, sizeof(unsigned), st));
+    return cuda_status(launch_norm_ratio(g_dtype, w_dtype, n_layers, n, G, W, rel_step,
+                                         reinterpret_cast<double*>(ws + kStatusBytes),
+                                         norm_ratio_blocks(n_layers, n), out, st));
+}
+
 int32_t fpo_testing_gemm_bf16(int64_t M, int64_t N, int64_t K, int32_t a_mn, int32_t b_mn,
                               const void* A, const void* B, float* C, void* workspace,
                               size_t workspace_bytes, void* stream) {
