@@ -543,8 +543,10 @@ def run_fpo(args, wl):
             "norm_ratio": ({"ratio": ratio_out[:, 2].tolist(),
                             "implied_sgd_lr_1pct": ratio_out[:, 3].tolist()} if ratio else None),
             "algo": algo_name,
-            "gemm_kernel": "cta-pair 256x256 (tcgen05 cta_group::2)" if variant == 1
-                           else "single-cta 128x256 (tcgen05 cta_group::1)",
+            "gemm_kernel": {0: "single-cta 128x256 (tcgen05 cta_group::1)",
+                            1: "cta-pair 256x256 (tcgen05 cta_group::2)",
+                            2: "cta-pair 256x256, projection 256x512 (tcgen05 cta_group::2)"
+                            }[variant],
             "cpu_baseline": cpu,
             "e2e": e2e,
             "gpu_launches": launches_per_step * args.steps,
@@ -627,9 +629,9 @@ def main():
                     help="device input sets of the end-to-end loop (copies run depth-1 steps ahead)")
     ap.add_argument("--band", type=int, default=0,
                     help="GEMM rasterisation band height in tiles (0: library default; tuning)")
-    ap.add_argument("--gemm-variant", type=int, choices=(-1, 0, 1), default=-1,
+    ap.add_argument("--gemm-variant", type=int, choices=(-1, 0, 1, 2), default=-1,
                     help="tensor-core GEMM kernel: 0 single-CTA tiles, 1 CTA-pair tiles, "
-                         "-1 library default")
+                         "2 CTA-pair tiles with a 256x512 projection, -1 library default")
     ap.add_argument("--shape", default=None,
                     help="T,d,d_ff,V,layers override of the workload's shape (small ncu cases)")
     ap.add_argument("--cpu-tokens", type=int, default=16, help="oracle sample size (tokens)")

@@ -32,8 +32,10 @@ int32_t fpo_testing_gemm_bf16(int64_t M, int64_t N, int64_t K, int32_t a_mn, int
 /*
  * Select the tensor-core GEMM kernel every later call uses (process-wide):
  * 0 = one CTA per 128 x 256 output tile, 1 = a CTA pair (tcgen05 cta_group::2)
- * per 256 x 256 tile (the default).  Returns the previous setting.  Both compute the same
- * sums in the same order per output element.
+ * per 256 x 256 tile, 2 = as 1 but 256 x 512 pair tiles for the projection
+ * g = E W_U (one accumulator, a quarter less operand traffic; the default).
+ * Returns the previous setting.  All compute the same sums in the same order per
+ * output element.
  */
 int32_t fpo_testing_set_gemm_variant(int32_t variant);
 

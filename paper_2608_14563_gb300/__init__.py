@@ -121,8 +121,9 @@ def set_wait_limit_ns(ns: int) -> None:
 
 
 def set_gemm_variant(variant: int) -> int:
-    """fpo_testing_set_gemm_variant: 0 single-CTA, 1 CTA-pair tiles; a negative value only
-    reads the current setting.  Returns the setting in force before the call."""
+    """fpo_testing_set_gemm_variant: 0 single-CTA, 1 CTA-pair tiles, 2 CTA-pair tiles with a
+    256 x 512 projection; a negative value only reads the current setting.  Returns the
+    setting in force before the call."""
     if variant < 0:
         cur = _lib.fpo_testing_set_gemm_variant(0)
         _lib.fpo_testing_set_gemm_variant(cur)

@@ -146,10 +146,15 @@ cudaError_t run_gemm_pair(const GemmMaps<MAXG>& maps, const typename Epi::Params
 
 constexpr int kPairStages = 6;
 
-std::atomic<int> g_gemm_variant{1};  // 0 = single-CTA tiles, 1 = CTA-pair tiles (default)
+// 0 = single-CTA tiles, 1 = CTA-pair tiles, 2 = CTA-pair tiles with 256 x 512 tiles for
+// the projection (default: its K loop runs over the whole vocabulary, so the epilogue
+// that the single accumulator cannot overlap costs ~1%, while a quarter less operand
+// traffic per FLOP made the projection 6-7% faster)
+std::atomic<int> g_gemm_variant{2};
 std::atomic<int> g_band_override{0};  // > 0: rasterisation band height (tests / tuning)
 
-bool use_pair() { return g_gemm_variant.load(std::memory_order_relaxed) == 1; }
+bool use_pair() { return g_gemm_variant.load(std::memory_order_relaxed) >= 1; }
+bool wide_proj() { return g_gemm_variant.load(std::memory_order_relaxed) == 2; }
 
 // Rasterisation band in tile rows, unless overridden: 16 tile rows, i.e. 2048
 // output rows of single-CTA tiles and 4096 of pair tiles.  With pair tiles the
@@ -165,7 +170,9 @@ int band_for(bool) {
 
 void set_band_override(int b) { g_band_override.store(b > 0 ? b : 0, std::memory_order_relaxed); }
 
-void set_gemm_variant(int v) { g_gemm_variant.store(v == 1 ? 1 : 0, std::memory_order_relaxed); }
+void set_gemm_variant(int v) {
+    g_gemm_variant.store(v >= 0 && v <= 2 ? v : 0, std::memory_order_relaxed);
+}
 int gemm_variant() { return g_gemm_variant.load(std::memory_order_relaxed); }
 
 constexpr int kLseBN = 256;
@@ -259,6 +266,8 @@ cudaError_t launch_lse_prob_bf16(const void* yhat, const void* W_U, const int32_
 
 constexpr int kProjBN = 256;
 constexpr int kProjStages = 4;
+constexpr int kWideBN = 512;     // pair tiles 256 x 512: 48 KB stages
+constexpr int kWideStages = 4;
 
 cudaError_t launch_proj_direct_bf16(const void* P, const void* W_U, const int32_t* y,
                                     const float* alpha, const float* beta, int Tc, int d, int V,
@@ -274,6 +283,9 @@ cudaError_t launch_proj_direct_bf16(const void* P, const void* W_U, const int32_
     ep.W_U = static_cast<const __nv_bfloat16*>(W_U);
     ep.M = Tc;
     ep.N = d;
+    if (wide_proj())
+        return run_gemm_pair<kWideBN, false, true, kWideStages, 1, EpiProjDirect>(
+            maps, ep, make_shape(Tc, d, V, kWideBN, 1, band_for(true), kPairBM), status, st);
     if (use_pair())
         return run_gemm_pair<kProjBN, false, true, kPairStages, 1, EpiProjDirect>(
             maps, ep, make_shape(Tc, d, V, kProjBN, 1, band_for(true), kPairBM), status, st);
@@ -290,6 +302,9 @@ cudaError_t launch_proj_bf16(const void* E, const void* W_U, int Tc, int d, int 
     if (!map_out_f32(&ep.Cmap, g, Tc, d)) return cudaErrorInvalidValue;
     ep.M = Tc;
     ep.N = d;
+    if (wide_proj())
+        return run_gemm_pair<kWideBN, false, true, kWideStages, 1, EpiStoreF32>(
+            maps, ep, make_shape(Tc, d, V, kWideBN, 1, band_for(true), kPairBM), status, st);
     if (use_pair())
         return run_gemm_pair<kProjBN, false, true, kPairStages, 1, EpiStoreF32>(
             maps, ep, make_shape(Tc, d, V, kProjBN, 1, band_for(true), kPairBM), status, st);
@@ -401,6 +416,19 @@ cudaError_t launch_test_gemm_bf16(int M, int N, int K, bool a_mn, bool b_mn, con
     if (!map_out_f32(&ep.Cmap, C, M, N)) return cudaErrorInvalidValue;
     ep.M = M;
     ep.N = N;
+    if (wide_proj()) {  // every layout on 256 x 512 pair tiles
+        const GemmShape sh = make_shape(M, N, K, kWideBN, 1, band_for(true), kPairBM);
+        if (!a_mn && !b_mn)
+            return run_gemm_pair<kWideBN, false, false, kWideStages, 1, EpiStoreF32>(maps, ep, sh,
+                                                                                    status, st);
+        if (!a_mn && b_mn)
+            return run_gemm_pair<kWideBN, false, true, kWideStages, 1, EpiStoreF32>(maps, ep, sh,
+                                                                                   status, st);
+        if (a_mn && b_mn)
+            return run_gemm_pair<kWideBN, true, true, kWideStages, 1, EpiStoreF32>(maps, ep, sh,
+                                                                                  status, st);
+        return cudaErrorInvalidValue;
+    }
     if (pair) {
         const GemmShape sh = make_shape(M, N, K, 256, 1, band_for(true), kPairBM);
         if (!a_mn && !b_mn)

@@ -13,7 +13,12 @@
 //                       accumulator-ready barriers of BOTH CTAs (multicast)
 //   both CTAs, warps 2-5  epilogue on the CTA's 128 rows; arrive on the
 //                       leader's accumulator-empty barrier (8 arrivals)
-// TMEM (2 x BN columns) is allocated collectively by warp 1 of both CTAs.
+// TMEM (512 columns) is allocated collectively by warp 1 of both CTAs.
+//
+// BN is 256 (two accumulator buffers of 256 columns: the epilogue of one tile
+// overlaps the mainloop of the next) or 512 (two N=256 MMAs per K slice into
+// one 512-column accumulator: a quarter less operand traffic per FLOP, but the
+// next tile waits for the epilogue; for GEMMs with a long K loop).
 // All waits are bounded as in the single-CTA kernel; the pair meets at a
 // cluster barrier before TMEM is freed and before either CTA exits.
 #pragma once
@@ -91,10 +96,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     tc_gemm_pair_kernel(const __grid_constant__ GemmMaps<MAXG> maps,
                         const __grid_constant__ typename Epi::Params ep, const GemmShape sh,
                         unsigned int* status, unsigned long long wait_limit_ns) {
+    static_assert(BN == 256 || BN == 512, "pair tiles are 256 or 512 columns wide");
     using L = GemmPairSmem<BN, STAGES>;
-    constexpr int kBHalf = BN / 2;
-    constexpr uint32_t kIdesc = idesc_bf16_f32(kPairBM, BN, A_MN, B_MN);
-    constexpr int kTmemCols = 2 * BN;
+    constexpr int kNSub = BN / 256;                // N = 256 MMAs per K slice
+    constexpr int kAccBufs = kNSub == 1 ? 2 : 1;   // accumulator buffers in TMEM
+    constexpr int kBSub = 128;                     // B columns per CTA per N = 256 MMA
+    constexpr uint32_t kBSubBytes = kBSub * kBK * 2;
+    constexpr uint32_t kIdesc = idesc_bf16_f32(kPairBM, 256, A_MN, B_MN);
+    constexpr int kTmemCols = kAccBufs * BN;       // 512 either way
     constexpr uint16_t kBoth = 0x3;
 
     extern __shared__ uint8_t smem_raw[];
@@ -159,7 +168,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
                 const CUtensorMap* amap = &maps.a[MAXG == 1 ? 0 : g];
                 const CUtensorMap* bmap = &maps.b[MAXG == 1 ? 0 : g];
                 const int a_row = mp * kPairBM + 128 * static_cast<int>(rank);
-                const int b_row = nb * BN + kBHalf * static_cast<int>(rank);
+                const int b_row = nb * BN + kBSub * static_cast<int>(rank);
                 for (int kb = 0; kb < sh.k_blocks; ++kb) {
                     if (!mbar_wait_cl(empty_bar(stage), phase ^ 1u, guard)) { ok = false; break; }
                     const uint32_t sa = sbase + stage * L::kStageBytes;
@@ -167,7 +176,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
                     const uint32_t fb = mapa_shared(full_bar(stage), 0);
                     if (leader) mbar_arrive_expect_tx(full_bar(stage), 2 * L::kStageBytes);
                     load_operand_pair<A_MN, 128>(amap, sa, fb, a_row, kb * kBK);
-                    load_operand_pair<B_MN, kBHalf>(bmap, sb, fb, b_row, kb * kBK);
+#pragma unroll
+                    for (int h = 0; h < kNSub; ++h)
+                        load_operand_pair<B_MN, kBSub>(bmap, sb + h * kBSubBytes, fb,
+                                                       b_row + 256 * h, kb * kBK);
                     issued_mask |= 1u << stage;
                     issued_parity = (issued_parity & ~(1u << stage)) | (phase << stage);
                     if (++stage == STAGES) { stage = 0; phase ^= 1u; }
@@ -201,15 +213,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
                     const uint32_t sb = sa + L::kABytes;
 #pragma unroll
                     for (int kk = 0; kk < kBK / kUmmaK; ++kk)
-                        tc_mma_bf16_pair(d_tmem, operand_desc<A_MN>(sa, kk),
-                                         operand_desc<B_MN>(sb, kk), kIdesc, (kb | kk) != 0 ? 1u : 0u);
+#pragma unroll
+                        for (int h = 0; h < kNSub; ++h)
+                            tc_mma_bf16_pair(d_tmem + 256u * h, operand_desc<A_MN>(sa, kk),
+                                             operand_desc<B_MN>(sb + h * kBSubBytes, kk), kIdesc,
+                                             (kb | kk) != 0 ? 1u : 0u);
                     issued_any = true;
                     tc_commit_pair_multicast(empty_bar(stage), kBoth);
                     if (++stage == STAGES) { stage = 0; phase ^= 1u; }
                 }
                 if (!ok) break;
                 tc_commit_pair_multicast(tfull_bar(acc), kBoth);
-                if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
+                if (++acc == kAccBufs) { acc = 0; acc_phase ^= 1u; }
             }
             if (!ok && issued_any) {
                 tc_commit_pair_multicast(drain_bar, 0x1);
@@ -251,7 +266,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
                 else
                     mbar_arrive_cluster(mapa_shared(tempty_bar(acc), 0));
             }
-            if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
+            if (++acc == kAccBufs) { acc = 0; acc_phase ^= 1u; }
         }
         if (lane == 0) bulk_wait_group_all();
         __syncwarp();

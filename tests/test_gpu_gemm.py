@@ -16,9 +16,10 @@ pytestmark = pytest.mark.gpu
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 
-@pytest.fixture(scope="module", params=[0, 1], ids=["cta", "cta_pair"])
+@pytest.fixture(scope="module", params=[0, 1, 2], ids=["cta", "cta_pair", "cta_pair_wide"])
 def tlib(fpo, request):
-    """The test entry points, with the GEMM kernel variant selected (single CTA / CTA pair)."""
+    """The test entry points, with the GEMM kernel variant selected (single CTA, CTA pair, CTA
+    pair with 256 x 512 tiles)."""
     lib = ctypes.CDLL(os.path.join(ROOT, "paper_2608_14563_gb300", "libfpo.so"))
     vp = ctypes.c_void_p
     lib.fpo_testing_gemm_bf16.argtypes = [ctypes.c_int64] * 3 + [ctypes.c_int32] * 2 + [vp] * 4 + [
