@@ -159,3 +159,27 @@ def test_rows_outside_the_anchor_window_are_fixed(fpo):
     assert np.max(np.abs(g[50:100] - G[50:100])) < 1e-30
     assert np.max(np.abs(f64(outs[0]["lse"]) - ref["lse"]) / np.maximum(1, np.abs(ref["lse"]))) < 1e-5
     assert abs(outs[0]["loss"].item() - oracle.mean_ce(ref["lse"], ref["zy"])) < 1e-4 * np.mean(ce)
+
+
+@pytest.mark.parametrize("variant", [0, 1, 2])
+@pytest.mark.parametrize("algo", [1, 2, 3])  # recompute, stored logits, direct
+def test_results_do_not_depend_on_workspace_contents(fpo, ragged, variant, algo):
+    """Every workspace byte a call reads it writes first: a workspace full of 0xFF (NaN
+    bit patterns) gives the same bits as a zeroed one, for every kernel variant."""
+    inp, _ = ragged
+    h, w, W_U, y = (inp[k].cuda() for k in ("h", "w", "W_U", "y"))
+    prev = fpo.set_gemm_variant(variant)
+    try:
+        desc = fpo.error_signal_desc(*h.shape, W_U.shape[0], fpo.BF16, algo=algo, t_chunk=128)
+        n = fpo.error_signal_workspace(desc)
+        outs = []
+        for fill in (0x00, 0xFF):
+            ws = torch.full((n,), fill, dtype=torch.uint8, device="cuda")
+            g = torch.empty_like(h)
+            loss = torch.empty(1, dtype=torch.float32, device="cuda")
+            fpo.error_signal(h, w, W_U, y, g, loss_out=loss, workspace=ws, algo=algo, t_chunk=128)
+            assert fpo.get_device_status(ws) == fpo.OK
+            outs.append((g, loss))
+    finally:
+        fpo.set_gemm_variant(prev)
+    assert torch.equal(outs[0][0], outs[1][0]) and torch.equal(outs[0][1], outs[1][1])
