@@ -318,6 +318,8 @@ def run_fpo(args, wl):
         launches_per_step += wl.layers + 1
     if args.norm_ratio:  # partial sums over all layers + the per-layer final
         launches_per_step += 2
+    if args.cosine or wl.name.startswith("diag"):  # grouped partial sums + final
+        launches_per_step += 2
 
     # The tensors one step reads that come from the forward pass / the data: the
     # end-to-end loop below copies them from host memory every step.
@@ -326,24 +328,41 @@ def run_fpo(args, wl):
           "x": gu_x if gate_up else []}
 
     ratio = args.norm_ratio
-    if ratio:  # App. C update-magnitude ratio on each step's G_l (bf16) and fp32 masters
-        if optimize:
-            raise SystemExit("--norm-ratio reads G_l from the fused update (--optimizer fused-sgd)")
+    # Sec. 2.2 diagnostic: cos(G_l, G~_l) per target layer against a 'true' gradient G~_l
+    # (a seeded stand-in drawn once: the timing does not depend on its values), on by
+    # default for the diag workload
+    cosine = args.cosine or wl.name.startswith("diag")
+    if (ratio or cosine) and optimize:
+        raise SystemExit("--norm-ratio / --cosine read G_l from the fused update "
+                         "(--optimizer fused-sgd)")
+    if ratio or cosine:
         Go = [torch.empty(wl.d, wl.d_ff, dtype=torch.bfloat16, device=dev)
               for _ in range(wl.layers)]
+    if ratio:  # App. C update-magnitude ratio on each step's G_l (bf16) and fp32 masters
         ratio_out = torch.empty(wl.layers, 4, dtype=torch.float64, device=dev)
         ws_nr = torch.empty(fpo.norm_ratio_workspace(wl.layers, wl.d * wl.d_ff),
                             dtype=torch.uint8, device=dev)
+    if cosine:
+        n_el = wl.d * wl.d_ff
+        G_true = [synth.make_noise(n_el, seed=wl_r.seed, layer=l, device=dev).mul_(1e-3)
+                  .to(torch.bfloat16) for l in range(wl.layers)]
+        cos_out = torch.empty(wl.layers, 4, dtype=torch.float64, device=dev)
+        ws_cos = torch.empty(fpo.cosine_grouped_workspace(wl.layers, n_el), dtype=torch.uint8,
+                             device=dev)
+        Go_flat = [x.view(-1) for x in Go]
 
     def update(X):
         signals = g_l if post else [g] * wl.layers
-        G_outs = Go if ratio else None
+        G_outs = Go if (ratio or cosine) else None
         if optimize:
             fpo.layer_optimize_grouped(signals, X["A"], opt, Wm, W_outs=Wo, states1=st1,
                                        states2=st2, workspace=ws_up)
         elif post:
             fpo.layer_update_grouped_signals(g_l, X["A"], wl.lr, W_masters=Wm, W_outs=Wo,
                                              G_outs=G_outs, workspace=ws_up)
+        elif wl.lr == 0.0 and G_outs is not None:
+            # the diagnostic's step: G_l only (no master to move at lr = 0)
+            fpo.layer_update_grouped(g, X["A"], 0.0, G_outs=G_outs, workspace=ws_up)
         else:
             fpo.layer_update_grouped(g, X["A"], wl.lr, W_masters=Wm, W_outs=Wo, G_outs=G_outs,
                                      workspace=ws_up)
@@ -381,6 +400,12 @@ def run_fpo(args, wl):
             fpo.norm_ratio(Go, Wm, rel_step=0.01, out=ratio_out, workspace=ws_nr)
             if upd_events:
                 upd_events[5].record(stream)
+        if cosine:
+            if upd_events:
+                upd_events[6].record(stream)
+            fpo.cosine_grouped(Go_flat, G_true, out=cos_out, workspace=ws_cos)
+            if upd_events:
+                upd_events[7].record(stream)
 
     for _ in range(args.warmup):
         step(X0)
@@ -390,7 +415,7 @@ def run_fpo(args, wl):
     # per-stage events for every timed step (recorded once so their handles exist)
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(fpo.STAGE_EVENTS)]
           for _ in range(args.steps)]
-    uev = [[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(args.steps)]
+    uev = [[torch.cuda.Event(enable_timing=True) for _ in range(8)] for _ in range(args.steps)]
     for e in [x for row in ev + uev for x in row]:
         e.record(stream)
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -427,6 +452,9 @@ def run_fpo(args, wl):
     if ratio:
         stage_ms["norm_ratio"] = statistics.mean(uev[i][4].elapsed_time(uev[i][5])
                                                  for i in range(args.steps))
+    if cosine:
+        stage_ms["cosine"] = statistics.mean(uev[i][6].elapsed_time(uev[i][7])
+                                             for i in range(args.steps))
 
     # ------------------------------------------------ end to end through the public API
     # Every step copies its inputs (h, targets, every A_l, and the per-layer caches of the
@@ -538,8 +566,11 @@ def run_fpo(args, wl):
             "kernels_ms": stage_ms,
             "kernels_tflops": {k: per_kernel_flops[k] / (stage_ms[k] / 1e3) / 1e12
                                for k in per_kernel_flops},
-            "kernels_gbs": ({"norm_ratio": wl.layers * wl.d * wl.d_ff * (2 + 4)
-                             / (stage_ms["norm_ratio"] / 1e3) / 1e9} if ratio else {}),
+            "kernels_gbs": {**({"norm_ratio": wl.layers * wl.d * wl.d_ff * (2 + 4)
+                                / (stage_ms["norm_ratio"] / 1e3) / 1e9} if ratio else {}),
+                            **({"cosine": wl.layers * wl.d * wl.d_ff * (2 + 2)
+                                / (stage_ms["cosine"] / 1e3) / 1e9} if cosine else {})},
+            "cosine": cos_out[:, 3].tolist() if cosine else None,
             "norm_ratio": ({"ratio": ratio_out[:, 2].tolist(),
                             "implied_sgd_lr_1pct": ratio_out[:, 3].tolist()} if ratio else None),
             "algo": algo_name,
@@ -623,6 +654,9 @@ def main():
                     help="compose each layer's post-FFN RMSNorm VJP (OLMo-2 layout) in the step")
     ap.add_argument("--algo", choices=("auto", "recompute", "stored", "direct"), default="auto",
                     help="how the error matrix is formed (fpo_es_algo)")
+    ap.add_argument("--cosine", action="store_true",
+                    help="add the Sec. 2.2 diagnostic cosine of every layer's G_l to each step "
+                         "(always on for the diag workload)")
     ap.add_argument("--norm-ratio", action="store_true",
                     help="add the App. C update-magnitude ratio ||G_l||/||W_l|| to every step")
     ap.add_argument("--e2e-depth", type=int, default=3,

@@ -350,6 +350,24 @@ int32_t fpo_cosine(int64_t n, int32_t dtype, const void* X, const void* Y, doubl
 int32_t fpo_cosine_noalloc(int64_t n, int32_t dtype, const void* X, const void* Y, double* out,
                            void* stream);
 
+/* Bytes of workspace fpo_cosine_grouped needs (0 for an invalid n_layers or n). */
+size_t fpo_cosine_grouped_workspace(int32_t n_layers, int64_t n);
+
+/*
+ * fpo_cosine_grouped -- fpo_cosine (Sec. 2.2, Eq. (cosine)) for n_layers pairs
+ * of equal size in one launch pair, e.g. every target layer's pseudogradient
+ * against its true gradient in the layer-viability diagnostic:
+ *   out[4 l + {0,1,2,3}] = <X_l, Y_l>, ||X_l||^2, ||Y_l||^2, cos_l (0 if a norm is 0)
+ * X, Y: host arrays of n_layers device pointers to n elements of dtype, 16-byte
+ * aligned; out: device, 4 x n_layers fp64, 8-byte aligned; 1 <= n_layers <=
+ * FPO_MAX_GROUPED_LAYERS.  Sums run in fp32 over runs of at most 128 elements and
+ * in fp64 after that, in a fixed order (repeat calls give identical bits; the
+ * order differs from fpo_cosine's, so the two agree to rounding, not bitwise).
+ */
+int32_t fpo_cosine_grouped(int32_t n_layers, int64_t n, int32_t dtype, const void* const* X,
+                           const void* const* Y, double* out, void* workspace,
+                           size_t workspace_bytes, void* stream);
+
 /* Bytes of workspace fpo_norm_ratio needs (0 for an invalid n_layers or n). */
 size_t fpo_norm_ratio_workspace(int32_t n_layers, int64_t n);
 

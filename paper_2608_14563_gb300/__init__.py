@@ -91,6 +91,11 @@ _lib.fpo_cosine.argtypes = [_i64, _i32, _vp, _vp, _vp, _vp, _sz, _vp]
 _lib.fpo_cosine.restype = _i32
 _lib.fpo_get_device_status.argtypes = [_vp, _vp]
 _lib.fpo_get_device_status.restype = _i32
+_lib.fpo_cosine_grouped_workspace.argtypes = [_i32, _i64]
+_lib.fpo_cosine_grouped_workspace.restype = _sz
+_lib.fpo_cosine_grouped.argtypes = [_i32, _i64, _i32, ctypes.POINTER(_vp), ctypes.POINTER(_vp),
+                                    _vp, _vp, _sz, _vp]
+_lib.fpo_cosine_grouped.restype = _i32
 _lib.fpo_norm_ratio_workspace.argtypes = [_i32, _i64]
 _lib.fpo_norm_ratio_workspace.restype = _sz
 _lib.fpo_norm_ratio.argtypes = [_i32, _i64, _i32, ctypes.POINTER(_vp), _i32, ctypes.POINTER(_vp),
@@ -337,6 +342,33 @@ def cosine(X, Y, out=None, *, workspace=None, stream=None):
     rc = _lib.fpo_cosine(n, _dtype_code(X), _ptr(X), _ptr(Y), _ptr(out), _ptr(workspace),
                          workspace.numel(), _stream(stream))
     _check(rc, "fpo_cosine")
+    return out
+
+
+def cosine_grouped_workspace(n_layers: int, n: int) -> int:
+    return int(_lib.fpo_cosine_grouped_workspace(int(n_layers), int(n)))
+
+
+def cosine_grouped(X, Y, out=None, *, workspace=None, stream=None):
+    """fpo_cosine_grouped: per layer [<X_l,Y_l>, |X_l|^2, |Y_l|^2, cos_l] as a device fp64
+    tensor [len(X), 4]; X and Y are lists of same-size tensors of one dtype."""
+    n_layers = len(X)
+    if n_layers != len(Y) or n_layers == 0:
+        raise ValueError("X and Y need one tensor per layer")
+    n = X[0].numel()
+    if any(t.numel() != n for t in list(X) + list(Y)):
+        raise ValueError("every X_l and Y_l must have the same number of elements")
+    if any(t.dtype != X[0].dtype for t in list(X) + list(Y)):
+        raise TypeError("X and Y share one dtype")
+    if out is None:
+        out = torch.empty(n_layers, 4, dtype=torch.float64, device=X[0].device)
+    if workspace is None:
+        workspace = _workspace(cosine_grouped_workspace(n_layers, n), X[0].device)
+    xarr = (_vp * n_layers)(*[_ptr(t) for t in X])
+    yarr = (_vp * n_layers)(*[_ptr(t) for t in Y])
+    rc = _lib.fpo_cosine_grouped(n_layers, n, _dtype_code(X[0]), xarr, yarr, _ptr(out),
+                                 _ptr(workspace), workspace.numel(), _stream(stream))
+    _check(rc, "fpo_cosine_grouped")
     return out
 
 

@@ -555,7 +555,7 @@ int32_t fpo_cosine(int64_t n, int32_t dtype, const void* X, const void* Y, doubl
 size_t fpo_norm_ratio_workspace(int32_t n_layers, int64_t n) {
     if (n_layers < 1 || n_layers > FPO_MAX_GROUPED_LAYERS || n < 0) return 0;
     return kStatusBytes +
-           align_up(static_cast<size_t>(n_layers) * norm_ratio_blocks(n_layers, n) * 2 *
+           align_up(static_cast<size_t>(n_layers) * norm_ratio_blocks(n_layers, n) * 3 *
                     sizeof(double));
 }
 
@@ -582,6 +582,34 @@ int32_t fpo_norm_ratio(int32_t n_layers, int64_t n, int32_t g_dtype, const void*
     return cuda_status(launch_norm_ratio(g_dtype, w_dtype, n_layers, n, G, W, rel_step,
                                          reinterpret_cast<double*>(ws + kStatusBytes),
                                          norm_ratio_blocks(n_layers, n), out, st));
+}
+
+size_t fpo_cosine_grouped_workspace(int32_t n_layers, int64_t n) {
+    return fpo_norm_ratio_workspace(n_layers, n);  // same partial layout
+}
+
+int32_t fpo_cosine_grouped(int32_t n_layers, int64_t n, int32_t dtype, const void* const* X,
+                           const void* const* Y, double* out, void* workspace,
+                           size_t workspace_bytes, void* stream) {
+    if (dtype != FPO_F32 && dtype != FPO_BF16) return FPO_ERR_DTYPE;
+    if (n_layers < 1 || n_layers > FPO_MAX_GROUPED_LAYERS || n < 0) return FPO_ERR_SHAPE;
+    if (!X || !Y || !out) return FPO_ERR_NULL;
+    for (int l = 0; l < n_layers; ++l) {
+        if (n > 0 && (!X[l] || !Y[l])) return FPO_ERR_NULL;
+        if (!aligned16(X[l]) || !aligned16(Y[l])) return FPO_ERR_ALIGN;
+    }
+    if (reinterpret_cast<uintptr_t>(out) & 7u) return FPO_ERR_ALIGN;
+    if (!workspace) return FPO_ERR_WORKSPACE;
+    if ((reinterpret_cast<uintptr_t>(workspace) % kAlign) != 0) return FPO_ERR_ALIGN;
+    if (workspace_bytes < fpo_cosine_grouped_workspace(n_layers, n)) return FPO_ERR_WORKSPACE;
+    int32_t rc = check_arch();
+    if (rc != FPO_OK) return rc;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    uint8_t* ws = static_cast<uint8_t*>(workspace);
+    FPO_TRY(cudaMemsetAsync(ws, 0, sizeof(unsigned), st));
+    return cuda_status(launch_cosine_grouped(dtype, n_layers, n, X, Y,
+                                             reinterpret_cast<double*>(ws + kStatusBytes),
+                                             norm_ratio_blocks(n_layers, n), out, st));
 }
 
 int32_t fpo_testing_gemm_bf16(int64_t M, int64_t N, int64_t K, int32_t a_mn, int32_t b_mn,

@@ -133,15 +133,19 @@ cudaError_t launch_rmsnorm_vjp_at(int dtype, const void* g, const void* x, const
 // One block waiting on an mbarrier nothing arrives on, bounded by limit_ns.
 cudaError_t launch_wait_timeout(unsigned* status, uint64_t limit_ns, cudaStream_t st);
 
-// ------------------------------------------------------------ update-magnitude ratio
+// ------------------------------------------------------------ grouped per-layer reductions
 constexpr int kNrMaxLayers = 64;
-// Blocks per layer of the first pass; partial needs n_layers * blocks * 2 doubles.
+// Blocks per layer of the first pass; partial needs n_layers * blocks * 3 doubles.
 int norm_ratio_blocks(int n_layers, int64_t n);
 // out[4 l ..] = ||G_l||^2, ||W_l||^2, ||G_l|| / ||W_l||, rel / ratio (device, fp64);
 // dtypes 0 = fp32, 1 = bf16.
 cudaError_t launch_norm_ratio(int g_dtype, int w_dtype, int n_layers, int64_t n,
                               const void* const* G, const void* const* W, double rel,
                               double* partial, int blocks, double* out, cudaStream_t st);
+// out[4 l ..] = <X_l,Y_l>, ||X_l||^2, ||Y_l||^2, cos_l for every layer (dtype of both).
+cudaError_t launch_cosine_grouped(int dtype, int n_layers, int64_t n, const void* const* X,
+                                  const void* const* Y, double* partial, int blocks, double* out,
+                                  cudaStream_t st);
 
 // ------------------------------------------------------------ cosine
 int cosine_blocks(int64_t n);
