@@ -306,58 +306,102 @@ __global__ void __launch_bounds__(kRowThreads)
     }
 }
 
-// Rows outside the anchor window, one (row, vocabulary tile) per work item:
-// z_tj = <yhat_t, W_U[j]> in fp32 (one warp per column), then the tile of P is
-// rewritten as p_tj = exp(z_tj - lse_t) in bf16 (target zero) and sx[t, tile]
-// as the sum of the rounded values.  The row count is read on the device, so
-// the launch is the same whether or not any row needs it.
-constexpr int kFixTile = 256;  // vocabulary columns per work item (the logits tile width)
+// Rows outside the anchor window, in groups of up to kFixRows rows per work item
+// (group, vocabulary tile): the group's yhat rows are staged in shared memory (or
+// read from global memory when d is too large to stage), and each warp takes tile
+// columns j in turn, reading W_U[j] once for the whole group:
+//   z_rj = <yhat_r, W_U[j]> (fp32),  P[r, j] = bf16(exp(z_rj - lse_r)) (target 0),
+// and per row the sum of the tile's rounded values goes to sx[row, tile].  The row
+// count is read on the device, so the launch is the same whether or not any row
+// needs it; with none it returns at once.
+constexpr int kFixTile = 256;        // vocabulary columns per work item (the logits tile width)
+constexpr int kFixRows = 8;          // rows per group: one W_U read serves all of them
+constexpr int kFixStageMax = 192 * 1024;  // shared memory for staged yhat rows
 
-template <int VEC>
+template <bool kStage>
 __global__ void __launch_bounds__(kRowThreads)
     direct_fixup_kernel(const __nv_bfloat16* __restrict__ yhat,
                         const __nv_bfloat16* __restrict__ W_U, const int32_t* __restrict__ y,
                         const float* __restrict__ lse, const int* __restrict__ fix,
                         const int* __restrict__ fix_count, int d, int V, int n_tiles,
                         __nv_bfloat16* __restrict__ P, float* __restrict__ sx) {
-    __shared__ float part_sum[kRowThreads / 32];
+    extern __shared__ __align__(16) uint8_t fx_smem[];
+    __nv_bfloat16* xs = reinterpret_cast<__nv_bfloat16*>(fx_smem);  // [kFixRows][d] if staged
+    __shared__ float wsum[kRowThreads / 32][kFixRows];
     const int lane = threadIdx.x & 31;
     const int warp = threadIdx.x >> 5;
-    const long long items = static_cast<long long>(*fix_count) * n_tiles;
+    const int count = *fix_count;
+    const long long groups = (count + kFixRows - 1) / kFixRows;
+    const long long items = groups * n_tiles;
     for (long long it = blockIdx.x; it < items; it += gridDim.x) {
-        const int row = fix[it / n_tiles];
+        const int r0 = static_cast<int>(it / n_tiles) * kFixRows;
         const int tile = static_cast<int>(it % n_tiles);
-        const int t = y[row];
-        const float l = lse[row];
-        const __nv_bfloat16* xr = yhat + static_cast<size_t>(row) * d;
-        float acc = 0.f;
+        const int nr = count - r0 < kFixRows ? count - r0 : kFixRows;
+        const __nv_bfloat16* xr[kFixRows];
+        __syncthreads();  // the previous item is done with the staged rows and wsum
+        if constexpr (kStage) {
+            const int v8 = d / 8;
+            for (int idx = threadIdx.x; idx < nr * v8; idx += kRowThreads) {
+                const int r = idx / v8, k = (idx - r * v8) * 8;
+                *reinterpret_cast<uint4*>(xs + static_cast<size_t>(r) * d + k) =
+                    *reinterpret_cast<const uint4*>(yhat + static_cast<size_t>(fix[r0 + r]) * d + k);
+            }
+            __syncthreads();
+#pragma unroll
+            for (int r = 0; r < kFixRows; ++r) xr[r] = xs + static_cast<size_t>(r) * d;
+        } else {
+#pragma unroll
+            for (int r = 0; r < kFixRows; ++r)
+                xr[r] = yhat + static_cast<size_t>(fix[r0 + (r < nr ? r : 0)]) * d;
+        }
+        float acc[kFixRows];
+#pragma unroll
+        for (int r = 0; r < kFixRows; ++r) acc[r] = 0.f;
         for (int c = warp; c < kFixTile; c += kRowThreads / 32) {
             const int j = tile * kFixTile + c;
             if (j >= V) break;
             const __nv_bfloat16* ur = W_U + static_cast<size_t>(j) * d;
-            float z = 0.f;
-            for (int k = lane * VEC; k < d; k += 32 * VEC) {
-                float a[VEC], b[VEC];
-                ld_vec<VEC>(xr + k, a);
-                ld_vec<VEC>(ur + k, b);
+            float z[kFixRows];
 #pragma unroll
-                for (int q = 0; q < VEC; ++q) z = fmaf(a[q], b[q], z);
+            for (int r = 0; r < kFixRows; ++r) z[r] = 0.f;
+            for (int k = lane * 8; k < d; k += 32 * 8) {
+                float b[8];
+                ld_vec<8>(ur + k, b);
+#pragma unroll
+                for (int r = 0; r < kFixRows; ++r) {
+                    if (r < nr) {
+                        float a[8];
+                        ld_vec<8>(xr[r] + k, a);
+#pragma unroll
+                        for (int q = 0; q < 8; ++q) z[r] = fmaf(a[q], b[q], z[r]);
+                    }
+                }
             }
-            z = warp_sum(z);
+#pragma unroll
+            for (int r = 0; r < kFixRows; ++r) z[r] = warp_sum(z[r]);
             if (lane == 0) {
-                const __nv_bfloat16 p = __float2bfloat16_rn(j == t ? 0.f : expf(z - l));
-                P[static_cast<size_t>(row) * V + j] = p;
-                acc += __bfloat162float(p);
+#pragma unroll
+                for (int r = 0; r < kFixRows; ++r) {
+                    if (r < nr) {
+                        const int row = fix[r0 + r];
+                        const __nv_bfloat16 p =
+                            __float2bfloat16_rn(j == y[row] ? 0.f : expf(z[r] - lse[row]));
+                        P[static_cast<size_t>(row) * V + j] = p;
+                        acc[r] += __bfloat162float(p);
+                    }
+                }
             }
         }
-        if (lane == 0) part_sum[warp] = acc;
-        __syncthreads();
-        if (threadIdx.x == 0) {
-            float S = 0.f;
-            for (int i = 0; i < kRowThreads / 32; ++i) S += part_sum[i];
-            sx[static_cast<size_t>(row) * n_tiles + tile] = S;
+        if (lane == 0) {
+#pragma unroll
+            for (int r = 0; r < kFixRows; ++r) wsum[warp][r] = acc[r];
         }
         __syncthreads();
+        if (threadIdx.x < nr) {
+            float S = 0.f;
+            for (int w = 0; w < kRowThreads / 32; ++w) S += wsum[w][threadIdx.x];
+            sx[static_cast<size_t>(fix[r0 + threadIdx.x]) * n_tiles + tile] = S;
+        }
     }
 }
 
@@ -522,9 +566,20 @@ cudaError_t launch_direct_fixup(const void* yhat, const void* W_U, const int32_t
                                 float* beta, cudaStream_t st) {
     DevInfo di;
     const int sms = current_device_info(&di) ? di.sm_count : 148;
-    direct_fixup_kernel<8><<<sms * 4, kRowThreads, 0, st>>>(
-        static_cast<const __nv_bfloat16*>(yhat), static_cast<const __nv_bfloat16*>(W_U), y, lse,
-        fix, fix_count, d, V, n_tiles, static_cast<__nv_bfloat16*>(P), sx);
+    const size_t stage = static_cast<size_t>(kFixRows) * d * 2;
+    const auto* yh = static_cast<const __nv_bfloat16*>(yhat);
+    const auto* wu = static_cast<const __nv_bfloat16*>(W_U);
+    auto* pp = static_cast<__nv_bfloat16*>(P);
+    if (stage <= static_cast<size_t>(kFixStageMax)) {
+        static const cudaError_t attr = cudaFuncSetAttribute(
+            direct_fixup_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, kFixStageMax);
+        if (attr != cudaSuccess) return attr;
+        direct_fixup_kernel<true><<<2 * sms, kRowThreads, stage, st>>>(yh, wu, y, lse, fix, fix_count,
+                                                                   d, V, n_tiles, pp, sx);
+    } else {
+        direct_fixup_kernel<false><<<sms * 4, kRowThreads, 0, st>>>(yh, wu, y, lse, fix, fix_count,
+                                                                    d, V, n_tiles, pp, sx);
+    }
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     direct_fixup_factors_kernel<<<sms, kRowThreads, 0, st>>>(sx, fix, fix_count, n_tiles, s, alpha,

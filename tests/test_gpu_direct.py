@@ -183,3 +183,35 @@ def test_results_do_not_depend_on_workspace_contents(fpo, ragged, variant, algo)
     finally:
         fpo.set_gemm_variant(prev)
     assert torch.equal(outs[0][0], outs[1][0]) and torch.equal(outs[0][1], outs[1][1])
+
+
+def test_many_rows_outside_the_window(fpo):
+    """Logits ~30x the usual scale (exact +-1 hidden states, W_U x 64): most tokens have
+    cross-entropy far beyond the window and go through the grouped fixup (8 rows per
+    group, a partial last group); the rows match the oracle and the count matches the
+    fp64 window test of S'_t."""
+    T, d, V = 1000, 512, 4096
+    wl = Workload("many-fixed", T=T, d=d, d_ff=8, V=V, layers=1, targets="uniform", eps=0.0)
+    w = synth.make_norm_w(wl)
+    W_U = synth.make_W_U(wl) * 64
+    h = torch.sign(synth.normal((T, d), seed=5, tensor="h"))
+    h[h == 0] = 1.0
+    h = h.to(torch.bfloat16)
+    y = synth.make_targets(wl)
+    z = (f64(h) * f64(w)[None, :]) @ f64(W_U).T
+    zo = z.copy()
+    zo[np.arange(T), y.numpy()] = -np.inf
+    mo = zo.max(axis=1)
+    log2_S = (mo - z[np.arange(T), y.numpy()] + np.log(np.exp(zo - mo[:, None]).sum(axis=1))) \
+        / np.log(2.0)
+    sure = int(np.sum(np.abs(log2_S) > 80.5))
+    maybe = int(np.sum(np.abs(log2_S) > 79.5))
+    assert sure > T // 2
+    out = run(fpo, h, w, W_U, y, eps=0.0, algo=fpo.ES_DIRECT)
+    assert sure <= out["fixed"] <= maybe
+    ref = reference(h, w, W_U, y, eps=0.0, s=1.0 / T)
+    g, G = f64(out["g"]), ref["g_tilde"]
+    assert rel_frob(g, G) < TOL and cos(g, G) >= COS_MIN
+    for t in range(0, T, 37):
+        assert rel_frob(g[t], G[t]) < TOL, t
+    assert np.max(np.abs(f64(out["lse"]) - ref["lse"]) / np.maximum(1, np.abs(ref["lse"]))) < 1e-5
