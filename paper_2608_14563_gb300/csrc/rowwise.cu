@@ -12,7 +12,9 @@
 //   rmsnorm_vjp   App. E Eq. (rmsnorm-vjp) with the min-RMS clamp:
 //                 g~ = (w (.) g - xhat <xhat, w (.) g> / d) / max(rho, rho_min)
 //
-// One warp per token row, 16-byte vector loads, warp-shuffle reductions.
+// bf16 rows of up to 8192 elements: one block per row, the row kept in registers
+// (each input read once); otherwise one warp per row (two passes over the row),
+// 16-byte vector loads, shuffle reductions.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <math.h>
@@ -145,6 +147,210 @@ __global__ void __launch_bounds__(kRowThreads)
             if (anchor) anchor[row] = zt;
         }
     }
+}
+
+// ---------------------------------------------------------------------------
+// One block per row (bf16, d <= 256 EPT): the row stays in registers, so each
+// input is read from HBM once (the warp-per-row kernels above read the row twice:
+// a reduction pass, then the output pass).  Element k of thread j's v-th vector is
+// (v * 256 + j) * 8 + i: every vector load of the block is one contiguous 4 KB span.
+constexpr int kBlkThreads = 256;
+
+// Block-wide sum of two values; every thread gets both results.
+__device__ __forceinline__ float2 block_sum2(float a, float b) {
+    __shared__ float2 red[kBlkThreads / 32];
+    a = warp_sum(a);
+    b = warp_sum(b);
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    __syncthreads();  // the previous call's readers are done with red
+    if (lane == 0) red[wid] = make_float2(a, b);
+    __syncthreads();
+    float2 t = make_float2(0.f, 0.f);
+#pragma unroll
+    for (int i = 0; i < kBlkThreads / 32; ++i) {
+        t.x += red[i].x;
+        t.y += red[i].y;
+    }
+    return t;
+}
+
+template <int EPT>
+__global__ void __launch_bounds__(kBlkThreads)
+    rmsnorm_fwd_row_kernel(const __nv_bfloat16* __restrict__ h, const __nv_bfloat16* __restrict__ w,
+                           int T, int d, float eps, __nv_bfloat16* __restrict__ yhat,
+                           float* __restrict__ rho, const int32_t* __restrict__ y, int V,
+                           unsigned* status, const __nv_bfloat16* __restrict__ W_U,
+                           float* __restrict__ anchor) {
+    constexpr int NV = EPT / 8;
+    for (int row = blockIdx.x; row < T; row += gridDim.x) {
+        const __nv_bfloat16* hr = h + static_cast<size_t>(row) * d;
+        const int t = y[row];
+        const bool t_ok = t >= 0 && t < V;
+        // the target's unembedding row, read only for an in-range target, loaded with h
+        const __nv_bfloat16* ur = (anchor && t_ok) ? W_U + static_cast<size_t>(t) * d : nullptr;
+        uint4 hx[NV], ux[NV];
+#pragma unroll
+        for (int v = 0; v < NV; ++v) {
+            const int k = (v * kBlkThreads + threadIdx.x) * 8;
+            hx[v] = k < d ? *reinterpret_cast<const uint4*>(hr + k) : make_uint4(0, 0, 0, 0);
+            ux[v] = (ur && k < d) ? *reinterpret_cast<const uint4*>(ur + k) : make_uint4(0, 0, 0, 0);
+        }
+        float ss = 0.f;
+#pragma unroll
+        for (int v = 0; v < NV; ++v) {
+            const uint32_t q4[4] = {hx[v].x, hx[v].y, hx[v].z, hx[v].w};
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const float lo = __uint_as_float(q4[q] << 16), hi = __uint_as_float(q4[q] & 0xffff0000u);
+                ss = fmaf(lo, lo, ss);
+                ss = fmaf(hi, hi, ss);
+            }
+        }
+        const float r = sqrtf(block_sum2(ss, 0.f).x / static_cast<float>(d) + eps);
+        const float inv = 1.0f / r;
+        __nv_bfloat16* yr = yhat + static_cast<size_t>(row) * d;
+        float zt = 0.f;
+#pragma unroll
+        for (int v = 0; v < NV; ++v) {
+            const int k = (v * kBlkThreads + threadIdx.x) * 8;
+            if (k < d) {
+                float wv[8], o[8];
+                ld_vec<8>(w + k, wv);
+                const uint32_t q4[4] = {hx[v].x, hx[v].y, hx[v].z, hx[v].w};
+                const uint32_t u4[4] = {ux[v].x, ux[v].y, ux[v].z, ux[v].w};
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    o[2 * q] = wv[2 * q] * (__uint_as_float(q4[q] << 16) * inv);
+                    o[2 * q + 1] = wv[2 * q + 1] * (__uint_as_float(q4[q] & 0xffff0000u) * inv);
+                    zt = fmaf(round_to<__nv_bfloat16>(o[2 * q]), __uint_as_float(u4[q] << 16), zt);
+                    zt = fmaf(round_to<__nv_bfloat16>(o[2 * q + 1]),
+                              __uint_as_float(u4[q] & 0xffff0000u), zt);
+                }
+                st_vec<8>(yr + k, o);
+            }
+        }
+        if (anchor) zt = block_sum2(zt, 0.f).x;
+        if (threadIdx.x == 0) {
+            rho[row] = r;
+            if (!t_ok) atomicOr(status, kDevTargetRange);
+            if (anchor) anchor[row] = zt;
+        }
+    }
+}
+
+template <int EPT>
+__global__ void __launch_bounds__(kBlkThreads)
+    rmsnorm_vjp_row_kernel(const float* __restrict__ g, const __nv_bfloat16* __restrict__ h,
+                           const __nv_bfloat16* __restrict__ w, const float* __restrict__ rho,
+                           int T, int d, float min_rms, __nv_bfloat16* __restrict__ out) {
+    constexpr int NV = EPT / 8;
+    for (int row = blockIdx.x; row < T; row += gridDim.x) {
+        const float r = rho[row];
+        const float inv_r = 1.0f / r;
+        const float* gr = g + static_cast<size_t>(row) * d;
+        const __nv_bfloat16* hr = h + static_cast<size_t>(row) * d;
+        float wg[EPT], xh[EPT];
+        float c = 0.f;
+#pragma unroll
+        for (int v = 0; v < NV; ++v) {
+            const int k = (v * kBlkThreads + threadIdx.x) * 8;
+            float gv[8], x[8], wv[8];
+            if (k < d) {
+                ld_vec<8>(gr + k, gv);
+                ld_vec<8>(hr + k, x);
+                ld_vec<8>(w + k, wv);
+            } else {
+#pragma unroll
+                for (int q = 0; q < 8; ++q) gv[q] = x[q] = wv[q] = 0.f;
+            }
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                wg[8 * v + q] = wv[q] * gv[q];
+                xh[8 * v + q] = x[q] * inv_r;
+                c = fmaf(xh[8 * v + q], wg[8 * v + q], c);
+            }
+        }
+        const float kd = block_sum2(c, 0.f).x / static_cast<float>(d);
+        const float pref = 1.0f / fmaxf(r, min_rms);
+        __nv_bfloat16* orow = out + static_cast<size_t>(row) * d;
+#pragma unroll
+        for (int v = 0; v < NV; ++v) {
+            const int k = (v * kBlkThreads + threadIdx.x) * 8;
+            if (k < d) {
+                float o[8];
+#pragma unroll
+                for (int q = 0; q < 8; ++q) o[q] = (wg[8 * v + q] - xh[8 * v + q] * kd) * pref;
+                st_vec<8>(orow + k, o);
+            }
+        }
+    }
+}
+
+template <int EPT>
+__global__ void __launch_bounds__(kBlkThreads)
+    rmsnorm_vjp_at_row_kernel(const __nv_bfloat16* __restrict__ g,
+                              const __nv_bfloat16* __restrict__ x,
+                              const __nv_bfloat16* __restrict__ gamma, int T, int d, float eps,
+                              float min_rms, __nv_bfloat16* __restrict__ out) {
+    constexpr int NV = EPT / 8;
+    for (int row = blockIdx.x; row < T; row += gridDim.x) {
+        const __nv_bfloat16* gr = g + static_cast<size_t>(row) * d;
+        const __nv_bfloat16* xr = x + static_cast<size_t>(row) * d;
+        float wg[EPT], xv[EPT];
+        float ss = 0.f, xg = 0.f;
+#pragma unroll
+        for (int v = 0; v < NV; ++v) {
+            const int k = (v * kBlkThreads + threadIdx.x) * 8;
+            float gv[8], xx[8], wv[8];
+            if (k < d) {
+                ld_vec<8>(gr + k, gv);
+                ld_vec<8>(xr + k, xx);
+                ld_vec<8>(gamma + k, wv);
+            } else {
+#pragma unroll
+                for (int q = 0; q < 8; ++q) gv[q] = xx[q] = wv[q] = 0.f;
+            }
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                wg[8 * v + q] = wv[q] * gv[q];
+                xv[8 * v + q] = xx[q];
+                ss = fmaf(xx[q], xx[q], ss);
+                xg = fmaf(xx[q], wg[8 * v + q], xg);
+            }
+        }
+        const float2 sums = block_sum2(ss, xg);
+        const float r = sqrtf(sums.x / static_cast<float>(d) + eps);
+        const float inv_r = 1.0f / r;
+        const float kd = (sums.y * inv_r) / static_cast<float>(d);
+        const float pref = 1.0f / fmaxf(r, min_rms);
+        __nv_bfloat16* orow = out + static_cast<size_t>(row) * d;
+#pragma unroll
+        for (int v = 0; v < NV; ++v) {
+            const int k = (v * kBlkThreads + threadIdx.x) * 8;
+            if (k < d) {
+                float o[8];
+#pragma unroll
+                for (int q = 0; q < 8; ++q)
+                    o[q] = (wg[8 * v + q] - (xv[8 * v + q] * inv_r) * kd) * pref;
+                st_vec<8>(orow + k, o);
+            }
+        }
+    }
+}
+
+// Elements per thread of the block-per-row kernels for a bf16 row of d, or 0 when
+// the row does not fit (the warp-per-row kernels take it).
+int row_ept(int d) {
+    if (d <= 8 * kBlkThreads) return 8;
+    if (d <= 16 * kBlkThreads) return 16;
+    if (d <= 32 * kBlkThreads) return 32;
+    return 0;
+}
+
+int blk_grid(int T) {
+    DevInfo di;
+    const int sms = current_device_info(&di) ? di.sm_count : 148;
+    return T < sms * 8 ? T : sms * 8;
 }
 
 template <typename TT, int VEC>
@@ -533,7 +739,22 @@ cudaError_t launch_rmsnorm_fwd(int dtype, const void* h, const void* w, int T, i
                                cudaStream_t st, const void* W_U, float* anchor) {
     if (T <= 0) return cudaSuccess;
     const int grid = row_grid(T);
-    if (dtype == 1) {
+    const int ept = dtype == 1 ? row_ept(d) : 0;
+    if (ept) {
+        const auto* hh = static_cast<const __nv_bfloat16*>(h);
+        const auto* ww = static_cast<const __nv_bfloat16*>(w);
+        auto* yy = static_cast<__nv_bfloat16*>(yhat);
+        const auto* wu = static_cast<const __nv_bfloat16*>(W_U);
+        if (ept == 8)
+            rmsnorm_fwd_row_kernel<8><<<blk_grid(T), kBlkThreads, 0, st>>>(
+                hh, ww, T, d, eps, yy, rho, y, V, status, wu, anchor);
+        else if (ept == 16)
+            rmsnorm_fwd_row_kernel<16><<<blk_grid(T), kBlkThreads, 0, st>>>(
+                hh, ww, T, d, eps, yy, rho, y, V, status, wu, anchor);
+        else
+            rmsnorm_fwd_row_kernel<32><<<blk_grid(T), kBlkThreads, 0, st>>>(
+                hh, ww, T, d, eps, yy, rho, y, V, status, wu, anchor);
+    } else if (dtype == 1) {
         rmsnorm_fwd_kernel<__nv_bfloat16, 8><<<grid, kRowThreads, 0, st>>>(
             static_cast<const __nv_bfloat16*>(h), static_cast<const __nv_bfloat16*>(w), T, d, eps,
             static_cast<__nv_bfloat16*>(yhat), rho, y, V, status,
@@ -592,7 +813,21 @@ cudaError_t launch_rmsnorm_vjp(int dtype, const float* g, const void* h, const v
                                cudaStream_t st) {
     if (T <= 0) return cudaSuccess;
     const int grid = row_grid(T);
-    if (dtype == 1) {
+    const int ept = dtype == 1 ? row_ept(d) : 0;
+    if (ept) {
+        const auto* hh = static_cast<const __nv_bfloat16*>(h);
+        const auto* ww = static_cast<const __nv_bfloat16*>(w);
+        auto* oo = static_cast<__nv_bfloat16*>(out);
+        if (ept == 8)
+            rmsnorm_vjp_row_kernel<8><<<blk_grid(T), kBlkThreads, 0, st>>>(g, hh, ww, rho, T, d,
+                                                                        min_rms, oo);
+        else if (ept == 16)
+            rmsnorm_vjp_row_kernel<16><<<blk_grid(T), kBlkThreads, 0, st>>>(g, hh, ww, rho, T, d,
+                                                                         min_rms, oo);
+        else
+            rmsnorm_vjp_row_kernel<32><<<blk_grid(T), kBlkThreads, 0, st>>>(g, hh, ww, rho, T, d,
+                                                                         min_rms, oo);
+    } else if (dtype == 1) {
         rmsnorm_vjp_kernel<__nv_bfloat16, 8><<<grid, kRowThreads, 0, st>>>(
             g, static_cast<const __nv_bfloat16*>(h), static_cast<const __nv_bfloat16*>(w), rho, T,
             d, min_rms, static_cast<__nv_bfloat16*>(out));
@@ -642,7 +877,22 @@ cudaError_t launch_rmsnorm_vjp_at(int dtype, const void* g, const void* x, const
                                   cudaStream_t st) {
     if (T <= 0) return cudaSuccess;
     const int grid = row_grid(T);
-    if (dtype == 1) {
+    const int ept = dtype == 1 ? row_ept(d) : 0;
+    if (ept) {
+        const auto* gg = static_cast<const __nv_bfloat16*>(g);
+        const auto* xx = static_cast<const __nv_bfloat16*>(x);
+        const auto* ga = static_cast<const __nv_bfloat16*>(gamma);
+        auto* oo = static_cast<__nv_bfloat16*>(out);
+        if (ept == 8)
+            rmsnorm_vjp_at_row_kernel<8><<<blk_grid(T), kBlkThreads, 0, st>>>(gg, xx, ga, T, d, eps,
+                                                                           min_rms, oo);
+        else if (ept == 16)
+            rmsnorm_vjp_at_row_kernel<16><<<blk_grid(T), kBlkThreads, 0, st>>>(gg, xx, ga, T, d,
+                                                                            eps, min_rms, oo);
+        else
+            rmsnorm_vjp_at_row_kernel<32><<<blk_grid(T), kBlkThreads, 0, st>>>(gg, xx, ga, T, d,
+                                                                            eps, min_rms, oo);
+    } else if (dtype == 1) {
         rmsnorm_vjp_at_kernel<__nv_bfloat16, 8><<<grid, kRowThreads, 0, st>>>(
             static_cast<const __nv_bfloat16*>(g), static_cast<const __nv_bfloat16*>(x),
             static_cast<const __nv_bfloat16*>(gamma), T, d, eps, min_rms,
