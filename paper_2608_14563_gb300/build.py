@@ -33,7 +33,7 @@ def _nvcc() -> str:
 
 def _headers_mtime() -> float:
     hs = glob.glob(os.path.join(CSRC, "*.cuh")) + glob.glob(os.path.join(CSRC, "*.h"))
-    hs.append(os.path.join(ROOT, "include", "fpo.h"))
+    hs += glob.glob(os.path.join(ROOT, "include", "*.h"))
     return max(os.path.getmtime(h) for h in hs)
 
 
