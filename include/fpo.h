@@ -11,7 +11,13 @@
  *     (or one fpo_layer_update_grouped call for all target layers)
  *
  * and the layer-viability diagnostic of Sec. 2.2 reduces pairs of gradients
- * with fpo_cosine.
+ * with fpo_cosine (one pair) or fpo_cosine_grouped (every layer in one call).
+ * Further entry points cover the rest of the method around that step: the
+ * post-FFN RMSNorm VJP and per-layer signals (fpo_rmsnorm_vjp,
+ * fpo_layer_update_grouped_signals), optimizers with the relative clip
+ * (fpo_layer_optimize_grouped), the gate/up signals through the cached
+ * W3_init (fpo_gate_up_signals) and the App. C update-magnitude ratio
+ * (fpo_norm_ratio).
  *
  * Conventions (all entry points)
  * ------------------------------
