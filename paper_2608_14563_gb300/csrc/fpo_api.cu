@@ -73,7 +73,8 @@ int32_t cuda_status(cudaError_t e) { return e == cudaSuccess ? FPO_OK : FPO_ERR_
 
 // ------------------------------------------------------------------ error signal
 struct EsLayout {
-    size_t yhat, rho, lse, zy, ce, part, g, E, z, anchor, sx, alpha, beta, fix, fix_count, total;
+    size_t yhat, rho, lse, zy, ce, part, g, E, z, anchor, sx, alpha, beta, fix, fix_count, sk,
+        total;
     int n_tiles;
     int64_t Tc;
     int algo;  // the algorithm that runs: FPO_ES_RECOMPUTE, _STORED_LOGITS or _DIRECT
@@ -128,6 +129,8 @@ EsLayout es_layout(const fpo_error_signal_desc* d) {
     L.beta = off;      off = align_up(off + Tdir * 4);
     L.fix = off;       off = align_up(off + Tcdir * 4);
     L.fix_count = off; off = align_up(off + (direct ? 4 : 0));
+    // the projection's stream-K tail (cut tiles' partial sums), bf16 tensor-core path
+    L.sk = off;        off = align_up(off + (d->dtype == FPO_BF16 ? proj_sk_scratch_bytes() : 0));
     L.total = off;
     return L;
 }
@@ -200,6 +203,7 @@ int32_t fpo_error_signal(const fpo_error_signal_desc* desc, const void* h, const
     float2* part = reinterpret_cast<float2*>(ws + L.part);
     float* g = reinterpret_cast<float*>(ws + L.g);
     void* E = ws + L.E;
+    float* sk = reinterpret_cast<float*>(ws + L.sk);
 
     auto mark = [&](int i) -> cudaError_t {
         if (!desc->stage_events || !desc->stage_events[i]) return cudaSuccess;
@@ -243,7 +247,7 @@ int32_t fpo_error_signal(const fpo_error_signal_desc* desc, const void* h, const
                                         st));
             if (last) FPO_TRY(mark(4));
             FPO_TRY(launch_proj_direct_bf16(E, W_U, targets + c0, alpha + c0, beta + c0, tc, d, V,
-                                            g + c0 * d, status, st));
+                                            g + c0 * d, sk, status, st));
         }
     } else if (L.algo == FPO_ES_RECOMPUTE) {
         // 2. logits pass over all tokens: per-vocabulary-tile (max, sum exp) partials -> lse
@@ -266,7 +270,7 @@ int32_t fpo_error_signal(const fpo_error_signal_desc* desc, const void* h, const
                 FPO_TRY(launch_error_bf16(yh, W_U, targets + c0, lse + c0, tc, d, V,
                                           desc->loss_scale, E, status, st));
                 if (c0 + tc >= T) FPO_TRY(mark(4));
-                FPO_TRY(launch_proj_bf16(E, W_U, tc, d, V, g + c0 * d, status, st));
+                FPO_TRY(launch_proj_bf16(E, W_U, tc, d, V, g + c0 * d, sk, status, st));
             } else {
                 FPO_TRY(launch_error_f32(static_cast<const float*>(yh),
                                          static_cast<const float*>(W_U), targets + c0, lse + c0,
@@ -301,7 +305,7 @@ int32_t fpo_error_signal(const fpo_error_signal_desc* desc, const void* h, const
                                              desc->loss_scale, E, st));
             if (last) FPO_TRY(mark(4));
             if (bf16)
-                FPO_TRY(launch_proj_bf16(E, W_U, tc, d, V, g + c0 * d, status, st));
+                FPO_TRY(launch_proj_bf16(E, W_U, tc, d, V, g + c0 * d, sk, status, st));
             else
                 FPO_TRY(launch_proj_f32(static_cast<const float*>(E), static_cast<const float*>(W_U),
                                         tc, d, V, g + c0 * d, st));

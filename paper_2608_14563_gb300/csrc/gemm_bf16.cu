@@ -91,6 +91,9 @@ GemmShape make_shape(int M, int N, int K, int BN, int groups, int band, int BM =
     sh.groups = groups;
     sh.band = band;
     sh.tiles = static_cast<long long>(groups) * sh.m_blocks * sh.n_blocks;
+    sh.tail_tiles = 0;
+    sh.tail_split = 0;
+    sh.sk_scratch = nullptr;
     return sh;
 }
 
@@ -126,10 +129,46 @@ int pair_clusters(Kern kern, int smem_bytes, int sm_count) {
     return n;
 }
 
+// Split-K tail of one launch: tail_tiles tiles, each in tail_split k ranges (0: whole).
+struct SkPlan {
+    long long tail_tiles = 0;
+    int tail_split = 0;
+};
+
+// Units of split tail tiles a scratch area must hold: up to three waves of pair clusters.
+constexpr int kTailWaves = 3;
+
+// The split of the last partial wave of `tiles` tiles over `clusters` clusters: R tail
+// tiles in S k ranges, S chosen so that the R S units fill whole waves as nearly as
+// possible (at most kTailWaves waves, at least 8 k-blocks per range); none if no split
+// beats the plain partial wave.
+SkPlan tail_plan(long long tiles, long long clusters, int k_blocks) {
+    SkPlan p;
+    const long long R = tiles % clusters;
+    if (tiles < clusters || R == 0) return p;
+    double best = static_cast<double>(R) / clusters;  // busy fraction of the plain last wave
+    for (int S = 2; S <= 64; ++S) {
+        if (R * S > kTailWaves * clusters || k_blocks / S < 8) break;
+        const long long waves = (R * S + clusters - 1) / clusters;
+        const double eff = static_cast<double>(R * S) / (waves * clusters);
+        if (eff > best + 1e-9) {
+            best = eff;
+            p.tail_tiles = R;
+            p.tail_split = S;
+        }
+    }
+    return p;
+}
+
+// With sk_scratch non-null, the tiles of the last partial wave are split by tail_plan
+// (SegCursor); the caller then runs sk_fixup over them (plan->tail_tiles > 0).
+// sk_scratch holds kTailWaves x clusters x 256 x BN fp32.
 template <int BN, bool A_MN, bool B_MN, int STAGES, int MAXG, class Epi>
 cudaError_t run_gemm_pair(const GemmMaps<MAXG>& maps, const typename Epi::Params& ep,
-                          const GemmShape& sh, unsigned* status, cudaStream_t st) {
-    if (sh.tiles <= 0 || sh.k_blocks <= 0) return cudaSuccess;
+                          const GemmShape& sh_in, unsigned* status, cudaStream_t st,
+                          float* sk_scratch = nullptr, SkPlan* plan = nullptr) {
+    if (plan) *plan = SkPlan{};
+    if (sh_in.tiles <= 0 || sh_in.k_blocks <= 0) return cudaSuccess;
     using L = GemmPairSmem<BN, STAGES>;
     auto kern = tc_gemm_pair_kernel<BN, A_MN, B_MN, STAGES, MAXG, Epi>;
     static cudaError_t attr_err =
@@ -138,13 +177,90 @@ cudaError_t run_gemm_pair(const GemmMaps<MAXG>& maps, const typename Epi::Params
     DevInfo di;
     if (!current_device_info(&di)) return cudaErrorUnknown;
     static int max_clusters = pair_clusters(kern, L::kBytes, di.sm_count);
-    const long long clusters = sh.tiles < max_clusters ? sh.tiles : max_clusters;
+    const long long clusters = sh_in.tiles < max_clusters ? sh_in.tiles : max_clusters;
+    GemmShape sh = sh_in;
+    if (sk_scratch) {
+        const SkPlan p = tail_plan(sh.tiles, clusters, sh.k_blocks);
+        if (p.tail_tiles > 0) {
+            sh.tail_tiles = p.tail_tiles;
+            sh.tail_split = p.tail_split;
+            sh.sk_scratch = sk_scratch;
+            if (plan) *plan = p;
+        }
+    }
     kern<<<static_cast<unsigned>(2 * clusters), kGemmThreads, L::kBytes, st>>>(maps, ep, sh, status,
                                                                               wait_limit_ns());
     return cudaGetLastError();
 }
 
+// Sum the tail_split k-range partials of every split tail tile in range order, then the
+// projection epilogue: C[row, n] = alpha_row * sum + beta_row * W_U[y_row, n]
+// (alpha == nullptr: the plain sum), as EpiProjDirect / EpiStoreF32 form whole tiles.
+// Grid (tail tiles, 256 rows / rows per block): one thread per 4 columns of a row.
+constexpr int kFixupThreads = 256;
+
+template <int BN>
+__global__ void __launch_bounds__(kFixupThreads)
+    sk_fixup_kernel(const GemmShape sh, const float* __restrict__ scratch,
+                    float* __restrict__ C, const float* __restrict__ alpha,
+                    const float* __restrict__ beta, const int* __restrict__ y,
+                    const __nv_bfloat16* __restrict__ W_U) {
+    constexpr int kThreadsPerRow = BN / 4;
+    constexpr int kRowsPerBlock = kFixupThreads / kThreadsPerRow;
+    const long long R = sh.tail_tiles;
+    const long long r_tile = blockIdx.x;
+    const int r = blockIdx.y * kRowsPerBlock + threadIdx.x / kThreadsPerRow;
+    const int col = (threadIdx.x % kThreadsPerRow) * 4;
+    int g, mp, nb;
+    tile_coords(sh.tiles - R + r_tile, sh, g, mp, nb);
+    const int row = mp * kPairBM + r;
+    const int n = nb * BN + col;
+    if (row >= sh.M || n >= sh.N) return;  // N % 8 == 0: whole float4s
+    float s4[4] = {0.f, 0.f, 0.f, 0.f};
+    for (int q = 0; q < sh.tail_split; ++q) {
+        const float4 u = *reinterpret_cast<const float4*>(
+            scratch + ((static_cast<size_t>(q) * R + r_tile) * kPairBM + r) * BN + col);
+        s4[0] += u.x;
+        s4[1] += u.y;
+        s4[2] += u.z;
+        s4[3] += u.w;
+    }
+    const float a = alpha ? alpha[row] : 1.f;
+    const float bb = alpha ? beta[row] : 0.f;
+    const __nv_bfloat16* wy =
+        (a != 0.f && bb != 0.f) ? W_U + static_cast<long long>(y[row]) * sh.N : nullptr;
+    float o[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        if (a == 0.f)
+            o[j] = 0.f;
+        else if (wy)
+            o[j] = fmaf(a, s4[j], bb * __bfloat162float(wy[n + j]));
+        else
+            o[j] = a * s4[j];
+    }
+    *reinterpret_cast<float4*>(C + static_cast<size_t>(row) * sh.N + n) =
+        make_float4(o[0], o[1], o[2], o[3]);
+}
+
+template <int BN>
+cudaError_t launch_sk_fixup(const SkPlan& plan, const GemmShape& sh_in, const float* scratch,
+                            float* C, const float* alpha, const float* beta, const int* y,
+                            const void* W_U, cudaStream_t st) {
+    if (plan.tail_tiles <= 0) return cudaSuccess;
+    GemmShape sh = sh_in;
+    sh.tail_tiles = plan.tail_tiles;
+    sh.tail_split = plan.tail_split;
+    constexpr int kRowsPerBlock = kFixupThreads / (BN / 4);
+    const dim3 grid(static_cast<unsigned>(plan.tail_tiles), kPairBM / kRowsPerBlock);
+    sk_fixup_kernel<BN><<<grid, kFixupThreads, 0, st>>>(sh, scratch, C, alpha, beta, y,
+                                                        static_cast<const __nv_bfloat16*>(W_U));
+    return cudaGetLastError();
+}
+
 constexpr int kPairStages = 6;
+constexpr int kWideBN = 512;     // pair tiles 256 x 512: 48 KB stages
+constexpr int kWideStages = 4;
 
 // 0 = single-CTA tiles, 1 = CTA-pair tiles, 2 = CTA-pair tiles with 256 x 512 tiles for
 // the projection (default: its K loop runs over the whole vocabulary, so the epilogue
@@ -174,6 +290,24 @@ void set_gemm_variant(int v) {
     g_gemm_variant.store(v >= 0 && v <= 2 ? v : 0, std::memory_order_relaxed);
 }
 int gemm_variant() { return g_gemm_variant.load(std::memory_order_relaxed); }
+
+size_t proj_sk_scratch_bytes() {
+    // kTailWaves x clusters units of 256 x 512 fp32; clusters of the 256 x 512 pair kernel
+    // on this device, or an upper bound of 128 without one
+    static const size_t bytes = [] {
+        using L = GemmPairSmem<kWideBN, kWideStages>;
+        auto kern = tc_gemm_pair_kernel<kWideBN, false, true, kWideStages, 1, EpiProjDirect>;
+        DevInfo di;
+        long long c = 128;
+        if (current_device_info(&di) &&
+            cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::kBytes) ==
+                cudaSuccess)
+            c = pair_clusters(kern, L::kBytes, di.sm_count);
+        cudaGetLastError();
+        return static_cast<size_t>(kTailWaves) * c * kPairBM * kWideBN * sizeof(float);
+    }();
+    return bytes;
+}
 
 constexpr int kLseBN = 256;
 constexpr int kLseStages = 4;
@@ -266,12 +400,11 @@ cudaError_t launch_lse_prob_bf16(const void* yhat, const void* W_U, const int32_
 
 constexpr int kProjBN = 256;
 constexpr int kProjStages = 4;
-constexpr int kWideBN = 512;     // pair tiles 256 x 512: 48 KB stages
-constexpr int kWideStages = 4;
 
 cudaError_t launch_proj_direct_bf16(const void* P, const void* W_U, const int32_t* y,
                                     const float* alpha, const float* beta, int Tc, int d, int V,
-                                    float* g, unsigned* status, cudaStream_t st) {
+                                    float* g, float* sk_scratch, unsigned* status,
+                                    cudaStream_t st) {
     GemmMaps<1> maps;
     if (!map_kmajor(&maps.a[0], P, Tc, V, kBM) || !map_mnmajor(&maps.b[0], W_U, V, d))
         return cudaErrorInvalidValue;
@@ -283,9 +416,14 @@ cudaError_t launch_proj_direct_bf16(const void* P, const void* W_U, const int32_
     ep.W_U = static_cast<const __nv_bfloat16*>(W_U);
     ep.M = Tc;
     ep.N = d;
-    if (wide_proj())
-        return run_gemm_pair<kWideBN, false, true, kWideStages, 1, EpiProjDirect>(
-            maps, ep, make_shape(Tc, d, V, kWideBN, 1, band_for(true), kPairBM), status, st);
+    if (wide_proj()) {
+        const GemmShape sh = make_shape(Tc, d, V, kWideBN, 1, band_for(true), kPairBM);
+        SkPlan plan;
+        cudaError_t e = run_gemm_pair<kWideBN, false, true, kWideStages, 1, EpiProjDirect>(
+            maps, ep, sh, status, st, sk_scratch, &plan);
+        if (e != cudaSuccess) return e;
+        return launch_sk_fixup<kWideBN>(plan, sh, sk_scratch, g, alpha, beta, y, W_U, st);
+    }
     if (use_pair())
         return run_gemm_pair<kProjBN, false, true, kPairStages, 1, EpiProjDirect>(
             maps, ep, make_shape(Tc, d, V, kProjBN, 1, band_for(true), kPairBM), status, st);
@@ -294,7 +432,7 @@ cudaError_t launch_proj_direct_bf16(const void* P, const void* W_U, const int32_
 }
 
 cudaError_t launch_proj_bf16(const void* E, const void* W_U, int Tc, int d, int V, float* g,
-                             unsigned* status, cudaStream_t st) {
+                             float* sk_scratch, unsigned* status, cudaStream_t st) {
     GemmMaps<1> maps;
     if (!map_kmajor(&maps.a[0], E, Tc, V, kBM) || !map_mnmajor(&maps.b[0], W_U, V, d))
         return cudaErrorInvalidValue;
@@ -302,9 +440,15 @@ cudaError_t launch_proj_bf16(const void* E, const void* W_U, int Tc, int d, int 
     if (!map_out_f32(&ep.Cmap, g, Tc, d)) return cudaErrorInvalidValue;
     ep.M = Tc;
     ep.N = d;
-    if (wide_proj())
-        return run_gemm_pair<kWideBN, false, true, kWideStages, 1, EpiStoreF32>(
-            maps, ep, make_shape(Tc, d, V, kWideBN, 1, band_for(true), kPairBM), status, st);
+    if (wide_proj()) {
+        const GemmShape sh = make_shape(Tc, d, V, kWideBN, 1, band_for(true), kPairBM);
+        SkPlan plan;
+        cudaError_t e = run_gemm_pair<kWideBN, false, true, kWideStages, 1, EpiStoreF32>(
+            maps, ep, sh, status, st, sk_scratch, &plan);
+        if (e != cudaSuccess) return e;
+        return launch_sk_fixup<kWideBN>(plan, sh, sk_scratch, g, nullptr, nullptr, nullptr,
+                                        nullptr, st);
+    }
     if (use_pair())
         return run_gemm_pair<kProjBN, false, true, kPairStages, 1, EpiStoreF32>(
             maps, ep, make_shape(Tc, d, V, kProjBN, 1, band_for(true), kPairBM), status, st);

@@ -36,9 +36,11 @@ cudaError_t launch_error_bf16(const void* yhat, const void* W_U, const int32_t* 
                               int Tc, int d, int V, float s, void* E, unsigned* status,
                               cudaStream_t st);
 
-// Projection: g[Tc, d] = E[Tc, V] W_U (fp32 out).
+// Projection: g[Tc, d] = E[Tc, V] W_U (fp32 out).  sk_scratch: proj_sk_scratch_bytes() of
+// device memory for the split-K tail of the 256 x 512 kernel (or null: whole tiles only).
 cudaError_t launch_proj_bf16(const void* E, const void* W_U, int Tc, int d, int V, float* g,
-                             unsigned* status, cudaStream_t st);
+                             float* sk_scratch, unsigned* status, cudaStream_t st);
+size_t proj_sk_scratch_bytes();
 
 // Direct algorithm, logits pass: as launch_lse_partial_bf16 (z never stored), plus
 // P[T, V] = exp(z - anchor) in bf16 with the target column zero, and sx[T, part_ld]
@@ -50,7 +52,8 @@ cudaError_t launch_lse_prob_bf16(const void* yhat, const void* W_U, const int32_
 // Direct algorithm, projection: g[Tc, d] = alpha (.) (P W_U) + beta (.) W_U[y] (row-wise).
 cudaError_t launch_proj_direct_bf16(const void* P, const void* W_U, const int32_t* y,
                                     const float* alpha, const float* beta, int Tc, int d, int V,
-                                    float* g, unsigned* status, cudaStream_t st);
+                                    float* g, float* sk_scratch, unsigned* status,
+                                    cudaStream_t st);
 
 // Grouped pseudogradient update over n layers, layer l with signal g[l] (host array).
 cudaError_t launch_update_bf16(int n, int T, int d, int d_ff, const void* const* g,

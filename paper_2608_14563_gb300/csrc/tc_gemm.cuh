@@ -36,6 +36,12 @@ struct GemmShape {
     int groups;        // independent problems with equal shapes (target layers)
     int band;          // rasterisation band height in m-blocks (L2 reuse)
     long long tiles;   // groups * m_blocks * n_blocks
+    // Split-K tail (pair kernel only): the last tail_tiles tiles (less than one wave)
+    // are each split into tail_split equal k-block ranges, and every range leaves its
+    // fp32 sums in sk_scratch ([unit][256][BN]) for a fixup kernel.  0 = whole tiles.
+    long long tail_tiles;
+    int tail_split;
+    float* sk_scratch;
 };
 
 template <int MAXG>

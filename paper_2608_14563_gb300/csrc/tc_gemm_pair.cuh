@@ -78,6 +78,45 @@ __device__ __forceinline__ bool mbar_wait_cl_drain(uint32_t bar, uint32_t parity
     return true;
 }
 
+// The work of one pair cluster as a sequence of segments (tile, k-blocks [kb0, kb1)).
+// Tiles [0, tiles - tail_tiles) are whole and dealt round robin (cluster c takes c,
+// c + C, ...: concurrent tiles are neighbours in the rasterisation and stream the same
+// k-blocks, sharing operands in L2).  The tail_tiles = R tiles of the last, partial
+// wave are each split into S = tail_split equal k-block ranges; the R S units, ordered
+// by range then tile (so concurrent units stream the same k-blocks), are dealt round
+// robin too, and unit u leaves its sums in slot u.  part = -1 marks a whole tile.
+// Every role of every CTA walks the same sequence.
+struct SegCursor {
+    long long C, t, u;
+
+    __device__ __forceinline__ SegCursor(const GemmShape&, long long c, long long C_)
+        : C(C_), t(c), u(c) {}
+
+    __device__ __forceinline__ bool next(const GemmShape& sh, long long& tile, int& kb0, int& kb1,
+                                         int& part, int& slot) {
+        const long long dp = sh.tiles - sh.tail_tiles;
+        if (t < dp) {
+            tile = t;
+            kb0 = 0;
+            kb1 = sh.k_blocks;
+            part = -1;
+            slot = -1;
+            t += C;
+            return true;
+        }
+        const long long R = sh.tail_tiles, S = sh.tail_split;
+        if (u >= R * S) return false;
+        const long long q = u / R;
+        tile = dp + (u - q * R);
+        kb0 = static_cast<int>((q * sh.k_blocks) / S);
+        kb1 = static_cast<int>(((q + 1) * sh.k_blocks) / S);
+        part = static_cast<int>(q);
+        slot = static_cast<int>(u);
+        u += C;
+        return true;
+    }
+};
+
 // One CTA's half of an operand k-block, counted on the leader's barrier.
 template <bool MN, int ROWS>
 __device__ __forceinline__ void load_operand_pair(const CUtensorMap* map, uint32_t dst,
@@ -162,14 +201,17 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
             uint32_t phase = 0;
             uint32_t issued_mask = 0, issued_parity = 0;
             bool ok = true;
-            for (long long t = cluster; t < sh.tiles && ok; t += n_clusters) {
+            SegCursor seg(sh, cluster, n_clusters);
+            long long t;
+            int kb0, kb1, part, slot;
+            while (ok && seg.next(sh, t, kb0, kb1, part, slot)) {
                 int g, mp, nb;
                 tile_coords(t, sh, g, mp, nb);
                 const CUtensorMap* amap = &maps.a[MAXG == 1 ? 0 : g];
                 const CUtensorMap* bmap = &maps.b[MAXG == 1 ? 0 : g];
                 const int a_row = mp * kPairBM + 128 * static_cast<int>(rank);
                 const int b_row = nb * BN + kBSub * static_cast<int>(rank);
-                for (int kb = 0; kb < sh.k_blocks; ++kb) {
+                for (int kb = kb0; kb < kb1; ++kb) {
                     if (!mbar_wait_cl(empty_bar(stage), phase ^ 1u, guard)) { ok = false; break; }
                     const uint32_t sa = sbase + stage * L::kStageBytes;
                     const uint32_t sb = sa + L::kABytes;
@@ -202,11 +244,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
             int acc = 0;
             uint32_t acc_phase = 0;
             bool ok = true, issued_any = false;
-            for (long long t = cluster; t < sh.tiles && ok; t += n_clusters) {
+            SegCursor seg(sh, cluster, n_clusters);
+            long long t;
+            int kb0, kb1, part, slot;
+            while (ok && seg.next(sh, t, kb0, kb1, part, slot)) {
                 if (!mbar_wait_cl(tempty_bar(acc), acc_phase ^ 1u, guard)) { ok = false; break; }
                 tc_fence_after();
                 const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * BN);
-                for (int kb = 0; kb < sh.k_blocks; ++kb) {
+                for (int kb = kb0; kb < kb1; ++kb) {
                     if (!mbar_wait_cl(full_bar(stage), phase, guard)) { ok = false; break; }
                     tc_fence_after();
                     const uint32_t sa = sbase + stage * L::kStageBytes;
@@ -217,7 +262,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
                         for (int h = 0; h < kNSub; ++h)
                             tc_mma_bf16_pair(d_tmem + 256u * h, operand_desc<A_MN>(sa, kk),
                                              operand_desc<B_MN>(sb + h * kBSubBytes, kk), kIdesc,
-                                             (kb | kk) != 0 ? 1u : 0u);
+                                             (kb != kb0 || kk != 0) ? 1u : 0u);
                     issued_any = true;
                     tc_commit_pair_multicast(empty_bar(stage), kBoth);
                     if (++stage == STAGES) { stage = 0; phase ^= 1u; }
@@ -240,24 +285,41 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
                  0, 0u};
         int acc = 0;
         uint32_t acc_phase = 0;
-        for (long long t = cluster; t < sh.tiles; t += n_clusters) {
+        SegCursor seg(sh, cluster, n_clusters);
+        long long t;
+        int kb0, kb1, part, slot;
+        while (seg.next(sh, t, kb0, kb1, part, slot)) {
             int g, mp, nb;
             tile_coords(t, sh, g, mp, nb);
             if (!mbar_wait_cl(tfull_bar(acc), acc_phase, guard)) break;
             tc_fence_after();
-            const int row = mp * kPairBM + r_in_tile;
-            const int n0 = nb * BN;
-            io.row0 = mp * kPairBM + 128 * static_cast<int>(rank) + q * 32;
-            Epi epi(ep, g, row, n0);
             const uint32_t t_row = tmem_base + (static_cast<uint32_t>(q * 32) << 16) +
                                    static_cast<uint32_t>(acc * BN);
+            if (part < 0) {
+                const int row = mp * kPairBM + r_in_tile;
+                const int n0 = nb * BN;
+                io.row0 = mp * kPairBM + 128 * static_cast<int>(rank) + q * 32;
+                Epi epi(ep, g, row, n0);
 #pragma unroll 1
-            for (int c = 0; c < BN / 32; ++c) {
-                float v[32];
-                tmem_ld_32x32b_x32(t_row + c * 32, v);
-                epi.chunk(ep, v, n0 + c * 32, c * 32, io);
+                for (int c = 0; c < BN / 32; ++c) {
+                    float v[32];
+                    tmem_ld_32x32b_x32(t_row + c * 32, v);
+                    epi.chunk(ep, v, n0 + c * 32, c * 32, io);
+                }
+                epi.finish(ep, nb);
+            } else {
+                // one k range of a split tile: its raw fp32 sums, row r_in_tile, to its slot
+                float* dst = sh.sk_scratch + (static_cast<size_t>(slot) * kPairBM + r_in_tile) * BN;
+#pragma unroll 1
+                for (int c = 0; c < BN / 32; ++c) {
+                    float v[32];
+                    tmem_ld_32x32b_x32(t_row + c * 32, v);
+                    float4* d4 = reinterpret_cast<float4*>(dst + c * 32);
+#pragma unroll
+                    for (int q4 = 0; q4 < 8; ++q4)
+                        d4[q4] = make_float4(v[4 * q4], v[4 * q4 + 1], v[4 * q4 + 2], v[4 * q4 + 3]);
+                }
             }
-            epi.finish(ep, nb);
             tc_fence_before();
             __syncwarp();
             if (lane == 0) {

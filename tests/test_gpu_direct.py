@@ -76,6 +76,8 @@ def test_auto_is_direct_for_bf16(fpo, ragged):
 
 
 def test_direct_is_bitwise_identical_across_token_chunks(fpo, ragged):
+    """Whole tiles only at this size (the projection's split-K tail needs at least one
+    wave of tiles; with it, split tiles depend on the chunk: see the split-K tail test)."""
     inp, _ = ragged
     runs = [run(fpo, inp["h"], inp["w"], inp["W_U"], inp["y"], eps=RAGGED.eps,
                 algo=fpo.ES_DIRECT, t_chunk=c) for c in (0, 128, 37)]
@@ -215,3 +217,33 @@ def test_many_rows_outside_the_window(fpo):
     for t in range(0, T, 37):
         assert rel_frob(g[t], G[t]) < TOL, t
     assert np.max(np.abs(f64(out["lse"]) - ref["lse"]) / np.maximum(1, np.abs(ref["lse"]))) < 1e-5
+
+
+@pytest.mark.parametrize("algo", [2, 3])  # stored logits, direct
+def test_projection_split_k_tail(fpo, algo):
+    """A projection of 20 x 8 tiles of 256 x 512 (T 5120, d 4096): 160 tiles are not a whole
+    number of waves of the pair clusters, so the tiles of the last partial wave are split
+    into k-block ranges and summed by the fixup kernel.  Checked against whole tiles (the
+    256 x 256 kernel), against the oracle, across chunkings and for repeatability."""
+    wl = Workload("sk", T=5120, d=4096, d_ff=8, V=2048, layers=1, targets="zipf")
+    inp = synth.make_all(wl)
+    h, w, W_U, y = inp["h"], inp["w"], inp["W_U"], inp["y"]
+    prev = fpo.set_gemm_variant(2)
+    try:
+        a = run(fpo, h, w, W_U, y, eps=wl.eps, algo=algo)
+        a2 = run(fpo, h, w, W_U, y, eps=wl.eps, algo=algo)
+        ac = run(fpo, h, w, W_U, y, eps=wl.eps, algo=algo, t_chunk=1000)
+        fpo.set_gemm_variant(1)
+        b = run(fpo, h, w, W_U, y, eps=wl.eps, algo=algo)
+    finally:
+        fpo.set_gemm_variant(prev)
+    assert torch.equal(a["g"], a2["g"])  # deterministic
+    ga, gb, gc = f64(a["g"]), f64(b["g"]), f64(ac["g"])
+    # g~ is bf16: summing a cut tile's two fp32 parts reassociates the K sum, which flips
+    # the bf16 rounding of a few elements (a wrong part would be off by O(1) on a tile)
+    for x, y_ in ((ga, gb), (gc, ga)):
+        assert rel_frob(x, y_) < 2e-4
+        row_err = np.linalg.norm(x - y_, axis=1) / np.linalg.norm(y_, axis=1)
+        assert np.max(row_err) < 5e-3
+    ref = reference(h, w, W_U, y, eps=wl.eps, s=wl.loss_scale)
+    assert rel_frob(ga, ref["g_tilde"]) < TOL and cos(ga, ref["g_tilde"]) >= COS_MIN
