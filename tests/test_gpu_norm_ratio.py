@@ -2,7 +2,6 @@
 relative step, Sec. C.2) against the oracle on the same seeded inputs."""
 import math
 
-import numpy as np
 import pytest
 import torch
 

@@ -5,7 +5,6 @@ Tolerances (Sec. 3.1 / App. A quantities):
   weights (and on the step dW = W' - W), cos(G_gpu, G_oracle) >= 0.9995.
 * fp32 path: relative Frobenius error <= 1e-5 on the same quantities.
 """
-import math
 
 import numpy as np
 import pytest
