@@ -486,8 +486,11 @@ def run_fpo(args, wl):
         def prefetch(b):
             copy_stream.wait_event(freed[b])
             with torch.cuda.stream(copy_stream):
-                for d_t, h_t in zip(flat(sets[b]), host):
-                    d_t.copy_(h_t, non_blocking=True)
+                if args.e2e_copy == "sm":
+                    fpo.h2d_copy(flat(sets[b]), host, stream=copy_stream)
+                else:
+                    for d_t, h_t in zip(flat(sets[b]), host):
+                        d_t.copy_(h_t, non_blocking=True)
                 ready[b].record(copy_stream)
 
         def e2e_step(i):
@@ -516,6 +519,8 @@ def run_fpo(args, wl):
         h2d = sum(t.numel() * t.element_size() for t in host)
         e2e = {"value": whole_job_tokens_per_s(wl.T, world, e2e_ms), "unit": "tokens/s",
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": 4, "ms_per_step": e2e_ms,
+               "copy": ("fpo_h2d_copy: SM loads of mapped pinned memory, one launch per step"
+                        if args.e2e_copy == "sm" else "copy engines: one cudaMemcpyAsync per tensor"),
                "pipeline": f"all step inputs H2D from pinned memory each step, {depth} device "
                            "sets: copies run on a copy stream up to "
                            f"{depth - 1} steps ahead of compute; loss D2H"}
@@ -661,6 +666,9 @@ def main():
                     help="add the App. C update-magnitude ratio ||G_l||/||W_l|| to every step")
     ap.add_argument("--e2e-depth", type=int, default=3,
                     help="device input sets of the end-to-end loop (copies run depth-1 steps ahead)")
+    ap.add_argument("--e2e-copy", choices=("sm", "ce"), default="sm",
+                    help="end-to-end input copies: sm = fpo_h2d_copy (SM loads of mapped pinned "
+                         "memory, one launch per step), ce = cudaMemcpyAsync per tensor")
     ap.add_argument("--band", type=int, default=0,
                     help="GEMM rasterisation band height in tiles (0: library default; tuning)")
     ap.add_argument("--gemm-variant", type=int, choices=(-1, 0, 1, 2), default=-1,

@@ -17,7 +17,7 @@
  * fpo_layer_update_grouped_signals), optimizers with the relative clip
  * (fpo_layer_optimize_grouped), the gate/up signals through the cached
  * W3_init (fpo_gate_up_signals) and the App. C update-magnitude ratio
- * (fpo_norm_ratio).
+ * (fpo_norm_ratio).  fpo_h2d_copy stages a step's inputs from host memory.
  *
  * Conventions (all entry points)
  * ------------------------------
@@ -56,6 +56,9 @@ extern "C" {
 
 /* Largest number of layers one fpo_layer_update_grouped call accepts. */
 #define FPO_MAX_GROUPED_LAYERS 64
+
+/* Largest number of buffers one fpo_h2d_copy call accepts. */
+#define FPO_MAX_COPY_BUFFERS 64
 
 typedef enum fpo_dtype {
     FPO_F32 = 0,
@@ -400,6 +403,30 @@ size_t fpo_norm_ratio_workspace(int32_t n_layers, int64_t n);
 int32_t fpo_norm_ratio(int32_t n_layers, int64_t n, int32_t g_dtype, const void* const* G,
                        int32_t w_dtype, const void* const* W, double rel_step, double* out,
                        void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * Host-to-device copy of n buffers by SM loads, for steps whose inputs (h, the
+ * targets, the cached activations A_l) arrive in host memory.  The paper has no
+ * counterpart.  One kernel launch copies every buffer; its threads read the host
+ * memory through its device mapping, so the copy does not use the copy engines
+ * and runs beside kernels on other streams (one 256-thread block per SM, no
+ * shared memory).
+ *
+ * src[i]    host, 16-byte aligned, inside page-locked memory that is mapped into
+ *           the device address space (cudaHostAlloc / cudaMallocHost memory, or
+ *           memory registered with cudaHostRegister and cudaHostRegisterMapped)
+ * dst[i]    device, 16-byte aligned, bytes[i] bytes; no overlap with any other
+ *           dst or src of the call
+ * bytes[i]  any size (a tail under 16 bytes is copied bytewise); 0 skips the pair
+ * 0 <= n <= FPO_MAX_COPY_BUFFERS; n == 0 enqueues nothing.  Host memory must stay
+ * valid and unchanged until the copy has completed on `stream`.
+ * Errors: FPO_ERR_SHAPE (n out of range), FPO_ERR_NULL, FPO_ERR_ALIGN, FPO_ERR_ARG
+ * (the first or last byte of src[i] is not in page-locked, device-mapped host memory
+ * -- pageable memory is rejected even where a kernel could read it -- or the two do
+ * not map to one contiguous device range).
+ */
+int32_t fpo_h2d_copy(int32_t n, void* const* dst, const void* const* src, const size_t* bytes,
+                     void* stream);
 
 /*
  * Synchronise `stream`, read the device status word of `workspace` (set by the

@@ -101,6 +101,9 @@ _lib.fpo_norm_ratio_workspace.restype = _sz
 _lib.fpo_norm_ratio.argtypes = [_i32, _i64, _i32, ctypes.POINTER(_vp), _i32, ctypes.POINTER(_vp),
                                 ctypes.c_double, _vp, _vp, _sz, _vp]
 _lib.fpo_norm_ratio.restype = _i32
+_lib.fpo_h2d_copy.argtypes = [_i32, ctypes.POINTER(_vp), ctypes.POINTER(_vp),
+                              ctypes.POINTER(_sz), _vp]
+_lib.fpo_h2d_copy.restype = _i32
 _lib.fpo_testing_direct_fixup_rows.argtypes = [ctypes.POINTER(ErrorSignalDesc), _vp, _vp]
 _lib.fpo_testing_direct_fixup_rows.restype = _i64
 _lib.fpo_testing_set_gemm_variant.argtypes = [_i32]
@@ -398,6 +401,29 @@ def norm_ratio(G, W, rel_step=0.01, out=None, *, workspace=None, stream=None):
                              _stream(stream))
     _check(rc, "fpo_norm_ratio")
     return out
+
+
+MAX_COPY_BUFFERS = 64
+
+
+def h2d_copy(dsts, srcs, *, stream=None):
+    """fpo_h2d_copy: copy page-locked host tensors srcs[i] into device tensors dsts[i]
+    (contiguous, equal byte sizes) by SM loads, one kernel launch per MAX_COPY_BUFFERS
+    pairs."""
+    if len(dsts) != len(srcs):
+        raise ValueError("h2d_copy takes as many destinations as sources")
+    for d_t, s_t in zip(dsts, srcs):
+        if s_t.is_cuda or not s_t.is_contiguous():
+            raise ValueError("h2d_copy sources are contiguous host tensors")
+        if d_t.numel() * d_t.element_size() != s_t.numel() * s_t.element_size():
+            raise ValueError("h2d_copy source and destination sizes differ")
+    for c in range(0, len(srcs), MAX_COPY_BUFFERS):
+        ds, ss = dsts[c:c + MAX_COPY_BUFFERS], srcs[c:c + MAX_COPY_BUFFERS]
+        n = len(ss)
+        darr = (_vp * n)(*[_ptr(t).value for t in ds])
+        sarr = (_vp * n)(*[t.data_ptr() for t in ss])
+        barr = (_sz * n)(*[t.numel() * t.element_size() for t in ss])
+        _check(_lib.fpo_h2d_copy(n, darr, sarr, barr, _stream(stream)), "fpo_h2d_copy")
 
 
 def get_device_status(workspace, stream=None) -> int:

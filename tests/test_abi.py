@@ -128,3 +128,17 @@ def test_layer_update_and_cosine_host_validation(L):
     assert lib.fpo_cosine(10, 1, None, fake, fake, fake, 1 << 20, None) == 1
     assert lib.fpo_cosine(10, 1, mis, fake, fake, fake, 1 << 20, None) == 4
     assert lib.fpo_get_device_status(None, None) == 5
+
+
+def test_h2d_copy_host_validation(L):
+    lib = L.lib
+    vp, sz = ctypes.c_void_p, ctypes.c_size_t
+    fake, mis = 1 << 20, (1 << 20) + 8
+    one = lambda *x: (vp * len(x))(*x)   # noqa: E731
+    assert lib.fpo_h2d_copy(-1, None, None, None, None) == 2
+    assert lib.fpo_h2d_copy(65, None, None, None, None) == 2
+    assert lib.fpo_h2d_copy(0, None, None, None, None) == 0
+    assert lib.fpo_h2d_copy(1, None, one(fake), (sz * 1)(16), None) == 1
+    assert lib.fpo_h2d_copy(1, one(fake), one(None), (sz * 1)(16), None) == 1
+    assert lib.fpo_h2d_copy(1, one(fake), one(mis), (sz * 1)(16), None) == 4
+    assert lib.fpo_h2d_copy(1, one(mis), one(fake), (sz * 1)(16), None) == 4
