@@ -561,7 +561,7 @@ def run_fpo(args, wl):
             "metric": METRIC, "value": tok_s, "unit": "tokens/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
-            "data": "synthetic (seeded; OLMo-2-7B shapes, random weights and activations)",
+            "data": f"synthetic (seeded; {wl.name} workload: random weights and activations)",
             "config": workload_config(wl, args),
             "tflops": {"algorithmic": alg_tf, "executed": exe_tf,
                        "frac_of_bf16_peak_burst": alg_tf / peaks.get("bf16_tflops", 1900.0),
