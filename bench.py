@@ -199,7 +199,7 @@ def run_reference(args, wl):
     world, rank, _ = dist_setup()
     if rank != 0:
         return
-    n_tok = args.cpu_tokens
+    n_tok = args.ref_tokens
     steps = []
     for i in range(args.warmup + args.steps):
         r = oracle_sample(wl, n_tok, seed=i)
@@ -676,7 +676,11 @@ def main():
                          "2 CTA-pair tiles with a 256x512 projection, -1 library default")
     ap.add_argument("--shape", default=None,
                     help="T,d,d_ff,V,layers override of the workload's shape (small ncu cases)")
-    ap.add_argument("--cpu-tokens", type=int, default=16, help="oracle sample size (tokens)")
+    ap.add_argument("--cpu-tokens", type=int, default=256,
+                    help="tokens of the oracle sample behind cpu_baseline (~10 s of CPU work "
+                         "at the OLMo shape on 16 cores)")
+    ap.add_argument("--ref-tokens", type=int, default=32,
+                    help="tokens of the oracle sample of each --impl reference step")
     ap.add_argument("--no-cpu", action="store_true", help="skip the oracle CPU baseline")
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end run")
     args = ap.parse_args()

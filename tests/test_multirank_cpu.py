@@ -37,7 +37,8 @@ def _worker(rank, world, port, q):
         m = b.max_over_ranks(ms)
         tok = b.whole_job_tokens_per_s(16384, world, m)
         # the reference arm prints only on rank 0
-        args = type("A", (), {"cpu_tokens": 1, "warmup": 0, "steps": 0, "gpus": world})()
+        args = type("A", (), {"cpu_tokens": 1, "ref_tokens": 1, "warmup": 0, "steps": 0,
+                              "gpus": world})()
         buf = io.StringIO()
         if rank != 0:
             with contextlib.redirect_stdout(buf):
