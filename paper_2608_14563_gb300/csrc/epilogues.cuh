@@ -432,17 +432,43 @@ struct EpiSwiglu {
         long long ld;
         int M, N;
     };
-    int row;
+    static constexpr int kTileN = 256;  // columns of the tiles it runs on (both GEMM kernels)
+    int row, n_end;
     bool valid, pair_out;
+    // a and b of the chunk the next chunk() call works on: loaded one chunk ahead, so
+    // their latency overlaps the arithmetic of the chunk before (the first chunk's loads
+    // are issued by the constructor)
+    uint4 ua[4], ub[4];
 
-    __device__ __forceinline__ EpiSwiglu(const Params& p, int, int row_, int) : row(row_) {
+    __device__ __forceinline__ void fetch(const Params& p, int col0) {
+        const int lim = p.N - col0;
+        const uint4* pa = reinterpret_cast<const uint4*>(p.a + row * p.ld + col0);
+        const uint4* pb = reinterpret_cast<const uint4*>(p.b + row * p.ld + col0);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const bool in = valid && q * 8 < lim;
+            ua[q] = in ? pa[q] : make_uint4(0, 0, 0, 0);
+            ub[q] = in ? pb[q] : make_uint4(0, 0, 0, 0);
+        }
+    }
+
+    __device__ __forceinline__ EpiSwiglu(const Params& p, int, int row_, int n0) : row(row_) {
         valid = row_ < p.M;
         pair_out = false;
+        n_end = n0 + kTileN;
+        fetch(p, n0);
     }
 
     __device__ __forceinline__ void chunk(const Params& p, const float (&v)[32], int col0, int c0,
                                           EpiIO& io) {
         const bool second = (c0 & 32) != 0;
+        uint4 ca[4], cb[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            ca[q] = ua[q];
+            cb[q] = ub[q];
+        }
+        if (col0 + 32 < n_end) fetch(p, col0 + 32);
         if (!second) {
             pair_out = col0 >= p.N || io.row0 >= p.M;
             if (pair_out) return;
@@ -450,37 +476,22 @@ struct EpiSwiglu {
             __syncwarp();
         }
         if (pair_out) return;
-        const int lim = p.N - col0;
-        float av[32], bv[32];
-        const uint4* pa = reinterpret_cast<const uint4*>(p.a + row * p.ld + col0);
-        const uint4* pb = reinterpret_cast<const uint4*>(p.b + row * p.ld + col0);
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            uint4 ua = make_uint4(0, 0, 0, 0), ub = make_uint4(0, 0, 0, 0);
-            if (valid && q * 8 < lim) {
-                ua = pa[q];
-                ub = pb[q];
-            }
-            const __nv_bfloat162* ha = reinterpret_cast<const __nv_bfloat162*>(&ua);
-            const __nv_bfloat162* hb = reinterpret_cast<const __nv_bfloat162*>(&ub);
-#pragma unroll
-            for (int k = 0; k < 4; ++k) {
-                const float2 fa = __bfloat1622float2(ha[k]), fb = __bfloat1622float2(hb[k]);
-                av[8 * q + 2 * k] = fa.x;
-                av[8 * q + 2 * k + 1] = fa.y;
-                bv[8 * q + 2 * k] = fb.x;
-                bv[8 * q + 2 * k + 1] = fb.y;
-            }
-        }
         uint32_t wa[16], wb[16];
 #pragma unroll
         for (int j = 0; j < 32; j += 2) {
+            const __nv_bfloat162 ha = reinterpret_cast<const __nv_bfloat162*>(&ca[j / 8])[(j % 8) / 2];
+            const __nv_bfloat162 hb = reinterpret_cast<const __nv_bfloat162*>(&cb[j / 8])[(j % 8) / 2];
+            const float2 fa = __bfloat1622float2(ha), fb = __bfloat1622float2(hb);
+            const float xa[2] = {fa.x, fa.y}, xb[2] = {fb.x, fb.y};
             float da[2], db[2];
 #pragma unroll
             for (int k = 0; k < 2; ++k) {
-                const float x = av[j + k];
-                const float sg = 1.f / (1.f + __expf(-x));
-                da[k] = v[j + k] * bv[j + k] * sg * fmaf(x, 1.f - sg, 1.f);
+                // sigmoid with the fast intrinsic divide: its few-ulp fp32 error is far
+                // below the bf16 rounding of dA and dB (for x < -87 it gives 0, as the
+                // exact value is below bf16's range there too)
+                const float x = xa[k];
+                const float sg = __fdividef(1.f, 1.f + __expf(-x));
+                da[k] = v[j + k] * xb[k] * sg * fmaf(x, 1.f - sg, 1.f);
                 db[k] = v[j + k] * x * sg;
             }
             wa[j / 2] = pack_bf16x2(da[0], da[1]);

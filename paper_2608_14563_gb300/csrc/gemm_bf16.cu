@@ -535,6 +535,7 @@ cudaError_t launch_swiglu_bf16(int T, int d, int d_ff, const void* g, const void
     GemmMaps<1> maps;
     if (!map_kmajor(&maps.a[0], g, T, d, kBM) || !map_mnmajor(&maps.b[0], W3, d, d_ff))
         return cudaErrorInvalidValue;
+    static_assert(EpiSwiglu::kTileN == 256, "the SwiGLU epilogue prefetches 256-column tiles");
     EpiSwiglu::Params ep;
     if (!map_out_bf16(&ep.dAmap, dA, T, d_ff) || !map_out_bf16(&ep.dBmap, dB, T, d_ff))
         return cudaErrorInvalidValue;
