@@ -111,3 +111,82 @@ def test_step_replays_bitwise_in_a_cuda_graph(dtype, shape, host_inputs):
             assert torch.equal(a, b)
     assert fpo.get_device_status(graphed.ws_es) == fpo.OK
     assert fpo.get_device_status(graphed.ws_up) == fpo.OK
+
+
+def test_full_configuration_step_replays_bitwise():
+    """The paper's OLMo-2 configuration: the error signal, a post-FFN norm VJP per layer,
+    AdamW with the 1% step clip on W3, and the W1/W2 updates through the cached W3_init.
+    (The optimizer's step index is a launch parameter, so a replay repeats the captured
+    one, as the eager calls here do.)"""
+    dtype = torch.bfloat16
+    T, d, d_ff, V, L = 600, 256, 768, 2112, 2
+    x = make(dtype, T, d, d_ff, V, L, seed=5)
+    g_ = torch.Generator(device="cuda").manual_seed(6)
+
+    def rn(*s, scale=1.0):
+        return (torch.randn(*s, device="cuda", generator=g_) * scale).to(dtype)
+
+    m_out = [rn(T, d) for _ in range(L)]
+    gamma = [(0.3 + 0.05 * torch.randn(d, device="cuda", generator=g_)).to(dtype)
+             for _ in range(L)]
+    W3i = [rn(d, d_ff, scale=0.02) for _ in range(L)]
+    ab = [(rn(T, d_ff), rn(T, d_ff)) for _ in range(L)]
+    xin = [rn(T, d) for _ in range(L)]
+    W12 = [0.02 * torch.randn(d_ff, d, device="cuda", generator=g_) for _ in range(2 * L)]
+    opt = fpo.optimizer_desc(fpo.OPT_ADAMW, lr=1e-3, clip=fpo.CLIP_STEP, step=3)
+    desc = fpo.error_signal_desc(T, d, V, fpo.BF16)
+
+    class Full:
+        def __init__(self):
+            self.g = torch.empty(T, d, dtype=dtype, device="cuda")
+            self.gl = [torch.empty(T, d, dtype=dtype, device="cuda") for _ in range(L)]
+            self.loss = torch.empty(1, device="cuda")
+            self.Wm = [t.clone() for t in x["Wm"]]
+            self.Wo = [torch.empty(d, d_ff, dtype=dtype, device="cuda") for _ in range(L)]
+            self.s1 = [torch.zeros(d, d_ff, device="cuda") for _ in range(L)]
+            self.s2 = [torch.zeros(d, d_ff, device="cuda") for _ in range(L)]
+            self.sig = [torch.empty(T, d_ff, dtype=dtype, device="cuda") for _ in range(2 * L)]
+            self.W12 = [t.clone() for t in W12]
+            self.W12o = [torch.empty(d_ff, d, dtype=dtype, device="cuda") for _ in range(2 * L)]
+            self.ws_es = torch.empty(fpo.error_signal_workspace(desc), dtype=torch.uint8,
+                                     device="cuda")
+            self.ws_opt = torch.empty(max(256, fpo.layer_optimize_workspace(L, d, d_ff)),
+                                      dtype=torch.uint8, device="cuda")
+            self.ws_up = torch.empty(max(256, fpo.layer_update_workspace()), dtype=torch.uint8,
+                                     device="cuda")
+
+        def __call__(self):
+            fpo.error_signal(x["h"], x["w"], x["W_U"], x["y"], self.g, loss_out=self.loss,
+                             workspace=self.ws_es)
+            for l in range(L):
+                fpo.rmsnorm_vjp(self.g, m_out[l], gamma[l], self.gl[l])
+            fpo.layer_optimize_grouped(self.gl, x["A"], opt, self.Wm, W_outs=self.Wo,
+                                       states1=self.s1, states2=self.s2, workspace=self.ws_opt)
+            for l in range(L):
+                fpo.gate_up_signals(self.gl[l], W3i[l], ab[l][0], ab[l][1], self.sig[2 * l],
+                                    self.sig[2 * l + 1], workspace=self.ws_up)
+            act = [t for t in xin for _ in range(2)]
+            fpo.layer_update_grouped_signals(self.sig, act, 1e-3, W_masters=self.W12,
+                                             W_outs=self.W12o, workspace=self.ws_up)
+
+        def outputs(self):
+            return ([self.g, self.loss] + self.gl + self.Wm + self.Wo + self.s1 + self.s2
+                    + self.sig + self.W12 + self.W12o)
+
+    eager, graphed = Full(), Full()
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        graphed()
+    torch.cuda.current_stream().wait_stream(side)
+    eager()
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        graphed()
+    for _ in range(2):
+        graph.replay()
+        eager()
+        torch.cuda.synchronize()
+        for a, b in zip(eager.outputs(), graphed.outputs()):
+            assert torch.equal(a, b)
