@@ -304,23 +304,6 @@ def run_fpo(args, wl):
                             dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream()
 
-    n_chunks = -(-wl.T // (args.t_chunk or wl.T))
-    # fwd, mean, vjp, update + per chunk (direct: logits, combine, fixup, fixup factors,
-    # projection; stored: logits, combine, E, projection; recompute: E pass, projection,
-    # plus one logits pass and one combine)
-    launches_per_step = 4 + {"direct": 5 * n_chunks, "stored-logits": 4 * n_chunks,
-                             "recompute": 2 + 2 * n_chunks}[algo_name]
-    if post:
-        launches_per_step += wl.layers
-    if args.optimizer != "fused-sgd":  # G GEMM + optimizer (norms, scale, apply with a clip)
-        launches_per_step += 3 if args.clip != "none" else 1
-    if args.gate_up:  # one error_h GEMM per layer + one grouped W1/W2 update
-        launches_per_step += wl.layers + 1
-    if args.norm_ratio:  # partial sums over all layers + the per-layer final
-        launches_per_step += 2
-    if args.cosine or wl.name.startswith("diag"):  # grouped partial sums + final
-        launches_per_step += 2
-
     # The tensors one step reads that come from the forward pass / the data: the
     # end-to-end loop below copies them from host memory every step.
     X0 = {"h": h, "y": y, "A": A, "m": m_out if post else [],
@@ -425,10 +408,12 @@ def run_fpo(args, wl):
     clocks = ClockSampler(local)
     clocks.start()
     time.sleep(0.3)
+    launches0 = fpo.kernel_launches()  # the library counts every kernel it launches
     start.record(stream)
     for i in range(args.steps):
         step(X0, ev[i], uev[i])
     end.record(stream)
+    launches = fpo.kernel_launches() - launches0
     torch.cuda.synchronize()
     clk = clocks.stop()
     if world > 1:
@@ -510,8 +495,10 @@ def run_fpo(args, wl):
             dist.barrier()
         s2, e2 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         s2.record(stream)
+        e2e_l0 = fpo.kernel_launches()
         for i in range(max(1, args.warmup), max(1, args.warmup) + args.steps):
             e2e_step(i)
+        e2e_launches = fpo.kernel_launches() - e2e_l0
         stream.wait_stream(copy_stream)
         e2.record(stream)
         torch.cuda.synchronize()
@@ -519,6 +506,7 @@ def run_fpo(args, wl):
         h2d = sum(t.numel() * t.element_size() for t in host)
         e2e = {"value": whole_job_tokens_per_s(wl.T, world, e2e_ms), "unit": "tokens/s",
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": 4, "ms_per_step": e2e_ms,
+               "gpu_launches": e2e_launches,
                "copy": ("fpo_h2d_copy: SM loads of mapped pinned memory, one launch per step"
                         if args.e2e_copy == "sm" else "copy engines: one cudaMemcpyAsync per tensor"),
                "pipeline": f"all step inputs H2D from pinned memory each step, {depth} device "
@@ -585,7 +573,7 @@ def run_fpo(args, wl):
                             }[variant],
             "cpu_baseline": cpu,
             "e2e": e2e,
-            "gpu_launches": launches_per_step * args.steps,
+            "gpu_launches": launches,
             "clocks": clk,
             "device_status": list(status),
         }

@@ -57,6 +57,13 @@ int64_t fpo_testing_direct_fixup_rows(const fpo_error_signal_desc* desc,
                                       const void* workspace, void* stream);
 
 /*
+ * Kernels this library has launched in this process, over every entry point and
+ * every thread (a launch the runtime rejected is counted too).  The difference of
+ * two readings around a region counts the library's kernels in it.
+ */
+uint64_t fpo_testing_kernel_launches(void);
+
+/*
  * Failure-detection check of the bounded waits every kernel uses: launches one
  * block that waits on a shared-memory mbarrier nothing ever arrives on, with
  * a limit of `limit_ns` nanoseconds.  The wait gives up, the kernel records

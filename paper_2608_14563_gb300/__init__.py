@@ -106,6 +106,8 @@ _lib.fpo_h2d_copy.argtypes = [_i32, ctypes.POINTER(_vp), ctypes.POINTER(_vp),
 _lib.fpo_h2d_copy.restype = _i32
 _lib.fpo_testing_direct_fixup_rows.argtypes = [ctypes.POINTER(ErrorSignalDesc), _vp, _vp]
 _lib.fpo_testing_direct_fixup_rows.restype = _i64
+_lib.fpo_testing_kernel_launches.argtypes = []
+_lib.fpo_testing_kernel_launches.restype = ctypes.c_uint64
 _lib.fpo_testing_set_gemm_variant.argtypes = [_i32]
 _lib.fpo_testing_set_gemm_variant.restype = _i32
 
@@ -126,6 +128,11 @@ def abi_version() -> int:
 
 def set_wait_limit_ns(ns: int) -> None:
     _lib.fpo_set_wait_limit_ns(int(ns))
+
+
+def kernel_launches() -> int:
+    """fpo_testing_kernel_launches: kernels this library has launched in this process."""
+    return int(_lib.fpo_testing_kernel_launches())
 
 
 def set_gemm_variant(variant: int) -> int:

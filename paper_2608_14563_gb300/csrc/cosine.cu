@@ -166,13 +166,15 @@ cudaError_t launch_cosine(int dtype, int64_t n, const void* X, const void* Y, do
                           int blocks, double* out, cudaStream_t st) {
     if (dtype == 1)
         cosine_partial_kernel<__nv_bfloat16><<<blocks, kCosThreads, 0, st>>>(
-            static_cast<const __nv_bfloat16*>(X), static_cast<const __nv_bfloat16*>(Y), n, partial);
+            static_cast<const __nv_bfloat16*>(X), static_cast<const __nv_bfloat16*>(Y), n, partial),
+            ::fpo::note_launch();
     else
         cosine_partial_kernel<float><<<blocks, kCosThreads, 0, st>>>(
-            static_cast<const float*>(X), static_cast<const float*>(Y), n, partial);
+            static_cast<const float*>(X), static_cast<const float*>(Y), n, partial),
+            ::fpo::note_launch();
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    cosine_final_kernel<<<1, kCosThreads, 0, st>>>(partial, blocks, out);
+    cosine_final_kernel<<<1, kCosThreads, 0, st>>>(partial, blocks, out), ::fpo::note_launch();
     return cudaGetLastError();
 }
 

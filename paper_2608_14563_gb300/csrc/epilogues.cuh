@@ -189,6 +189,59 @@ struct EpiLseProb {
 };
 
 // ---------------------------------------------------------------------------
+// Direct algorithm, rows outside the anchor window (Sec. 3.1 step 2 with the
+// anchor at lse_t): the GEMM's rows are the yhat rows gathered from fix[0, count);
+// each logit z of such a row becomes p~ = exp(z - lse_t), 0 at the target,
+// rounded to bf16 and stored into that row of P with plain 16-byte stores; the
+// row's sum of the rounded values over the tile goes to sx[row, tile].
+struct EpiFixProb {
+    struct Params {
+        __nv_bfloat16* P;    // [T, N] rows of the chunk, row stride N
+        float* sx;           // [T, n_tiles]
+        const int* fix;      // gathered row -> row of the chunk
+        const int* count;    // gathered rows (device)
+        const int32_t* y;    // [T] targets
+        const float* lse;    // [T]
+        int n_tiles, N;
+    };
+    int orig, yt;
+    float lse2, sxs;
+    bool valid;
+
+    __device__ __forceinline__ EpiFixProb(const Params& p, int, int row_, int) : sxs(0.f) {
+        valid = row_ < *p.count;
+        orig = valid ? p.fix[row_] : 0;
+        yt = valid ? p.y[orig] : -1;
+        lse2 = valid ? p.lse[orig] * kLog2e : 0.f;
+    }
+
+    __device__ __forceinline__ void chunk(const Params& p, const float (&v)[32], int col0, int,
+                                          EpiIO&) {
+        const int lim = p.N - col0;  // valid columns of the chunk
+        if (!valid || lim <= 0) return;
+        const int r = yt - col0;
+        uint32_t w[16];
+#pragma unroll
+        for (int j = 0; j < 32; j += 2) {
+            const float a = (j < lim && j != r) ? ex2_approx(fmaf(v[j], kLog2e, -lse2)) : 0.f;
+            const float b =
+                (j + 1 < lim && j + 1 != r) ? ex2_approx(fmaf(v[j + 1], kLog2e, -lse2)) : 0.f;
+            const uint32_t pk = pack_bf16x2(a, b);
+            sxs += __uint_as_float(pk << 16) + __uint_as_float(pk & 0xffff0000u);
+            w[j / 2] = pk;
+        }
+        uint4* dst = reinterpret_cast<uint4*>(p.P + static_cast<size_t>(orig) * p.N + col0);
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+            if (q * 8 < lim) dst[q] = make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
+    }
+
+    __device__ __forceinline__ void finish(const Params& p, int nb) {
+        if (valid) p.sx[static_cast<size_t>(orig) * p.n_tiles + nb] = sxs;
+    }
+};
+
+// ---------------------------------------------------------------------------
 // Recompute pass (Sec. 3.1 step 2): e = s (exp(z - lse) - [col == y]) rounded
 // to bf16 into the error matrix E [M, N]; two 32-column chunks fill one
 // 64-column bf16 staging row before each TMA store.

@@ -17,6 +17,7 @@ namespace fpo {
 
 namespace {
 std::atomic<uint64_t> g_wait_limit_ns{2000000000ull};
+std::atomic<uint64_t> g_launches{0};
 
 struct DevCache {
     std::once_flag once;
@@ -27,6 +28,10 @@ DevCache g_dev[64];
 }  // namespace
 
 uint64_t wait_limit_ns() { return g_wait_limit_ns.load(std::memory_order_relaxed); }
+
+void note_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
+
+uint64_t launches() { return g_launches.load(std::memory_order_relaxed); }
 
 bool current_device_info(DevInfo* out) {
     int dev = 0;
@@ -73,8 +78,8 @@ int32_t cuda_status(cudaError_t e) { return e == cudaSuccess ? FPO_OK : FPO_ERR_
 
 // ------------------------------------------------------------------ error signal
 struct EsLayout {
-    size_t yhat, rho, lse, zy, ce, part, g, E, z, anchor, sx, alpha, beta, fix, fix_count, sk,
-        total;
+    size_t yhat, rho, lse, zy, ce, part, g, E, z, anchor, sx, alpha, beta, fix, yfix, fix_count,
+        sk, total;
     int n_tiles;
     int64_t Tc;
     int algo;  // the algorithm that runs: FPO_ES_RECOMPUTE, _STORED_LOGITS or _DIRECT
@@ -128,6 +133,7 @@ EsLayout es_layout(const fpo_error_signal_desc* d) {
     L.alpha = off;     off = align_up(off + Tdir * 4);
     L.beta = off;      off = align_up(off + Tdir * 4);
     L.fix = off;       off = align_up(off + Tcdir * 4);
+    L.yfix = off;      off = align_up(off + Tcdir * D * esz);
     L.fix_count = off; off = align_up(off + (direct ? 4 : 0));
     // the projection's stream-K tail (cut tiles' partial sums), bf16 tensor-core path
     L.sk = off;        off = align_up(off + (d->dtype == FPO_BF16 ? proj_sk_scratch_bytes() : 0));
@@ -225,6 +231,7 @@ int32_t fpo_error_signal(const fpo_error_signal_desc* desc, const void* h, const
         float* beta = reinterpret_cast<float*>(ws + L.beta);
         int* fix = reinterpret_cast<int*>(ws + L.fix);
         int* fix_count = reinterpret_cast<int*>(ws + L.fix_count);
+        void* yfix = ws + L.yfix;
         float* zyd = reinterpret_cast<float*>(ws + L.zy);
         for (int64_t c0 = 0; c0 < T; c0 += L.Tc) {
             const int tc = static_cast<int>(L.Tc < T - c0 ? L.Tc : T - c0);
@@ -242,9 +249,11 @@ int32_t fpo_error_signal(const fpo_error_signal_desc* desc, const void* h, const
                                           beta + c0, fix, fix_count, st));
             if (last && loss_out) FPO_TRY(launch_mean(ce, T, loss_out, st));
             if (last) FPO_TRY(mark(3));
-            FPO_TRY(launch_direct_fixup(yh, W_U, targets + c0, lse + c0, fix, fix_count, d, V,
-                                        L.n_tiles, desc->loss_scale, E, sxc, alpha + c0, beta + c0,
-                                        st));
+            FPO_TRY(launch_gather_rows(yh, fix, fix_count, d, yfix, st));
+            FPO_TRY(launch_fixup_logits_bf16(yfix, W_U, fix, fix_count, targets + c0, lse + c0, tc,
+                                             d, V, E, sxc, L.n_tiles, status, st));
+            FPO_TRY(launch_direct_fixup_factors(sxc, fix, fix_count, L.n_tiles, desc->loss_scale,
+                                                alpha + c0, beta + c0, st));
             if (last) FPO_TRY(mark(4));
             FPO_TRY(launch_proj_direct_bf16(E, W_U, targets + c0, alpha + c0, beta + c0, tc, d, V,
                                             g + c0 * d, sk, status, st));
@@ -642,6 +651,8 @@ int32_t fpo_testing_set_gemm_variant(int32_t variant) {
 }
 
 void fpo_testing_set_band(int32_t band) { set_band_override(band); }
+
+uint64_t fpo_testing_kernel_launches(void) { return fpo::launches(); }
 
 int64_t fpo_testing_direct_fixup_rows(const fpo_error_signal_desc* desc, const void* workspace,
                                       void* stream) {

@@ -96,6 +96,7 @@ GemmShape make_shape(int M, int N, int K, int BN, int groups, int band, int BM =
     sh.tail_tiles = 0;
     sh.tail_split = 0;
     sh.sk_scratch = nullptr;
+    sh.m_dev = nullptr;
     return sh;
 }
 
@@ -112,7 +113,8 @@ cudaError_t run_gemm(const GemmMaps<MAXG>& maps, const typename Epi::Params& ep,
     if (!current_device_info(&di)) return cudaErrorUnknown;
     const long long grid = sh.tiles < di.sm_count ? sh.tiles : di.sm_count;
     kern<<<static_cast<unsigned>(grid), kGemmThreads, L::kBytes, st>>>(maps, ep, sh, status,
-                                                                      wait_limit_ns());
+                                                                      wait_limit_ns()),
+        ::fpo::note_launch();
     return cudaGetLastError();
 }
 
@@ -191,7 +193,8 @@ cudaError_t run_gemm_pair(const GemmMaps<MAXG>& maps, const typename Epi::Params
         }
     }
     kern<<<static_cast<unsigned>(2 * clusters), kGemmThreads, L::kBytes, st>>>(maps, ep, sh, status,
-                                                                              wait_limit_ns());
+                                                                              wait_limit_ns()),
+        ::fpo::note_launch();
     return cudaGetLastError();
 }
 
@@ -256,7 +259,8 @@ cudaError_t launch_sk_fixup(const SkPlan& plan, const GemmShape& sh_in, const fl
     constexpr int kRowsPerBlock = kFixupThreads / (BN / 4);
     const dim3 grid(static_cast<unsigned>(plan.tail_tiles), kPairBM / kRowsPerBlock);
     sk_fixup_kernel<BN><<<grid, kFixupThreads, 0, st>>>(sh, scratch, C, alpha, beta, y,
-                                                        static_cast<const __nv_bfloat16*>(W_U));
+                                                        static_cast<const __nv_bfloat16*>(W_U)),
+        ::fpo::note_launch();
     return cudaGetLastError();
 }
 
@@ -398,6 +402,30 @@ cudaError_t launch_lse_prob_bf16(const void* yhat, const void* W_U, const int32_
         return run_gemm_pair<kLseBN, false, false, kPairStages, 1, EpiLseProb>(maps, ep, sh, status,
                                                                                st);
     return run_gemm<kLseBN, false, false, kLseStages, 1, EpiLseProb>(maps, ep, sh, status, st);
+}
+
+// The same GEMM as the logits pass on the gathered rows outside the anchor window.
+// Always the pair kernel (the only one that reads its row count on the device): the
+// recomputed rows are identical whichever kernel variant the other GEMMs use.
+cudaError_t launch_fixup_logits_bf16(const void* yfix, const void* W_U, const int* fix,
+                                     const int* fix_count, const int32_t* y, const float* lse,
+                                     int Tc, int d, int V, void* P, float* sx, int n_tiles,
+                                     unsigned* status, cudaStream_t st) {
+    GemmMaps<1> maps;
+    if (!map_kmajor(&maps.a[0], yfix, Tc, d, kBM) || !map_kmajor(&maps.b[0], W_U, V, d, kLseBN / 2))
+        return cudaErrorInvalidValue;
+    EpiFixProb::Params ep;
+    ep.P = static_cast<__nv_bfloat16*>(P);
+    ep.sx = sx;
+    ep.fix = fix;
+    ep.count = fix_count;
+    ep.y = y;
+    ep.lse = lse;
+    ep.n_tiles = n_tiles;
+    ep.N = V;
+    GemmShape sh = make_shape(Tc, V, d, kLseBN, 1, band_for(true), kPairBM);
+    sh.m_dev = fix_count;
+    return run_gemm_pair<kLseBN, false, false, kPairStages, 1, EpiFixProb>(maps, ep, sh, status, st);
 }
 
 constexpr int kProjBN = 256;

@@ -200,11 +200,11 @@ cudaError_t run(const NrPtrs& ptrs, int n_layers, int64_t n, int blocks, int mod
                 double* partial, double* out, cudaStream_t st) {
     grouped_partial_kernel<TG, TW, kDot>
         <<<dim3(static_cast<unsigned>(blocks), static_cast<unsigned>(n_layers)), kNrThreads, 0,
-           st>>>(ptrs, n, partial);
+           st>>>(ptrs, n, partial), ::fpo::note_launch();
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     grouped_final_kernel<<<(n_layers + 63) / 64, 64, 0, st>>>(partial, blocks, n_layers, mode,
-                                                              rel, out);
+                                                              rel, out), ::fpo::note_launch();
     return cudaGetLastError();
 }
 

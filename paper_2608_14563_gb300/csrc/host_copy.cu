@@ -121,6 +121,6 @@ extern "C" int32_t fpo_h2d_copy(int32_t n, void* const* dst, const void* const* 
                              cudaSharedmemCarveoutMaxShared) != cudaSuccess)
         return FPO_ERR_CUDA;
     fpo::h2d_copy_kernel<<<di.sm_count, fpo::kCopyThreads, 0, static_cast<cudaStream_t>(stream)>>>(
-        list);
+        list), ::fpo::note_launch();
     return cudaGetLastError() == cudaSuccess ? FPO_OK : FPO_ERR_CUDA;
 }

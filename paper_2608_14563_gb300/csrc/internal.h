@@ -23,6 +23,10 @@ bool current_device_info(DevInfo* out);
 
 uint64_t wait_limit_ns();
 
+// Counts one kernel launch of this library (process-wide); launches() reads the count.
+void note_launch();
+uint64_t launches();
+
 // ------------------------------------------------------------ bf16 (tcgen05)
 // Logits pass: part[T, n_tiles] (max, sum exp), zy[T] (target logits) and, when z is
 // non-null, the fp32 logits z[T, V] (stored-logits algorithm).
@@ -49,6 +53,14 @@ cudaError_t launch_lse_prob_bf16(const void* yhat, const void* W_U, const int32_
                                  const float* anchor, int T, int d, int V, float2* part, float* sx,
                                  int part_ld, float* zy, void* P, unsigned* status,
                                  cudaStream_t st);
+// Direct algorithm, rows outside the anchor window: the logits of the gathered rows
+// yfix[*fix_count, d] (capacity Tc rows) on the tensor cores; P[fix[i], :] = exp(z - lse)
+// in bf16 with the target column zero, sx[fix[i], tile] the per-tile sums of the rounded
+// values.  The row count is read on the device (none: the kernel returns at once).
+cudaError_t launch_fixup_logits_bf16(const void* yfix, const void* W_U, const int* fix,
+                                     const int* fix_count, const int32_t* y, const float* lse,
+                                     int Tc, int d, int V, void* P, float* sx, int n_tiles,
+                                     unsigned* status, cudaStream_t st);
 // Direct algorithm, projection: g[Tc, d] = alpha (.) (P W_U) + beta (.) W_U[y] (row-wise).
 cudaError_t launch_proj_direct_bf16(const void* P, const void* W_U, const int32_t* y,
                                     const float* alpha, const float* beta, int Tc, int d, int V,
@@ -111,11 +123,14 @@ cudaError_t launch_direct_combine(const float2* part, const float* sx, int n_til
                                   const int32_t* y, const float* anchor, const float* zy, float s,
                                   float* lse, float* ce, float* alpha, float* beta, int* fix,
                                   int* fix_count, cudaStream_t st);
-// Recompute the P rows, sx partials and row factors of the listed rows, anchored at lse.
-cudaError_t launch_direct_fixup(const void* yhat, const void* W_U, const int32_t* y,
-                                const float* lse, const int* fix, const int* fix_count, int d,
-                                int V, int n_tiles, float s, void* P, float* sx, float* alpha,
-                                float* beta, cudaStream_t st);
+// Rows outside the anchor window: out[i, :] = yhat[fix[i], :] for i < *fix_count (bf16,
+// d a multiple of 8), then (launch_fixup_logits_bf16) their P rows and sx partials
+// recomputed anchored at lse, then their row factors alpha = s, beta = -s S'.
+cudaError_t launch_gather_rows(const void* yhat, const int* fix, const int* fix_count, int d,
+                               void* out, cudaStream_t st);
+cudaError_t launch_direct_fixup_factors(const float* sx, const int* fix, const int* fix_count,
+                                        int n_tiles, float s, float* alpha, float* beta,
+                                        cudaStream_t st);
 cudaError_t launch_lse_combine(const float2* part, int n_tiles, int T, const float* zy,
                                float* lse, float* ce, cudaStream_t st);
 cudaError_t launch_mean(const float* x, int n, float* out, cudaStream_t st);

@@ -175,19 +175,23 @@ cudaError_t launch_optimizer(int dtype, int n_layers, size_t n_elem, const Optim
     const int bpl = blocks_per_layer(n_layers);
     const dim3 grid(bpl, n_layers);
     if (op.clip != 0) {
-        optim_norms_kernel<<<grid, kOptThreads, 0, st>>>(lp, n_elem, op, partials);
+        optim_norms_kernel<<<grid, kOptThreads, 0, st>>>(lp, n_elem, op, partials),
+            ::fpo::note_launch();
         cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return e;
-        optim_scale_kernel<<<n_layers, 32, 0, st>>>(partials, bpl, op, scales);
+        optim_scale_kernel<<<n_layers, 32, 0, st>>>(partials, bpl, op, scales),
+            ::fpo::note_launch();
         e = cudaGetLastError();
         if (e != cudaSuccess) return e;
     }
     if (dtype == 1)
         optim_apply_kernel<true><<<grid, kOptThreads, 0, st>>>(lp, n_elem, op,
-                                                               op.clip != 0 ? scales : nullptr);
+                                                               op.clip != 0 ? scales : nullptr),
+            ::fpo::note_launch();
     else
         optim_apply_kernel<false><<<grid, kOptThreads, 0, st>>>(lp, n_elem, op,
-                                                                op.clip != 0 ? scales : nullptr);
+                                                                op.clip != 0 ? scales : nullptr),
+            ::fpo::note_launch();
     return cudaGetLastError();
 }
 

@@ -7,7 +7,8 @@
 //   lse_combine   lse_t from the per-vocabulary-tile (max, sum exp) partials
 //   direct_combine  the same, plus the direct algorithm's row factors
 //                 alpha_t, beta_t and the list of rows outside the anchor window
-//   direct_fixup  recomputes the P rows of those rows, anchored at lse_t
+//   gather_rows   gathers the yhat rows of those rows for their tensor-core
+//                 recomputation anchored at lse_t (gemm_bf16.cu)
 //   mean          mean of a vector in a fixed order (the mean cross-entropy)
 //   rmsnorm_vjp   App. E Eq. (rmsnorm-vjp) with the min-RMS clamp:
 //                 g~ = (w (.) g - xhat <xhat, w (.) g> / d) / max(rho, rho_min)
@@ -512,102 +513,17 @@ __global__ void __launch_bounds__(kRowThreads)
     }
 }
 
-// Rows outside the anchor window, in groups of up to kFixRows rows per work item
-// (group, vocabulary tile): the group's yhat rows are staged in shared memory (or
-// read from global memory when d is too large to stage), and each warp takes tile
-// columns j in turn, reading W_U[j] once for the whole group:
-//   z_rj = <yhat_r, W_U[j]> (fp32),  P[r, j] = bf16(exp(z_rj - lse_r)) (target 0),
-// and per row the sum of the tile's rounded values goes to sx[row, tile].  The row
-// count is read on the device, so the launch is the same whether or not any row
-// needs it; with none it returns at once.
-constexpr int kFixTile = 256;        // vocabulary columns per work item (the logits tile width)
-constexpr int kFixRows = 8;          // rows per group: one W_U read serves all of them
-constexpr int kFixStageMax = 192 * 1024;  // shared memory for staged yhat rows
-
-template <bool kStage>
+// Rows outside the anchor window: their yhat rows gathered into a compact [count, d]
+// matrix for the tensor-core recomputation (16-byte vectors; the row count is read on
+// the device, so with no such row the launch returns at once).
 __global__ void __launch_bounds__(kRowThreads)
-    direct_fixup_kernel(const __nv_bfloat16* __restrict__ yhat,
-                        const __nv_bfloat16* __restrict__ W_U, const int32_t* __restrict__ y,
-                        const float* __restrict__ lse, const int* __restrict__ fix,
-                        const int* __restrict__ fix_count, int d, int V, int n_tiles,
-                        __nv_bfloat16* __restrict__ P, float* __restrict__ sx) {
-    extern __shared__ __align__(16) uint8_t fx_smem[];
-    __nv_bfloat16* xs = reinterpret_cast<__nv_bfloat16*>(fx_smem);  // [kFixRows][d] if staged
-    __shared__ float wsum[kRowThreads / 32][kFixRows];
-    const int lane = threadIdx.x & 31;
-    const int warp = threadIdx.x >> 5;
-    const int count = *fix_count;
-    const long long groups = (count + kFixRows - 1) / kFixRows;
-    const long long items = groups * n_tiles;
-    for (long long it = blockIdx.x; it < items; it += gridDim.x) {
-        const int r0 = static_cast<int>(it / n_tiles) * kFixRows;
-        const int tile = static_cast<int>(it % n_tiles);
-        const int nr = count - r0 < kFixRows ? count - r0 : kFixRows;
-        const __nv_bfloat16* xr[kFixRows];
-        __syncthreads();  // the previous item is done with the staged rows and wsum
-        if constexpr (kStage) {
-            const int v8 = d / 8;
-            for (int idx = threadIdx.x; idx < nr * v8; idx += kRowThreads) {
-                const int r = idx / v8, k = (idx - r * v8) * 8;
-                *reinterpret_cast<uint4*>(xs + static_cast<size_t>(r) * d + k) =
-                    *reinterpret_cast<const uint4*>(yhat + static_cast<size_t>(fix[r0 + r]) * d + k);
-            }
-            __syncthreads();
-#pragma unroll
-            for (int r = 0; r < kFixRows; ++r) xr[r] = xs + static_cast<size_t>(r) * d;
-        } else {
-#pragma unroll
-            for (int r = 0; r < kFixRows; ++r)
-                xr[r] = yhat + static_cast<size_t>(fix[r0 + (r < nr ? r : 0)]) * d;
-        }
-        float acc[kFixRows];
-#pragma unroll
-        for (int r = 0; r < kFixRows; ++r) acc[r] = 0.f;
-        for (int c = warp; c < kFixTile; c += kRowThreads / 32) {
-            const int j = tile * kFixTile + c;
-            if (j >= V) break;
-            const __nv_bfloat16* ur = W_U + static_cast<size_t>(j) * d;
-            float z[kFixRows];
-#pragma unroll
-            for (int r = 0; r < kFixRows; ++r) z[r] = 0.f;
-            for (int k = lane * 8; k < d; k += 32 * 8) {
-                float b[8];
-                ld_vec<8>(ur + k, b);
-#pragma unroll
-                for (int r = 0; r < kFixRows; ++r) {
-                    if (r < nr) {
-                        float a[8];
-                        ld_vec<8>(xr[r] + k, a);
-#pragma unroll
-                        for (int q = 0; q < 8; ++q) z[r] = fmaf(a[q], b[q], z[r]);
-                    }
-                }
-            }
-#pragma unroll
-            for (int r = 0; r < kFixRows; ++r) z[r] = warp_sum(z[r]);
-            if (lane == 0) {
-#pragma unroll
-                for (int r = 0; r < kFixRows; ++r) {
-                    if (r < nr) {
-                        const int row = fix[r0 + r];
-                        const __nv_bfloat16 p =
-                            __float2bfloat16_rn(j == y[row] ? 0.f : expf(z[r] - lse[row]));
-                        P[static_cast<size_t>(row) * V + j] = p;
-                        acc[r] += __bfloat162float(p);
-                    }
-                }
-            }
-        }
-        if (lane == 0) {
-#pragma unroll
-            for (int r = 0; r < kFixRows; ++r) wsum[warp][r] = acc[r];
-        }
-        __syncthreads();
-        if (threadIdx.x < nr) {
-            float S = 0.f;
-            for (int w = 0; w < kRowThreads / 32; ++w) S += wsum[w][threadIdx.x];
-            sx[static_cast<size_t>(fix[r0 + threadIdx.x]) * n_tiles + tile] = S;
-        }
+    gather_rows_kernel(const uint4* __restrict__ src, const int* __restrict__ fix,
+                       const int* __restrict__ count, int v8, uint4* __restrict__ dst) {
+    const long long n = static_cast<long long>(*count) * v8;
+    for (long long i = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x; i < n;
+         i += static_cast<long long>(gridDim.x) * blockDim.x) {
+        const long long r = i / v8;
+        dst[i] = src[static_cast<long long>(fix[r]) * v8 + (i - r * v8)];
     }
 }
 
@@ -747,26 +663,28 @@ cudaError_t launch_rmsnorm_fwd(int dtype, const void* h, const void* w, int T, i
         const auto* wu = static_cast<const __nv_bfloat16*>(W_U);
         if (ept == 8)
             rmsnorm_fwd_row_kernel<8><<<blk_grid(T), kBlkThreads, 0, st>>>(
-                hh, ww, T, d, eps, yy, rho, y, V, status, wu, anchor);
+                hh, ww, T, d, eps, yy, rho, y, V, status, wu, anchor), ::fpo::note_launch();
         else if (ept == 16)
             rmsnorm_fwd_row_kernel<16><<<blk_grid(T), kBlkThreads, 0, st>>>(
-                hh, ww, T, d, eps, yy, rho, y, V, status, wu, anchor);
+                hh, ww, T, d, eps, yy, rho, y, V, status, wu, anchor), ::fpo::note_launch();
         else
             rmsnorm_fwd_row_kernel<32><<<blk_grid(T), kBlkThreads, 0, st>>>(
-                hh, ww, T, d, eps, yy, rho, y, V, status, wu, anchor);
+                hh, ww, T, d, eps, yy, rho, y, V, status, wu, anchor), ::fpo::note_launch();
     } else if (dtype == 1) {
         rmsnorm_fwd_kernel<__nv_bfloat16, 8><<<grid, kRowThreads, 0, st>>>(
             static_cast<const __nv_bfloat16*>(h), static_cast<const __nv_bfloat16*>(w), T, d, eps,
             static_cast<__nv_bfloat16*>(yhat), rho, y, V, status,
-            static_cast<const __nv_bfloat16*>(W_U), anchor);
+            static_cast<const __nv_bfloat16*>(W_U), anchor), ::fpo::note_launch();
     } else if (d % 4 == 0) {
         rmsnorm_fwd_kernel<float, 4><<<grid, kRowThreads, 0, st>>>(
             static_cast<const float*>(h), static_cast<const float*>(w), T, d, eps,
-            static_cast<float*>(yhat), rho, y, V, status, static_cast<const float*>(W_U), anchor);
+            static_cast<float*>(yhat), rho, y, V, status, static_cast<const float*>(W_U), anchor),
+            ::fpo::note_launch();
     } else {
         rmsnorm_fwd_kernel<float, 1><<<grid, kRowThreads, 0, st>>>(
             static_cast<const float*>(h), static_cast<const float*>(w), T, d, eps,
-            static_cast<float*>(yhat), rho, y, V, status, static_cast<const float*>(W_U), anchor);
+            static_cast<float*>(yhat), rho, y, V, status, static_cast<const float*>(W_U), anchor),
+            ::fpo::note_launch();
     }
     return cudaGetLastError();
 }
@@ -777,34 +695,28 @@ cudaError_t launch_direct_combine(const float2* part, const float* sx, int n_til
                                   int* fix_count, cudaStream_t st) {
     if (T <= 0) return cudaSuccess;
     direct_combine_kernel<<<row_grid(T), kRowThreads, 0, st>>>(
-        part, sx, n_tiles, T, V, y, anchor, zy, s, lse, ce, alpha, beta, fix, fix_count);
+        part, sx, n_tiles, T, V, y, anchor, zy, s, lse, ce, alpha, beta, fix, fix_count),
+        ::fpo::note_launch();
     return cudaGetLastError();
 }
 
-cudaError_t launch_direct_fixup(const void* yhat, const void* W_U, const int32_t* y,
-                                const float* lse, const int* fix, const int* fix_count, int d,
-                                int V, int n_tiles, float s, void* P, float* sx, float* alpha,
-                                float* beta, cudaStream_t st) {
+cudaError_t launch_gather_rows(const void* yhat, const int* fix, const int* fix_count, int d,
+                               void* out, cudaStream_t st) {
     DevInfo di;
     const int sms = current_device_info(&di) ? di.sm_count : 148;
-    const size_t stage = static_cast<size_t>(kFixRows) * d * 2;
-    const auto* yh = static_cast<const __nv_bfloat16*>(yhat);
-    const auto* wu = static_cast<const __nv_bfloat16*>(W_U);
-    auto* pp = static_cast<__nv_bfloat16*>(P);
-    if (stage <= static_cast<size_t>(kFixStageMax)) {
-        static const cudaError_t attr = cudaFuncSetAttribute(
-            direct_fixup_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, kFixStageMax);
-        if (attr != cudaSuccess) return attr;
-        direct_fixup_kernel<true><<<2 * sms, kRowThreads, stage, st>>>(yh, wu, y, lse, fix, fix_count,
-                                                                   d, V, n_tiles, pp, sx);
-    } else {
-        direct_fixup_kernel<false><<<sms * 4, kRowThreads, 0, st>>>(yh, wu, y, lse, fix, fix_count,
-                                                                    d, V, n_tiles, pp, sx);
-    }
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
+    gather_rows_kernel<<<4 * sms, kRowThreads, 0, st>>>(static_cast<const uint4*>(yhat), fix,
+                                                        fix_count, d / 8, static_cast<uint4*>(out)),
+        ::fpo::note_launch();
+    return cudaGetLastError();
+}
+
+cudaError_t launch_direct_fixup_factors(const float* sx, const int* fix, const int* fix_count,
+                                        int n_tiles, float s, float* alpha, float* beta,
+                                        cudaStream_t st) {
+    DevInfo di;
+    const int sms = current_device_info(&di) ? di.sm_count : 148;
     direct_fixup_factors_kernel<<<sms, kRowThreads, 0, st>>>(sx, fix, fix_count, n_tiles, s, alpha,
-                                                            beta);
+                                                            beta), ::fpo::note_launch();
     return cudaGetLastError();
 }
 
@@ -820,25 +732,28 @@ cudaError_t launch_rmsnorm_vjp(int dtype, const float* g, const void* h, const v
         auto* oo = static_cast<__nv_bfloat16*>(out);
         if (ept == 8)
             rmsnorm_vjp_row_kernel<8><<<blk_grid(T), kBlkThreads, 0, st>>>(g, hh, ww, rho, T, d,
-                                                                        min_rms, oo);
+                                                                        min_rms, oo),
+                ::fpo::note_launch();
         else if (ept == 16)
             rmsnorm_vjp_row_kernel<16><<<blk_grid(T), kBlkThreads, 0, st>>>(g, hh, ww, rho, T, d,
-                                                                         min_rms, oo);
+                                                                         min_rms, oo),
+                ::fpo::note_launch();
         else
             rmsnorm_vjp_row_kernel<32><<<blk_grid(T), kBlkThreads, 0, st>>>(g, hh, ww, rho, T, d,
-                                                                         min_rms, oo);
+                                                                         min_rms, oo),
+                ::fpo::note_launch();
     } else if (dtype == 1) {
         rmsnorm_vjp_kernel<__nv_bfloat16, 8><<<grid, kRowThreads, 0, st>>>(
             g, static_cast<const __nv_bfloat16*>(h), static_cast<const __nv_bfloat16*>(w), rho, T,
-            d, min_rms, static_cast<__nv_bfloat16*>(out));
+            d, min_rms, static_cast<__nv_bfloat16*>(out)), ::fpo::note_launch();
     } else if (d % 4 == 0) {
         rmsnorm_vjp_kernel<float, 4><<<grid, kRowThreads, 0, st>>>(
             g, static_cast<const float*>(h), static_cast<const float*>(w), rho, T, d, min_rms,
-            static_cast<float*>(out));
+            static_cast<float*>(out)), ::fpo::note_launch();
     } else {
         rmsnorm_vjp_kernel<float, 1><<<grid, kRowThreads, 0, st>>>(
             g, static_cast<const float*>(h), static_cast<const float*>(w), rho, T, d, min_rms,
-            static_cast<float*>(out));
+            static_cast<float*>(out)), ::fpo::note_launch();
     }
     return cudaGetLastError();
 }
@@ -847,7 +762,7 @@ cudaError_t launch_cast_f32(int dtype, const float* src, size_t n, void* dst, cu
     if (n == 0) return cudaSuccess;
     if (dtype != 1) return cudaMemcpyAsync(dst, src, n * sizeof(float), cudaMemcpyDeviceToDevice, st);
     cast_f32_kernel<<<row_grid(static_cast<int>((n + 255) / 256 * 8)), kRowThreads, 0, st>>>(
-        src, n, static_cast<__nv_bfloat16*>(dst));
+        src, n, static_cast<__nv_bfloat16*>(dst)), ::fpo::note_launch();
     return cudaGetLastError();
 }
 
@@ -858,17 +773,20 @@ cudaError_t launch_error_from_logits(int dtype, const float* z, const float* lse
     const int sms = current_device_info(&di) ? di.sm_count : 148;
     const int grid = M < sms * 8 ? M : sms * 8;
     if (dtype == 1)
-        error_from_logits_kernel<true><<<grid, kErrThreads, 0, st>>>(z, lse, y, M, V, s, E);
+        error_from_logits_kernel<true><<<grid, kErrThreads, 0, st>>>(z, lse, y, M, V, s, E),
+            ::fpo::note_launch();
     else if (V % 8 == 0)
-        error_from_logits_kernel<false><<<grid, kErrThreads, 0, st>>>(z, lse, y, M, V, s, E);
+        error_from_logits_kernel<false><<<grid, kErrThreads, 0, st>>>(z, lse, y, M, V, s, E),
+            ::fpo::note_launch();
     else
         error_from_logits_scalar_kernel<<<grid, kErrThreads, 0, st>>>(z, lse, y, M, V, s,
-                                                                      static_cast<float*>(E));
+                                                                      static_cast<float*>(E)),
+            ::fpo::note_launch();
     return cudaGetLastError();
 }
 
 cudaError_t launch_wait_timeout(unsigned* status, uint64_t limit_ns, cudaStream_t st) {
-    wait_timeout_kernel<<<1, 32, 0, st>>>(status, limit_ns);
+    wait_timeout_kernel<<<1, 32, 0, st>>>(status, limit_ns), ::fpo::note_launch();
     return cudaGetLastError();
 }
 
@@ -885,26 +803,31 @@ cudaError_t launch_rmsnorm_vjp_at(int dtype, const void* g, const void* x, const
         auto* oo = static_cast<__nv_bfloat16*>(out);
         if (ept == 8)
             rmsnorm_vjp_at_row_kernel<8><<<blk_grid(T), kBlkThreads, 0, st>>>(gg, xx, ga, T, d, eps,
-                                                                           min_rms, oo);
+                                                                           min_rms, oo),
+                ::fpo::note_launch();
         else if (ept == 16)
             rmsnorm_vjp_at_row_kernel<16><<<blk_grid(T), kBlkThreads, 0, st>>>(gg, xx, ga, T, d,
-                                                                            eps, min_rms, oo);
+                                                                            eps, min_rms, oo),
+                ::fpo::note_launch();
         else
             rmsnorm_vjp_at_row_kernel<32><<<blk_grid(T), kBlkThreads, 0, st>>>(gg, xx, ga, T, d,
-                                                                            eps, min_rms, oo);
+                                                                            eps, min_rms, oo),
+                ::fpo::note_launch();
     } else if (dtype == 1) {
         rmsnorm_vjp_at_kernel<__nv_bfloat16, 8><<<grid, kRowThreads, 0, st>>>(
             static_cast<const __nv_bfloat16*>(g), static_cast<const __nv_bfloat16*>(x),
             static_cast<const __nv_bfloat16*>(gamma), T, d, eps, min_rms,
-            static_cast<__nv_bfloat16*>(out));
+            static_cast<__nv_bfloat16*>(out)), ::fpo::note_launch();
     } else if (d % 4 == 0) {
         rmsnorm_vjp_at_kernel<float, 4><<<grid, kRowThreads, 0, st>>>(
             static_cast<const float*>(g), static_cast<const float*>(x),
-            static_cast<const float*>(gamma), T, d, eps, min_rms, static_cast<float*>(out));
+            static_cast<const float*>(gamma), T, d, eps, min_rms, static_cast<float*>(out)),
+            ::fpo::note_launch();
     } else {
         rmsnorm_vjp_at_kernel<float, 1><<<grid, kRowThreads, 0, st>>>(
             static_cast<const float*>(g), static_cast<const float*>(x),
-            static_cast<const float*>(gamma), T, d, eps, min_rms, static_cast<float*>(out));
+            static_cast<const float*>(gamma), T, d, eps, min_rms, static_cast<float*>(out)),
+            ::fpo::note_launch();
     }
     return cudaGetLastError();
 }
@@ -912,13 +835,14 @@ cudaError_t launch_rmsnorm_vjp_at(int dtype, const void* g, const void* x, const
 cudaError_t launch_lse_combine(const float2* part, int n_tiles, int T, const float* zy, float* lse,
                                float* ce, cudaStream_t st) {
     if (T <= 0) return cudaSuccess;
-    lse_combine_kernel<<<row_grid(T), kRowThreads, 0, st>>>(part, n_tiles, T, zy, lse, ce);
+    lse_combine_kernel<<<row_grid(T), kRowThreads, 0, st>>>(part, n_tiles, T, zy, lse, ce),
+        ::fpo::note_launch();
     return cudaGetLastError();
 }
 
 cudaError_t launch_mean(const float* x, int n, float* out, cudaStream_t st) {
     if (n <= 0) return cudaSuccess;
-    mean_kernel<<<1, kMeanThreads, 0, st>>>(x, n, out);
+    mean_kernel<<<1, kMeanThreads, 0, st>>>(x, n, out), ::fpo::note_launch();
     return cudaGetLastError();
 }
 

@@ -177,7 +177,7 @@ template <class Epi>
 cudaError_t run(const SimtOps& ops, const Epi& ep, int groups, cudaStream_t st) {
     if (ops.M <= 0 || ops.N <= 0) return cudaSuccess;
     dim3 grid((ops.N + kT - 1) / kT, (ops.M + kT - 1) / kT, groups);
-    simt_gemm_kernel<Epi><<<grid, kThreads, 0, st>>>(ops, ep);
+    simt_gemm_kernel<Epi><<<grid, kThreads, 0, st>>>(ops, ep), ::fpo::note_launch();
     return cudaGetLastError();
 }
 

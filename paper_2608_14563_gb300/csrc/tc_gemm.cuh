@@ -42,6 +42,10 @@ struct GemmShape {
     long long tail_tiles;
     int tail_split;
     float* sk_scratch;
+    // Pair kernel only: when set, the number of rows of A is read here on the device at
+    // kernel start (at most M; the tensor maps cover M rows) and the tiles beyond it are
+    // dropped; with no rows the kernel returns before it sets anything up.
+    const int* m_dev;
 };
 
 template <int MAXG>

@@ -133,7 +133,7 @@ __device__ __forceinline__ void load_operand_pair(const CUtensorMap* map, uint32
 template <int BN, bool A_MN, bool B_MN, int STAGES, int MAXG, class Epi>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     tc_gemm_pair_kernel(const __grid_constant__ GemmMaps<MAXG> maps,
-                        const __grid_constant__ typename Epi::Params ep, const GemmShape sh,
+                        const __grid_constant__ typename Epi::Params ep, const GemmShape sh_in,
                         unsigned int* status, unsigned long long wait_limit_ns) {
     static_assert(BN == 256 || BN == 512, "pair tiles are 256 or 512 columns wide");
     using L = GemmPairSmem<BN, STAGES>;
@@ -144,6 +144,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     constexpr uint32_t kIdesc = idesc_bf16_f32(kPairBM, 256, A_MN, B_MN);
     constexpr int kTmemCols = kAccBufs * BN;       // 512 either way
     constexpr uint16_t kBoth = 0x3;
+
+    GemmShape sh = sh_in;
+    if (sh.m_dev) {  // rows counted on the device (every thread reads the same value)
+        const int m = min(*sh.m_dev, sh.M);
+        if (m <= 0) return;
+        sh.M = m;
+        sh.m_blocks = (m + kPairBM - 1) / kPairBM;
+        sh.tiles = static_cast<long long>(sh.groups) * sh.m_blocks * sh.n_blocks;
+        sh.tail_tiles = 0;
+    }
 
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);

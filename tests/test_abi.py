@@ -66,10 +66,11 @@ def test_error_signal_workspace_query(L):
     small = fpo.error_signal_desc(128, 64, 512, fpo.F32)
     assert fpo.error_signal_workspace(small) > 0
     # per token of the chunk: recompute holds a bf16 row of E; stored logits add an fp32
-    # row of logits; direct (the bf16 default) holds a bf16 row of P and one fixup-list entry
-    V = 151936
+    # row of logits; direct (the bf16 default) holds a bf16 row of P, one fixup-list entry
+    # and a bf16 row of d for the gathered rows of the fixup
+    V, d = 151936, 4096
     for algo, per in ((fpo.ES_RECOMPUTE, 2 * V), (fpo.ES_STORED_LOGITS, 6 * V),
-                      (fpo.ES_DIRECT, 2 * V + 4), (fpo.ES_AUTO, 2 * V + 4)):
+                      (fpo.ES_DIRECT, 2 * V + 4 + 2 * d), (fpo.ES_AUTO, 2 * V + 4 + 2 * d)):
         chunked = fpo.error_signal_desc(4096, 4096, V, fpo.BF16, t_chunk=1024, algo=algo)
         full = fpo.error_signal_desc(4096, 4096, V, fpo.BF16, algo=algo)
         diff = fpo.error_signal_workspace(full) - fpo.error_signal_workspace(chunked)
@@ -142,3 +143,14 @@ def test_h2d_copy_host_validation(L):
     assert lib.fpo_h2d_copy(1, one(fake), one(None), (sz * 1)(16), None) == 1
     assert lib.fpo_h2d_copy(1, one(fake), one(mis), (sz * 1)(16), None) == 4
     assert lib.fpo_h2d_copy(1, one(mis), one(fake), (sz * 1)(16), None) == 4
+
+
+def test_rejected_calls_launch_no_kernel(L):
+    """Host-side argument errors return before anything is enqueued: the library's
+    launch counter does not move."""
+    lib = L.lib
+    n0 = L.fpo.kernel_launches()
+    fake = ctypes.c_void_p(1 << 20)
+    assert lib.fpo_cosine(10, 1, None, fake, fake, fake, 1 << 20, None) == 1
+    assert lib.fpo_h2d_copy(-1, None, None, None, None) == 2
+    assert L.fpo.kernel_launches() == n0

@@ -189,9 +189,9 @@ def test_results_do_not_depend_on_workspace_contents(fpo, ragged, variant, algo)
 
 def test_many_rows_outside_the_window(fpo):
     """Logits ~30x the usual scale (exact +-1 hidden states, W_U x 64): most tokens have
-    cross-entropy far beyond the window and go through the grouped fixup (8 rows per
-    group, a partial last group); the rows match the oracle and the count matches the
-    fp64 window test of S'_t."""
+    cross-entropy far beyond the window and go through the tensor-core fixup (several
+    256-row tiles of gathered rows, a partial last one); the rows match the oracle and the
+    count matches the fp64 window test of S'_t."""
     T, d, V = 1000, 512, 4096
     wl = Workload("many-fixed", T=T, d=d, d_ff=8, V=V, layers=1, targets="uniform", eps=0.0)
     w = synth.make_norm_w(wl)
