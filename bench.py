@@ -468,21 +468,39 @@ def run_fpo(args, wl):
         for e in freed:
             e.record(stream)
 
-        def prefetch(b):
+        # "sm": the copy of a step's inputs in two halves by bytes, each started at a stage
+        # boundary of the current step so that it runs beside one long GEMM (the logits
+        # pass, then the projection) and not beside the short bandwidth-bound kernels
+        # between them, which the copy's host loads slow down most
+        nbytes = [t.numel() * t.element_size() for t in host]
+        half = 0
+        while half < len(host) and sum(nbytes[:half]) < sum(nbytes) / 2:
+            half += 1
+        sev = [torch.cuda.Event() for _ in range(fpo.STAGE_EVENTS)]
+        for e in sev:
+            e.record(stream)
+
+        def prefetch(b, after=None):
             copy_stream.wait_event(freed[b])
             with torch.cuda.stream(copy_stream):
-                if args.e2e_copy == "sm":
-                    fpo.h2d_copy(flat(sets[b]), host, stream=copy_stream)
+                dst = flat(sets[b])
+                if args.e2e_copy == "sm" and after is not None:
+                    copy_stream.wait_event(after[1])      # the RMSNorm forward is done
+                    fpo.h2d_copy(dst[:half], host[:half], stream=copy_stream)
+                    copy_stream.wait_event(after[4])      # the projection starts
+                    fpo.h2d_copy(dst[half:], host[half:], stream=copy_stream)
+                elif args.e2e_copy in ("sm", "sm1"):
+                    fpo.h2d_copy(dst, host, stream=copy_stream)
                 else:
-                    for d_t, h_t in zip(flat(sets[b]), host):
+                    for d_t, h_t in zip(dst, host):
                         d_t.copy_(h_t, non_blocking=True)
                 ready[b].record(copy_stream)
 
         def e2e_step(i):
             b = i % depth
-            prefetch((i + depth - 1) % depth)  # the inputs of step i + depth - 1
             stream.wait_event(ready[b])
-            step(sets[b])
+            step(sets[b], sev)
+            prefetch((i + depth - 1) % depth, sev)  # the inputs of step i + depth - 1
             freed[b].record(stream)
             loss_host.copy_(loss, non_blocking=True)
 
@@ -507,8 +525,11 @@ def run_fpo(args, wl):
         e2e = {"value": whole_job_tokens_per_s(wl.T, world, e2e_ms), "unit": "tokens/s",
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": 4, "ms_per_step": e2e_ms,
                "gpu_launches": e2e_launches,
-               "copy": ("fpo_h2d_copy: SM loads of mapped pinned memory, one launch per step"
-                        if args.e2e_copy == "sm" else "copy engines: one cudaMemcpyAsync per tensor"),
+               "copy": {"sm": "fpo_h2d_copy (SM loads of mapped pinned memory): two launches "
+                              "per step, beside the logits pass and the projection",
+                        "sm1": "fpo_h2d_copy (SM loads of mapped pinned memory): one launch per "
+                               "step",
+                        "ce": "copy engines: one cudaMemcpyAsync per tensor"}[args.e2e_copy],
                "pipeline": f"all step inputs H2D from pinned memory each step, {depth} device "
                            "sets: copies run on a copy stream up to "
                            f"{depth - 1} steps ahead of compute; loss D2H"}
@@ -654,9 +675,10 @@ def main():
                     help="add the App. C update-magnitude ratio ||G_l||/||W_l|| to every step")
     ap.add_argument("--e2e-depth", type=int, default=3,
                     help="device input sets of the end-to-end loop (copies run depth-1 steps ahead)")
-    ap.add_argument("--e2e-copy", choices=("sm", "ce"), default="sm",
+    ap.add_argument("--e2e-copy", choices=("sm", "sm1", "ce"), default="sm",
                     help="end-to-end input copies: sm = fpo_h2d_copy (SM loads of mapped pinned "
-                         "memory, one launch per step), ce = cudaMemcpyAsync per tensor")
+                         "memory) in two halves beside the two long GEMMs of the error signal, "
+                         "sm1 = one fpo_h2d_copy per step, ce = cudaMemcpyAsync per tensor")
     ap.add_argument("--band", type=int, default=0,
                     help="GEMM rasterisation band height in tiles (0: library default; tuning)")
     ap.add_argument("--gemm-variant", type=int, choices=(-1, 0, 1, 2), default=-1,
