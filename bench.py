@@ -232,7 +232,9 @@ def workload_config(wl, args):
             "optimizer": ("plain SGD fused in the update GEMM epilogue" if args.optimizer == "fused-sgd"
                           else f"{args.optimizer} on fp32 masters, clip={args.clip} (1% of ||W||_F)"),
             "l2": "inputs larger than L2 (W_U %.0f MB, A_l %.2f GB per step); no flush"
-                  % (wl.V * wl.d * 2 / 1e6, wl.layers * wl.T * wl.d_ff * 2 / 1e9)}
+                  % (wl.V * wl.d * 2 / 1e6, wl.layers * wl.T * wl.d_ff * 2 / 1e9),
+            **({"inputs": "window stress: +-1 hidden states, W_U x 64"}
+               if getattr(args, "window_stress", False) else {})}
 
 
 # --------------------------------------------------------------------------- GPU arm
@@ -261,6 +263,11 @@ def run_fpo(args, wl):
     w = synth.make_norm_w(wl_r, dev)
     W_U = synth.make_W_U(wl_r, dev)
     y = synth.make_targets(wl_r, dev)
+    if args.window_stress:
+        # logits ~30x the usual scale (+-1 hidden states, W_U x 64): most tokens fall
+        # outside the direct algorithm's anchor window and are recomputed by its fixup
+        h = torch.where(h >= 0, 1.0, -1.0).to(h.dtype)
+        W_U = (W_U.float() * 64).to(W_U.dtype)
     A = [synth.make_A(wl_r, l, dev) for l in range(wl.layers)]
     Wm = [synth.make_W_master(wl_r, l, dev) for l in range(wl.layers)]
     Wo = [torch.empty(wl.d, wl.d_ff, dtype=torch.bfloat16, device=dev) for _ in range(wl.layers)]
@@ -420,6 +427,9 @@ def run_fpo(args, wl):
         dist.barrier()
     ms = start.elapsed_time(end) / args.steps
     status = (fpo.get_device_status(ws_es), fpo.get_device_status(ws_up))
+    # rows of the last step the direct algorithm recomputed outside its anchor window
+    fixup_rows = (fpo.direct_fixup_rows(X0["h"], W_U, ws_es, t_chunk=args.t_chunk, algo=algo)
+                  if algo_name == "direct" else None)
 
     names = ["rmsnorm_fwd", "logits_lse_pass", "lse_combine",
              {"direct": "direct_fixup", "stored-logits": "logits_to_error",
@@ -588,6 +598,7 @@ def run_fpo(args, wl):
             "norm_ratio": ({"ratio": ratio_out[:, 2].tolist(),
                             "implied_sgd_lr_1pct": ratio_out[:, 3].tolist()} if ratio else None),
             "algo": algo_name,
+            "direct_fixup_rows": fixup_rows,
             "gemm_kernel": {0: "single-cta 128x256 (tcgen05 cta_group::1)",
                             1: "cta-pair 256x256 (tcgen05 cta_group::2)",
                             2: "cta-pair 256x256, projection 256x512 (tcgen05 cta_group::2)"
@@ -684,6 +695,9 @@ def main():
     ap.add_argument("--gemm-variant", type=int, choices=(-1, 0, 1, 2), default=-1,
                     help="tensor-core GEMM kernel: 0 single-CTA tiles, 1 CTA-pair tiles, "
                          "2 CTA-pair tiles with a 256x512 projection, -1 library default")
+    ap.add_argument("--window-stress", action="store_true",
+                    help="+-1 hidden states and W_U x 64: most tokens fall outside the direct "
+                         "algorithm's anchor window (its worst case); reports the rows recomputed")
     ap.add_argument("--shape", default=None,
                     help="T,d,d_ff,V,layers override of the workload's shape (small ncu cases)")
     ap.add_argument("--cpu-tokens", type=int, default=256,
