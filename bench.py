@@ -684,8 +684,10 @@ def main():
                          "(always on for the diag workload)")
     ap.add_argument("--norm-ratio", action="store_true",
                     help="add the App. C update-magnitude ratio ||G_l||/||W_l|| to every step")
-    ap.add_argument("--e2e-depth", type=int, default=3,
-                    help="device input sets of the end-to-end loop (copies run depth-1 steps ahead)")
+    ap.add_argument("--e2e-depth", type=int, default=6,
+                    help="device input sets of the end-to-end loop (copies run up to depth-1 steps "
+                         "ahead, so a stall of the host link shorter than that many steps is "
+                         "absorbed)")
     ap.add_argument("--e2e-copy", choices=("sm", "sm1", "ce"), default="sm",
                     help="end-to-end input copies: sm = fpo_h2d_copy (SM loads of mapped pinned "
                          "memory) in two halves beside the two long GEMMs of the error signal, "
