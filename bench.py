@@ -569,7 +569,11 @@ def run_fpo(args, wl):
         peak_sus = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
         achieved = per_kernel_flops[dom] / (stage_ms[dom] / 1e3) / 1e12
         roofline = {"bound": "tensor", "achieved": achieved, "peak": peak_sus, "unit": "TFLOP/s",
-                    "frac": achieved / peak_sus, "traffic": load_traffic(dom),
+                    "frac": achieved / peak_sus,
+                    "traffic": load_traffic(dom, {"workload": wl.name, "algo": algo_name,
+                                                  "gemm_variant": variant,
+                                                  "t_chunk": args.t_chunk or wl.T,
+                                                  "window_stress": bool(args.window_stress)}),
                     "kernel": dom, "peak_kind": f"bf16 sustained ({peaks_src})"}
         cpu = None
         if world == 1 and not args.no_cpu:
@@ -625,14 +629,17 @@ KERNEL_SOURCES = {
 }
 
 
-def load_traffic(kernel):
+def load_traffic(kernel, run_config):
     """Per-launch DRAM bytes of `kernel` from the committed ncu summary, or None when that
-    summary is missing or was taken on different sources of that kernel."""
+    summary is missing, was taken on another configuration (workload, algorithm, kernel
+    variant, token chunk, inputs) or on different sources of that kernel."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     if not os.path.exists(path) or kernel not in KERNEL_SOURCES:
         return None
     with open(path) as f:
         tr = json.load(f)
+    if tr.get("_config") != run_config:
+        return None
     ent = tr.get(kernel)
     if not ent or ent.get("sources_sha256") != sources_digest(KERNEL_SOURCES[kernel]):
         return None
