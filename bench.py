@@ -605,7 +605,9 @@ def run_fpo(args, wl):
             "direct_fixup_rows": fixup_rows,
             "gemm_kernel": {0: "single-cta 128x256 (tcgen05 cta_group::1)",
                             1: "cta-pair 256x256 (tcgen05 cta_group::2)",
-                            2: "cta-pair 256x256, projection 256x512 (tcgen05 cta_group::2)"
+                            2: "cta-pair 256x256, projection 256x512 (tcgen05 cta_group::2)",
+                            3: "two cta-pairs sharing B (TMA multicast) for the logits pass and "
+                               "the update, projection 256x512 (tcgen05 cta_group::2)"
                             }[variant],
             "cpu_baseline": cpu,
             "e2e": e2e,
@@ -705,9 +707,11 @@ def main():
                          "sm1 = one fpo_h2d_copy per step, ce = cudaMemcpyAsync per tensor")
     ap.add_argument("--band", type=int, default=0,
                     help="GEMM rasterisation band height in tiles (0: library default; tuning)")
-    ap.add_argument("--gemm-variant", type=int, choices=(-1, 0, 1, 2), default=-1,
+    ap.add_argument("--gemm-variant", type=int, choices=(-1, 0, 1, 2, 3), default=-1,
                     help="tensor-core GEMM kernel: 0 single-CTA tiles, 1 CTA-pair tiles, "
-                         "2 CTA-pair tiles with a 256x512 projection, -1 library default")
+                         "2 CTA-pair tiles with a 256x512 projection, 3 as 2 with two CTA pairs "
+                         "sharing each B tile in the logits pass and the update, -1 library "
+                         "default")
     ap.add_argument("--window-stress", action="store_true",
                     help="+-1 hidden states and W_U x 64: most tokens fall outside the direct "
                          "algorithm's anchor window (its worst case); reports the rows recomputed")

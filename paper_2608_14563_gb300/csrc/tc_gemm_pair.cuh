@@ -130,12 +130,25 @@ __device__ __forceinline__ void load_operand_pair(const CUtensorMap* map, uint32
     }
 }
 
-template <int BN, bool A_MN, bool B_MN, int STAGES, int MAXG, class Epi>
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
+// 64 rows (M or N) x one k-block of an operand, multicast to the CTAs of cta_mask:
+// K-major one box {64 (K), 64 rows}, MN-major one box {64 (M or N), 64 (K)}.
+template <bool MN>
+__device__ __forceinline__ void load_operand_pair_mc(const CUtensorMap* map, uint32_t dst,
+                                                     uint32_t bar_leader, int row0, int k0,
+                                                     uint16_t cta_mask) {
+    if constexpr (!MN)
+        tma_load_2d_pair_mc(map, dst, bar_leader, k0, row0, cta_mask);
+    else
+        tma_load_2d_pair_mc(map, dst, bar_leader, row0, k0, cta_mask);
+}
+
+template <int BN, bool A_MN, bool B_MN, int STAGES, int MAXG, class Epi, int kPairs = 1>
+__global__ void __cluster_dims__(2 * kPairs, 1, 1) __launch_bounds__(kGemmThreads, 1)
     tc_gemm_pair_kernel(const __grid_constant__ GemmMaps<MAXG> maps,
                         const __grid_constant__ typename Epi::Params ep, const GemmShape sh_in,
                         unsigned int* status, unsigned long long wait_limit_ns) {
     static_assert(BN == 256 || BN == 512, "pair tiles are 256 or 512 columns wide");
+    static_assert(kPairs == 1 || (kPairs == 2 && BN == 256), "two pairs share 256-wide B tiles");
     using L = GemmPairSmem<BN, STAGES>;
     constexpr int kNSub = BN / 256;                // N = 256 MMAs per K slice
     constexpr int kAccBufs = kNSub == 1 ? 2 : 1;   // accumulator buffers in TMEM
@@ -143,14 +156,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     constexpr uint32_t kBSubBytes = kBSub * kBK * 2;
     constexpr uint32_t kIdesc = idesc_bf16_f32(kPairBM, 256, A_MN, B_MN);
     constexpr int kTmemCols = kAccBufs * BN;       // 512 either way
-    constexpr uint16_t kBoth = 0x3;
+    constexpr int kCta = 2 * kPairs;                  // CTAs of the cluster
+    constexpr uint16_t kAll = (1u << kCta) - 1u;      // every CTA of the cluster
+    constexpr int kClusterBM = kPairBM * kPairs;      // output rows of one cluster tile
 
     GemmShape sh = sh_in;
     if (sh.m_dev) {  // rows counted on the device (every thread reads the same value)
         const int m = min(*sh.m_dev, sh.M);
         if (m <= 0) return;
         sh.M = m;
-        sh.m_blocks = (m + kPairBM - 1) / kPairBM;
+        sh.m_blocks = (m + kClusterBM - 1) / kClusterBM;
         sh.tiles = static_cast<long long>(sh.groups) * sh.m_blocks * sh.n_blocks;
         sh.tail_tiles = 0;
     }
@@ -162,9 +177,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     const uint32_t sbase = raw + pad;
 
     const uint32_t rank = cluster_ctarank();
-    const bool leader = rank == 0;
-    const long long cluster = blockIdx.x >> 1;
-    const long long n_clusters = gridDim.x >> 1;
+    const uint32_t prank = rank & 1u;        // position in the CTA pair
+    const uint32_t pair = rank >> 1;         // which pair of the cluster
+    const uint32_t lrank = rank & ~1u;       // the pair's leader (issues its MMAs)
+    const bool leader = prank == 0;
+    const uint16_t pair_mask = static_cast<uint16_t>(0x3u << lrank);
+    const long long cluster = blockIdx.x / kCta;
+    const long long n_clusters = gridDim.x / kCta;
 
     const uint32_t bar0 = sbase + L::kBarOffset;
     auto full_bar = [&](int s) { return bar0 + 8u * s; };
@@ -181,7 +200,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(full_bar(s), 1);   // leader's: one expect_tx arrival, both CTAs' bytes
-            mbar_init(empty_bar(s), 1);  // one multicast commit from the leader
+            mbar_init(empty_bar(s), kPairs);  // one multicast commit from each pair leader
         }
         for (int a = 0; a < 2; ++a) {
             mbar_init(tfull_bar(a), 1);
@@ -219,19 +238,30 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
                 tile_coords(t, sh, g, mp, nb);
                 const CUtensorMap* amap = &maps.a[MAXG == 1 ? 0 : g];
                 const CUtensorMap* bmap = &maps.b[MAXG == 1 ? 0 : g];
-                const int a_row = mp * kPairBM + 128 * static_cast<int>(rank);
-                const int b_row = nb * BN + kBSub * static_cast<int>(rank);
+                const int a_row = (mp * kPairs + static_cast<int>(pair)) * kPairBM +
+                                  128 * static_cast<int>(prank);
+                const int b_row = nb * BN + kBSub * static_cast<int>(prank);
                 for (int kb = kb0; kb < kb1; ++kb) {
                     if (!mbar_wait_cl(empty_bar(stage), phase ^ 1u, guard)) { ok = false; break; }
                     const uint32_t sa = sbase + stage * L::kStageBytes;
                     const uint32_t sb = sa + L::kABytes;
-                    const uint32_t fb = mapa_shared(full_bar(stage), 0);
+                    const uint32_t fb = mapa_shared(full_bar(stage), lrank);
                     if (leader) mbar_arrive_expect_tx(full_bar(stage), 2 * L::kStageBytes);
                     load_operand_pair<A_MN, 128>(amap, sa, fb, a_row, kb * kBK);
+                    if constexpr (kPairs == 1) {
 #pragma unroll
-                    for (int h = 0; h < kNSub; ++h)
-                        load_operand_pair<B_MN, kBSub>(bmap, sb + h * kBSubBytes, fb,
-                                                       b_row + 256 * h, kb * kBK);
+                        for (int h = 0; h < kNSub; ++h)
+                            load_operand_pair<B_MN, kBSub>(bmap, sb + h * kBSubBytes, fb,
+                                                           b_row + 256 * h, kb * kBK);
+                    } else {
+                        // the pairs share the B tile: this CTA loads the 64 rows of its
+                        // half of B at position `pair` and multicasts them to the CTA
+                        // holding the same half in the other pair; each destination
+                        // pair's leader counts the bytes
+                        load_operand_pair_mc<B_MN>(
+                            bmap, sb + pair * (64u * kBK * 2u), fb, b_row + 64 * static_cast<int>(pair),
+                            kb * kBK, static_cast<uint16_t>((1u << prank) | (1u << (prank + 2))));
+                    }
                     issued_mask |= 1u << stage;
                     issued_parity = (issued_parity & ~(1u << stage)) | (phase << stage);
                     if (++stage == STAGES) { stage = 0; phase ^= 1u; }
@@ -274,15 +304,17 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
                                              operand_desc<B_MN>(sb + h * kBSubBytes, kk), kIdesc,
                                              (kb != kb0 || kk != 0) ? 1u : 0u);
                     issued_any = true;
-                    tc_commit_pair_multicast(empty_bar(stage), kBoth);
+                    // the stage is free in every CTA once every pair has consumed it (the
+                    // other pair's B rows were written into this pair's stage too)
+                    tc_commit_pair_multicast(empty_bar(stage), kAll);
                     if (++stage == STAGES) { stage = 0; phase ^= 1u; }
                 }
                 if (!ok) break;
-                tc_commit_pair_multicast(tfull_bar(acc), kBoth);
+                tc_commit_pair_multicast(tfull_bar(acc), pair_mask);
                 if (++acc == kAccBufs) { acc = 0; acc_phase ^= 1u; }
             }
             if (!ok && issued_any) {
-                tc_commit_pair_multicast(drain_bar, 0x1);
+                tc_commit_pair_multicast(drain_bar, static_cast<uint16_t>(1u << lrank));
                 mbar_wait_cl_drain(drain_bar, 0, wait_limit_ns);
             }
         }
@@ -290,7 +322,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     } else {
         // ------------------------------------------------------- epilogue (both CTAs)
         const int q = warp & 3;
-        const int r_in_tile = 128 * static_cast<int>(rank) + q * 32 + lane;
+        const int r_in_tile = 128 * static_cast<int>(prank) + q * 32 + lane;
         EpiIO io{sbase + L::kOutOffset + static_cast<uint32_t>((warp - 2) * kOutBytesPerWarp), lane,
                  0, 0u};
         int acc = 0;
@@ -306,9 +338,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
             const uint32_t t_row = tmem_base + (static_cast<uint32_t>(q * 32) << 16) +
                                    static_cast<uint32_t>(acc * BN);
             if (part < 0) {
-                const int row = mp * kPairBM + r_in_tile;
+                const int tile_row0 = (mp * kPairs + static_cast<int>(pair)) * kPairBM;
+                const int row = tile_row0 + r_in_tile;
                 const int n0 = nb * BN;
-                io.row0 = mp * kPairBM + 128 * static_cast<int>(rank) + q * 32;
+                io.row0 = tile_row0 + 128 * static_cast<int>(prank) + q * 32;
                 Epi epi(ep, g, row, n0);
 #pragma unroll 1
                 for (int c = 0; c < BN / 32; ++c) {
@@ -336,7 +369,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
                 if (leader)
                     mbar_arrive(tempty_bar(acc));
                 else
-                    mbar_arrive_cluster(mapa_shared(tempty_bar(acc), 0));
+                    mbar_arrive_cluster(mapa_shared(tempty_bar(acc), lrank));
             }
             if (++acc == kAccBufs) { acc = 0; acc_phase ^= 1u; }
         }
@@ -346,7 +379,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
 
     tc_fence_before();
     __syncthreads();
-    cluster_sync();  // neither CTA frees TMEM or exits while the pair may still touch it
+    cluster_sync();  // no CTA frees TMEM or exits while another may still touch it
     if (warp == 1) {
         tc_fence_after();
         tmem_dealloc_pair<kTmemCols>(tmem_base);

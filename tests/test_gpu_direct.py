@@ -92,7 +92,7 @@ def test_direct_is_bitwise_identical_across_gemm_kernels(fpo, ragged):
     prev = fpo.set_gemm_variant(0)
     outs = []
     try:
-        for v in (0, 1, 2):
+        for v in (0, 1, 2, 3):
             fpo.set_gemm_variant(v)
             outs.append(run(fpo, inp["h"], inp["w"], inp["W_U"], inp["y"], eps=RAGGED.eps,
                             algo=fpo.ES_DIRECT))
@@ -163,7 +163,7 @@ def test_rows_outside_the_anchor_window_are_fixed(fpo):
     assert abs(outs[0]["loss"].item() - oracle.mean_ce(ref["lse"], ref["zy"])) < 1e-4 * np.mean(ce)
 
 
-@pytest.mark.parametrize("variant", [0, 1, 2])
+@pytest.mark.parametrize("variant", [0, 1, 2, 3])
 @pytest.mark.parametrize("algo", [1, 2, 3])  # recompute, stored logits, direct
 def test_results_do_not_depend_on_workspace_contents(fpo, ragged, variant, algo):
     """Every workspace byte a call reads it writes first: a workspace full of 0xFF (NaN
@@ -247,3 +247,31 @@ def test_projection_split_k_tail(fpo, algo):
         assert np.max(row_err) < 5e-3
     ref = reference(h, w, W_U, y, eps=wl.eps, s=wl.loss_scale)
     assert rel_frob(ga, ref["g_tilde"]) < TOL and cos(ga, ref["g_tilde"]) >= COS_MIN
+
+
+@pytest.mark.parametrize("shape", [(700, 320, 840, 3), (1024, 512, 768, 2), (300, 1024, 264, 4)])
+def test_update_is_bitwise_identical_across_gemm_kernels(fpo, shape):
+    """The grouped update (G_l, the fp32 master step, the bf16 weights) computes the same
+    sums in the same order per element under every GEMM kernel variant: single CTA, CTA
+    pair, and two CTA pairs sharing each B tile by multicast (ragged T and d)."""
+    T, d, d_ff, L = shape
+    gen = torch.Generator(device="cuda").manual_seed(T + d)
+    g = (torch.randn(T, d, device="cuda", generator=gen) * 1e-2).to(torch.bfloat16)
+    A = [torch.randn(T, d_ff, device="cuda", generator=gen).to(torch.bfloat16) for _ in range(L)]
+    W0 = [0.02 * torch.randn(d, d_ff, device="cuda", generator=gen) for _ in range(L)]
+    prev = fpo.set_gemm_variant(0)
+    outs = []
+    try:
+        for v in (0, 1, 2, 3):
+            fpo.set_gemm_variant(v)
+            Wm = [w.clone() for w in W0]
+            Wo = [torch.empty(d, d_ff, dtype=torch.bfloat16, device="cuda") for _ in range(L)]
+            Go = [torch.empty(d, d_ff, dtype=torch.bfloat16, device="cuda") for _ in range(L)]
+            ws = fpo.layer_update_grouped(g, A, 1e-3, W_masters=Wm, W_outs=Wo, G_outs=Go)
+            assert fpo.get_device_status(ws) == fpo.OK
+            outs.append(Wm + Wo + Go)
+    finally:
+        fpo.set_gemm_variant(prev)
+    for o in outs[1:]:
+        for a, b in zip(outs[0], o):
+            assert torch.equal(a, b)

@@ -31,7 +31,7 @@ def _shapes(n, seed=2024):
 SHAPES = _shapes(12)
 
 
-@pytest.mark.parametrize("variant", [0, 1, 2])
+@pytest.mark.parametrize("variant", [0, 1, 2, 3])
 @pytest.mark.parametrize("algo", [1, 2, 3])  # recompute, stored logits, direct
 @pytest.mark.parametrize("shape", SHAPES, ids=[f"T{t}d{d}V{v}f{f}" for t, d, v, f in SHAPES])
 def test_random_ragged_shapes(fpo, shape, algo, variant):
