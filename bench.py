@@ -228,7 +228,8 @@ def workload_config(wl, args):
             "error_matrix": {"auto": "direct (auto)", "recompute": "recompute",
                              "stored": "stored-logits", "direct": "direct"}[args.algo],
             "norms_composed": "final + post-FFN per layer" if args.post_ffn_norm else "final",
-            "weights_updated": "W3, W1, W2 (W1/W2 via W3_init feedback)" if args.gate_up else "W3",
+            "weights_updated": ("W3, W1, W2 (W1/W2 via W3_init feedback, the same optimizer)"
+                                if args.gate_up else "W3"),
             "optimizer": ("plain SGD fused in the update GEMM epilogue" if args.optimizer == "fused-sgd"
                           else f"{args.optimizer} on fp32 masters, clip={args.clip} (1% of ||W||_F)"),
             "l2": "inputs larger than L2 (W_U %.0f MB, A_l %.2f GB per step); no flush"
@@ -309,6 +310,13 @@ def run_fpo(args, wl):
                if kind == fpo.OPT_ADAMW else None)
         ws_up = torch.empty(fpo.layer_optimize_workspace(wl.layers, wl.d, wl.d_ff),
                             dtype=torch.uint8, device=dev)
+        if gate_up:  # the same optimizer and clip on W1 and W2 of every target layer
+            gu_st1 = ([torch.zeros(wl.d_ff, wl.d, device=dev) for _ in range(2 * wl.layers)]
+                      if kind != fpo.OPT_SGD else None)
+            gu_st2 = ([torch.zeros(wl.d_ff, wl.d, device=dev) for _ in range(2 * wl.layers)]
+                      if kind == fpo.OPT_ADAMW else None)
+            ws_gu_opt = torch.empty(fpo.layer_optimize_workspace(2 * wl.layers, wl.d_ff, wl.d),
+                                    dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream()
 
     # The tensors one step reads that come from the forward pass / the data: the
@@ -363,8 +371,12 @@ def run_fpo(args, wl):
                                 X["ab"][2 * l + 1], gu_sig[2 * l], gu_sig[2 * l + 1],
                                 workspace=ws_gu)
         gu_act = [x for x in X["x"] for _ in range(2)]
-        fpo.layer_update_grouped_signals(gu_sig, gu_act, wl.lr, W_masters=gu_W12, W_outs=gu_out,
-                                         workspace=ws_gu)
+        if optimize:
+            fpo.layer_optimize_grouped(gu_sig, gu_act, opt, gu_W12, W_outs=gu_out,
+                                       states1=gu_st1, states2=gu_st2, workspace=ws_gu_opt)
+        else:
+            fpo.layer_update_grouped_signals(gu_sig, gu_act, wl.lr, W_masters=gu_W12,
+                                             W_outs=gu_out, workspace=ws_gu)
 
     def step(X, stage_events=None, upd_events=None):
         fpo.error_signal(X["h"], w, W_U, X["y"], g, eps=wl.eps, min_rms=wl.min_rms,
