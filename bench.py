@@ -188,6 +188,19 @@ def cores():
         return os.cpu_count()
 
 
+def cpu_model():
+    """The host CPU's model name (lscpu), for the CPU-baseline record."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.strip().startswith("Model name:"):
+                return line.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    import platform
+    return platform.processor() or platform.machine()
+
+
 def sample_text(r, wl):
     return (f"{r['n_tok']} of {wl.T} tokens through the oracle (error signal {r['es_s']:.2f} s, "
             f"G for 1 of {wl.layers} layers {r['G_s']:.2f} s, one weight update {r['upd_s']:.2f} s),"
@@ -213,7 +226,8 @@ def run_reference(args, wl):
         "ms_per_step": step_s * 1e3, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": workload_config(wl, args),
-        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores(), "kind": "oracle",
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores(),
+                         "cpu_model": cpu_model(), "kind": "oracle",
                          "sample": sample_text(steps[-1], wl)},
         "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
@@ -591,6 +605,7 @@ def run_fpo(args, wl):
         if world == 1 and not args.no_cpu:
             r = oracle_sample(wl, args.cpu_tokens)
             cpu = {"value": r["tokens_per_s"], "unit": "tokens/s", "cores": cores(),
+                   "cpu_model": cpu_model(),
                    "kind": "oracle", "sample": sample_text(r, wl)}
         line = {
             "metric": METRIC, "value": tok_s, "unit": "tokens/s", "n_gpus": world,
