@@ -238,7 +238,8 @@ def run_reference(args, wl):
 def workload_config(wl, args):
     return {"workload": wl.name, "T": wl.T, "d": wl.d, "d_ff": wl.d_ff, "V": wl.V,
             "target_layers": wl.layers, "targets": "zipf(1.1)" if wl.targets == "zipf" else wl.targets,
-            "lr": wl.lr, "t_chunk": args.t_chunk or wl.T, "global_batch_tokens": wl.T * args.gpus,
+            "lr": wl.lr, "t_chunk": min(args.t_chunk or AUTO_T_CHUNK, wl.T),
+            "global_batch_tokens": wl.T * args.gpus,
             "error_matrix": {"auto": "direct (auto)", "recompute": "recompute",
                              "stored": "stored-logits", "direct": "direct"}[args.algo],
             "norms_composed": "final + post-FFN per layer" if args.post_ffn_norm else "final",
@@ -392,10 +393,10 @@ def run_fpo(args, wl):
             fpo.layer_update_grouped_signals(gu_sig, gu_act, wl.lr, W_masters=gu_W12,
                                              W_outs=gu_out, workspace=ws_gu)
 
-    def step(X, stage_events=None, upd_events=None):
+    def step(X, stage_events=None, upd_events=None, per_chunk=False):
         fpo.error_signal(X["h"], w, W_U, X["y"], g, eps=wl.eps, min_rms=wl.min_rms,
                          t_chunk=args.t_chunk, loss_out=loss, workspace=ws_es,
-                         stage_events=stage_events, algo=algo)
+                         stage_events=stage_events, algo=algo, per_chunk_events=per_chunk)
         if post:
             if upd_events:
                 upd_events[2].record(stream)
@@ -428,9 +429,14 @@ def run_fpo(args, wl):
     torch.cuda.synchronize()
     assert fpo.get_device_status(ws_es) == fpo.OK and fpo.get_device_status(ws_up) == fpo.OK
 
-    # per-stage events for every timed step (recorded once so their handles exist)
-    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(fpo.STAGE_EVENTS)]
-          for _ in range(args.steps)]
+    # per-stage events of every token chunk, for every timed step (recorded once so their
+    # handles exist): 0 start, 1 after the RMSNorm forward, per chunk c the ends of its
+    # logits pass (2+4c), combine (3+4c), fixup / E stage (4+4c) and projection (5+4c), and
+    # the end of the VJP (2+4n)
+    n_ev = fpo.stage_event_count(fpo.error_signal_desc(
+        wl.T, wl.d, wl.V, fpo.BF16, t_chunk=args.t_chunk, algo=algo, per_chunk_events=True))
+    n_chunks = (n_ev - 3) // 4
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(n_ev)] for _ in range(args.steps)]
     uev = [[torch.cuda.Event(enable_timing=True) for _ in range(8)] for _ in range(args.steps)]
     for e in [x for row in ev + uev for x in row]:
         e.record(stream)
@@ -444,7 +450,7 @@ def run_fpo(args, wl):
     launches0 = fpo.kernel_launches()  # the library counts every kernel it launches
     start.record(stream)
     for i in range(args.steps):
-        step(X0, ev[i], uev[i])
+        step(X0, ev[i], uev[i], per_chunk=True)
     end.record(stream)
     launches = fpo.kernel_launches() - launches0
     torch.cuda.synchronize()
@@ -453,14 +459,26 @@ def run_fpo(args, wl):
         dist.barrier()
     ms = start.elapsed_time(end) / args.steps
     status = (fpo.get_device_status(ws_es), fpo.get_device_status(ws_up))
-    # rows of the last step the direct algorithm recomputed outside its anchor window
+    # rows of the last step's last token chunk that the direct algorithm recomputed
+    # outside its anchor window
     fixup_rows = (fpo.direct_fixup_rows(X0["h"], W_U, ws_es, t_chunk=args.t_chunk, algo=algo)
                   if algo_name == "direct" else None)
 
     names = ["rmsnorm_fwd", "logits_lse_pass", "lse_combine",
              {"direct": "direct_fixup", "stored-logits": "logits_to_error",
               "recompute": "recompute_error_pass"}[algo_name], "projection", "rmsnorm_vjp"]
-    stage_ms = {n: statistics.mean(ev[i][k].elapsed_time(ev[i][k + 1]) for i in range(args.steps))
+    def stage_sum(e, k):  # one kernel stage summed over the token chunks (k: 1..4)
+        if k == 0:
+            return e[0].elapsed_time(e[1])
+        if k == 5:
+            return e[5 + 4 * (n_chunks - 1)].elapsed_time(e[2 + 4 * n_chunks])
+        total = 0.0
+        for c in range(n_chunks):
+            a = (1 if c == 0 else 5 + 4 * (c - 1)) if k == 1 else k + 4 * c
+            total += e[a].elapsed_time(e[k + 1 + 4 * c])
+        return total
+
+    stage_ms = {n: statistics.mean(stage_sum(ev[i], k) for i in range(args.steps))
                 for k, n in enumerate(names)}
     stage_ms["layer_update"] = statistics.mean(uev[i][0].elapsed_time(uev[i][1])
                                                for i in range(args.steps))
@@ -598,7 +616,8 @@ def run_fpo(args, wl):
                     "frac": achieved / peak_sus,
                     "traffic": load_traffic(dom, {"workload": wl.name, "algo": algo_name,
                                                   "gemm_variant": variant,
-                                                  "t_chunk": args.t_chunk or wl.T,
+                                                  "t_chunk": min(args.t_chunk or AUTO_T_CHUNK,
+                                                                 wl.T),
                                                   "window_stress": bool(args.window_stress)}),
                     "kernel": dom, "peak_kind": f"bf16 sustained ({peaks_src})"}
         cpu = None
@@ -629,7 +648,7 @@ def run_fpo(args, wl):
             "norm_ratio": ({"ratio": ratio_out[:, 2].tolist(),
                             "implied_sgd_lr_1pct": ratio_out[:, 3].tolist()} if ratio else None),
             "algo": algo_name,
-            "direct_fixup_rows": fixup_rows,
+            "direct_fixup_rows_last_chunk": fixup_rows,
             "gemm_kernel": {0: "single-cta 128x256 (tcgen05 cta_group::1)",
                             1: "cta-pair 256x256 (tcgen05 cta_group::2)",
                             2: "cta-pair 256x256, projection 256x512 (tcgen05 cta_group::2)",
@@ -646,6 +665,9 @@ def run_fpo(args, wl):
     if world > 1:
         dist.destroy_process_group()
 
+
+# The library's token chunk when --t-chunk is 0 (FPO_AUTO_T_CHUNK in include/fpo.h).
+AUTO_T_CHUNK = 8192
 
 # Files that define each kernel whose DRAM traffic profiles/traffic.json records.
 GEMM_SOURCES = ("tc_gemm.cuh", "tc_gemm_pair.cuh", "epilogues.cuh", "error_math.cuh", "ptx.cuh",

@@ -52,7 +52,7 @@
 extern "C" {
 #endif
 
-#define FPO_ABI_VERSION 1
+#define FPO_ABI_VERSION 2
 
 /* Largest number of layers one fpo_layer_update_grouped call accepts. */
 #define FPO_MAX_GROUPED_LAYERS 64
@@ -102,15 +102,22 @@ typedef enum fpo_status {
  *                        bf16 once like E, and saves the E pass: T_chunk x V x 2
  *                        bytes of workspace.  Rows with S'_t outside
  *                        [2^-80, 2^80] (token cross-entropy beyond ~55 nats, or
- *                        1 - p_target below ~1e-24) are recomputed by an fp32
- *                        SIMT kernel anchored at lse_t before the projection.
+ *                        1 - p_target below ~1e-24) are gathered and recomputed
+ *                        by the same tensor-core logits GEMM anchored at lse_t
+ *                        before the projection (its row count read on the device).
  *  FPO_ES_AUTO           the library's choice: FPO_ES_DIRECT for bf16,
  *                        FPO_ES_STORED_LOGITS for fp32 (where DIRECT also runs
  *                        the stored-logits algorithm).
  * RECOMPUTE and STORED_LOGITS compute every value with the same arithmetic:
  * their outputs are bit-identical.  DIRECT agrees with them to the bf16
- * rounding of the probabilities, and is bit-identical across t_chunk values.
+ * rounding of the probabilities.  Results are deterministic; across t_chunk
+ * values they are bit-identical while the projection has whole tiles (fewer
+ * than one wave), and otherwise agree to rounding (its last partial wave is
+ * split into k ranges).
  */
+
+/* Tokens per error-matrix chunk when fpo_error_signal_desc.t_chunk is 0. */
+#define FPO_AUTO_T_CHUNK 8192
 typedef enum fpo_es_algo {
     FPO_ES_AUTO = 0,
     FPO_ES_RECOMPUTE = 1,
@@ -128,10 +135,13 @@ typedef struct fpo_error_signal_desc {
     float min_rms;      /* floor on rho in the 1/rho prefactor of the VJP (0.5)  */
     float loss_scale;   /* s in e = s (softmax(z) - 1_y); 1/T = mean-reduced CE */
     int32_t algo;       /* fpo_es_algo                                            */
-    int64_t t_chunk;    /* tokens per error-matrix chunk; 0 = all T at once       */
-    void* const* stage_events;  /* NULL, or FPO_STAGE_EVENTS caller-created
-                                   cudaEvent_t recorded on the stream at the stage
-                                   boundaries (profiling; see below)              */
+    int64_t t_chunk;    /* tokens per error-matrix chunk; 0 = FPO_AUTO_T_CHUNK    */
+    void* const* stage_events;  /* NULL, or caller-created cudaEvent_t recorded on
+                                   the stream at the stage boundaries (profiling;
+                                   see below)                                     */
+    int32_t stage_events_per_chunk; /* 0: FPO_STAGE_EVENTS events; 1: the stages of
+                                   every token chunk, fpo_error_signal_stage_events()
+                                   events (see below)                             */
 } fpo_error_signal_desc;
 
 /*
@@ -144,8 +154,19 @@ typedef struct fpo_error_signal_desc {
  * after the projection of the last token chunk, 6 after the final-norm VJP.
  * With one chunk, consecutive events bracket one kernel each (plus the loss
  * mean in [2]-[3]).
+ * With stage_events_per_chunk = 1 and n token chunks the events are 3 + 4 n:
+ * 0 start, 1 after the RMSNorm forward, then for chunk c = 0 .. n-1:
+ * 2 + 4c after its logits pass, 3 + 4c after its combine (and, last chunk, the
+ * loss mean), 4 + 4c after its E / fixup stage, 5 + 4c after its projection;
+ * and 2 + 4n after the VJP.  (FPO_ES_RECOMPUTE runs one logits pass and one
+ * combine over all tokens: they fill chunk 0's first two slots; the other
+ * chunks record those two at the chunk's start.)
  */
 #define FPO_STAGE_EVENTS 7
+
+/* Number of stage events `desc` asks for (FPO_STAGE_EVENTS, or 3 + 4 n with
+ * stage_events_per_chunk), or 0 on a bad desc. */
+int32_t fpo_error_signal_stage_events(const fpo_error_signal_desc* desc);
 
 /* Bytes of workspace fpo_error_signal needs for `desc` (0 on a bad desc). */
 size_t fpo_error_signal_workspace(const fpo_error_signal_desc* desc);

@@ -23,6 +23,7 @@ OK = 0
 MAX_GROUPED_LAYERS = 64
 STAGE_EVENTS = 7
 ES_AUTO, ES_RECOMPUTE, ES_STORED_LOGITS, ES_DIRECT = 0, 1, 2, 3
+AUTO_T_CHUNK = 8192  # FPO_AUTO_T_CHUNK: tokens per error-matrix chunk when t_chunk is 0
 
 if not os.path.exists(LIB_PATH):
     raise ImportError(f"libfpo.so is not built ({LIB_PATH} missing); run "
@@ -37,7 +38,7 @@ class ErrorSignalDesc(ctypes.Structure):
     """Mirror of fpo_error_signal_desc."""
     _fields_ = [("T", _i64), ("d", _i64), ("V", _i64), ("dtype", _i32), ("eps", _f32),
                 ("min_rms", _f32), ("loss_scale", _f32), ("algo", _i32), ("t_chunk", _i64),
-                ("stage_events", ctypes.POINTER(_vp))]
+                ("stage_events", ctypes.POINTER(_vp)), ("stage_events_per_chunk", _i32)]
 
 
 _lib.fpo_abi_version.restype = _i32
@@ -45,6 +46,8 @@ _lib.fpo_status_string.argtypes = [_i32]
 _lib.fpo_status_string.restype = ctypes.c_char_p
 _lib.fpo_set_wait_limit_ns.argtypes = [ctypes.c_uint64]
 _lib.fpo_set_wait_limit_ns.restype = None
+_lib.fpo_error_signal_stage_events.argtypes = [ctypes.POINTER(ErrorSignalDesc)]
+_lib.fpo_error_signal_stage_events.restype = _i32
 _lib.fpo_error_signal_workspace.argtypes = [ctypes.POINTER(ErrorSignalDesc)]
 _lib.fpo_error_signal_workspace.restype = _sz
 _lib.fpo_error_signal.argtypes = [ctypes.POINTER(ErrorSignalDesc), _vp, _vp, _vp, _vp, _vp, _vp,
@@ -181,19 +184,26 @@ def _workspace(nbytes: int, device) -> torch.Tensor:
 
 # --------------------------------------------------------------------------- error signal
 def error_signal_desc(T, d, V, dtype=BF16, *, eps=1e-6, min_rms=0.5, loss_scale=None, t_chunk=0,
-                      stage_events=None, algo=ES_AUTO):
-    """fpo_error_signal_desc; ``stage_events`` is None or STAGE_EVENTS torch.cuda.Event objects
-    that have been recorded once (so their CUDA handles exist)."""
+                      stage_events=None, algo=ES_AUTO, per_chunk_events=False):
+    """fpo_error_signal_desc; ``stage_events`` is None or torch.cuda.Event objects that have
+    been recorded once (so their CUDA handles exist): STAGE_EVENTS of them, or with
+    ``per_chunk_events`` stage_event_count() of them (every token chunk's stages)."""
     s = (1.0 / T if T > 0 else 1.0) if loss_scale is None else loss_scale
-    ev = None
-    if stage_events is not None:
-        if len(stage_events) != STAGE_EVENTS:
-            raise ValueError(f"stage_events needs {STAGE_EVENTS} events")
-        ev = (_vp * STAGE_EVENTS)(*[e.cuda_event for e in stage_events])
     d = ErrorSignalDesc(int(T), int(d), int(V), int(dtype), float(eps), float(min_rms), float(s),
-                        int(algo), int(t_chunk), ev)
-    d._keep = ev
+                        int(algo), int(t_chunk), None, 1 if per_chunk_events else 0)
+    if stage_events is not None:
+        need = stage_event_count(d)
+        if len(stage_events) != need:
+            raise ValueError(f"stage_events needs {need} events")
+        ev = (_vp * need)(*[e.cuda_event for e in stage_events])
+        d.stage_events = ctypes.cast(ev, ctypes.POINTER(_vp))
+        d._keep = ev
     return d
+
+
+def stage_event_count(desc: ErrorSignalDesc) -> int:
+    """fpo_error_signal_stage_events: events the descriptor's stage-event layout needs."""
+    return int(_lib.fpo_error_signal_stage_events(ctypes.byref(desc)))
 
 
 def error_signal_workspace(desc: ErrorSignalDesc) -> int:
@@ -202,7 +212,7 @@ def error_signal_workspace(desc: ErrorSignalDesc) -> int:
 
 def error_signal(h, norm_w, W_U, targets, g_out, *, eps=1e-6, min_rms=0.5, loss_scale=None,
                  t_chunk=0, lse_out=None, loss_out=None, workspace=None, stream=None,
-                 stage_events=None, algo=ES_AUTO):
+                 stage_events=None, algo=ES_AUTO, per_chunk_events=False):
     """fpo_error_signal: g~ = final-RMSNorm VJP of (softmax(z) - 1_y) W_U into ``g_out``.
 
     Returns the workspace tensor (its first word holds the device status).
@@ -211,7 +221,7 @@ def error_signal(h, norm_w, W_U, targets, g_out, *, eps=1e-6, min_rms=0.5, loss_
     V = W_U.shape[0]
     desc = error_signal_desc(T, d, V, _dtype_code(h), eps=eps, min_rms=min_rms,
                              loss_scale=loss_scale, t_chunk=t_chunk, stage_events=stage_events,
-                             algo=algo)
+                             algo=algo, per_chunk_events=per_chunk_events)
     need = error_signal_workspace(desc)
     if workspace is None:
         workspace = _workspace(need, h.device)

@@ -43,7 +43,7 @@ def test_library_exports_every_declared_symbol():
 
 def test_binding_loads_and_reports_version():
     import paper_2608_14563_gb300 as fpo
-    assert fpo.abi_version() == 1
+    assert fpo.abi_version() == 2
     assert fpo.status_string(0) == "FPO_OK"
     assert "TARGET_RANGE" in fpo.status_string(8)
     assert fpo.status_string(12345) == "unknown fpo status"

@@ -53,10 +53,10 @@ def test_gpu_arm_prints_the_contract_line():
     assert d["gpu_launches"] % 3 == 0 and 30 <= d["gpu_launches"] <= 33
     assert e["gpu_launches"] >= d["gpu_launches"]   # plus the input copies
     assert {"sm_mhz", "sm_max_mhz", "reasons"} <= set(d["clocks"])
-    assert d["direct_fixup_rows"] == 0
+    assert d["direct_fixup_rows_last_chunk"] == 0
 
 
 def test_window_stress_goes_through_the_fixup():
     d = run_bench("--window-stress", "--no-e2e", "--no-cpu")
-    assert d["direct_fixup_rows"] > 2048 // 2
+    assert d["direct_fixup_rows_last_chunk"] > 2048 // 2
     assert d["config"]["inputs"].startswith("window stress")
