@@ -522,27 +522,33 @@ def run_fpo(args, wl):
         for e in freed:
             e.record(stream)
 
-        # "sm": the copy of a step's inputs in two halves by bytes, each started at a stage
-        # boundary of the current step so that it runs beside one long GEMM (the logits
-        # pass, then the projection) and not beside the short bandwidth-bound kernels
-        # between them, which the copy's host loads slow down most
-        nbytes = [t.numel() * t.element_size() for t in host]
-        half = 0
-        while half < len(host) and sum(nbytes[:half]) < sum(nbytes) / 2:
-            half += 1
-        sev = [torch.cuda.Event() for _ in range(fpo.STAGE_EVENTS)]
+        # "sm": the copy of a step's inputs in one part per long GEMM phase of the error
+        # signal (each token chunk's logits pass and projection), parts split by bytes,
+        # each started at the stage boundary where its phase begins, so that the copies
+        # run beside long GEMMs and not beside the short bandwidth-bound kernels between
+        # them, which the copy's host loads slow down most
+        sev = [torch.cuda.Event() for _ in range(n_ev)]
         for e in sev:
             e.record(stream)
+        starts = [1 if c == 0 else 5 + 4 * (c - 1) for c in range(n_chunks)]  # logits begin
+        triggers = sorted(starts + [4 + 4 * c for c in range(n_chunks)])        # + projections
+        nbytes = [t.numel() * t.element_size() for t in host]
+        cuts, acc, total = [0], 0, sum(nbytes)
+        for j, nb in enumerate(nbytes):
+            acc += nb
+            if len(cuts) < len(triggers) and acc >= total * len(cuts) / len(triggers):
+                cuts.append(j + 1)
+        cuts.append(len(host))
+        parts = [(a, b) for a, b in zip(cuts[:-1], cuts[1:]) if b > a]
 
         def prefetch(b, after=None):
             copy_stream.wait_event(freed[b])
             with torch.cuda.stream(copy_stream):
                 dst = flat(sets[b])
                 if args.e2e_copy == "sm" and after is not None:
-                    copy_stream.wait_event(after[1])      # the RMSNorm forward is done
-                    fpo.h2d_copy(dst[:half], host[:half], stream=copy_stream)
-                    copy_stream.wait_event(after[4])      # the projection starts
-                    fpo.h2d_copy(dst[half:], host[half:], stream=copy_stream)
+                    for (p0, p1), k in zip(parts, triggers):
+                        copy_stream.wait_event(after[k])  # this part's GEMM phase begins
+                        fpo.h2d_copy(dst[p0:p1], host[p0:p1], stream=copy_stream)
                 elif args.e2e_copy in ("sm", "sm1"):
                     fpo.h2d_copy(dst, host, stream=copy_stream)
                 else:
@@ -553,7 +559,7 @@ def run_fpo(args, wl):
         def e2e_step(i):
             b = i % depth
             stream.wait_event(ready[b])
-            step(sets[b], sev)
+            step(sets[b], sev, per_chunk=True)
             prefetch((i + depth - 1) % depth, sev)  # the inputs of step i + depth - 1
             freed[b].record(stream)
             loss_host.copy_(loss, non_blocking=True)
@@ -579,8 +585,9 @@ def run_fpo(args, wl):
         e2e = {"value": whole_job_tokens_per_s(wl.T, world, e2e_ms), "unit": "tokens/s",
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": 4, "ms_per_step": e2e_ms,
                "gpu_launches": e2e_launches,
-               "copy": {"sm": "fpo_h2d_copy (SM loads of mapped pinned memory): two launches "
-                              "per step, beside the logits pass and the projection",
+               "copy": {"sm": "fpo_h2d_copy (SM loads of mapped pinned memory): one launch per "
+                              "long GEMM phase of the error signal (each token chunk's logits "
+                              "pass and projection), started when the phase begins",
                         "sm1": "fpo_h2d_copy (SM loads of mapped pinned memory): one launch per "
                                "step",
                         "ce": "copy engines: one cudaMemcpyAsync per tensor"}[args.e2e_copy],
