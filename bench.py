@@ -541,15 +541,33 @@ def run_fpo(args, wl):
         cuts.append(len(host))
         parts = [(a, b) for a, b in zip(cuts[:-1], cuts[1:]) if b > a]
 
+        # one step's copy timed alone (the host link's own rate) decides the schedule: the
+        # per-phase parts pay off while the copy fits beside the error signal's GEMM phases
+        # (OLMo shape: e2e - device step 0.59 against 0.87 ms for one launch per step); a
+        # copy longer than those phases spills beside the update either way, and there
+        # one launch per step did better (Falcon shape: 3.7 against 6.4 ms)
+        link_ms = float("inf")
+        for _ in range(2):  # the first pass also maps the host pages
+            t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            t0.record(copy_stream)
+            fpo.h2d_copy(flat(sets[1]), host, stream=copy_stream)
+            t1.record(copy_stream)
+            torch.cuda.synchronize()
+            link_ms = min(link_ms, t0.elapsed_time(t1))
+        gemm_phase_ms = stage_ms["logits_lse_pass"] + stage_ms["projection"]
+        copy_mode = args.e2e_copy
+        if copy_mode == "auto":
+            copy_mode = "sm" if link_ms <= gemm_phase_ms else "sm1"
+
         def prefetch(b, after=None):
             copy_stream.wait_event(freed[b])
             with torch.cuda.stream(copy_stream):
                 dst = flat(sets[b])
-                if args.e2e_copy == "sm" and after is not None:
+                if copy_mode == "sm" and after is not None:
                     for (p0, p1), k in zip(parts, triggers):
                         copy_stream.wait_event(after[k])  # this part's GEMM phase begins
                         fpo.h2d_copy(dst[p0:p1], host[p0:p1], stream=copy_stream)
-                elif args.e2e_copy in ("sm", "sm1"):
+                elif copy_mode in ("sm", "sm1"):
                     fpo.h2d_copy(dst, host, stream=copy_stream)
                 else:
                     for d_t, h_t in zip(dst, host):
@@ -590,7 +608,8 @@ def run_fpo(args, wl):
                               "pass and projection), started when the phase begins",
                         "sm1": "fpo_h2d_copy (SM loads of mapped pinned memory): one launch per "
                                "step",
-                        "ce": "copy engines: one cudaMemcpyAsync per tensor"}[args.e2e_copy],
+                        "ce": "copy engines: one cudaMemcpyAsync per tensor"}[copy_mode],
+               "copy_alone_ms": link_ms, "error_signal_gemm_ms": gemm_phase_ms,
                "pipeline": f"all step inputs H2D from pinned memory each step, {depth} device "
                            "sets: copies run on a copy stream up to "
                            f"{depth - 1} steps ahead of compute; loss D2H"}
@@ -757,10 +776,12 @@ def main():
                     help="device input sets of the end-to-end loop (copies run up to depth-1 steps "
                          "ahead, so a stall of the host link shorter than that many steps is "
                          "absorbed)")
-    ap.add_argument("--e2e-copy", choices=("sm", "sm1", "ce"), default="sm",
+    ap.add_argument("--e2e-copy", choices=("auto", "sm", "sm1", "ce"), default="auto",
                     help="end-to-end input copies: sm = fpo_h2d_copy (SM loads of mapped pinned "
-                         "memory) in two halves beside the two long GEMMs of the error signal, "
-                         "sm1 = one fpo_h2d_copy per step, ce = cudaMemcpyAsync per tensor")
+                         "memory) in one part per long GEMM phase of the error signal, started "
+                         "as the phase begins; sm1 = one fpo_h2d_copy per step; ce = "
+                         "cudaMemcpyAsync per tensor; auto = sm when one step's copy, timed "
+                         "alone, is shorter than those GEMM phases, else sm1")
     ap.add_argument("--band", type=int, default=0,
                     help="GEMM rasterisation band height in tiles (0: library default; tuning)")
     ap.add_argument("--gemm-variant", type=int, choices=(-1, 0, 1, 2, 3), default=-1,
