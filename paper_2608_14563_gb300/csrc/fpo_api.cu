@@ -140,7 +140,7 @@ EsLayout es_layout(const fpo_error_signal_desc* d) {
     L.fix = off;       off = align_up(off + Tcdir * 4);
     L.yfix = off;      off = align_up(off + Tcdir * D * esz);
     L.fix_count = off; off = align_up(off + (direct ? 4 : 0));
-    // the projection's stream-K tail (cut tiles' partial sums), bf16 tensor-core path
+    // the projection's split-K tail (the fp32 partial sums of the last wave's split tiles)
     L.sk = off;        off = align_up(off + (d->dtype == FPO_BF16 ? proj_sk_scratch_bytes() : 0));
     L.total = off;
     return L;

@@ -65,7 +65,7 @@ class Workload:
         return 1.0 / self.T if self.T > 0 else 1.0
 
 
-# The five workloads of the benchmark set (shapes of the surveyed models,
+# The five workloads of the benchmark set (shapes of models the paper trains and probes,
 # packed 2048-token sequences, last 25% of layers as targets).
 WORKLOADS = {
     "tiny": Workload("tiny-f32", T=128, d=64, d_ff=256, V=512, layers=2, dtype="f32",
