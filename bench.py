@@ -212,7 +212,9 @@ def run_reference(args, wl):
     world, rank, _ = dist_setup()
     if rank != 0:
         return
-    n_tok = args.ref_tokens or max(4, min(32, 800 // max(1, args.warmup + args.steps)))
+    # the oracle runs one token per thread at a time, so a sample is a whole number of
+    # tokens per host thread (1 to 4, fewer for longer runs) to keep every core busy
+    n_tok = args.ref_tokens or cores() * max(1, min(4, 40 // max(1, args.warmup + args.steps)))
     steps = []
     for i in range(args.warmup + args.steps):
         r = oracle_sample(wl, n_tok, seed=i)
@@ -798,8 +800,9 @@ def main():
                     help="tokens of the oracle sample behind cpu_baseline (~10 s of CPU work "
                          "at the OLMo shape on 16 cores)")
     ap.add_argument("--ref-tokens", type=int, default=0,
-                    help="tokens of the oracle sample of each --impl reference step (0: 32, "
-                         "fewer when there are many steps, so the run stays within ~1 min)")
+                    help="tokens of the oracle sample of each --impl reference step (0: one to "
+                         "four per host thread, fewer for longer runs, so that every core works "
+                         "and the run stays within a few minutes)")
     ap.add_argument("--no-cpu", action="store_true", help="skip the oracle CPU baseline")
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end run")
     args = ap.parse_args()
