@@ -93,6 +93,10 @@ def test_reference_arm_prints_the_contract_line():
     assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["cores"] >= 1
     assert d["e2e"]["value"] == d["value"] and d["e2e"]["h2d_bytes_per_step"] == 0
     assert d["config"]["workload"] == "tiny-f32"
+    # the oracle runs one token per host thread at a time: the sample keeps every thread
+    # busy (four tokens per thread for a 6-step run, capped at the workload's 128 tokens)
+    n = int(d["cpu_baseline"]["sample"].split(" of ")[0])
+    assert n == min(128, 4 * d["cpu_baseline"]["cores"])
 
 
 def test_bench_rejects_fewer_than_three_warmups():
