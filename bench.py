@@ -181,6 +181,15 @@ def oracle_sample(wl, n_tok, seed=0):
             "n_tok": n_tok, "es_s": t1 - t0, "G_s": t2 - t1, "upd_s": t3 - t2}
 
 
+def copy_schedule(requested, copy_alone_ms, gemm_phase_ms):
+    """The end-to-end input-copy schedule: `requested` unless it is "auto", which takes
+    the per-phase parts ("sm") when one step's copy, timed alone, fits in the error
+    signal's GEMM phases, else one copy launch per step ("sm1")."""
+    if requested != "auto":
+        return requested
+    return "sm" if copy_alone_ms <= gemm_phase_ms else "sm1"
+
+
 def cores():
     try:
         return len(os.sched_getaffinity(0))
@@ -557,9 +566,7 @@ def run_fpo(args, wl):
             torch.cuda.synchronize()
             link_ms = min(link_ms, t0.elapsed_time(t1))
         gemm_phase_ms = stage_ms["logits_lse_pass"] + stage_ms["projection"]
-        copy_mode = args.e2e_copy
-        if copy_mode == "auto":
-            copy_mode = "sm" if link_ms <= gemm_phase_ms else "sm1"
+        copy_mode = copy_schedule(args.e2e_copy, link_ms, gemm_phase_ms)
 
         def prefetch(b, after=None):
             copy_stream.wait_event(freed[b])

@@ -1,4 +1,4 @@
-"""The N>1 replica path of bench.py on CPU: two gloo ranks (127.0.0.1), each with its
+"""bench.py host logic on CPU.  The N>1 replica path: two gloo ranks (127.0.0.1), each with its
 own step time; the reported time is the max over ranks and the throughput counts the
 tokens of every replica.  The reference arm runs on rank 0 only."""
 import importlib.util
@@ -106,3 +106,15 @@ def test_bench_rejects_fewer_than_three_warmups():
                           "--workload", "tiny", "--steps", "1", "--warmup", "2"],
                          capture_output=True, text=True, timeout=120, cwd=ROOT)
     assert out.returncode != 0 and "warmup" in out.stderr
+
+
+def test_end_to_end_copy_schedule():
+    """Per-phase copies while a step's copy fits beside the error signal's GEMMs (the
+    OLMo shape: 14.4 ms of copy, 16.3 ms of GEMMs), else one launch per step (the Falcon
+    shape: 51 ms of copy, 34 ms of GEMMs); an explicit choice is kept."""
+    b = _bench()
+    assert b.copy_schedule("auto", 14.4, 16.3) == "sm"
+    assert b.copy_schedule("auto", 51.1, 33.4) == "sm1"
+    assert b.copy_schedule("auto", 16.3, 16.3) == "sm"
+    for m in ("sm", "sm1", "ce"):
+        assert b.copy_schedule(m, 51.1, 33.4) == m
