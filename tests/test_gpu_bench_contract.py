@@ -60,3 +60,14 @@ def test_window_stress_goes_through_the_fixup():
     d = run_bench("--window-stress", "--no-e2e", "--no-cpu")
     assert d["direct_fixup_rows_last_chunk"] > 2048 // 2
     assert d["config"]["inputs"].startswith("window stress")
+
+
+@pytest.mark.parametrize("mode,parts", [("sm1", 1), ("sm", 2)])
+def test_e2e_copy_schedules_launch_one_copy_per_part(mode, parts):
+    """The end-to-end loop issues, every step, the step's kernels plus one input-copy
+    launch per part: one for `sm1`; for `sm` one per long GEMM phase of the error signal,
+    i.e. the logits pass and the projection of the shape's single token chunk."""
+    d = run_bench("--no-cpu", "--e2e-copy", mode)
+    e = d["e2e"]
+    assert e["gpu_launches"] - d["gpu_launches"] == parts * d["steps"]
+    assert e["h2d_bytes_per_step"] == 2048 * 1024 * 2 + 2048 * 4 + 2 * 2048 * 2816 * 2
