@@ -127,7 +127,8 @@ typedef enum fpo_es_algo {
 
 /* Error-signal problem description (Sec. 3.1 steps 2-4, App. E). */
 typedef struct fpo_error_signal_desc {
-    int64_t T;          /* tokens (B x L flattened), >= 0; T = 0 enqueues nothing */
+    int64_t T;          /* tokens (B x L flattened), >= 0; T = 0 launches no
+                           kernel (the status word and loss_out are zeroed)      */
     int64_t d;          /* model width (RMSNorm size, unembedding input)          */
     int64_t V;          /* vocabulary size                                        */
     int32_t dtype;      /* fpo_dtype of h, norm_w, W_U and g_out                  */
