@@ -29,6 +29,11 @@ if not os.path.exists(LIB_PATH):
     raise ImportError(f"libfpo.so is not built ({LIB_PATH} missing); run "
                       "`python -m paper_2608_14563_gb300.build` first")
 _lib = ctypes.CDLL(LIB_PATH)
+ABI_VERSION = 2  # FPO_ABI_VERSION of include/fpo.h that the structures below mirror
+_lib.fpo_abi_version.restype = ctypes.c_int32
+if _lib.fpo_abi_version() != ABI_VERSION:
+    raise ImportError(f"libfpo.so reports ABI version {_lib.fpo_abi_version()}, this binding "
+                      f"needs {ABI_VERSION}; rebuild it (`python -m paper_2608_14563_gb300.build`)")
 
 _vp, _i64, _i32, _f32, _sz = (ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32, ctypes.c_float,
                               ctypes.c_size_t)
@@ -69,6 +74,8 @@ _lib.fpo_layer_update_grouped_signals.argtypes = [_i32, _i64, _i64, _i64, _i32,
 _lib.fpo_layer_update_grouped_signals.restype = _i32
 _lib.fpo_rmsnorm_vjp.argtypes = [_i64, _i64, _i32, _vp, _vp, _vp, _f32, _f32, _vp, _vp]
 _lib.fpo_rmsnorm_vjp.restype = _i32
+
+
 class OptimizerDesc(ctypes.Structure):
     """Mirror of fpo_optimizer_desc."""
     _fields_ = [("kind", _i32), ("clip", _i32), ("lr", _f32), ("momentum", _f32),

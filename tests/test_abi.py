@@ -49,6 +49,29 @@ def test_binding_loads_and_reports_version():
     assert fpo.status_string(12345) == "unknown fpo status"
 
 
+def test_binding_constants_match_the_header():
+    """The binding's copies of the header's constants and enums equal the header's."""
+    import paper_2608_14563_gb300 as fpo
+    with open(os.path.join(ROOT, "include", "fpo.h")) as f:
+        hdr = f.read()
+    defines = dict(re.findall(r"#define (FPO_\w+) (\d+)", hdr))
+    assert int(defines["FPO_ABI_VERSION"]) == fpo.ABI_VERSION == fpo.abi_version()
+    assert int(defines["FPO_MAX_GROUPED_LAYERS"]) == fpo.MAX_GROUPED_LAYERS
+    assert int(defines["FPO_MAX_COPY_BUFFERS"]) == fpo.MAX_COPY_BUFFERS
+    assert int(defines["FPO_STAGE_EVENTS"]) == fpo.STAGE_EVENTS
+    assert int(defines["FPO_AUTO_T_CHUNK"]) == fpo.AUTO_T_CHUNK
+    enums = dict((k, int(v)) for k, v in re.findall(r"(FPO_\w+) = (\d+)", hdr))
+    for name, value in [("FPO_F32", fpo.F32), ("FPO_BF16", fpo.BF16), ("FPO_OK", fpo.OK),
+                        ("FPO_ES_AUTO", fpo.ES_AUTO), ("FPO_ES_RECOMPUTE", fpo.ES_RECOMPUTE),
+                        ("FPO_ES_STORED_LOGITS", fpo.ES_STORED_LOGITS),
+                        ("FPO_ES_DIRECT", fpo.ES_DIRECT), ("FPO_OPT_SGD", fpo.OPT_SGD),
+                        ("FPO_OPT_SGD_MOMENTUM", fpo.OPT_SGD_MOMENTUM),
+                        ("FPO_OPT_ADAMW", fpo.OPT_ADAMW), ("FPO_CLIP_NONE", fpo.CLIP_NONE),
+                        ("FPO_CLIP_STEP", fpo.CLIP_STEP),
+                        ("FPO_CLIP_GRADIENT", fpo.CLIP_GRADIENT)]:
+        assert enums[name] == value, name
+
+
 class _Lib:
     def __init__(self):
         import paper_2608_14563_gb300 as fpo
