@@ -185,6 +185,10 @@ def _stream(stream):
     return ctypes.c_void_p(s.cuda_stream)
 
 
+def _nbytes(t: torch.Tensor) -> int:
+    return t.numel() * t.element_size()
+
+
 def _workspace(nbytes: int, device) -> torch.Tensor:
     return torch.empty(max(int(nbytes), 256), dtype=torch.uint8, device=device)
 
@@ -234,7 +238,7 @@ def error_signal(h, norm_w, W_U, targets, g_out, *, eps=1e-6, min_rms=0.5, loss_
         workspace = _workspace(need, h.device)
     rc = _lib.fpo_error_signal(ctypes.byref(desc), _ptr(h), _ptr(norm_w), _ptr(W_U), _ptr(targets),
                                _ptr(g_out), _ptr(lse_out), _ptr(loss_out), _ptr(workspace),
-                               workspace.numel() * workspace.element_size(), _stream(stream))
+                               _nbytes(workspace), _stream(stream))
     _check(rc, "fpo_error_signal")
     return workspace
 
@@ -261,7 +265,7 @@ def layer_update(g, A, lr, *, W_master=None, W_out=None, G_out=None, workspace=N
         workspace = _workspace(layer_update_workspace(), g.device)
     rc = _lib.fpo_layer_update(T, d, d_ff, _dtype_code(g), _ptr(g), _ptr(A), float(lr),
                                _ptr(W_master), _ptr(W_out), _ptr(G_out), _ptr(workspace),
-                               workspace.numel(), _stream(stream))
+                               _nbytes(workspace), _stream(stream))
     _check(rc, "fpo_layer_update")
     return workspace
 
@@ -285,7 +289,7 @@ def layer_update_grouped(g, As, lr, *, W_masters=None, W_outs=None, G_outs=None,
         workspace = _workspace(layer_update_workspace(), g.device)
     rc = _lib.fpo_layer_update_grouped(n, T, d, d_ff, _dtype_code(g), _ptr(g), _ptr_array(As, n),
                                        float(lr), _ptr_array(W_masters, n), _ptr_array(W_outs, n),
-                                       _ptr_array(G_outs, n), _ptr(workspace), workspace.numel(),
+                                       _ptr_array(G_outs, n), _ptr(workspace), _nbytes(workspace),
                                        _stream(stream))
     _check(rc, "fpo_layer_update_grouped")
     return workspace
@@ -302,7 +306,7 @@ def layer_update_grouped_signals(gs, As, lr, *, W_masters=None, W_outs=None, G_o
     rc = _lib.fpo_layer_update_grouped_signals(
         n, T, d, d_ff, _dtype_code(gs[0]), _ptr_array(gs, n), _ptr_array(As, n), float(lr),
         _ptr_array(W_masters, n), _ptr_array(W_outs, n), _ptr_array(G_outs, n), _ptr(workspace),
-        workspace.numel(), _stream(stream))
+        _nbytes(workspace), _stream(stream))
     _check(rc, "fpo_layer_update_grouped_signals")
     return workspace
 
@@ -328,7 +332,7 @@ def layer_optimize_grouped(gs, As, opt, W_masters, *, W_outs=None, states1=None,
     rc = _lib.fpo_layer_optimize_grouped(
         n, T, d, d_ff, _dtype_code(gs[0]), _ptr_array(gs, n), _ptr_array(As, n), ctypes.byref(opt),
         _ptr_array(W_masters, n), _ptr_array(W_outs, n), _ptr_array(states1, n),
-        _ptr_array(states2, n), _ptr(workspace), workspace.numel(), _stream(stream))
+        _ptr_array(states2, n), _ptr(workspace), _nbytes(workspace), _stream(stream))
     _check(rc, "fpo_layer_optimize_grouped")
     return workspace
 
@@ -340,7 +344,7 @@ def gate_up_signals(g, W3_init, a, b, dA, dB, *, workspace=None, stream=None):
     if workspace is None:
         workspace = _workspace(layer_update_workspace(), g.device)
     rc = _lib.fpo_gate_up_signals(T, d, d_ff, _dtype_code(g), _ptr(g), _ptr(W3_init), _ptr(a),
-                                  _ptr(b), _ptr(dA), _ptr(dB), _ptr(workspace), workspace.numel(),
+                                  _ptr(b), _ptr(dA), _ptr(dB), _ptr(workspace), _nbytes(workspace),
                                   _stream(stream))
     _check(rc, "fpo_gate_up_signals")
     return workspace
@@ -368,7 +372,7 @@ def cosine(X, Y, out=None, *, workspace=None, stream=None):
     if workspace is None:
         workspace = _workspace(cosine_workspace(n), X.device)
     rc = _lib.fpo_cosine(n, _dtype_code(X), _ptr(X), _ptr(Y), _ptr(out), _ptr(workspace),
-                         workspace.numel(), _stream(stream))
+                         _nbytes(workspace), _stream(stream))
     _check(rc, "fpo_cosine")
     return out
 
@@ -395,7 +399,7 @@ def cosine_grouped(X, Y, out=None, *, workspace=None, stream=None):
     xarr = (_vp * n_layers)(*[_ptr(t) for t in X])
     yarr = (_vp * n_layers)(*[_ptr(t) for t in Y])
     rc = _lib.fpo_cosine_grouped(n_layers, n, _dtype_code(X[0]), xarr, yarr, _ptr(out),
-                                 _ptr(workspace), workspace.numel(), _stream(stream))
+                                 _ptr(workspace), _nbytes(workspace), _stream(stream))
     _check(rc, "fpo_cosine_grouped")
     return out
 
@@ -422,7 +426,7 @@ def norm_ratio(G, W, rel_step=0.01, out=None, *, workspace=None, stream=None):
     garr = (_vp * n_layers)(*[_ptr(t) for t in G])
     warr = (_vp * n_layers)(*[_ptr(t) for t in W])
     rc = _lib.fpo_norm_ratio(n_layers, n, _dtype_code(G[0]), garr, _dtype_code(W[0]), warr,
-                             float(rel_step), _ptr(out), _ptr(workspace), workspace.numel(),
+                             float(rel_step), _ptr(out), _ptr(workspace), _nbytes(workspace),
                              _stream(stream))
     _check(rc, "fpo_norm_ratio")
     return out
