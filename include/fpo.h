@@ -372,7 +372,8 @@ int32_t fpo_cosine(int64_t n, int32_t dtype, const void* X, const void* Y, doubl
  *
  * - The first call on each device looks up the array's device address
  *   (cudaGetSymbolAddress) with that device current; make that first call
- *   before any stream capture.
+ *   before any stream capture.  A lookup that fails returns FPO_ERR_CUDA and is
+ *   retried by the next call; only a successful one is kept.
  * - All calls on a device share the one array, which keeps the last call's
  *   partials.  Every slot a call reads is written by the same call first, so
  *   nothing needs clearing, but two calls that overlap on the GPU (different

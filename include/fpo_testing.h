@@ -33,10 +33,8 @@ int32_t fpo_testing_gemm_bf16(int64_t M, int64_t N, int64_t K, int32_t a_mn, int
  * Select the tensor-core GEMM kernel every later call uses (process-wide):
  * 0 = one CTA per 128 x 256 output tile, 1 = a CTA pair (tcgen05 cta_group::2)
  * per 256 x 256 tile, 2 = as 1 but 256 x 512 pair tiles for the projection
- * g = E W_U (one accumulator, a quarter less operand traffic; the default),
- * 3 = as 2, and the logits pass and the update on clusters of two CTA pairs that
- * share each B tile by TMA multicast (512 x 256 tiles per cluster).
- * Returns the previous setting.  All compute the same sums in the same order per
+ * g = E W_U (one accumulator, a quarter less operand traffic; the default).
+ * Any other value selects 0.  Returns the previous setting.  All compute the same sums in the same order per
  * output element.
  */
 int32_t fpo_testing_set_gemm_variant(int32_t variant);

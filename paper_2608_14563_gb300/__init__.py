@@ -147,8 +147,7 @@ def kernel_launches() -> int:
 
 def set_gemm_variant(variant: int) -> int:
     """fpo_testing_set_gemm_variant: 0 single-CTA, 1 CTA-pair tiles, 2 CTA-pair tiles with a
-    256 x 512 projection, 3 as 2 with two CTA pairs sharing each B tile in the logits pass
-    and the update; a negative value only reads the current setting.  Returns the setting in
+    256 x 512 projection (the default); a negative value only reads the current setting.  Returns the setting in
     force before the call."""
     if variant < 0:
         cur = _lib.fpo_testing_set_gemm_variant(0)

@@ -199,29 +199,30 @@ constexpr int kNoAllocSlots = 1024;
 // 24 KiB of device memory, held by every GPU that loads the library until exit.
 static __device__ __align__(256) double g_cosine_noalloc_scratch[3 * kNoAllocSlots];
 
-struct NoAllocScratch {
-    std::once_flag once;
-    double* ptr = nullptr;
-    cudaError_t err = cudaSuccess;
-};
-NoAllocScratch g_noalloc_scratch[64];
+// Device address of the static scratch per device, once looked up successfully.
+std::mutex g_noalloc_mu;
+double* g_noalloc_scratch[64] = {};
 
 // Device address of the static scratch on the current device.  In host code the
-// array's name is only a host-side stand-in, so the address is looked up once per
-// device, with that device current.
+// array's name is only a host-side stand-in, so the address is looked up with that
+// device current.  Only a successful lookup is kept: a failed one (e.g. a first call
+// made during a stream capture) is retried on the next call.
 cudaError_t noalloc_scratch(double** out) {
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-    NoAllocScratch& s = g_noalloc_scratch[dev];
-    std::call_once(s.once, [&s] {
+    std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    if (!g_noalloc_scratch[dev]) {
         void* p = nullptr;
-        s.err = cudaGetSymbolAddress(&p, g_cosine_noalloc_scratch);
-        s.ptr = static_cast<double*>(p);
-    });
-    if (s.err != cudaSuccess) return s.err;
-    *out = s.ptr;
+        e = cudaGetSymbolAddress(&p, g_cosine_noalloc_scratch);
+        if (e != cudaSuccess) {
+            cudaGetLastError();  // leave no sticky-free error behind for the caller
+            return e;
+        }
+        g_noalloc_scratch[dev] = static_cast<double*>(p);
+    }
+    *out = g_noalloc_scratch[dev];
     return cudaSuccess;
 }
 

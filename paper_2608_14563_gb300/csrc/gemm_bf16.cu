@@ -168,24 +168,20 @@ SkPlan tail_plan(long long tiles, long long clusters, int k_blocks) {
 // With sk_scratch non-null, the tiles of the last partial wave are split by tail_plan
 // (SegCursor); the caller then runs sk_fixup over them (plan->tail_tiles > 0).
 // sk_scratch holds kTailWaves x clusters x 256 x BN fp32.
-// kPairs = 2: clusters of two CTA pairs sharing each B tile (tiles of 512 output rows;
-// the shape is built with that row-tile height; no split tail).
-template <int BN, bool A_MN, bool B_MN, int STAGES, int MAXG, class Epi, int kPairs = 1>
+template <int BN, bool A_MN, bool B_MN, int STAGES, int MAXG, class Epi>
 cudaError_t run_gemm_pair(const GemmMaps<MAXG>& maps, const typename Epi::Params& ep,
                           const GemmShape& sh_in, unsigned* status, cudaStream_t st,
                           float* sk_scratch = nullptr, SkPlan* plan = nullptr) {
     if (plan) *plan = SkPlan{};
     if (sh_in.tiles <= 0 || sh_in.k_blocks <= 0) return cudaSuccess;
-    static_assert(kPairs == 1 || kPairs == 2, "one or two CTA pairs per cluster");
-    if (kPairs == 2 && sk_scratch) return cudaErrorInvalidValue;
     using L = GemmPairSmem<BN, STAGES>;
-    auto kern = tc_gemm_pair_kernel<BN, A_MN, B_MN, STAGES, MAXG, Epi, kPairs>;
+    auto kern = tc_gemm_pair_kernel<BN, A_MN, B_MN, STAGES, MAXG, Epi>;
     static cudaError_t attr_err =
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::kBytes);
     if (attr_err != cudaSuccess) return attr_err;
     DevInfo di;
     if (!current_device_info(&di)) return cudaErrorUnknown;
-    static int max_clusters = pair_clusters(kern, L::kBytes, di.sm_count, 2 * kPairs);
+    static int max_clusters = pair_clusters(kern, L::kBytes, di.sm_count, 2);
     const long long clusters = sh_in.tiles < max_clusters ? sh_in.tiles : max_clusters;
     GemmShape sh = sh_in;
     if (sk_scratch) {
@@ -197,7 +193,7 @@ cudaError_t run_gemm_pair(const GemmMaps<MAXG>& maps, const typename Epi::Params
             if (plan) *plan = p;
         }
     }
-    kern<<<static_cast<unsigned>(2 * kPairs * clusters), kGemmThreads, L::kBytes, st>>>(maps, ep, sh, status,
+    kern<<<static_cast<unsigned>(2 * clusters), kGemmThreads, L::kBytes, st>>>(maps, ep, sh, status,
                                                                               wait_limit_ns()),
         ::fpo::note_launch();
     return cudaGetLastError();
@@ -282,9 +278,6 @@ std::atomic<int> g_band_override{0};  // > 0: rasterisation band height (tests /
 
 bool use_pair() { return g_gemm_variant.load(std::memory_order_relaxed) >= 1; }
 bool wide_proj() { return g_gemm_variant.load(std::memory_order_relaxed) >= 2; }
-// 3: as 2, and the logits pass and the update on clusters of two CTA pairs that share
-// each B tile by TMA multicast (a quarter less operand traffic from L2 per FLOP)
-bool shared_b() { return g_gemm_variant.load(std::memory_order_relaxed) == 3; }
 
 // Rasterisation band in tile rows, unless overridden: 16 tile rows, i.e. 2048
 // output rows of single-CTA tiles and 4096 of pair tiles.  With pair tiles the
@@ -295,15 +288,13 @@ int band_for(bool) {
     const int o = g_band_override.load(std::memory_order_relaxed);
     return o > 0 ? o : kBandTiles;
 }
-// The same rows per band for tiles of two pairs (512 rows): half as many tile rows.
-int quad_band() { return band_for(true) > 1 ? band_for(true) / 2 : 1; }
 
 }  // namespace
 
 void set_band_override(int b) { g_band_override.store(b > 0 ? b : 0, std::memory_order_relaxed); }
 
 void set_gemm_variant(int v) {
-    g_gemm_variant.store(v >= 0 && v <= 3 ? v : 0, std::memory_order_relaxed);
+    g_gemm_variant.store(v >= 0 && v <= 2 ? v : 0, std::memory_order_relaxed);
 }
 int gemm_variant() { return g_gemm_variant.load(std::memory_order_relaxed); }
 
@@ -392,10 +383,10 @@ cudaError_t launch_lse_prob_bf16(const void* yhat, const void* W_U, const int32_
                                  const float* anchor, int T, int d, int V, float2* part, float* sx,
                                  int part_ld, float* zy, void* P, unsigned* status,
                                  cudaStream_t st) {
-    const bool pair = use_pair(), quad = shared_b();
+    const bool pair = use_pair();
     GemmMaps<1> maps;
     if (!map_kmajor(&maps.a[0], yhat, T, d, kBM) ||
-        !map_kmajor(&maps.b[0], W_U, V, d, quad ? kLseBN / 4 : pair ? kLseBN / 2 : kLseBN))
+        !map_kmajor(&maps.b[0], W_U, V, d, pair ? kLseBN / 2 : kLseBN))
         return cudaErrorInvalidValue;
     EpiLseProb::Params ep;
     if (!map_out_bf16(&ep.pmap, P, T, V)) return cudaErrorInvalidValue;
@@ -407,9 +398,6 @@ cudaError_t launch_lse_prob_bf16(const void* yhat, const void* W_U, const int32_
     ep.anchor = anchor;
     ep.M = T;
     ep.N = V;
-    if (quad)
-        return run_gemm_pair<kLseBN, false, false, kPairStages, 1, EpiLseProb, 2>(
-            maps, ep, make_shape(T, V, d, kLseBN, 1, quad_band(), 2 * kPairBM), status, st);
     const GemmShape sh = make_shape(T, V, d, kLseBN, 1, band_for(pair), pair ? kPairBM : kBM);
     if (pair)
         return run_gemm_pair<kLseBN, false, false, kPairStages, 1, EpiLseProb>(maps, ep, sh, status,
@@ -532,9 +520,6 @@ cudaError_t launch_update_bf16(int n, int T, int d, int d_ff, const void* const*
     ep.M = d;
     ep.N = d_ff;
     ep.neg_lr = -lr;
-    if (shared_b())
-        return run_gemm_pair<kUpdBN, true, true, kPairStages, kMaxGroups, EpiUpdate, 2>(
-            maps, ep, make_shape(d, d_ff, T, kUpdBN, n, quad_band(), 2 * kPairBM), status, st);
     if (use_pair())
         return run_gemm_pair<kUpdBN, true, true, kPairStages, kMaxGroups, EpiUpdate>(
             maps, ep, make_shape(d, d_ff, T, kUpdBN, n, band_for(true), kPairBM), status, st);

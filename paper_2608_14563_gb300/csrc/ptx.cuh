@@ -179,19 +179,18 @@ __device__ __forceinline__ void tma_load_2d_pair(const CUtensorMap* map, uint32_
         : "memory");
 }
 
-// TMA load multicast to the CTAs of `cta_mask` (same shared-memory offset in each),
-// for a pair-MMA cluster: each destination CTA's bytes are counted on the mbarrier at
-// the offset of `bar_cluster_addr` in the leader of that CTA's pair (the address given
-// is this CTA's pair leader's).
-__device__ __forceinline__ void tma_load_2d_pair_mc(const CUtensorMap* map, uint32_t smem_dst,
-                                                    uint32_t bar_cluster_addr, int x, int y,
-                                                    uint16_t cta_mask) {
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
-        ".multicast::cluster.cta_group::2 [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(smem_dst),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(bar_cluster_addr), "r"(x), "r"(y),
-        "h"(cta_mask)
-        : "memory");
+// Complete `bytes` of the current phase's expected transaction count of an mbarrier
+// of this CTA without a copy (the accounting of a copy that will never be issued).
+__device__ __forceinline__ void mbar_complete_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.complete_tx.relaxed.cta.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(bytes)
+                 : "memory");
+}
+
+// 32-bit load from the shared memory of another CTA of the cluster (shared::cluster address).
+__device__ __forceinline__ uint32_t ld_shared_cluster_u32(uint32_t cluster_addr) {
+    uint32_t v;
+    asm volatile("ld.shared::cluster.u32 %0, [%1];" : "=r"(v) : "r"(cluster_addr) : "memory");
+    return v;
 }
 
 // ----------------------------------------------------------------- tcgen05

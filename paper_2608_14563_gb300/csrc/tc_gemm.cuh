@@ -16,8 +16,8 @@
 // are loaded by the TMA engine with the 128-byte swizzle and described to the
 // tensor core by the matching shared-memory descriptor.  Every wait is bounded
 // (WaitGuard); on a timeout all roles stop issuing, in-flight copies and MMAs
-// are drained with a second bounded wait, TMEM is freed and the kernel returns
-// with the timeout bit set in the status word.
+// are drained with a second wait of a fixed, generous limit (kDrainLimitNs), TMEM
+// is freed and the kernel returns with the timeout bit set in the status word.
 #pragma once
 
 #include "ptx.cuh"
@@ -29,6 +29,9 @@ constexpr int kBK = 64;        // k-block: 64 bf16 = one 128-byte swizzle row
 constexpr int kUmmaK = 16;     // K of one tcgen05.mma.kind::f16
 constexpr int kGemmThreads = 192;
 constexpr int kMaxGroups = 64;
+// Limit of the teardown waits for copies and MMAs already issued (they complete in
+// microseconds); fixed, so that a short wait limit cannot cut them off.
+constexpr uint64_t kDrainLimitNs = 1000000000ull;
 
 struct GemmShape {
     int M, N, K;
@@ -241,12 +244,12 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                     if (++stage == STAGES) { stage = 0; phase ^= 1u; }
                 }
             }
-            if (!ok) {
-                // Do not leave copies landing in shared memory after exit.
-                for (int s = 0; s < STAGES; ++s)
-                    if (issued_mask & (1u << s))
-                        mbar_wait_drain(full_bar(s), (issued_parity >> s) & 1u, wait_limit_ns);
-            }
+            // Do not leave copies landing in shared memory after exit: the last copy of
+            // every stage is awaited (at once when it was consumed), also when another
+            // role gave up first.
+            for (int s = 0; s < STAGES; ++s)
+                if (issued_mask & (1u << s))
+                    mbar_wait_drain(full_bar(s), (issued_parity >> s) & 1u, kDrainLimitNs);
         }
         __syncwarp();
     } else if (warp == 1) {
@@ -279,10 +282,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 tc_commit(tfull_bar(acc));
                 if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
             }
-            if (!ok && issued_any) {
-                // Wait for the MMAs already issued before TMEM and smem go away.
+            if (issued_any) {
+                // Wait for the MMAs already issued before TMEM and smem go away (also
+                // when only the epilogue gave up).
                 tc_commit(drain_bar);
-                mbar_wait_drain(drain_bar, 0, wait_limit_ns);
+                mbar_wait_drain(drain_bar, 0, kDrainLimitNs);
             }
         }
         __syncwarp();

@@ -19,8 +19,11 @@
 // overlaps the mainloop of the next) or 512 (two N=256 MMAs per K slice into
 // one 512-column accumulator: a quarter less operand traffic per FLOP, but the
 // next tile waits for the epilogue; for GEMMs with a long K loop).
-// All waits are bounded as in the single-CTA kernel; the pair meets at a
-// cluster barrier before TMEM is freed and before either CTA exits.
+// All waits are bounded as in the single-CTA kernel.  Teardown: the pair meets at
+// a cluster barrier, the leader waits (with a separate, fixed limit) for every
+// operand copy either CTA issued into the last ring positions, which its full
+// barriers count, and the pair meets again before TMEM is freed and before either
+// CTA exits (pair_drain_copies below).
 #pragma once
 
 #include "tc_gemm.cuh"
@@ -40,6 +43,10 @@ struct GemmPairSmem {
     static constexpr int kMiscOffset = kBarOffset + kNumBars * 8;
     static constexpr int kBytes = kMiscOffset + 16 + 1024;
 };
+
+// Misc words of the pair kernel's shared memory: TMEM base address, abort flag,
+// and the number of k-blocks this CTA's producer issued.
+constexpr int kMiscTmem = 0, kMiscAbort = 4, kMiscIssued = 8;
 
 __device__ __forceinline__ bool mbar_try_wait_cluster(uint32_t bar, uint32_t parity) {
     uint32_t ok;
@@ -130,25 +137,36 @@ __device__ __forceinline__ void load_operand_pair(const CUtensorMap* map, uint32
     }
 }
 
-// 64 rows (M or N) x one k-block of an operand, multicast to the CTAs of cta_mask:
-// K-major one box {64 (K), 64 rows}, MN-major one box {64 (M or N), 64 (K)}.
-template <bool MN>
-__device__ __forceinline__ void load_operand_pair_mc(const CUtensorMap* map, uint32_t dst,
-                                                     uint32_t bar_leader, int row0, int k0,
-                                                     uint16_t cta_mask) {
-    if constexpr (!MN)
-        tma_load_2d_pair_mc(map, dst, bar_leader, k0, row0, cta_mask);
-    else
-        tma_load_2d_pair_mc(map, dst, bar_leader, row0, k0, cta_mask);
+// Teardown of the pair (leader's producer thread, after both producers have stopped
+// and published their issued k-block counts n_self and n_peer): every copy either CTA
+// issued must have landed before the CTAs exit.  The k-block with index i sits in
+// stage i % STAGES, phase parity (i / STAGES) & 1, and its leader full barrier counts
+// both halves (2 x half_bytes, armed by the leader's expect_tx).  Every k-block below
+// max(n_self, n_peer) - STAGES was consumed by an MMA, so both halves landed; for the
+// last STAGES indices the barrier is still in that k-block's phase, and the side that
+// did not issue it is accounted for here: a missing peer half by completing its
+// bytes, a missing leader expect_tx by arming the barrier for the peer's half only.
+// Each such phase is then awaited with the fixed drain limit.
+template <int STAGES>
+__device__ __forceinline__ void pair_drain_copies(uint32_t bar0, long long n_self, long long n_peer,
+                                                  uint32_t half_bytes) {
+    const long long hi = n_self > n_peer ? n_self : n_peer;
+    for (long long i = hi - STAGES > 0 ? hi - STAGES : 0; i < hi; ++i) {
+        const uint32_t bar = bar0 + 8u * static_cast<uint32_t>(i % STAGES);
+        const uint32_t parity = static_cast<uint32_t>((i / STAGES) & 1);
+        const bool mine = i < n_self, peer = i < n_peer;
+        if (mine && !peer) mbar_complete_tx(bar, half_bytes);
+        if (!mine && peer) mbar_arrive_expect_tx(bar, half_bytes);
+        mbar_wait_cl_drain(bar, parity, kDrainLimitNs);
+    }
 }
 
-template <int BN, bool A_MN, bool B_MN, int STAGES, int MAXG, class Epi, int kPairs = 1>
-__global__ void __cluster_dims__(2 * kPairs, 1, 1) __launch_bounds__(kGemmThreads, 1)
+template <int BN, bool A_MN, bool B_MN, int STAGES, int MAXG, class Epi>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     tc_gemm_pair_kernel(const __grid_constant__ GemmMaps<MAXG> maps,
                         const __grid_constant__ typename Epi::Params ep, const GemmShape sh_in,
                         unsigned int* status, unsigned long long wait_limit_ns) {
     static_assert(BN == 256 || BN == 512, "pair tiles are 256 or 512 columns wide");
-    static_assert(kPairs == 1 || (kPairs == 2 && BN == 256), "two pairs share 256-wide B tiles");
     using L = GemmPairSmem<BN, STAGES>;
     constexpr int kNSub = BN / 256;                // N = 256 MMAs per K slice
     constexpr int kAccBufs = kNSub == 1 ? 2 : 1;   // accumulator buffers in TMEM
@@ -156,16 +174,14 @@ __global__ void __cluster_dims__(2 * kPairs, 1, 1) __launch_bounds__(kGemmThread
     constexpr uint32_t kBSubBytes = kBSub * kBK * 2;
     constexpr uint32_t kIdesc = idesc_bf16_f32(kPairBM, 256, A_MN, B_MN);
     constexpr int kTmemCols = kAccBufs * BN;       // 512 either way
-    constexpr int kCta = 2 * kPairs;                  // CTAs of the cluster
-    constexpr uint16_t kAll = (1u << kCta) - 1u;      // every CTA of the cluster
-    constexpr int kClusterBM = kPairBM * kPairs;      // output rows of one cluster tile
+    constexpr uint16_t kBoth = 0x3;                // both CTAs of the pair
 
     GemmShape sh = sh_in;
     if (sh.m_dev) {  // rows counted on the device (every thread reads the same value)
         const int m = min(*sh.m_dev, sh.M);
         if (m <= 0) return;
         sh.M = m;
-        sh.m_blocks = (m + kClusterBM - 1) / kClusterBM;
+        sh.m_blocks = (m + kPairBM - 1) / kPairBM;
         sh.tiles = static_cast<long long>(sh.groups) * sh.m_blocks * sh.n_blocks;
         sh.tail_tiles = 0;
     }
@@ -176,14 +192,10 @@ __global__ void __cluster_dims__(2 * kPairs, 1, 1) __launch_bounds__(kGemmThread
     uint8_t* smem = smem_raw + pad;
     const uint32_t sbase = raw + pad;
 
-    const uint32_t rank = cluster_ctarank();
-    const uint32_t prank = rank & 1u;        // position in the CTA pair
-    const uint32_t pair = rank >> 1;         // which pair of the cluster
-    const uint32_t lrank = rank & ~1u;       // the pair's leader (issues its MMAs)
-    const bool leader = prank == 0;
-    const uint16_t pair_mask = static_cast<uint16_t>(0x3u << lrank);
-    const long long cluster = blockIdx.x / kCta;
-    const long long n_clusters = gridDim.x / kCta;
+    const uint32_t rank = cluster_ctarank();  // position in the CTA pair
+    const bool leader = rank == 0;            // the leader issues the pair's MMAs
+    const long long cluster = blockIdx.x / 2;
+    const long long n_clusters = gridDim.x / 2;
 
     const uint32_t bar0 = sbase + L::kBarOffset;
     auto full_bar = [&](int s) { return bar0 + 8u * s; };
@@ -191,8 +203,9 @@ __global__ void __cluster_dims__(2 * kPairs, 1, 1) __launch_bounds__(kGemmThread
     auto tfull_bar = [&](int a) { return bar0 + 8u * (2 * STAGES + a); };
     auto tempty_bar = [&](int a) { return bar0 + 8u * (2 * STAGES + 2 + a); };
     const uint32_t drain_bar = bar0 + 8u * (2 * STAGES + 4);
-    uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(smem + L::kMiscOffset);
-    volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::kMiscOffset + 4);
+    uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(smem + L::kMiscOffset + kMiscTmem);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::kMiscOffset + kMiscAbort);
+    uint32_t* issued_word = reinterpret_cast<uint32_t*>(smem + L::kMiscOffset + kMiscIssued);
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -200,7 +213,7 @@ __global__ void __cluster_dims__(2 * kPairs, 1, 1) __launch_bounds__(kGemmThread
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(full_bar(s), 1);   // leader's: one expect_tx arrival, both CTAs' bytes
-            mbar_init(empty_bar(s), kPairs);  // one multicast commit from each pair leader
+            mbar_init(empty_bar(s), 1);  // one multicast commit from the leader
         }
         for (int a = 0; a < 2; ++a) {
             mbar_init(tfull_bar(a), 1);
@@ -208,6 +221,7 @@ __global__ void __cluster_dims__(2 * kPairs, 1, 1) __launch_bounds__(kGemmThread
         }
         mbar_init(drain_bar, 1);
         *abort_flag = 0;
+        *issued_word = 0;
         fence_mbar_init();
         tma_prefetch_desc(&maps.a[0]);
     }
@@ -228,7 +242,7 @@ __global__ void __cluster_dims__(2 * kPairs, 1, 1) __launch_bounds__(kGemmThread
         if (lane == 0) {
             int stage = 0;
             uint32_t phase = 0;
-            uint32_t issued_mask = 0, issued_parity = 0;
+            uint32_t issued = 0;  // k-blocks issued: k-block i used stage i % STAGES
             bool ok = true;
             SegCursor seg(sh, cluster, n_clusters);
             long long t;
@@ -238,42 +252,24 @@ __global__ void __cluster_dims__(2 * kPairs, 1, 1) __launch_bounds__(kGemmThread
                 tile_coords(t, sh, g, mp, nb);
                 const CUtensorMap* amap = &maps.a[MAXG == 1 ? 0 : g];
                 const CUtensorMap* bmap = &maps.b[MAXG == 1 ? 0 : g];
-                const int a_row = (mp * kPairs + static_cast<int>(pair)) * kPairBM +
-                                  128 * static_cast<int>(prank);
-                const int b_row = nb * BN + kBSub * static_cast<int>(prank);
+                const int a_row = mp * kPairBM + 128 * static_cast<int>(rank);
+                const int b_row = nb * BN + kBSub * static_cast<int>(rank);
                 for (int kb = kb0; kb < kb1; ++kb) {
                     if (!mbar_wait_cl(empty_bar(stage), phase ^ 1u, guard)) { ok = false; break; }
                     const uint32_t sa = sbase + stage * L::kStageBytes;
                     const uint32_t sb = sa + L::kABytes;
-                    const uint32_t fb = mapa_shared(full_bar(stage), lrank);
+                    const uint32_t fb = mapa_shared(full_bar(stage), 0);
                     if (leader) mbar_arrive_expect_tx(full_bar(stage), 2 * L::kStageBytes);
                     load_operand_pair<A_MN, 128>(amap, sa, fb, a_row, kb * kBK);
-                    if constexpr (kPairs == 1) {
 #pragma unroll
-                        for (int h = 0; h < kNSub; ++h)
-                            load_operand_pair<B_MN, kBSub>(bmap, sb + h * kBSubBytes, fb,
-                                                           b_row + 256 * h, kb * kBK);
-                    } else {
-                        // the pairs share the B tile: this CTA loads the 64 rows of its
-                        // half of B at position `pair` and multicasts them to the CTA
-                        // holding the same half in the other pair; each destination
-                        // pair's leader counts the bytes
-                        load_operand_pair_mc<B_MN>(
-                            bmap, sb + pair * (64u * kBK * 2u), fb, b_row + 64 * static_cast<int>(pair),
-                            kb * kBK, static_cast<uint16_t>((1u << prank) | (1u << (prank + 2))));
-                    }
-                    issued_mask |= 1u << stage;
-                    issued_parity = (issued_parity & ~(1u << stage)) | (phase << stage);
+                    for (int h = 0; h < kNSub; ++h)
+                        load_operand_pair<B_MN, kBSub>(bmap, sb + h * kBSubBytes, fb,
+                                                       b_row + 256 * h, kb * kBK);
+                    ++issued;
                     if (++stage == STAGES) { stage = 0; phase ^= 1u; }
                 }
             }
-            if (!ok && leader) {
-                // The leader's full barriers count both CTAs' bytes: wait for the
-                // copies in flight before the pair meets at the final barrier.
-                for (int s = 0; s < STAGES; ++s)
-                    if (issued_mask & (1u << s))
-                        mbar_wait_cl_drain(full_bar(s), (issued_parity >> s) & 1u, wait_limit_ns);
-            }
+            *issued_word = issued;  // read by the leader at teardown
         }
         __syncwarp();
     } else if (warp == 1) {
@@ -304,25 +300,26 @@ __global__ void __cluster_dims__(2 * kPairs, 1, 1) __launch_bounds__(kGemmThread
                                              operand_desc<B_MN>(sb + h * kBSubBytes, kk), kIdesc,
                                              (kb != kb0 || kk != 0) ? 1u : 0u);
                     issued_any = true;
-                    // the stage is free in every CTA once every pair has consumed it (the
-                    // other pair's B rows were written into this pair's stage too)
-                    tc_commit_pair_multicast(empty_bar(stage), kAll);
+                    // the stage is free in both CTAs once the MMAs reading it completed
+                    tc_commit_pair_multicast(empty_bar(stage), kBoth);
                     if (++stage == STAGES) { stage = 0; phase ^= 1u; }
                 }
                 if (!ok) break;
-                tc_commit_pair_multicast(tfull_bar(acc), pair_mask);
+                tc_commit_pair_multicast(tfull_bar(acc), kBoth);
                 if (++acc == kAccBufs) { acc = 0; acc_phase ^= 1u; }
             }
-            if (!ok && issued_any) {
-                tc_commit_pair_multicast(drain_bar, static_cast<uint16_t>(1u << lrank));
-                mbar_wait_cl_drain(drain_bar, 0, wait_limit_ns);
+            if (issued_any) {
+                // every MMA issued, which reads both CTAs' stages and writes their TMEM,
+                // completes before teardown (also when only the epilogue gave up)
+                tc_commit_pair_multicast(drain_bar, 0x1);
+                mbar_wait_cl_drain(drain_bar, 0, kDrainLimitNs);
             }
         }
         __syncwarp();
     } else {
         // ------------------------------------------------------- epilogue (both CTAs)
         const int q = warp & 3;
-        const int r_in_tile = 128 * static_cast<int>(prank) + q * 32 + lane;
+        const int r_in_tile = 128 * static_cast<int>(rank) + q * 32 + lane;
         EpiIO io{sbase + L::kOutOffset + static_cast<uint32_t>((warp - 2) * kOutBytesPerWarp), lane,
                  0, 0u};
         int acc = 0;
@@ -338,10 +335,10 @@ __global__ void __cluster_dims__(2 * kPairs, 1, 1) __launch_bounds__(kGemmThread
             const uint32_t t_row = tmem_base + (static_cast<uint32_t>(q * 32) << 16) +
                                    static_cast<uint32_t>(acc * BN);
             if (part < 0) {
-                const int tile_row0 = (mp * kPairs + static_cast<int>(pair)) * kPairBM;
+                const int tile_row0 = mp * kPairBM;
                 const int row = tile_row0 + r_in_tile;
                 const int n0 = nb * BN;
-                io.row0 = tile_row0 + 128 * static_cast<int>(prank) + q * 32;
+                io.row0 = tile_row0 + 128 * static_cast<int>(rank) + q * 32;
                 Epi epi(ep, g, row, n0);
 #pragma unroll 1
                 for (int c = 0; c < BN / 32; ++c) {
@@ -369,7 +366,7 @@ __global__ void __cluster_dims__(2 * kPairs, 1, 1) __launch_bounds__(kGemmThread
                 if (leader)
                     mbar_arrive(tempty_bar(acc));
                 else
-                    mbar_arrive_cluster(mapa_shared(tempty_bar(acc), lrank));
+                    mbar_arrive_cluster(mapa_shared(tempty_bar(acc), 0));
             }
             if (++acc == kAccBufs) { acc = 0; acc_phase ^= 1u; }
         }
@@ -377,7 +374,18 @@ __global__ void __cluster_dims__(2 * kPairs, 1, 1) __launch_bounds__(kGemmThread
         __syncwarp();
     }
 
+    // Teardown.  Every role has stopped; both producers have published their issued
+    // k-block counts.  After the first pair barrier the leader waits for each copy of
+    // either CTA that no MMA consumed (pair_drain_copies: a no-op wait on completed
+    // phases when nothing gave up); the second barrier keeps both CTAs, and their
+    // shared memory and TMEM, alive until then.
     tc_fence_before();
+    __syncthreads();
+    cluster_sync();
+    if (leader && threadIdx.x == 0)
+        pair_drain_copies<STAGES>(bar0, *issued_word,
+                                  ld_shared_cluster_u32(mapa_shared(smem_u32(issued_word), 1)),
+                                  L::kStageBytes);
     __syncthreads();
     cluster_sync();  // no CTA frees TMEM or exits while another may still touch it
     if (warp == 1) {

@@ -2,7 +2,8 @@
 
 This module only draws inputs; it contains none of the method's arithmetic,
 and it is the one piece of code that both the CUDA path's tests and the oracle
-tests use.  It stands in for the paper's forward-pass caches (Sec. 3.1 step 1:
+tests use.  It sits outside the library package, so importing it loads no
+native code: the oracle-only benchmark arm uses it without touching libfpo.  It stands in for the paper's forward-pass caches (Sec. 3.1 step 1:
 the final pre-norm residual and each target layer's down-projection input)
 and for its adaptation corpora (Sec. 4: packed 2048-token sequences), which
 are not available here.

@@ -32,10 +32,9 @@ _ensure_built()
 @pytest.fixture(scope="session")
 def fpo():
     """The CUDA library through its Python binding; skips when no GPU is present.
-    FPO_TEST_GEMM_VARIANT=0|1|2|3 runs the suite on the single-CTA GEMM, the CTA-pair
-    GEMM with 256 x 256 tiles only, the CTA pair with the 256 x 512 projection (the
-    library default), or that with two CTA pairs sharing each B tile by multicast in the
-    logits pass and the update."""
+    FPO_TEST_GEMM_VARIANT=0|1|2 runs the suite on the single-CTA GEMM, the CTA-pair
+    GEMM with 256 x 256 tiles only, or the CTA pair with the 256 x 512 projection (the
+    library default)."""
     import torch
     if not torch.cuda.is_available():
         pytest.skip("no CUDA device")

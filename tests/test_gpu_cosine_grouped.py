@@ -7,7 +7,7 @@ import pytest
 import torch
 
 import oracle
-from paper_2608_14563_gb300 import synth
+import synth
 
 pytestmark = pytest.mark.gpu
 

@@ -21,8 +21,8 @@ import torch
 
 import oracle
 from helpers import cos, f64, rel_frob
-from paper_2608_14563_gb300 import synth
-from paper_2608_14563_gb300.synth import Workload
+import synth
+from synth import Workload
 
 pytestmark = pytest.mark.gpu
 
@@ -92,7 +92,7 @@ def test_direct_is_bitwise_identical_across_gemm_kernels(fpo, ragged):
     prev = fpo.set_gemm_variant(0)
     outs = []
     try:
-        for v in (0, 1, 2, 3):
+        for v in (0, 1, 2):
             fpo.set_gemm_variant(v)
             outs.append(run(fpo, inp["h"], inp["w"], inp["W_U"], inp["y"], eps=RAGGED.eps,
                             algo=fpo.ES_DIRECT))
@@ -163,7 +163,7 @@ def test_rows_outside_the_anchor_window_are_fixed(fpo):
     assert abs(outs[0]["loss"].item() - oracle.mean_ce(ref["lse"], ref["zy"])) < 1e-4 * np.mean(ce)
 
 
-@pytest.mark.parametrize("variant", [0, 1, 2, 3])
+@pytest.mark.parametrize("variant", [0, 1, 2])
 @pytest.mark.parametrize("algo", [1, 2, 3])  # recompute, stored logits, direct
 def test_results_do_not_depend_on_workspace_contents(fpo, ragged, variant, algo):
     """Every workspace byte a call reads it writes first: a workspace full of 0xFF (NaN
@@ -252,8 +252,8 @@ def test_projection_split_k_tail(fpo, algo):
 @pytest.mark.parametrize("shape", [(700, 320, 840, 3), (1024, 512, 768, 2), (300, 1024, 264, 4)])
 def test_update_is_bitwise_identical_across_gemm_kernels(fpo, shape):
     """The grouped update (G_l, the fp32 master step, the bf16 weights) computes the same
-    sums in the same order per element under every GEMM kernel variant: single CTA, CTA
-    pair, and two CTA pairs sharing each B tile by multicast (ragged T and d)."""
+    sums in the same order per element under every GEMM kernel variant: single CTA and CTA
+    pair (ragged T and d)."""
     T, d, d_ff, L = shape
     gen = torch.Generator(device="cuda").manual_seed(T + d)
     g = (torch.randn(T, d, device="cuda", generator=gen) * 1e-2).to(torch.bfloat16)
@@ -262,7 +262,7 @@ def test_update_is_bitwise_identical_across_gemm_kernels(fpo, shape):
     prev = fpo.set_gemm_variant(0)
     outs = []
     try:
-        for v in (0, 1, 2, 3):
+        for v in (0, 1, 2):
             fpo.set_gemm_variant(v)
             Wm = [w.clone() for w in W0]
             Wo = [torch.empty(d, d_ff, dtype=torch.bfloat16, device="cuda") for _ in range(L)]

@@ -6,8 +6,8 @@ import pytest
 import torch
 
 import oracle
-from paper_2608_14563_gb300 import synth
-from paper_2608_14563_gb300.synth import WORKLOADS
+import synth
+from synth import WORKLOADS
 
 pytestmark = pytest.mark.gpu
 

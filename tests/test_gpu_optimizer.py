@@ -6,8 +6,8 @@ import torch
 
 import oracle
 from helpers import f64, rel_frob
-from paper_2608_14563_gb300 import synth
-from paper_2608_14563_gb300.synth import Workload
+import synth
+from synth import Workload
 
 pytestmark = pytest.mark.gpu
 

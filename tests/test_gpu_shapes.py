@@ -8,8 +8,8 @@ import torch
 
 import oracle
 from helpers import cos, f64, rel_frob
-from paper_2608_14563_gb300 import synth
-from paper_2608_14563_gb300.synth import Workload
+import synth
+from synth import Workload
 
 pytestmark = pytest.mark.gpu
 
@@ -31,7 +31,7 @@ def _shapes(n, seed=2024):
 SHAPES = _shapes(12)
 
 
-@pytest.mark.parametrize("variant", [0, 1, 2, 3])
+@pytest.mark.parametrize("variant", [0, 1, 2])
 @pytest.mark.parametrize("algo", [1, 2, 3])  # recompute, stored logits, direct
 @pytest.mark.parametrize("shape", SHAPES, ids=[f"T{t}d{d}V{v}f{f}" for t, d, v, f in SHAPES])
 def test_random_ragged_shapes(fpo, shape, algo, variant):
