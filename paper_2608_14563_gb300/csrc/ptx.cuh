@@ -63,14 +63,13 @@ struct WaitGuard {
 
 // Wait until the phase with parity `parity` of `bar` has completed.  Returns
 // false (and raises the abort flag / timeout status) when the limit ran out,
-// or when another thread of the CTA already gave up.
+// or when another thread of the CTA already gave up.  try_wait may suspend the
+// thread for a while by itself, so the limit is checked after every try.
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, const WaitGuard& g) {
     if (mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = global_timer_ns();
     while (true) {
-#pragma unroll 1
-        for (int i = 0; i < 32; ++i)
-            if (mbar_try_wait(bar, parity)) return true;
+        if (mbar_try_wait(bar, parity)) return true;
         if (*g.abort_flag) return false;
         if (global_timer_ns() - t0 > g.limit_ns) {
             *g.abort_flag = 1;

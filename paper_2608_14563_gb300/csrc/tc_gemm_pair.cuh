@@ -66,9 +66,7 @@ __device__ __forceinline__ bool mbar_wait_cl(uint32_t bar, uint32_t parity, cons
     if (mbar_try_wait_cluster(bar, parity)) return true;
     const uint64_t t0 = global_timer_ns();
     while (true) {
-#pragma unroll 1
-        for (int i = 0; i < 32; ++i)
-            if (mbar_try_wait_cluster(bar, parity)) return true;
+        if (mbar_try_wait_cluster(bar, parity)) return true;
         if (*g.abort_flag) return false;
         if (global_timer_ns() - t0 > g.limit_ns) {
             *g.abort_flag = 1;
