@@ -496,6 +496,8 @@ def run_fpo(args, wl):
     fixup_rows = (fpo.direct_fixup_rows(X0["h"], W_U, ws_es, t_chunk=args.t_chunk, algo=algo)
                   if algo_name == "direct" else None)
 
+    # the direct algorithm's projection epilogue applies the final-norm VJP itself: its
+    # "projection" stage includes the VJP and its "rmsnorm_vjp" stage is empty
     names = ["rmsnorm_fwd", "logits_lse_pass", "lse_combine",
              {"direct": "direct_fixup", "stored-logits": "logits_to_error",
               "recompute": "recompute_error_pass"}[algo_name], "projection", "rmsnorm_vjp"]
@@ -702,6 +704,9 @@ def run_fpo(args, wl):
                        "peaks": peaks_src},
             "roofline": roofline,
             "kernels_ms": stage_ms,
+            "kernels_note": ("the projection's epilogue applies the final-norm VJP (direct "
+                             "algorithm): rmsnorm_vjp is an empty stage"
+                             if algo_name == "direct" else None),
             "kernels_tflops": {k: per_kernel_flops[k] / (stage_ms[k] / 1e3) / 1e12
                                for k in per_kernel_flops},
             "kernels_gbs": {**({"norm_ratio": wl.layers * wl.d * wl.d_ff * (2 + 4)

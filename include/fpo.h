@@ -94,17 +94,25 @@ typedef enum fpo_status {
  *                        <xhat_t (.) norm_w, W_U[y_t]> (the target logit, from the
  *                        RMSNorm forward), the logits pass writes
  *                        P_tj = exp(z_tj - c_t) in bf16 with the target column 0,
- *                        and the projection forms
+ *                        lse_t = c_t + log(1 + sum_j P_tj) before rounding, and
+ *                        the projection forms
  *                          g_t = s e^{c_t - lse_t} (P_t W_U - S'_t W_U[y_t]),
- *                        S'_t the sum of row t of the rounded P.  This equals
- *                        e_t W_U exactly in real arithmetic (the target entry of
- *                        e_t is -sum of the others), rounds each probability to
- *                        bf16 once like E, and saves the E pass: T_chunk x V x 2
- *                        bytes of workspace.  Rows with S'_t outside
- *                        [2^-80, 2^80] (token cross-entropy beyond ~55 nats, or
- *                        1 - p_target below ~1e-24) are gathered and recomputed
- *                        by the same tensor-core logits GEMM anchored at lse_t
- *                        before the projection (its row count read on the device).
+ *                        S'_t the sum of row t of the rounded P.
+ *                        This equals e_t W_U exactly in real arithmetic (the
+ *                        target entry of e_t is -sum of the others), rounds each
+ *                        probability to bf16 once like E, and saves the E pass:
+ *                        T_chunk x V x 2 bytes of workspace.  The projection's
+ *                        epilogue also applies the final-norm VJP, writing g~
+ *                        directly: the row term <xhat_t, norm_w (.) g_t> is
+ *                        s e^{c_t - lse_t} sum_j P_tj (z_tj - c_t), with sums the
+ *                        logits pass keeps (<yhat_t, W_U[j]> = z_tj).  Rows
+ *                        with S'_t outside [2^-80, 2^80] (token cross-entropy
+ *                        beyond ~55 nats, or 1 - p_target below ~1e-24) are
+ *                        gathered and recomputed by the same tensor-core logits
+ *                        GEMM, first for a max-based lse_t, then anchored at
+ *                        lse_t, before the projection (their row count read on
+ *                        the device).  A row with an out-of-range target gets
+ *                        g~ = 0, and lse 0 and loss term 0.
  *  FPO_ES_AUTO           the library's choice: FPO_ES_DIRECT for bf16,
  *                        FPO_ES_STORED_LOGITS for fp32 (where DIRECT also runs
  *                        the stored-logits algorithm).
@@ -151,14 +159,16 @@ typedef struct fpo_error_signal_desc {
  * the last token chunk for FPO_ES_STORED_LOGITS), 3 after the log-sum-exp
  * combine (and loss), 4 after the recompute pass (FPO_ES_RECOMPUTE), the
  * logits-to-E conversion (FPO_ES_STORED_LOGITS) or the anchor-window fixup
- * (FPO_ES_DIRECT) of the last token chunk, 5
- * after the projection of the last token chunk, 6 after the final-norm VJP.
+ * (FPO_ES_DIRECT; with the loss mean) of the last token chunk, 5
+ * after the projection of the last token chunk, 6 after the final-norm VJP
+ * (under FPO_ES_DIRECT the projection applies the VJP: 5 to 6 is empty).
  * With one chunk, consecutive events bracket one kernel each (plus the loss
  * mean in [2]-[3]).
  * With stage_events_per_chunk = 1 and n token chunks the events are 3 + 4 n:
  * 0 start, 1 after the RMSNorm forward, then for chunk c = 0 .. n-1:
- * 2 + 4c after its logits pass, 3 + 4c after its combine (and, last chunk, the
- * loss mean), 4 + 4c after its E / fixup stage, 5 + 4c after its projection;
+ * 2 + 4c after its logits pass, 3 + 4c after its combine (and, last chunk and
+ * not FPO_ES_DIRECT, the loss mean), 4 + 4c after its E / fixup stage (and,
+ * last chunk and FPO_ES_DIRECT, the loss mean), 5 + 4c after its projection;
  * and 2 + 4n after the VJP.  (FPO_ES_RECOMPUTE runs one logits pass and one
  * combine over all tokens: they fill chunk 0's first two slots; the other
  * chunks record those two at the chunk's start.)

@@ -90,45 +90,71 @@ using EpiLseStoreZ = EpiLsePartialT<true>;
 
 // ---------------------------------------------------------------------------
 // Logits pass of the direct algorithm (Sec. 3.1 step 2 rewritten around a
-// per-token anchor c_t): besides the (max, sum exp) partial and the target
-// logit of EpiLsePartial, every valid non-target logit leaves
-//   p~_tj = exp(z_tj - c_t) = exp(z_tj - m) exp(m - c_t)   (m: the running max)
+// per-token anchor c_t, the target logit): every valid non-target logit leaves
+//   p~_tj = exp(z_tj - c_t)
 // rounded to bf16 into P [M, N] (the target column and the overhang are written
-// as 0), and the tile's sum of those rounded values, S'_t partial, goes to
-// sx [M, part_ld].  Two 32-column chunks fill one 64-column bf16 staging row
-// before each TMA store.
-struct EpiLseProb {
+// as 0), and per (row, 256-column tile) three sums:
+//   su = sum_j p~_tj          (unrounded: lse_t = c_t + log(1 + S_t), the target's
+//                              own term being exp(0) = 1)
+//   sx = sum_j p^_tj          (p^ the rounded values: the tile's part of S'_t, which
+//                              makes the target entry of e the exact negative sum)
+//   qz = sum_j p^_tj z_tj     (for the final-norm VJP fused into the projection:
+//                              <yhat_t, g_t> = sum_v e_tv z_tv = alpha_t (Qz_t - c_t S'_t))
+// No running maximum is kept: a row whose S'_t leaves the window [2^-80, 2^80]
+// (where the anchored sums could overflow, or hold no significant digit) is
+// recomputed by the fixup path, which takes its lse from a max-based pass
+// (EpiFixLse, then EpiFixProb).
+// Chunks that hold neither a target nor the vocabulary's ragged end (all but a few
+// per row) take a branch-free path on packed f32x2 arithmetic; two 32-column chunks
+// fill one 64-column bf16 staging row before each TMA store.
+struct EpiAnchorProb {
     struct Params {
         CUtensorMap pmap;     // bf16 P [M, N], box 64 x 32
-        float2* part;         // [M, part_ld] (max, sum exp(z - max))
+        float* su;            // [M, part_ld] sum of p~ over the tile
         float* sx;            // [M, part_ld] sum of the rounded p~ of the tile
+        float* qz;            // [M, part_ld] sum of the rounded p~ times z over the tile
         int part_ld;
-        float* zy;            // [M] target logit, or null
         const int* y;         // [M] targets
         const float* anchor;  // [M] c_t
         int M, N;
     };
-    float m, s, zt, sxs, c2;
-    int yoff;
-    int row;
-    bool valid, has_t, pair_out;
+    float2 u0, u1, s0, s1, q0, q1;  // two accumulators each: shorter dependency chains
+    float2 nc2;             // (-c_t log2 e) twice
+    int yoff, row;
+    bool valid, pair_out;
     uint32_t w[32];
 
-    __device__ __forceinline__ EpiLseProb(const Params& p, int, int row_, int n0)
-        : m(-INFINITY), s(0.f), zt(0.f), sxs(0.f), row(row_), has_t(false), pair_out(false) {
+    __device__ __forceinline__ EpiAnchorProb(const Params& p, int, int row_, int n0)
+        : row(row_), pair_out(false) {
         valid = row_ < p.M;
         yoff = valid ? __ldg(p.y + row_) - n0 : -1;
-        c2 = valid ? __ldg(p.anchor + row_) * kLog2e : 0.f;
+        const float nc = valid ? -__ldg(p.anchor + row_) * kLog2e : 0.f;
+        nc2 = make_float2(nc, nc);
+        u0 = u1 = s0 = s1 = q0 = q1 = make_float2(0.f, 0.f);
     }
 
-    // p~ of logits j, j+1 of the chunk from their exponentials e relative to the running
-    // max (0 for the target and for columns >= lim, where e is 0), scaled by
-    // f = exp(max - c); packed to bf16, the rounded values added to the tile sum.
-    __device__ __forceinline__ uint32_t prob_pair(const float (&e)[32], float f, int j, int r) {
-        const float a = j != r ? e[j] * f : 0.f;
-        const float b = j + 1 != r ? e[j + 1] * f : 0.f;
-        const uint32_t pk = pack_bf16x2(a, b);
-        sxs += __uint_as_float(pk << 16) + __uint_as_float(pk & 0xffff0000u);
+    // p^ of the pair (j, j + 1) and its contribution to the sums; kMask: zero the
+    // target (position r) and the columns >= lim.
+    template <bool kMask>
+    __device__ __forceinline__ uint32_t pair(const float (&v)[32], int j, int r, int lim) {
+        const float2 z = make_float2(v[j], v[j + 1]);
+        const float2 arg = __ffma2_rn(z, make_float2(kLog2e, kLog2e), nc2);
+        float pa = ex2_approx(arg.x), pb = ex2_approx(arg.y);
+        if constexpr (kMask) {
+            pa = (j < lim && j != r) ? pa : 0.f;
+            pb = (j + 1 < lim && j + 1 != r) ? pb : 0.f;
+        }
+        const uint32_t pk = pack_bf16x2(pa, pb);
+        const float2 rp = make_float2(__uint_as_float(pk << 16), __uint_as_float(pk & 0xffff0000u));
+        if ((j / 2) & 1) {
+            u1 = __fadd2_rn(u1, make_float2(pa, pb));
+            s1 = __fadd2_rn(s1, rp);
+            q1 = __ffma2_rn(rp, z, q1);
+        } else {
+            u0 = __fadd2_rn(u0, make_float2(pa, pb));
+            s0 = __fadd2_rn(s0, rp);
+            q0 = __ffma2_rn(rp, z, q0);
+        }
         return pk;
     }
 
@@ -138,41 +164,22 @@ struct EpiLseProb {
         if (!second) pair_out = col0 >= p.N || io.row0 >= p.M;
         const int lim = p.N - col0;  // valid columns in this chunk (may be <= 0)
         const int r = yoff - c0;     // target position in this chunk, if in [0, 32)
-        float e[32];
-        float f = 0.f;
-        if (lim > 0) {
-            float cm = -INFINITY;
+        uint32_t pk[16];
+        // warp-uniform: a chunk holding any lane's target, or the ragged end, is masked
+        if (lim < 32 || __any_sync(0xffffffffu, static_cast<unsigned>(r) < 32u)) {
 #pragma unroll
-            for (int j = 0; j < 32; ++j)
-                if (j < lim) cm = fmaxf(cm, v[j]);
-            const float nm = fmaxf(m, cm);
-            const float nml = nm * kLog2e;
-            float acc = (m == -INFINITY) ? 0.f : s * ex2_approx(m * kLog2e - nml);
-#pragma unroll
-            for (int j = 0; j < 32; ++j) {
-                e[j] = j < lim ? ex2_approx(fmaf(v[j], kLog2e, -nml)) : 0.f;
-                acc += e[j];
-            }
-            s = acc;
-            m = nm;
-            f = ex2_approx(nml - c2);
-            if (static_cast<unsigned>(r) < 32u) {
-#pragma unroll
-                for (int j = 0; j < 32; ++j)
-                    if (j == r) zt = v[j];
-                has_t = true;
-            }
+            for (int j = 0; j < 32; j += 2) pk[j / 2] = pair<true>(v, j, r, lim);
         } else {
 #pragma unroll
-            for (int j = 0; j < 32; ++j) e[j] = 0.f;
+            for (int j = 0; j < 32; j += 2) pk[j / 2] = pair<false>(v, j, r, lim);
         }
         if (pair_out) return;
         if (!second) {
 #pragma unroll
-            for (int j = 0; j < 32; j += 2) w[j / 2] = prob_pair(e, f, j, r);
+            for (int i = 0; i < 16; ++i) w[i] = pk[i];
         } else {
 #pragma unroll
-            for (int j = 0; j < 32; j += 2) w[16 + j / 2] = prob_pair(e, f, j, r);
+            for (int i = 0; i < 16; ++i) w[16 + i] = pk[i];
             const uint32_t buf = out_acquire(io);
             out_stage_row(buf, io.lane, w);
             out_commit(io, &p.pmap, buf, col0 - 32, io.row0);
@@ -182,22 +189,71 @@ struct EpiLseProb {
     __device__ __forceinline__ void finish(const Params& p, int nb) {
         if (!valid) return;
         const long long o = static_cast<long long>(row) * p.part_ld + nb;
-        p.part[o] = make_float2(m, s);
-        p.sx[o] = sxs;
-        if (has_t && p.zy) p.zy[row] = zt;
+        const float2 u = __fadd2_rn(u0, u1), s = __fadd2_rn(s0, s1), q = __fadd2_rn(q0, q1);
+        p.su[o] = u.x + u.y;
+        p.sx[o] = s.x + s.y;
+        p.qz[o] = q.x + q.y;
     }
 };
 
 // ---------------------------------------------------------------------------
-// Direct algorithm, rows outside the anchor window (Sec. 3.1 step 2 with the
-// anchor at lse_t): the GEMM's rows are the yhat rows gathered from fix[0, count);
-// each logit z of such a row becomes p~ = exp(z - lse_t), 0 at the target,
-// rounded to bf16 and stored into that row of P with plain 16-byte stores; the
-// row's sum of the rounded values over the tile goes to sx[row, tile].
+// Direct algorithm, rows outside the anchor window, first pass: the logits of the
+// gathered rows (the GEMM's rows are fix[0, count)) reduced to a running max and
+// sum of exponentials per (row, 256-column tile), written to part[row of the chunk,
+// tile], from which lse is formed before the second pass (EpiFixProb).
+struct EpiFixLse {
+    struct Params {
+        float2* part;        // [T, part_ld] (max, sum exp(z - max))
+        int part_ld;
+        const int* fix;      // gathered row -> row of the chunk
+        const int* count;    // gathered rows (device)
+        int N;
+    };
+    float m, s;
+    int orig;
+    bool valid;
+
+    __device__ __forceinline__ EpiFixLse(const Params& p, int, int row_, int)
+        : m(-INFINITY), s(0.f) {
+        valid = row_ < *p.count;
+        orig = valid ? p.fix[row_] : 0;
+    }
+
+    __device__ __forceinline__ void chunk(const Params& p, const float (&v)[32], int col0, int,
+                                          EpiIO&) {
+        const int lim = p.N - col0;
+        if (!valid || lim <= 0) return;
+        float cm = -INFINITY;
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+            if (j < lim) cm = fmaxf(cm, v[j]);
+        const float nm = fmaxf(m, cm);
+        const float nml = nm * kLog2e;
+        float acc = (m == -INFINITY) ? 0.f : s * ex2_approx(m * kLog2e - nml);
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+            if (j < lim) acc += ex2_approx(fmaf(v[j], kLog2e, -nml));
+        s = acc;
+        m = nm;
+    }
+
+    __device__ __forceinline__ void finish(const Params& p, int nb) {
+        if (valid) p.part[static_cast<size_t>(orig) * p.part_ld + nb] = make_float2(m, s);
+    }
+};
+
+// ---------------------------------------------------------------------------
+// Direct algorithm, rows outside the anchor window, second pass (Sec. 3.1 step 2
+// with the anchor at lse_t): the GEMM's rows are the yhat rows gathered from
+// fix[0, count); each logit z of such a row becomes p~ = exp(z - lse_t), 0 at the
+// target, rounded to bf16 and stored into that row of P with plain 16-byte stores;
+// the row's sums over the tile of the rounded values and of the rounded values
+// times z go to sx[row, tile] and qz[row, tile], as EpiAnchorProb leaves them.
 struct EpiFixProb {
     struct Params {
         __nv_bfloat16* P;    // [T, N] rows of the chunk, row stride N
         float* sx;           // [T, n_tiles]
+        float* qz;           // [T, n_tiles]
         const int* fix;      // gathered row -> row of the chunk
         const int* count;    // gathered rows (device)
         const int32_t* y;    // [T] targets
@@ -205,10 +261,11 @@ struct EpiFixProb {
         int n_tiles, N;
     };
     int orig, yt;
-    float lse2, sxs;
+    float lse2, sxs, qs;
     bool valid;
 
-    __device__ __forceinline__ EpiFixProb(const Params& p, int, int row_, int) : sxs(0.f) {
+    __device__ __forceinline__ EpiFixProb(const Params& p, int, int row_, int)
+        : sxs(0.f), qs(0.f) {
         valid = row_ < *p.count;
         orig = valid ? p.fix[row_] : 0;
         yt = valid ? p.y[orig] : -1;
@@ -227,7 +284,10 @@ struct EpiFixProb {
             const float b =
                 (j + 1 < lim && j + 1 != r) ? ex2_approx(fmaf(v[j + 1], kLog2e, -lse2)) : 0.f;
             const uint32_t pk = pack_bf16x2(a, b);
-            sxs += __uint_as_float(pk << 16) + __uint_as_float(pk & 0xffff0000u);
+            const float ra = __uint_as_float(pk << 16), rb = __uint_as_float(pk & 0xffff0000u);
+            sxs += ra + rb;
+            qs = fmaf(ra, v[j], qs);
+            qs = fmaf(rb, v[j + 1], qs);
             w[j / 2] = pk;
         }
         uint4* dst = reinterpret_cast<uint4*>(p.P + static_cast<size_t>(orig) * p.N + col0);
@@ -237,7 +297,10 @@ struct EpiFixProb {
     }
 
     __device__ __forceinline__ void finish(const Params& p, int nb) {
-        if (valid) p.sx[static_cast<size_t>(orig) * p.n_tiles + nb] = sxs;
+        if (valid) {
+            p.sx[static_cast<size_t>(orig) * p.n_tiles + nb] = sxs;
+            p.qz[static_cast<size_t>(orig) * p.n_tiles + nb] = qs;
+        }
     }
 };
 
@@ -314,62 +377,118 @@ struct EpiStoreF32 {
 };
 
 // ---------------------------------------------------------------------------
-// Projection of the direct algorithm: with acc = P W_U (target column of P
-// zero), the unnormalised error signal of token t is
+// Projection of the direct algorithm with the final-norm VJP (App. E,
+// Eq. rmsnorm-vjp) fused in.  With acc = P W_U (target column of P zero), the
+// unnormalised error signal of token t is
 //   g_t = alpha_t acc_t + beta_t W_U[y_t],   alpha_t = s exp(c_t - lse_t),
 //   beta_t = -alpha_t S'_t,
-// which is s (softmax(z_t) - 1_{y_t}) W_U written with the anchor c_t.  A row
-// with alpha_t == 0 is written as zeros (rows the fixup kernel recomputes, or
-// s == 0); beta_t == 0 skips the read of the target's W_U row.
-struct EpiProjDirect {
+// which is s (softmax(z_t) - 1_{y_t}) W_U written with the anchor c_t, and the
+// epilogue writes, in bf16,
+//   g~_t = (w (.) g_t - x^_t k_t) / max(rho_t, rho_min),   x^_t = h_t / rho_t,
+// where k_t = <x^_t, w (.) g_t> / d arrives as cv_t / d: cv_t = alpha_t (Qz_t - c_t S'_t)
+// from the logits pass (EpiAnchorProb), the same inner product taken through the
+// logits (<yhat_t, W_U[v]> = z_tv), so no tile needs the whole row of g.
+// A row with alpha_t == 0 is written as zeros (s == 0, or an out-of-range
+// target); beta_t == 0 skips the read of the target's W_U row.  The h, w and
+// W_U[y] values of the next 32-column chunk are loaded while the current one is
+// processed; two chunks fill one 64-column bf16 staging row per TMA store.
+struct EpiProjVjp {
     struct Params {
-        CUtensorMap Cmap;  // fp32 g [M, N], box 32 x 32
-        const float* alpha;
-        const float* beta;
-        const int* y;
-        const __nv_bfloat16* W_U;  // [V, N]
+        CUtensorMap omap;           // bf16 g~ [M, N], box 64 x 32
+        const float* alpha;         // [M]
+        const float* beta;          // [M]
+        const float* cv;            // [M] <yhat_t, g_t>
+        const float* rho;           // [M] RMS of h_t (forward pass)
+        const int* y;               // [M]
+        const __nv_bfloat16* W_U;   // [V, N]
+        const __nv_bfloat16* h;     // [M, N] pre-norm residual
+        const __nv_bfloat16* w;     // [N] final RMSNorm weight
+        float min_rms, inv_d;
         int M, N;
+        int tile_n;                 // columns of the kernel's tiles (one epilogue object each)
     };
-    float a, b;
+    float a, b, inv_r, kd, pref;
     const __nv_bfloat16* wy;
+    const __nv_bfloat16* hr;
+    bool valid, pair_out;
+    int n_end;
+    uint4 uh[4], uw[4], uy[4];  // h, w, W_U[y] of the chunk the next chunk() call uses
+    uint32_t o[32];
 
-    __device__ __forceinline__ EpiProjDirect(const Params& p, int, int row, int) {
-        const bool valid = row < p.M;
-        a = valid ? __ldg(p.alpha + row) : 0.f;
-        b = valid ? __ldg(p.beta + row) : 0.f;
-        wy = (a != 0.f && b != 0.f) ? p.W_U + static_cast<long long>(__ldg(p.y + row)) * p.N
-                                    : nullptr;
+    __device__ __forceinline__ void fetch(const Params& p, int col0) {
+        const int lim = p.N - col0;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const bool in = q * 8 < lim;
+            uh[q] = (valid && in) ? __ldg(reinterpret_cast<const uint4*>(hr + col0) + q)
+                                  : make_uint4(0, 0, 0, 0);
+            uw[q] = in ? __ldg(reinterpret_cast<const uint4*>(p.w + col0) + q)
+                       : make_uint4(0, 0, 0, 0);
+            uy[q] = (wy && in) ? __ldg(reinterpret_cast<const uint4*>(wy + col0) + q)
+                               : make_uint4(0, 0, 0, 0);
+        }
     }
 
-    __device__ __forceinline__ void chunk(const Params& p, const float (&v)[32], int col0, int,
+    __device__ __forceinline__ EpiProjVjp(const Params& p, int, int row, int n0)
+        : pair_out(false) {
+        valid = row < p.M;
+        a = valid ? __ldg(p.alpha + row) : 0.f;
+        b = valid ? __ldg(p.beta + row) : 0.f;
+        const float r = valid ? __ldg(p.rho + row) : 1.f;
+        inv_r = 1.0f / r;
+        kd = valid ? __ldg(p.cv + row) * p.inv_d : 0.f;
+        pref = 1.0f / fmaxf(r, p.min_rms);
+        wy = (a != 0.f && b != 0.f) ? p.W_U + static_cast<long long>(__ldg(p.y + row)) * p.N
+                                    : nullptr;
+        hr = p.h + static_cast<long long>(valid ? row : 0) * p.N;
+        n_end = min(n0 + p.tile_n, p.N);
+        if (n0 < p.N) fetch(p, n0);
+    }
+
+    __device__ __forceinline__ void chunk(const Params& p, const float (&v)[32], int col0, int c0,
                                           EpiIO& io) {
-        if (col0 >= p.N || io.row0 >= p.M) return;
-        const int lim = p.N - col0;  // a multiple of 8: N % 8 == 0 and col0 % 32 == 0
-        uint32_t o[32];
-        if (a == 0.f) {
+        const bool second = (c0 & 32) != 0;
+        uint4 ch[4], cw[4], cy[4];
 #pragma unroll
-            for (int j = 0; j < 32; ++j) o[j] = 0u;
-        } else if (wy) {
+        for (int q = 0; q < 4; ++q) {
+            ch[q] = uh[q];
+            cw[q] = uw[q];
+            cy[q] = uy[q];
+        }
+        if (col0 + 32 < n_end) fetch(p, col0 + 32);
+        if (!second) pair_out = col0 >= p.N || io.row0 >= p.M;
+        if (pair_out) return;
+        uint32_t r[16];
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                uint4 u = make_uint4(0, 0, 0, 0);
-                if (q * 8 < lim) u = __ldg(reinterpret_cast<const uint4*>(wy + col0) + q);
-                const uint32_t h[4] = {u.x, u.y, u.z, u.w};
+        for (int q = 0; q < 4; ++q) {
+            const uint32_t hh[4] = {ch[q].x, ch[q].y, ch[q].z, ch[q].w};
+            const uint32_t ww[4] = {cw[q].x, cw[q].y, cw[q].z, cw[q].w};
+            const uint32_t yy[4] = {cy[q].x, cy[q].y, cy[q].z, cy[q].w};
 #pragma unroll
-                for (int k = 0; k < 4; ++k) {
-                    const int j = 8 * q + 2 * k;
-                    o[j] = __float_as_uint(fmaf(a, v[j], b * __uint_as_float(h[k] << 16)));
-                    o[j + 1] =
-                        __float_as_uint(fmaf(a, v[j + 1], b * __uint_as_float(h[k] & 0xffff0000u)));
+            for (int k = 0; k < 4; ++k) {
+                const int j = 8 * q + 2 * k;
+                float gv[2], out[2];
+                const float hv[2] = {__uint_as_float(hh[k] << 16), __uint_as_float(hh[k] & 0xffff0000u)};
+                const float wv[2] = {__uint_as_float(ww[k] << 16), __uint_as_float(ww[k] & 0xffff0000u)};
+                const float uv[2] = {__uint_as_float(yy[k] << 16), __uint_as_float(yy[k] & 0xffff0000u)};
+#pragma unroll
+                for (int e = 0; e < 2; ++e) {
+                    gv[e] = a == 0.f ? 0.f : fmaf(a, v[j + e], b * uv[e]);
+                    out[e] = (wv[e] * gv[e] - (hv[e] * inv_r) * kd) * pref;
                 }
+                r[j / 2] = pack_bf16x2(out[0], out[1]);
             }
+        }
+        if (!second) {
+#pragma unroll
+            for (int i = 0; i < 16; ++i) o[i] = r[i];
         } else {
 #pragma unroll
-            for (int j = 0; j < 32; ++j) o[j] = __float_as_uint(a * v[j]);
+            for (int i = 0; i < 16; ++i) o[16 + i] = r[i];
+            const uint32_t buf = out_acquire(io);
+            out_stage_row(buf, io.lane, o);
+            out_commit(io, &p.omap, buf, col0 - 32, io.row0);
         }
-        const uint32_t buf = out_acquire(io);
-        out_stage_row(buf, io.lane, o);
-        out_commit(io, &p.Cmap, buf, col0, io.row0);
     }
 
     __device__ __forceinline__ void finish(const Params&, int) {}
@@ -406,10 +525,21 @@ struct EpiUpdate {
         if (wm) {
             float4* wp = reinterpret_cast<float4*>(wm + off);
             uint4* op = reinterpret_cast<uint4*>(wo + off);
+            // every master load of the chunk is issued before the first store (which the
+            // compiler cannot reorder across, as W_out might alias W_master): one memory
+            // round trip per chunk instead of four
+            float4 ma[4], mb[4];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                if (q * 8 < lim) {
+                    ma[q] = wp[2 * q];
+                    mb[q] = wp[2 * q + 1];
+                }
+            }
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
                 if (q * 8 >= lim) break;
-                float4 a = wp[2 * q], b = wp[2 * q + 1];
+                float4 a = ma[q], b = mb[q];
                 a.x = fmaf(p.neg_lr, v[8 * q + 0], a.x);
                 a.y = fmaf(p.neg_lr, v[8 * q + 1], a.y);
                 a.z = fmaf(p.neg_lr, v[8 * q + 2], a.z);

@@ -78,8 +78,8 @@ int32_t cuda_status(cudaError_t e) { return e == cudaSuccess ? FPO_OK : FPO_ERR_
 
 // ------------------------------------------------------------------ error signal
 struct EsLayout {
-    size_t yhat, rho, lse, zy, ce, part, g, E, z, anchor, sx, alpha, beta, fix, yfix, fix_count,
-        sk, total;
+    size_t yhat, rho, lse, zy, ce, part, g, E, z, anchor, su, sx, q, alpha, beta, cv, fix, yfix,
+        fix_count, sk, total;
     int n_tiles;
     int64_t Tc;
     int algo;  // the algorithm that runs: FPO_ES_RECOMPUTE, _STORED_LOGITS or _DIRECT
@@ -127,16 +127,20 @@ EsLayout es_layout(const fpo_error_signal_desc* d) {
     L.zy = off;   off = align_up(off + T * 4);
     L.ce = off;   off = align_up(off + T * 4);
     L.part = off; off = align_up(off + T * static_cast<size_t>(L.n_tiles) * 8);
-    L.g = off;    off = align_up(off + T * D * 4);
-    L.E = off;    off = align_up(off + static_cast<size_t>(L.Tc) * V * esz);
     L.algo = es_algo(d);
     const bool stored = L.algo == FPO_ES_STORED_LOGITS, direct = L.algo == FPO_ES_DIRECT;
+    // g in fp32 for the separate VJP (the direct algorithm writes g~ from the projection)
+    L.g = off;    off = align_up(off + (direct ? 0 : T * D * 4));
+    L.E = off;    off = align_up(off + static_cast<size_t>(L.Tc) * V * esz);
     L.z = off;    off = align_up(off + (stored ? static_cast<size_t>(L.Tc) * V * 4 : 0));
     const size_t Tdir = direct ? T : 0, Tcdir = direct ? static_cast<size_t>(L.Tc) : 0;
     L.anchor = off;    off = align_up(off + Tdir * 4);
+    L.su = off;        off = align_up(off + Tdir * static_cast<size_t>(L.n_tiles) * 4);
     L.sx = off;        off = align_up(off + Tdir * static_cast<size_t>(L.n_tiles) * 4);
+    L.q = off;         off = align_up(off + Tdir * static_cast<size_t>(L.n_tiles) * 4);
     L.alpha = off;     off = align_up(off + Tdir * 4);
     L.beta = off;      off = align_up(off + Tdir * 4);
+    L.cv = off;        off = align_up(off + Tdir * 4);
     L.fix = off;       off = align_up(off + Tcdir * 4);
     L.yfix = off;      off = align_up(off + Tcdir * D * esz);
     L.fix_count = off; off = align_up(off + (direct ? 4 : 0));
@@ -247,39 +251,54 @@ int32_t fpo_error_signal(const fpo_error_signal_desc* desc, const void* h, const
                                status, st, direct ? W_U : nullptr, direct ? anchor : nullptr));
     FPO_TRY(mark(1));
     if (direct) {
-        // 2.-4. per token chunk: logits pass writing P = exp(z - c) -> lse and row
-        //       factors -> fixup of rows outside the anchor window -> g = alpha P W_U + beta W_U[y]
+        // 2.-5. per token chunk: logits pass anchored at the target logit, writing
+        //       P = exp(z - c) and the per-tile sums -> lse, loss and row factors -> the
+        //       rows outside the anchor window: their lse by a max-based pass, then P
+        //       anchored at lse -> g = alpha P W_U + beta W_U[y] with the final-norm VJP
+        //       in the projection's epilogue -> g~
+        float* su = reinterpret_cast<float*>(ws + L.su);
         float* sx = reinterpret_cast<float*>(ws + L.sx);
+        float* qz = reinterpret_cast<float*>(ws + L.q);
         float* alpha = reinterpret_cast<float*>(ws + L.alpha);
         float* beta = reinterpret_cast<float*>(ws + L.beta);
+        float* cv = reinterpret_cast<float*>(ws + L.cv);
         int* fix = reinterpret_cast<int*>(ws + L.fix);
         int* fix_count = reinterpret_cast<int*>(ws + L.fix_count);
         void* yfix = ws + L.yfix;
-        float* zyd = reinterpret_cast<float*>(ws + L.zy);
         for (int64_t c0 = 0, ci = 0; c0 < T; c0 += L.Tc, ++ci) {
             const int tc = static_cast<int>(L.Tc < T - c0 ? L.Tc : T - c0);
             const bool last = c0 + tc >= T;
             const void* yh = static_cast<const uint8_t*>(yhat) + static_cast<size_t>(c0) * d * esz;
             float2* pc = part + static_cast<size_t>(c0) * L.n_tiles;
+            float* suc = su + static_cast<size_t>(c0) * L.n_tiles;
             float* sxc = sx + static_cast<size_t>(c0) * L.n_tiles;
+            float* qc = qz + static_cast<size_t>(c0) * L.n_tiles;
             float* cec = ce ? ce + c0 : nullptr;
             FPO_TRY(cudaMemsetAsync(fix_count, 0, sizeof(int), st));
-            FPO_TRY(launch_lse_prob_bf16(yh, W_U, targets + c0, anchor + c0, tc, d, V, pc, sxc,
-                                         L.n_tiles, zyd + c0, E, status, st));
+            FPO_TRY(launch_anchor_prob_bf16(yh, W_U, targets + c0, anchor + c0, tc, d, V, suc, sxc,
+                                            qc, L.n_tiles, E, status, st));
             FPO_TRY(cmark(ci, 2));
-            FPO_TRY(launch_direct_combine(pc, sxc, L.n_tiles, tc, V, targets + c0, anchor + c0,
-                                          zyd + c0, desc->loss_scale, lse + c0, cec, alpha + c0,
-                                          beta + c0, fix, fix_count, st));
-            if (last && loss_out) FPO_TRY(launch_mean(ce, T, loss_out, st));
+            FPO_TRY(launch_direct_combine(suc, sxc, qc, L.n_tiles, tc, V, targets + c0, anchor + c0,
+                                          desc->loss_scale, lse + c0, cec, alpha + c0, beta + c0,
+                                          cv + c0, fix, fix_count, st));
             FPO_TRY(cmark(ci, 3));
             FPO_TRY(launch_gather_rows(yh, fix, fix_count, d, yfix, st));
+            FPO_TRY(launch_fixup_lse_bf16(yfix, W_U, fix, fix_count, tc, d, V, pc, L.n_tiles,
+                                          status, st));
+            FPO_TRY(launch_direct_fixup_lse(pc, fix, fix_count, L.n_tiles, anchor + c0, lse + c0,
+                                            cec, st));
             FPO_TRY(launch_fixup_logits_bf16(yfix, W_U, fix, fix_count, targets + c0, lse + c0, tc,
-                                             d, V, E, sxc, L.n_tiles, status, st));
-            FPO_TRY(launch_direct_fixup_factors(sxc, fix, fix_count, L.n_tiles, desc->loss_scale,
-                                                alpha + c0, beta + c0, st));
+                                             d, V, E, sxc, qc, L.n_tiles, status, st));
+            FPO_TRY(launch_direct_fixup_factors(sxc, qc, fix, fix_count, L.n_tiles, anchor + c0,
+                                                desc->loss_scale, alpha + c0, beta + c0, cv + c0,
+                                                st));
+            if (last && loss_out) FPO_TRY(launch_mean(ce, T, loss_out, st));
             FPO_TRY(cmark(ci, 4));
-            FPO_TRY(launch_proj_direct_bf16(E, W_U, targets + c0, alpha + c0, beta + c0, tc, d, V,
-                                            g + c0 * d, sk, status, st));
+            FPO_TRY(launch_proj_vjp_bf16(
+                E, W_U, targets + c0, alpha + c0, beta + c0, cv + c0, rho + c0,
+                static_cast<const uint8_t*>(h) + static_cast<size_t>(c0) * d * esz, norm_w,
+                desc->min_rms, tc, d, V,
+                static_cast<uint8_t*>(g_out) + static_cast<size_t>(c0) * d * esz, sk, status, st));
             FPO_TRY(cmark(ci, 5));
         }
     } else if (L.algo == FPO_ES_RECOMPUTE) {
@@ -350,8 +369,11 @@ int32_t fpo_error_signal(const fpo_error_signal_desc* desc, const void* h, const
             FPO_TRY(cmark(ci, 5));
         }
     }
-    // 5. final-norm VJP with the min-RMS clamp -> g~
-    FPO_TRY(launch_rmsnorm_vjp(desc->dtype, g, h, norm_w, rho, T, d, desc->min_rms, g_out, st));
+    // 5. final-norm VJP with the min-RMS clamp -> g~ (already in the direct algorithm's
+    //    projection epilogue; the stage is then empty)
+    if (!direct)
+        FPO_TRY(launch_rmsnorm_vjp(desc->dtype, g, h, norm_w, rho, T, d, desc->min_rms, g_out,
+                                   st));
     FPO_TRY(per_chunk ? ev(2 + 4 * n_chunks) : mark(6));
     return FPO_OK;
 }

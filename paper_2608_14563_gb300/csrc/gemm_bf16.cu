@@ -4,7 +4,8 @@
 //   recompute pass   same GEMM, epilogue writes E = s (softmax - onehot)
 //   direct logits    same GEMM, epilogue writes P = exp(z - c) (target zero)
 //   projection       g = E W_U           M=T  N=d    K=V   A K-major, B MN-major
-//                    (or g = alpha P W_U + beta W_U[y] in the direct algorithm)
+//                    (or g = alpha P W_U + beta W_U[y] in the direct algorithm, whose
+//                    epilogue applies the final-norm VJP and writes g~)
 //   update           G = g~^T A_l        M=d  N=d_ff K=T   A MN-major, B MN-major
 //
 // Tensor maps are encoded per call (a few microseconds of host work) through
@@ -199,18 +200,15 @@ cudaError_t run_gemm_pair(const GemmMaps<MAXG>& maps, const typename Epi::Params
     return cudaGetLastError();
 }
 
-// Sum the tail_split k-range partials of every split tail tile in range order, then the
-// projection epilogue: C[row, n] = alpha_row * sum + beta_row * W_U[y_row, n]
-// (alpha == nullptr: the plain sum), as EpiProjDirect / EpiStoreF32 form whole tiles.
+// Fixups of the split-K tail: sum the tail_split k-range partials of every split tail
+// tile in range order, then apply the epilogue the whole tiles got.
 // Grid (tail tiles, 256 rows / rows per block): one thread per 4 columns of a row.
 constexpr int kFixupThreads = 256;
 
+// The summed partials of this thread's 4 columns; false outside the matrix.
 template <int BN>
-__global__ void __launch_bounds__(kFixupThreads)
-    sk_fixup_kernel(const GemmShape sh, const float* __restrict__ scratch,
-                    float* __restrict__ C, const float* __restrict__ alpha,
-                    const float* __restrict__ beta, const int* __restrict__ y,
-                    const __nv_bfloat16* __restrict__ W_U) {
+__device__ __forceinline__ bool sk_tail_sum(const GemmShape& sh, const float* __restrict__ scratch,
+                                            int& row, int& n, float (&s4)[4]) {
     constexpr int kThreadsPerRow = BN / 4;
     constexpr int kRowsPerBlock = kFixupThreads / kThreadsPerRow;
     const long long R = sh.tail_tiles;
@@ -219,10 +217,10 @@ __global__ void __launch_bounds__(kFixupThreads)
     const int col = (threadIdx.x % kThreadsPerRow) * 4;
     int g, mp, nb;
     tile_coords(sh.tiles - R + r_tile, sh, g, mp, nb);
-    const int row = mp * kPairBM + r;
-    const int n = nb * BN + col;
-    if (row >= sh.M || n >= sh.N) return;  // N % 8 == 0: whole float4s
-    float s4[4] = {0.f, 0.f, 0.f, 0.f};
+    row = mp * kPairBM + r;
+    n = nb * BN + col;
+    if (row >= sh.M || n >= sh.N) return false;  // N % 8 == 0: whole groups of 4
+    s4[0] = s4[1] = s4[2] = s4[3] = 0.f;
     for (int q = 0; q < sh.tail_split; ++q) {
         const float4 u = *reinterpret_cast<const float4*>(
             scratch + ((static_cast<size_t>(q) * R + r_tile) * kPairBM + r) * BN + col);
@@ -231,36 +229,90 @@ __global__ void __launch_bounds__(kFixupThreads)
         s4[2] += u.z;
         s4[3] += u.w;
     }
-    const float a = alpha ? alpha[row] : 1.f;
-    const float bb = alpha ? beta[row] : 0.f;
+    return true;
+}
+
+// Plain fp32 sums, as EpiStoreF32 writes whole tiles (the projection g = E W_U).
+template <int BN>
+__global__ void __launch_bounds__(kFixupThreads)
+    sk_fixup_kernel(const GemmShape sh, const float* __restrict__ scratch, float* __restrict__ C) {
+    int row, n;
+    float s4[4];
+    if (!sk_tail_sum<BN>(sh, scratch, row, n, s4)) return;
+    *reinterpret_cast<float4*>(C + static_cast<size_t>(row) * sh.N + n) =
+        make_float4(s4[0], s4[1], s4[2], s4[3]);
+}
+
+// The direct algorithm's projection with the final-norm VJP fused in, as EpiProjVjp
+// writes whole tiles: g = alpha sum + beta W_U[y], out = bf16 of
+// (w g - (h / rho) cv / d) / max(rho, min_rms).
+struct VjpArgs {
+    const float* alpha;
+    const float* beta;
+    const float* cv;
+    const float* rho;
+    const int* y;
+    const __nv_bfloat16* W_U;
+    const __nv_bfloat16* h;
+    const __nv_bfloat16* w;
+    float min_rms, inv_d;
+};
+
+template <int BN>
+__global__ void __launch_bounds__(kFixupThreads)
+    sk_fixup_vjp_kernel(const GemmShape sh, const float* __restrict__ scratch,
+                        __nv_bfloat16* __restrict__ out, const VjpArgs va) {
+    int row, n;
+    float s4[4];
+    if (!sk_tail_sum<BN>(sh, scratch, row, n, s4)) return;
+    const float a = va.alpha[row], bb = va.beta[row];
+    const float rr = va.rho[row];
+    const float inv_r = 1.0f / rr;
+    const float kd = va.cv[row] * va.inv_d;
+    const float pref = 1.0f / fmaxf(rr, va.min_rms);
     const __nv_bfloat16* wy =
-        (a != 0.f && bb != 0.f) ? W_U + static_cast<long long>(y[row]) * sh.N : nullptr;
+        (a != 0.f && bb != 0.f) ? va.W_U + static_cast<long long>(va.y[row]) * sh.N : nullptr;
+    const __nv_bfloat16* hr = va.h + static_cast<long long>(row) * sh.N;
     float o[4];
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
-        if (a == 0.f)
-            o[j] = 0.f;
-        else if (wy)
-            o[j] = fmaf(a, s4[j], bb * __bfloat162float(wy[n + j]));
-        else
-            o[j] = a * s4[j];
+        const float yv = wy ? __bfloat162float(wy[n + j]) : 0.f;
+        const float gv = a == 0.f ? 0.f : fmaf(a, s4[j], bb * yv);
+        o[j] = (__bfloat162float(va.w[n + j]) * gv - (__bfloat162float(hr[n + j]) * inv_r) * kd) *
+               pref;
     }
-    *reinterpret_cast<float4*>(C + static_cast<size_t>(row) * sh.N + n) =
-        make_float4(o[0], o[1], o[2], o[3]);
+    *reinterpret_cast<uint2*>(out + static_cast<size_t>(row) * sh.N + n) =
+        make_uint2(pack_bf16x2(o[0], o[1]), pack_bf16x2(o[2], o[3]));
 }
 
 template <int BN>
-cudaError_t launch_sk_fixup(const SkPlan& plan, const GemmShape& sh_in, const float* scratch,
-                            float* C, const float* alpha, const float* beta, const int* y,
-                            const void* W_U, cudaStream_t st) {
-    if (plan.tail_tiles <= 0) return cudaSuccess;
+dim3 sk_fixup_grid(const SkPlan& plan) {
+    constexpr int kRowsPerBlock = kFixupThreads / (BN / 4);
+    return dim3(static_cast<unsigned>(plan.tail_tiles), kPairBM / kRowsPerBlock);
+}
+
+GemmShape sk_fixup_shape(const SkPlan& plan, const GemmShape& sh_in) {
     GemmShape sh = sh_in;
     sh.tail_tiles = plan.tail_tiles;
     sh.tail_split = plan.tail_split;
-    constexpr int kRowsPerBlock = kFixupThreads / (BN / 4);
-    const dim3 grid(static_cast<unsigned>(plan.tail_tiles), kPairBM / kRowsPerBlock);
-    sk_fixup_kernel<BN><<<grid, kFixupThreads, 0, st>>>(sh, scratch, C, alpha, beta, y,
-                                                        static_cast<const __nv_bfloat16*>(W_U)),
+    return sh;
+}
+
+template <int BN>
+cudaError_t launch_sk_fixup(const SkPlan& plan, const GemmShape& sh, const float* scratch,
+                            float* C, cudaStream_t st) {
+    if (plan.tail_tiles <= 0) return cudaSuccess;
+    sk_fixup_kernel<BN><<<sk_fixup_grid<BN>(plan), kFixupThreads, 0, st>>>(
+        sk_fixup_shape(plan, sh), scratch, C), ::fpo::note_launch();
+    return cudaGetLastError();
+}
+
+template <int BN>
+cudaError_t launch_sk_fixup_vjp(const SkPlan& plan, const GemmShape& sh, const float* scratch,
+                                void* out, const VjpArgs& va, cudaStream_t st) {
+    if (plan.tail_tiles <= 0) return cudaSuccess;
+    sk_fixup_vjp_kernel<BN><<<sk_fixup_grid<BN>(plan), kFixupThreads, 0, st>>>(
+        sk_fixup_shape(plan, sh), scratch, static_cast<__nv_bfloat16*>(out), va),
         ::fpo::note_launch();
     return cudaGetLastError();
 }
@@ -303,7 +355,7 @@ size_t proj_sk_scratch_bytes() {
     // on this device, or an upper bound of 128 without one
     static const size_t bytes = [] {
         using L = GemmPairSmem<kWideBN, kWideStages>;
-        auto kern = tc_gemm_pair_kernel<kWideBN, false, true, kWideStages, 1, EpiProjDirect>;
+        auto kern = tc_gemm_pair_kernel<kWideBN, false, true, kWideStages, 1, EpiProjVjp>;
         DevInfo di;
         long long c = 128;
         if (current_device_info(&di) &&
@@ -379,45 +431,63 @@ cudaError_t launch_error_bf16(const void* yhat, const void* W_U, const int32_t* 
     return run_gemm<kLseBN, false, false, kLseStages, 1, EpiError>(maps, ep, sh, status, st);
 }
 
-cudaError_t launch_lse_prob_bf16(const void* yhat, const void* W_U, const int32_t* y,
-                                 const float* anchor, int T, int d, int V, float2* part, float* sx,
-                                 int part_ld, float* zy, void* P, unsigned* status,
-                                 cudaStream_t st) {
+cudaError_t launch_anchor_prob_bf16(const void* yhat, const void* W_U, const int32_t* y,
+                                    const float* anchor, int T, int d, int V, float* su, float* sx,
+                                    float* qz, int part_ld, void* P, unsigned* status,
+                                    cudaStream_t st) {
     const bool pair = use_pair();
     GemmMaps<1> maps;
     if (!map_kmajor(&maps.a[0], yhat, T, d, kBM) ||
         !map_kmajor(&maps.b[0], W_U, V, d, pair ? kLseBN / 2 : kLseBN))
         return cudaErrorInvalidValue;
-    EpiLseProb::Params ep;
+    EpiAnchorProb::Params ep;
     if (!map_out_bf16(&ep.pmap, P, T, V)) return cudaErrorInvalidValue;
-    ep.part = part;
+    ep.su = su;
     ep.sx = sx;
+    ep.qz = qz;
     ep.part_ld = part_ld;
-    ep.zy = zy;
     ep.y = y;
     ep.anchor = anchor;
     ep.M = T;
     ep.N = V;
     const GemmShape sh = make_shape(T, V, d, kLseBN, 1, band_for(pair), pair ? kPairBM : kBM);
     if (pair)
-        return run_gemm_pair<kLseBN, false, false, kPairStages, 1, EpiLseProb>(maps, ep, sh, status,
-                                                                               st);
-    return run_gemm<kLseBN, false, false, kLseStages, 1, EpiLseProb>(maps, ep, sh, status, st);
+        return run_gemm_pair<kLseBN, false, false, kPairStages, 1, EpiAnchorProb>(maps, ep, sh,
+                                                                                  status, st);
+    return run_gemm<kLseBN, false, false, kLseStages, 1, EpiAnchorProb>(maps, ep, sh, status, st);
 }
 
-// The same GEMM as the logits pass on the gathered rows outside the anchor window.
-// Always the pair kernel (the only one that reads its row count on the device): the
-// recomputed rows are identical whichever kernel variant the other GEMMs use.
+// The fixup passes: the same GEMM as the logits pass on the gathered rows outside the
+// anchor window.  Always the pair kernel (the only one that reads its row count on the
+// device): the recomputed rows are identical whichever kernel variant the other GEMMs use.
+cudaError_t launch_fixup_lse_bf16(const void* yfix, const void* W_U, const int* fix,
+                                  const int* fix_count, int Tc, int d, int V, float2* part,
+                                  int part_ld, unsigned* status, cudaStream_t st) {
+    GemmMaps<1> maps;
+    if (!map_kmajor(&maps.a[0], yfix, Tc, d, kBM) || !map_kmajor(&maps.b[0], W_U, V, d, kLseBN / 2))
+        return cudaErrorInvalidValue;
+    EpiFixLse::Params ep;
+    ep.part = part;
+    ep.part_ld = part_ld;
+    ep.fix = fix;
+    ep.count = fix_count;
+    ep.N = V;
+    GemmShape sh = make_shape(Tc, V, d, kLseBN, 1, band_for(true), kPairBM);
+    sh.m_dev = fix_count;
+    return run_gemm_pair<kLseBN, false, false, kPairStages, 1, EpiFixLse>(maps, ep, sh, status, st);
+}
+
 cudaError_t launch_fixup_logits_bf16(const void* yfix, const void* W_U, const int* fix,
                                      const int* fix_count, const int32_t* y, const float* lse,
-                                     int Tc, int d, int V, void* P, float* sx, int n_tiles,
-                                     unsigned* status, cudaStream_t st) {
+                                     int Tc, int d, int V, void* P, float* sx, float* qz,
+                                     int n_tiles, unsigned* status, cudaStream_t st) {
     GemmMaps<1> maps;
     if (!map_kmajor(&maps.a[0], yfix, Tc, d, kBM) || !map_kmajor(&maps.b[0], W_U, V, d, kLseBN / 2))
         return cudaErrorInvalidValue;
     EpiFixProb::Params ep;
     ep.P = static_cast<__nv_bfloat16*>(P);
     ep.sx = sx;
+    ep.qz = qz;
     ep.fix = fix;
     ep.count = fix_count;
     ep.y = y;
@@ -432,33 +502,43 @@ cudaError_t launch_fixup_logits_bf16(const void* yfix, const void* W_U, const in
 constexpr int kProjBN = 256;
 constexpr int kProjStages = 4;
 
-cudaError_t launch_proj_direct_bf16(const void* P, const void* W_U, const int32_t* y,
-                                    const float* alpha, const float* beta, int Tc, int d, int V,
-                                    float* g, float* sk_scratch, unsigned* status,
-                                    cudaStream_t st) {
+cudaError_t launch_proj_vjp_bf16(const void* P, const void* W_U, const int32_t* y,
+                                 const float* alpha, const float* beta, const float* cv,
+                                 const float* rho, const void* h, const void* w, float min_rms,
+                                 int Tc, int d, int V, void* g_tilde, float* sk_scratch,
+                                 unsigned* status, cudaStream_t st) {
     GemmMaps<1> maps;
     if (!map_kmajor(&maps.a[0], P, Tc, V, kBM) || !map_mnmajor(&maps.b[0], W_U, V, d))
         return cudaErrorInvalidValue;
-    EpiProjDirect::Params ep;
-    if (!map_out_f32(&ep.Cmap, g, Tc, d)) return cudaErrorInvalidValue;
-    ep.alpha = alpha;
-    ep.beta = beta;
-    ep.y = y;
-    ep.W_U = static_cast<const __nv_bfloat16*>(W_U);
+    EpiProjVjp::Params ep;
+    if (!map_out_bf16(&ep.omap, g_tilde, Tc, d)) return cudaErrorInvalidValue;
+    VjpArgs va;
+    va.alpha = ep.alpha = alpha;
+    va.beta = ep.beta = beta;
+    va.cv = ep.cv = cv;
+    va.rho = ep.rho = rho;
+    va.y = ep.y = y;
+    va.W_U = ep.W_U = static_cast<const __nv_bfloat16*>(W_U);
+    va.h = ep.h = static_cast<const __nv_bfloat16*>(h);
+    va.w = ep.w = static_cast<const __nv_bfloat16*>(w);
+    va.min_rms = ep.min_rms = min_rms;
+    va.inv_d = ep.inv_d = 1.0f / static_cast<float>(d);
     ep.M = Tc;
     ep.N = d;
     if (wide_proj()) {
+        ep.tile_n = kWideBN;
         const GemmShape sh = make_shape(Tc, d, V, kWideBN, 1, band_for(true), kPairBM);
         SkPlan plan;
-        cudaError_t e = run_gemm_pair<kWideBN, false, true, kWideStages, 1, EpiProjDirect>(
+        cudaError_t e = run_gemm_pair<kWideBN, false, true, kWideStages, 1, EpiProjVjp>(
             maps, ep, sh, status, st, sk_scratch, &plan);
         if (e != cudaSuccess) return e;
-        return launch_sk_fixup<kWideBN>(plan, sh, sk_scratch, g, alpha, beta, y, W_U, st);
+        return launch_sk_fixup_vjp<kWideBN>(plan, sh, sk_scratch, g_tilde, va, st);
     }
+    ep.tile_n = kProjBN;
     if (use_pair())
-        return run_gemm_pair<kProjBN, false, true, kPairStages, 1, EpiProjDirect>(
+        return run_gemm_pair<kProjBN, false, true, kPairStages, 1, EpiProjVjp>(
             maps, ep, make_shape(Tc, d, V, kProjBN, 1, band_for(true), kPairBM), status, st);
-    return run_gemm<kProjBN, false, true, kProjStages, 1, EpiProjDirect>(
+    return run_gemm<kProjBN, false, true, kProjStages, 1, EpiProjVjp>(
         maps, ep, make_shape(Tc, d, V, kProjBN, 1, band_for(false)), status, st);
 }
 
@@ -477,8 +557,7 @@ cudaError_t launch_proj_bf16(const void* E, const void* W_U, int Tc, int d, int 
         cudaError_t e = run_gemm_pair<kWideBN, false, true, kWideStages, 1, EpiStoreF32>(
             maps, ep, sh, status, st, sk_scratch, &plan);
         if (e != cudaSuccess) return e;
-        return launch_sk_fixup<kWideBN>(plan, sh, sk_scratch, g, nullptr, nullptr, nullptr,
-                                        nullptr, st);
+        return launch_sk_fixup<kWideBN>(plan, sh, sk_scratch, g, st);
     }
     if (use_pair())
         return run_gemm_pair<kProjBN, false, true, kPairStages, 1, EpiStoreF32>(

@@ -46,26 +46,34 @@ cudaError_t launch_proj_bf16(const void* E, const void* W_U, int Tc, int d, int 
                              float* sk_scratch, unsigned* status, cudaStream_t st);
 size_t proj_sk_scratch_bytes();
 
-// Direct algorithm, logits pass: as launch_lse_partial_bf16 (z never stored), plus
-// P[T, V] = exp(z - anchor) in bf16 with the target column zero, and sx[T, part_ld]
-// the per-tile sums of the rounded P.
-cudaError_t launch_lse_prob_bf16(const void* yhat, const void* W_U, const int32_t* y,
-                                 const float* anchor, int T, int d, int V, float2* part, float* sx,
-                                 int part_ld, float* zy, void* P, unsigned* status,
-                                 cudaStream_t st);
-// Direct algorithm, rows outside the anchor window: the logits of the gathered rows
-// yfix[*fix_count, d] (capacity Tc rows) on the tensor cores; P[fix[i], :] = exp(z - lse)
-// in bf16 with the target column zero, sx[fix[i], tile] the per-tile sums of the rounded
-// values.  The row count is read on the device (none: the kernel returns at once).
+// Direct algorithm, logits pass anchored at c = anchor[t] (z never stored):
+// P[T, V] = exp(z - c) in bf16 with the target column zero, and per (row, 256-column
+// tile) the sums of P before rounding, su[T, part_ld], of the rounded P, sx[T, part_ld],
+// and of the rounded P times z, qz[T, part_ld].
+cudaError_t launch_anchor_prob_bf16(const void* yhat, const void* W_U, const int32_t* y,
+                                    const float* anchor, int T, int d, int V, float* su, float* sx,
+                                    float* qz, int part_ld, void* P, unsigned* status,
+                                    cudaStream_t st);
+// Direct algorithm, rows outside the anchor window (yfix[*fix_count, d], the gathered
+// yhat rows, capacity Tc; the row count is read on the device, none: the kernels return
+// at once).  First pass: part[fix[i], tile] = (max, sum exp(z - max)) of every tile.
+cudaError_t launch_fixup_lse_bf16(const void* yfix, const void* W_U, const int* fix,
+                                  const int* fix_count, int Tc, int d, int V, float2* part,
+                                  int part_ld, unsigned* status, cudaStream_t st);
+// Second pass, once lse is known: P[fix[i], :] = exp(z - lse) in bf16 with the target
+// column zero, and the sx, qz sums of those rows as the logits pass leaves them.
 cudaError_t launch_fixup_logits_bf16(const void* yfix, const void* W_U, const int* fix,
                                      const int* fix_count, const int32_t* y, const float* lse,
-                                     int Tc, int d, int V, void* P, float* sx, int n_tiles,
-                                     unsigned* status, cudaStream_t st);
-// Direct algorithm, projection: g[Tc, d] = alpha (.) (P W_U) + beta (.) W_U[y] (row-wise).
-cudaError_t launch_proj_direct_bf16(const void* P, const void* W_U, const int32_t* y,
-                                    const float* alpha, const float* beta, int Tc, int d, int V,
-                                    float* g, float* sk_scratch, unsigned* status,
-                                    cudaStream_t st);
+                                     int Tc, int d, int V, void* P, float* sx, float* qz,
+                                     int n_tiles, unsigned* status, cudaStream_t st);
+// Direct algorithm, projection with the final-norm VJP fused in: per row
+// g = alpha (.) (P W_U) + beta (.) W_U[y] and g~[Tc, d] (bf16) =
+// (w (.) g - (h / rho) cv / d) / max(rho, min_rms).
+cudaError_t launch_proj_vjp_bf16(const void* P, const void* W_U, const int32_t* y,
+                                 const float* alpha, const float* beta, const float* cv,
+                                 const float* rho, const void* h, const void* w, float min_rms,
+                                 int Tc, int d, int V, void* g_tilde, float* sk_scratch,
+                                 unsigned* status, cudaStream_t st);
 
 // Grouped pseudogradient update over n layers, layer l with signal g[l] (host array).
 cudaError_t launch_update_bf16(int n, int T, int d, int d_ff, const void* const* g,
@@ -117,19 +125,28 @@ cudaError_t launch_rmsnorm_fwd(int dtype, const void* h, const void* w, int T, i
                                void* yhat, float* rho, const int32_t* y, int V, unsigned* status,
                                cudaStream_t st, const void* W_U = nullptr,
                                float* anchor = nullptr);
-// Direct algorithm (bf16): lse, ce, the projection's row factors alpha, beta, and the
-// rows outside the anchor window (fix[0 .. *fix_count), appended atomically).
-cudaError_t launch_direct_combine(const float2* part, const float* sx, int n_tiles, int T, int V,
-                                  const int32_t* y, const float* anchor, const float* zy, float s,
-                                  float* lse, float* ce, float* alpha, float* beta, int* fix,
+// Direct algorithm (bf16), per token of a chunk with S = sum su, S' = sum sx and
+// Qz = sum qz over the tiles: rows inside the anchor window get lse = c + log(1 + S),
+// ce = log(1 + S), the projection's row factors alpha = s / (1 + S), beta = -alpha S'
+// and the VJP's row term cv = alpha (Qz - c S'); the others are appended to
+// fix[0 .. *fix_count) (atomically).
+cudaError_t launch_direct_combine(const float* su, const float* sx, const float* qz, int n_tiles,
+                                  int T, int V,
+                                  const int32_t* y, const float* anchor, float s, float* lse,
+                                  float* ce, float* alpha, float* beta, float* cv, int* fix,
                                   int* fix_count, cudaStream_t st);
 // Rows outside the anchor window: out[i, :] = yhat[fix[i], :] for i < *fix_count (bf16,
-// d a multiple of 8), then (launch_fixup_logits_bf16) their P rows and sx partials
-// recomputed anchored at lse, then their row factors alpha = s, beta = -s S'.
+// d a multiple of 8); after the first fixup pass their lse and ce from the (max, sum)
+// partials; after the second their row factors alpha = s, beta = -s S' and
+// cv = s (Qz - c S').
 cudaError_t launch_gather_rows(const void* yhat, const int* fix, const int* fix_count, int d,
                                void* out, cudaStream_t st);
-cudaError_t launch_direct_fixup_factors(const float* sx, const int* fix, const int* fix_count,
-                                        int n_tiles, float s, float* alpha, float* beta,
+cudaError_t launch_direct_fixup_lse(const float2* part, const int* fix, const int* fix_count,
+                                    int n_tiles, const float* anchor, float* lse, float* ce,
+                                    cudaStream_t st);
+cudaError_t launch_direct_fixup_factors(const float* sx, const float* qz, const int* fix,
+                                        const int* fix_count, int n_tiles, const float* anchor,
+                                        float s, float* alpha, float* beta, float* cv,
                                         cudaStream_t st);
 cudaError_t launch_lse_combine(const float2* part, int n_tiles, int T, const float* zy,
                                float* lse, float* ce, cudaStream_t st);

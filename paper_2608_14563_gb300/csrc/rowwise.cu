@@ -458,57 +458,66 @@ __global__ void __launch_bounds__(kRowThreads)
     }
 }
 
-// Direct algorithm, per token: lse_t and ce_t as lse_combine, S'_t = sum of the
-// tiles' rounded p~ (fixed order), and the row factors of the projection
-//   alpha_t = s exp(c_t - lse_t),  beta_t = -alpha_t S'_t.
-// The anchor window: with c_t the target logit, p~ = exp(z - c_t) holds every
-// probability that matters as a normal bf16 number, and the projection's fp32
-// sums stay finite, while 2^-80 <= S'_t <= 2^80.  A row outside it (or with a
-// non-finite S'_t) gets alpha_t = beta_t = 0 here and is appended to `fix` for
-// direct_fixup; a row with an out-of-range target gets zeros and no fixup.
-constexpr float kWindowHi = 1.2089258196146292e24f;   // 2^80
-constexpr float kWindowLo = 8.271806125530277e-25f;  // 2^-80
+// Direct algorithm, per token: S_t = sum of the tiles' p~ = exp(z - c_t) (target
+// excluded), S'_t the same sum of the bf16-rounded p~ and Qz_t = sum of the rounded
+// p~ times z, in a fixed order (fp32; the cancelling difference Qz_t - c_t S'_t and
+// the factors in fp64).  The target's own term is exp(0) = 1, so
+//   lse_t = c_t + log(1 + S_t),  ce_t = log(1 + S_t),
+// and the row factors of the projection are
+//   alpha_t = s exp(c_t - lse_t) = s / (1 + S_t),  beta_t = -alpha_t S'_t,
+// with the final-norm VJP's row term cv_t = <yhat_t, g_t> = alpha_t (Qz_t - c_t S'_t).
+// The anchor window: with c_t the target logit, p~ holds every probability that
+// matters as a normal bf16 number, and the projection's fp32 sums stay finite, while
+// 2^-80 <= S'_t <= 2^80.  A row outside it (or with a non-finite S'_t) gets
+// alpha_t = beta_t = 0 here and is appended to `fix` for the fixup passes, which also
+// form its lse and ce; a row with an out-of-range target gets zeros and no fixup.
+constexpr double kWindowHi = 1.2089258196146292e24;   // 2^80
+constexpr double kWindowLo = 8.271806125530277e-25;  // 2^-80
 
 __global__ void __launch_bounds__(kRowThreads)
-    direct_combine_kernel(const float2* __restrict__ part, const float* __restrict__ sx,
-                          int n_tiles, int T, int V, const int32_t* __restrict__ y,
-                          const float* __restrict__ anchor, const float* __restrict__ zy, float s,
-                          float* __restrict__ lse, float* __restrict__ ce,
-                          float* __restrict__ alpha, float* __restrict__ beta,
+    direct_combine_kernel(const float* __restrict__ su, const float* __restrict__ sx,
+                          const float* __restrict__ qz, int n_tiles, int T, int V,
+                          const int32_t* __restrict__ y,
+                          const float* __restrict__ anchor, float s, float* __restrict__ lse,
+                          float* __restrict__ ce, float* __restrict__ alpha,
+                          float* __restrict__ beta, float* __restrict__ cv,
                           int* __restrict__ fix, int* __restrict__ fix_count) {
     const int lane = threadIdx.x & 31;
     const int wpb = blockDim.x >> 5;
     for (int row = blockIdx.x * wpb + (threadIdx.x >> 5); row < T; row += gridDim.x * wpb) {
-        const float2* pr = part + static_cast<size_t>(row) * n_tiles;
+        const float* ur = su + static_cast<size_t>(row) * n_tiles;
         const float* xr = sx + static_cast<size_t>(row) * n_tiles;
-        float m = -INFINITY;
-        for (int i = lane; i < n_tiles; i += 32) m = fmaxf(m, pr[i].x);
-        m = warp_max(m);
-        float e = 0.f, S = 0.f;
+        const float* qr = qz + static_cast<size_t>(row) * n_tiles;
+        float su_ = 0.f, sx_ = 0.f, q_ = 0.f;
         for (int i = lane; i < n_tiles; i += 32) {
-            const float2 p = pr[i];
-            if (p.y > 0.f) e += p.y * expf(p.x - m);
-            S += xr[i];
+            su_ += ur[i];
+            sx_ += xr[i];
+            q_ += qr[i];
         }
-        e = warp_sum(e);
-        S = warp_sum(S);
-        const float l = m + logf(e);
+        const double Su = warp_sum(su_), S = warp_sum(sx_), Q = warp_sum(q_);
         if (lane == 0) {
-            lse[row] = l;
-            if (ce) ce[row] = l - zy[row];
             const int t = y[row];
-            float a = 0.f, b = 0.f;
+            float a = 0.f, b = 0.f, c = 0.f;
             if (t >= 0 && t < V) {
                 const bool inside = S <= kWindowHi && (S >= kWindowLo || V == 1);
                 if (inside) {
-                    a = s * expf(anchor[row] - l);
-                    b = -a * S;
+                    const float c_t = anchor[row];
+                    const float l1p = log1pf(static_cast<float>(Su));
+                    lse[row] = c_t + l1p;
+                    if (ce) ce[row] = l1p;
+                    a = s / (1.0f + static_cast<float>(Su));
+                    b = -a * static_cast<float>(S);
+                    c = a * static_cast<float>(Q - static_cast<double>(c_t) * S);
                 } else {
                     fix[atomicAdd(fix_count, 1)] = row;
                 }
+            } else {
+                lse[row] = 0.f;
+                if (ce) ce[row] = 0.f;
             }
             alpha[row] = a;
             beta[row] = b;
+            cv[row] = c;
         }
     }
 }
@@ -527,23 +536,62 @@ __global__ void __launch_bounds__(kRowThreads)
     }
 }
 
-// Row factors of the fixed rows (anchored at lse: alpha = s, beta = -s S').
+// lse and ce of the rows outside the anchor window, from the (max, sum exp) partials of
+// the first fixup pass: lse = m + log sum_tiles s_i exp(m_i - m), ce = lse - c.
 __global__ void __launch_bounds__(kRowThreads)
-    direct_fixup_factors_kernel(const float* __restrict__ sx, const int* __restrict__ fix,
-                                const int* __restrict__ fix_count, int n_tiles, float s,
-                                float* __restrict__ alpha, float* __restrict__ beta) {
+    direct_fixup_lse_kernel(const float2* __restrict__ part, const int* __restrict__ fix,
+                            const int* __restrict__ fix_count, int n_tiles,
+                            const float* __restrict__ anchor, float* __restrict__ lse,
+                            float* __restrict__ ce) {
+    const int lane = threadIdx.x & 31;
+    const int wpb = blockDim.x >> 5;
+    const int n = *fix_count;
+    for (int i = blockIdx.x * wpb + (threadIdx.x >> 5); i < n; i += gridDim.x * wpb) {
+        const int row = fix[i];
+        const float2* pr = part + static_cast<size_t>(row) * n_tiles;
+        float m = -INFINITY;
+        for (int k = lane; k < n_tiles; k += 32) m = fmaxf(m, pr[k].x);
+        m = warp_max(m);
+        float e = 0.f;
+        for (int k = lane; k < n_tiles; k += 32) {
+            const float2 p = pr[k];
+            if (p.y > 0.f) e += p.y * expf(p.x - m);
+        }
+        e = warp_sum(e);
+        if (lane == 0) {
+            const float l = m + logf(e);
+            lse[row] = l;
+            if (ce) ce[row] = l - anchor[row];
+        }
+    }
+}
+
+// Row factors of the fixed rows (anchored at lse: alpha = s, beta = -s S', and the
+// VJP's row term cv = s (Qz - c S')).
+__global__ void __launch_bounds__(kRowThreads)
+    direct_fixup_factors_kernel(const float* __restrict__ sx, const float* __restrict__ qz,
+                                const int* __restrict__ fix, const int* __restrict__ fix_count,
+                                int n_tiles, const float* __restrict__ anchor, float s,
+                                float* __restrict__ alpha, float* __restrict__ beta,
+                                float* __restrict__ cv) {
     const int lane = threadIdx.x & 31;
     const int wpb = blockDim.x >> 5;
     const int n = *fix_count;
     for (int i = blockIdx.x * wpb + (threadIdx.x >> 5); i < n; i += gridDim.x * wpb) {
         const int row = fix[i];
         const float* xr = sx + static_cast<size_t>(row) * n_tiles;
-        float S = 0.f;
-        for (int k = lane; k < n_tiles; k += 32) S += xr[k];
-        S = warp_sum(S);
+        const float* qr = qz + static_cast<size_t>(row) * n_tiles;
+        float sx_ = 0.f, q_ = 0.f;
+        for (int k = lane; k < n_tiles; k += 32) {
+            sx_ += xr[k];
+            q_ += qr[k];
+        }
+        const double S = warp_sum(sx_), Q = warp_sum(q_);
         if (lane == 0) {
             alpha[row] = s;
-            beta[row] = -s * S;
+            beta[row] = static_cast<float>(-static_cast<double>(s) * S);
+            cv[row] = static_cast<float>(static_cast<double>(s) *
+                                         (Q - static_cast<double>(anchor[row]) * S));
         }
     }
 }
@@ -689,13 +737,13 @@ cudaError_t launch_rmsnorm_fwd(int dtype, const void* h, const void* w, int T, i
     return cudaGetLastError();
 }
 
-cudaError_t launch_direct_combine(const float2* part, const float* sx, int n_tiles, int T, int V,
-                                  const int32_t* y, const float* anchor, const float* zy, float s,
-                                  float* lse, float* ce, float* alpha, float* beta, int* fix,
-                                  int* fix_count, cudaStream_t st) {
+cudaError_t launch_direct_combine(const float* su, const float* sx, const float* qz, int n_tiles,
+                                  int T, int V, const int32_t* y, const float* anchor, float s,
+                                  float* lse, float* ce, float* alpha, float* beta, float* cv,
+                                  int* fix, int* fix_count, cudaStream_t st) {
     if (T <= 0) return cudaSuccess;
     direct_combine_kernel<<<row_grid(T), kRowThreads, 0, st>>>(
-        part, sx, n_tiles, T, V, y, anchor, zy, s, lse, ce, alpha, beta, fix, fix_count),
+        su, sx, qz, n_tiles, T, V, y, anchor, s, lse, ce, alpha, beta, cv, fix, fix_count),
         ::fpo::note_launch();
     return cudaGetLastError();
 }
@@ -710,13 +758,25 @@ cudaError_t launch_gather_rows(const void* yhat, const int* fix, const int* fix_
     return cudaGetLastError();
 }
 
-cudaError_t launch_direct_fixup_factors(const float* sx, const int* fix, const int* fix_count,
-                                        int n_tiles, float s, float* alpha, float* beta,
+cudaError_t launch_direct_fixup_lse(const float2* part, const int* fix, const int* fix_count,
+                                    int n_tiles, const float* anchor, float* lse, float* ce,
+                                    cudaStream_t st) {
+    DevInfo di;
+    const int sms = current_device_info(&di) ? di.sm_count : 148;
+    direct_fixup_lse_kernel<<<sms, kRowThreads, 0, st>>>(part, fix, fix_count, n_tiles, anchor,
+                                                        lse, ce), ::fpo::note_launch();
+    return cudaGetLastError();
+}
+
+cudaError_t launch_direct_fixup_factors(const float* sx, const float* qz, const int* fix,
+                                        const int* fix_count, int n_tiles, const float* anchor,
+                                        float s, float* alpha, float* beta, float* cv,
                                         cudaStream_t st) {
     DevInfo di;
     const int sms = current_device_info(&di) ? di.sm_count : 148;
-    direct_fixup_factors_kernel<<<sms, kRowThreads, 0, st>>>(sx, fix, fix_count, n_tiles, s, alpha,
-                                                            beta), ::fpo::note_launch();
+    direct_fixup_factors_kernel<<<sms, kRowThreads, 0, st>>>(sx, qz, fix, fix_count, n_tiles,
+                                                            anchor, s, alpha, beta, cv),
+        ::fpo::note_launch();
     return cudaGetLastError();
 }
 

@@ -107,7 +107,9 @@ def test_direct_agrees_with_stored_logits(fpo, ragged):
     a = run(fpo, inp["h"], inp["w"], inp["W_U"], inp["y"], eps=RAGGED.eps, algo=fpo.ES_DIRECT)
     b = run(fpo, inp["h"], inp["w"], inp["W_U"], inp["y"], eps=RAGGED.eps,
             algo=fpo.ES_STORED_LOGITS)
-    assert torch.equal(a["lse"], b["lse"])  # same logits pass partials
+    # the direct algorithm takes lse = c + log(1 + S') from its bf16-rounded
+    # probabilities (S' off by at most 2^-9 relative), stored logits from fp32 sums
+    assert torch.max(torch.abs(a["lse"] - b["lse"])).item() < 2.0 ** -9
     assert rel_frob(f64(a["g"]), f64(b["g"])) < 1e-2
 
 
