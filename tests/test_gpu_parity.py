@@ -187,6 +187,42 @@ def test_min_rms_clamp_on_device(fpo):
     check(gpu, ref, inp, wl.lr, F32_TOL)
 
 
+def test_min_rms_clamp_in_the_fused_projection_epilogue(fpo):
+    """bf16, direct algorithm: the final-norm VJP runs in the projection's epilogue (and in
+    its split-tail fixup); tokens with rho ~ 0.2 < min_rms take the clamped prefactor
+    while x^ keeps the true rho, as the oracle defines it.  T = 4096, d = 4096: one chunk
+    has 128 projection tiles of 256 x 512, 1.7 waves of pair clusters, so its last wave is
+    split and the tail goes through the fixup kernel; chunks of 256 tokens have whole
+    tiles only."""
+    wl = Workload("clamp-bf16", T=4096, d=4096, d_ff=136, V=1032, layers=1, lr=1e-2)
+    inp = synth.make_all(wl)
+    inp["h"] = inp["h"].float()
+    inp["h"][::3] *= 0.2
+    inp["h"] = inp["h"].to(torch.bfloat16)
+    ref = oracle_step(wl, inp)
+    for t_chunk in (0, 256):
+        gpu = gpu_step(fpo, wl, inp, t_chunk=t_chunk)
+        check(gpu, ref, inp, wl.lr, BF16_TOL, BF16_COS)
+        g, G = f64(gpu["g"]), ref["g"]
+        rows = np.arange(0, wl.T, 3)  # every clamped token on its own
+        for t in rows:
+            assert rel_frob(g[t], G[t]) < BF16_TOL and cos(g[t], G[t]) >= BF16_COS, t
+
+
+def test_eps0_orthogonality_through_the_fused_vjp(fpo):
+    """bf16, direct algorithm, eps = 0: <g~_t, h_t> = 0 for every token up to the bf16
+    rounding of g~ (a relative size of ~2^-9 / sqrt(d)), with the VJP's row term taken
+    through the logits in the projection's epilogue."""
+    wl = Workload("eps0-bf16", T=300, d=1024, d_ff=64, V=4104, layers=1, eps=0.0)
+    inp = synth.make_all(wl)
+    gpu = gpu_step(fpo, wl, inp)
+    g, h = f64(gpu["g"]), f64(inp["h"])
+    rel = np.abs(np.sum(g * h, axis=1)) / (np.linalg.norm(g, axis=1) * np.linalg.norm(h, axis=1))
+    assert np.max(rel) < 1e-3
+    ref = oracle_step(wl, inp)
+    assert rel_frob(g, ref["g"]) < BF16_TOL
+
+
 def test_eps0_vjp_orthogonal_to_h_on_device(fpo):
     wl = Workload("eps0", T=96, d=256, d_ff=64, V=512, layers=1, dtype="f32", eps=0.0)
     inp = synth.make_all(wl)

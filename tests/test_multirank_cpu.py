@@ -99,6 +99,33 @@ def test_reference_arm_prints_the_contract_line():
     assert n == min(128, 4 * d["cpu_baseline"]["cores"])
 
 
+def test_reference_arm_loads_no_product_code():
+    """The oracle arm loads the oracle's library and nothing of the CUDA path: its inputs
+    come from synth.py, which sits outside the library package, and it never builds or
+    imports the binding (so libfpo.so is not mapped into the process)."""
+    import json
+    import subprocess
+    import sys
+    code = (
+        "import json, runpy, sys\n"
+        "sys.argv = ['bench.py', '--impl', 'reference', '--workload', 'tiny', '--steps', '1',"
+        " '--warmup', '3']\n"
+        "runpy.run_path('bench.py', run_name='__main__')\n"
+        "maps = open('/proc/self/maps').read().splitlines()\n"
+        "libs = sorted({l.split()[-1].rsplit('/', 1)[-1] for l in maps"
+        " if l.endswith('.so') and ('libfpo' in l or 'liboracle' in l)})\n"
+        "print('LOADED ' + json.dumps({'libs': libs, 'binding':"
+        " 'paper_2608_14563_gb300' in sys.modules}))\n")
+    out = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, timeout=300,
+                         cwd=ROOT)
+    assert out.returncode == 0, out.stderr[-2000:]
+    line = [l for l in out.stdout.splitlines() if l.startswith("LOADED ")][0]
+    d = json.loads(line[len("LOADED "):])
+    assert d == {"libs": ["liboracle.so"], "binding": False}, d
+    ref = json.loads([l for l in out.stdout.splitlines() if l.startswith("{")][0])
+    assert ref["ms_per_step_kind"] == "extrapolated" and "extrapolated" in ref["timing"]
+
+
 def test_bench_rejects_fewer_than_three_warmups():
     import subprocess
     import sys
