@@ -395,6 +395,14 @@ def run_fpo(args, wl):
         ws_cos = torch.empty(fpo.cosine_grouped_workspace(wl.layers, n_el), dtype=torch.uint8,
                              device=dev)
         Go_flat = [x.view(-1) for x in Go]
+    # the diagnostic's step (G_l only, no master to move) forms the cosines in the update
+    # GEMM's epilogue, so G_l is not read back, unless asked to run the two calls
+    fused_cos = (cosine and wl.lr == 0.0 and not (post or optimize or ratio or gate_up)
+                 and not args.cosine_separate)
+    if fused_cos:
+        G_true_2d = [x.view(wl.d, wl.d_ff) for x in G_true]
+        ws_gc = torch.empty(fpo.layer_grad_cosine_workspace(wl.layers, wl.d, wl.d_ff),
+                            dtype=torch.uint8, device=dev)
 
     def update(X):
         signals = g_l if post else [g] * wl.layers
@@ -405,6 +413,9 @@ def run_fpo(args, wl):
         elif post:
             fpo.layer_update_grouped_signals(g_l, X["A"], wl.lr, W_masters=Wm, W_outs=Wo,
                                              G_outs=G_outs, workspace=ws_up)
+        elif fused_cos:
+            # the diagnostic's step: G_l and its cosine against the true gradient
+            fpo.layer_grad_cosine_grouped(g, X["A"], G_true_2d, Go, out=cos_out, workspace=ws_gc)
         elif wl.lr == 0.0 and G_outs is not None:
             # the diagnostic's step: G_l only (no master to move at lr = 0)
             fpo.layer_update_grouped(g, X["A"], 0.0, G_outs=G_outs, workspace=ws_up)
@@ -452,14 +463,17 @@ def run_fpo(args, wl):
         if cosine:
             if upd_events:
                 upd_events[6].record(stream)
-            fpo.cosine_grouped(Go_flat, G_true, out=cos_out, workspace=ws_cos)
+            if not fused_cos:  # (fused: already formed by the update's epilogue)
+                fpo.cosine_grouped(Go_flat, G_true, out=cos_out, workspace=ws_cos)
             if upd_events:
                 upd_events[7].record(stream)
 
     for _ in range(args.warmup):
         step(X0)
     torch.cuda.synchronize()
-    assert fpo.get_device_status(ws_es) == fpo.OK and fpo.get_device_status(ws_up) == fpo.OK
+    ws_up_status = ws_gc if fused_cos else ws_up  # the update call's own status word
+    assert (fpo.get_device_status(ws_es) == fpo.OK
+            and fpo.get_device_status(ws_up_status) == fpo.OK)
 
     # per-stage events of every token chunk, for every timed step (recorded once so their
     # handles exist): 0 start, 1 after the RMSNorm forward, per chunk c the ends of its
@@ -490,7 +504,7 @@ def run_fpo(args, wl):
     if world > 1:
         dist.barrier()
     ms = start.elapsed_time(end) / args.steps
-    status = (fpo.get_device_status(ws_es), fpo.get_device_status(ws_up))
+    status = (fpo.get_device_status(ws_es), fpo.get_device_status(ws_up_status))
     # rows of the last step's last token chunk that the direct algorithm recomputed
     # outside its anchor window
     fixup_rows = (fpo.direct_fixup_rows(X0["h"], W_U, ws_es, t_chunk=args.t_chunk, algo=algo)
@@ -712,8 +726,13 @@ def run_fpo(args, wl):
             "kernels_gbs": {**({"norm_ratio": wl.layers * wl.d * wl.d_ff * (2 + 4)
                                 / (stage_ms["norm_ratio"] / 1e3) / 1e9} if ratio else {}),
                             **({"cosine": wl.layers * wl.d * wl.d_ff * (2 + 2)
-                                / (stage_ms["cosine"] / 1e3) / 1e9} if cosine else {})},
+                                / (stage_ms["cosine"] / 1e3) / 1e9}
+                               if cosine and not fused_cos else {})},
             "cosine": cos_out[:, 3].tolist() if cosine else None,
+            "cosine_mode": (None if not cosine else
+                            "fused: fpo_layer_grad_cosine_grouped forms the sums in the update "
+                            "GEMM's epilogue (the cosine stage is empty)" if fused_cos else
+                            "separate: fpo_cosine_grouped reads G_l and G~_l after the update"),
             "norm_ratio": ({"ratio": ratio_out[:, 2].tolist(),
                             "implied_sgd_lr_1pct": ratio_out[:, 3].tolist()} if ratio else None),
             "algo": algo_name,
@@ -811,6 +830,9 @@ def main():
     ap.add_argument("--cosine", action="store_true",
                     help="add the Sec. 2.2 diagnostic cosine of every layer's G_l to each step "
                          "(always on for the diag workload)")
+    ap.add_argument("--cosine-separate", action="store_true",
+                    help="diag workload: G_l by the grouped update, then fpo_cosine_grouped "
+                         "(two calls) instead of fpo_layer_grad_cosine_grouped")
     ap.add_argument("--norm-ratio", action="store_true",
                     help="add the App. C update-magnitude ratio ||G_l||/||W_l|| to every step")
     ap.add_argument("--e2e-depth", type=int, default=6,

@@ -410,6 +410,32 @@ int32_t fpo_cosine_grouped(int32_t n_layers, int64_t n, int32_t dtype, const voi
                            const void* const* Y, double* out, void* workspace,
                            size_t workspace_bytes, void* stream);
 
+/* Bytes of workspace fpo_layer_grad_cosine_grouped needs (0 on invalid sizes). */
+size_t fpo_layer_grad_cosine_workspace(int32_t n_layers, int64_t d, int64_t d_ff);
+
+/*
+ * fpo_layer_grad_cosine_grouped -- the layer-viability diagnostic in one grouped GEMM
+ * (Sec. 2.2, Eq. (cosine) over the pseudogradients of Eq. (w3update)): for every layer l
+ *   G_out[l] = g^T A_l                                   [d, d_ff] (dtype), as
+ *                                                        fpo_layer_update_grouped writes it
+ *   out[4 l + {0,1,2,3}] = <G_l, Y_l>, ||G_l||^2, ||Y_l||^2, cos_l   of the stored G_l
+ *                                                        (cos = 0 if a norm is 0)
+ * with Y_l [d, d_ff] (dtype) the gradient G_l is compared with.  bf16: the GEMM's
+ * epilogue adds up the three sums as it writes G_l (per tile and warp, in fp32 over a
+ * warp's 32 x 256 block, then in fp64 in a fixed order), so G_l is not read back; fp32:
+ * the update writes G_l and fpo_cosine_grouped reduces it.
+ * g [T, d], A_l [T, d_ff] (dtype); 1 <= n_layers <= FPO_MAX_GROUPED_LAYERS; pointers
+ * 16-byte aligned, out (device, 4 x n_layers fp64) 8-byte aligned; bf16 needs d and d_ff
+ * multiples of 8.  T = 0 gives G = 0 and cos 0.  workspace:
+ * fpo_layer_grad_cosine_workspace(n_layers, d, d_ff) bytes, 256-byte aligned (the device
+ * status word, then the partial sums).  Results are deterministic; they agree with
+ * fpo_layer_update_grouped + fpo_cosine_grouped bitwise on G and to rounding on the sums.
+ */
+int32_t fpo_layer_grad_cosine_grouped(int32_t n_layers, int64_t T, int64_t d, int64_t d_ff,
+                                      int32_t dtype, const void* g, const void* const* A,
+                                      const void* const* Y, void* const* G_out, double* out,
+                                      void* workspace, size_t workspace_bytes, void* stream);
+
 /* Bytes of workspace fpo_norm_ratio needs (0 for an invalid n_layers or n). */
 size_t fpo_norm_ratio_workspace(int32_t n_layers, int64_t n);
 

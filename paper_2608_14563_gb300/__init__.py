@@ -106,6 +106,12 @@ _lib.fpo_cosine_grouped_workspace.restype = _sz
 _lib.fpo_cosine_grouped.argtypes = [_i32, _i64, _i32, ctypes.POINTER(_vp), ctypes.POINTER(_vp),
                                     _vp, _vp, _sz, _vp]
 _lib.fpo_cosine_grouped.restype = _i32
+_lib.fpo_layer_grad_cosine_workspace.argtypes = [_i32, _i64, _i64]
+_lib.fpo_layer_grad_cosine_workspace.restype = _sz
+_lib.fpo_layer_grad_cosine_grouped.argtypes = [_i32, _i64, _i64, _i64, _i32, _vp,
+                                               ctypes.POINTER(_vp), ctypes.POINTER(_vp),
+                                               ctypes.POINTER(_vp), _vp, _vp, _sz, _vp]
+_lib.fpo_layer_grad_cosine_grouped.restype = _i32
 _lib.fpo_norm_ratio_workspace.argtypes = [_i32, _i64]
 _lib.fpo_norm_ratio_workspace.restype = _sz
 _lib.fpo_norm_ratio.argtypes = [_i32, _i64, _i32, ctypes.POINTER(_vp), _i32, ctypes.POINTER(_vp),
@@ -400,6 +406,30 @@ def cosine_grouped(X, Y, out=None, *, workspace=None, stream=None):
     rc = _lib.fpo_cosine_grouped(n_layers, n, _dtype_code(X[0]), xarr, yarr, _ptr(out),
                                  _ptr(workspace), _nbytes(workspace), _stream(stream))
     _check(rc, "fpo_cosine_grouped")
+    return out
+
+
+def layer_grad_cosine_workspace(n_layers: int, d: int, d_ff: int) -> int:
+    return int(_lib.fpo_layer_grad_cosine_workspace(int(n_layers), int(d), int(d_ff)))
+
+
+def layer_grad_cosine_grouped(g, As, Ys, G_outs, out=None, *, workspace=None, stream=None):
+    """fpo_layer_grad_cosine_grouped: G_outs[l] = g^T As[l] and, per layer,
+    [<G_l,Y_l>, |G_l|^2, |Y_l|^2, cos_l] as a device fp64 tensor [len(As), 4]."""
+    n = len(As)
+    if n == 0 or n != len(Ys) or n != len(G_outs):
+        raise ValueError("As, Ys and G_outs need one tensor per layer")
+    T, d = g.shape
+    d_ff = As[0].shape[1]
+    if out is None:
+        out = torch.empty(n, 4, dtype=torch.float64, device=g.device)
+    if workspace is None:
+        workspace = _workspace(layer_grad_cosine_workspace(n, d, d_ff), g.device)
+    arr = lambda ts: (_vp * n)(*[_ptr(t) for t in ts])  # noqa: E731
+    rc = _lib.fpo_layer_grad_cosine_grouped(n, T, d, d_ff, _dtype_code(g), _ptr(g), arr(As),
+                                            arr(Ys), arr(G_outs), _ptr(out), _ptr(workspace),
+                                            _nbytes(workspace), _stream(stream))
+    _check(rc, "fpo_layer_grad_cosine_grouped")
     return out
 
 

@@ -571,6 +571,97 @@ struct EpiUpdate {
 };
 
 // ---------------------------------------------------------------------------
+// Pseudogradients with the layer-viability diagnostic's cosine (Sec. 2.2 Eq. (cosine),
+// Eq. (w3update)): for group (layer) g, G_out[g] = bf16(G), and the three sums of the
+// cosine of that stored G against Y[g] (<G, Y>, ||G||^2, ||Y||^2) over the thread's
+// row of the tile, summed over the warp's 32 rows (a fixed butterfly) and written as one
+// triple per (layer, 256-row block, column tile, 32-row slot):
+//   part[(((g m256 + row / 256) n_blocks + nb) 8 + (row mod 256) / 32) 3 + {0, 1, 2}]
+// so the cosine needs no second pass over G.  The Y values of the next 32-column chunk
+// are loaded while the current one is processed.
+struct EpiGradCos {
+    struct Params {
+        __nv_bfloat16* G_out[kMaxGroups];
+        const __nv_bfloat16* Y[kMaxGroups];
+        float* part;     // [groups][m256][n_blocks][8][3]
+        long long ld;
+        int M, N;
+        int m256, n_blocks;
+    };
+    static constexpr int kTileN = 256;  // columns of the tiles it runs on (both GEMM kernels)
+    int row, g, n_end;
+    bool valid;
+    float2 s_gy, s_gg, s_yy;
+    uint4 uy[4];  // Y of the chunk the next chunk() call works on
+
+    __device__ __forceinline__ void fetch(const Params& p, int col0) {
+        const int lim = p.N - col0;
+        const uint4* py = reinterpret_cast<const uint4*>(p.Y[g] + row * p.ld + col0);
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+            uy[q] = (valid && q * 8 < lim) ? __ldg(py + q) : make_uint4(0, 0, 0, 0);
+    }
+
+    __device__ __forceinline__ EpiGradCos(const Params& p, int g_, int row_, int n0)
+        : row(row_), g(g_) {
+        valid = row_ < p.M;
+        n_end = n0 + kTileN;
+        s_gy = s_gg = s_yy = make_float2(0.f, 0.f);
+        if (n0 < p.N) fetch(p, n0);
+    }
+
+    __device__ __forceinline__ void chunk(const Params& p, const float (&v)[32], int col0, int,
+                                          EpiIO&) {
+        uint4 cy[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) cy[q] = uy[q];
+        if (col0 + 32 < n_end && col0 + 32 < p.N) fetch(p, col0 + 32);
+        const int lim = p.N - col0;
+        if (!valid || lim <= 0) return;
+        uint4* gp = reinterpret_cast<uint4*>(p.G_out[g] + row * p.ld + col0);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const uint32_t pk[4] = {pack_bf16x2(v[8 * q], v[8 * q + 1]),
+                                    pack_bf16x2(v[8 * q + 2], v[8 * q + 3]),
+                                    pack_bf16x2(v[8 * q + 4], v[8 * q + 5]),
+                                    pack_bf16x2(v[8 * q + 6], v[8 * q + 7])};
+            if (q * 8 < lim) gp[q] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+            // columns >= N: G is 0 there (zero-filled operand) and Y was loaded as 0
+            const uint32_t yk[4] = {cy[q].x, cy[q].y, cy[q].z, cy[q].w};
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const float2 gr = make_float2(__uint_as_float(pk[k] << 16),
+                                              __uint_as_float(pk[k] & 0xffff0000u));
+                const float2 yr = make_float2(__uint_as_float(yk[k] << 16),
+                                              __uint_as_float(yk[k] & 0xffff0000u));
+                s_gy = __ffma2_rn(gr, yr, s_gy);
+                s_gg = __ffma2_rn(gr, gr, s_gg);
+                s_yy = __ffma2_rn(yr, yr, s_yy);
+            }
+        }
+    }
+
+    __device__ __forceinline__ void finish(const Params& p, int nb) {
+        float gy = s_gy.x + s_gy.y, gg = s_gg.x + s_gg.y, yy = s_yy.x + s_yy.y;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            gy += __shfl_xor_sync(0xffffffffu, gy, o);
+            gg += __shfl_xor_sync(0xffffffffu, gg, o);
+            yy += __shfl_xor_sync(0xffffffffu, yy, o);
+        }
+        if ((threadIdx.x & 31) == 0) {
+            const long long slot =
+                ((static_cast<long long>(g) * p.m256 + row / 256) * p.n_blocks + nb) * 8 +
+                (row % 256) / 32;
+            float* o = p.part + slot * 3;
+            o[0] = gy;
+            o[1] = gg;
+            o[2] = yy;
+        }
+    }
+};
+
+// ---------------------------------------------------------------------------
 // Pseudogradient only, fp32, one output per group (layer): G[g] = g~^T A_l, for
 // the optimizers that need the whole G (and its norm) before they step.
 struct EpiStoreGroupF32 {

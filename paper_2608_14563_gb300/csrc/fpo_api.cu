@@ -444,6 +444,68 @@ int32_t fpo_layer_update_grouped(int32_t n_layers, int64_t T, int64_t d, int64_t
                                             W_out, G_out, workspace, workspace_bytes, stream);
 }
 
+size_t fpo_layer_grad_cosine_workspace(int32_t n_layers, int64_t d, int64_t d_ff) {
+    if (n_layers < 1 || n_layers > FPO_MAX_GROUPED_LAYERS || d <= 0 || d_ff <= 0 ||
+        d > INT_MAX || d_ff > INT_MAX)
+        return 0;
+    // bf16: the per-(tile, warp) triples of the fused epilogue; fp32: the partials of the
+    // separate grouped cosine (the larger of the two, so one size serves both)
+    const size_t fused = grad_cosine_partial_bytes(n_layers, static_cast<int>(d),
+                                                   static_cast<int>(d_ff));
+    const size_t sep = fpo_cosine_grouped_workspace(n_layers, d * d_ff);
+    return kStatusBytes + align_up(fused > sep ? fused : sep);
+}
+
+int32_t fpo_layer_grad_cosine_grouped(int32_t n_layers, int64_t T, int64_t d, int64_t d_ff,
+                                      int32_t dtype, const void* g, const void* const* A,
+                                      const void* const* Y, void* const* G_out, double* out,
+                                      void* workspace, size_t workspace_bytes, void* stream) {
+    if (dtype != FPO_F32 && dtype != FPO_BF16) return FPO_ERR_DTYPE;
+    if (n_layers < 1 || n_layers > FPO_MAX_GROUPED_LAYERS) return FPO_ERR_SHAPE;
+    if (T < 0 || d <= 0 || d_ff <= 0 || T > INT_MAX || d > INT_MAX || d_ff > INT_MAX)
+        return FPO_ERR_SHAPE;
+    if (dtype == FPO_BF16 && (d % 8 != 0 || d_ff % 8 != 0)) return FPO_ERR_SHAPE;
+    if (!A || !Y || !G_out || !out || (T > 0 && !g)) return FPO_ERR_NULL;
+    if (!aligned16(g) || (reinterpret_cast<uintptr_t>(out) & 7u)) return FPO_ERR_ALIGN;
+    for (int l = 0; l < n_layers; ++l) {
+        if ((T > 0 && !A[l]) || !Y[l] || !G_out[l]) return FPO_ERR_NULL;
+        if (!aligned16(A[l]) || !aligned16(Y[l]) || !aligned16(G_out[l])) return FPO_ERR_ALIGN;
+    }
+    if (!workspace || workspace_bytes < fpo_layer_grad_cosine_workspace(n_layers, d, d_ff))
+        return FPO_ERR_WORKSPACE;
+    if ((reinterpret_cast<uintptr_t>(workspace) % kAlign) != 0) return FPO_ERR_ALIGN;
+    int32_t rc = check_arch();
+    if (rc != FPO_OK) return rc;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    uint8_t* ws = static_cast<uint8_t*>(workspace);
+    unsigned* status = reinterpret_cast<unsigned*>(ws);
+    FPO_TRY(cudaMemsetAsync(status, 0, sizeof(unsigned), st));
+    const int Ti = static_cast<int>(T), di = static_cast<int>(d), fi = static_cast<int>(d_ff);
+    const size_t n = static_cast<size_t>(d) * static_cast<size_t>(d_ff);
+    if (T == 0) {
+        // G = 0: the cosine of every layer is 0, ||Y||^2 by the grouped reduction
+        for (int l = 0; l < n_layers; ++l)
+            FPO_TRY(cudaMemsetAsync(G_out[l], 0, n * (dtype == FPO_BF16 ? 2 : 4), st));
+        return cuda_status(launch_cosine_grouped(
+            dtype, n_layers, static_cast<int64_t>(n), const_cast<const void* const*>(G_out), Y,
+            reinterpret_cast<double*>(ws + kStatusBytes), norm_ratio_blocks(n_layers, n), out,
+            st));
+    }
+    const void* gs[FPO_MAX_GROUPED_LAYERS];
+    for (int l = 0; l < n_layers; ++l) gs[l] = g;
+    if (dtype == FPO_BF16)
+        return cuda_status(launch_grad_cosine_bf16(n_layers, Ti, di, fi, gs, A, Y, G_out,
+                                                   reinterpret_cast<float*>(ws + kStatusBytes),
+                                                   out, status, st));
+    // fp32: the SIMT update writes G, then the grouped cosine reads it back
+    FPO_TRY(launch_update_f32(n_layers, Ti, di, fi, reinterpret_cast<const float* const*>(gs),
+                              reinterpret_cast<const float* const*>(A), 0.f, nullptr, nullptr,
+                              reinterpret_cast<float* const*>(G_out), st));
+    return cuda_status(launch_cosine_grouped(
+        dtype, n_layers, static_cast<int64_t>(n), const_cast<const void* const*>(G_out), Y,
+        reinterpret_cast<double*>(ws + kStatusBytes), norm_ratio_blocks(n_layers, n), out, st));
+}
+
 size_t fpo_layer_optimize_workspace(int32_t n_layers, int64_t d, int64_t d_ff) {
     if (n_layers < 1 || n_layers > FPO_MAX_GROUPED_LAYERS || d <= 0 || d_ff <= 0) return 0;
     return kStatusBytes + align_up(static_cast<size_t>(n_layers) * static_cast<size_t>(d) *

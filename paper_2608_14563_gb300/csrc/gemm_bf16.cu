@@ -637,6 +637,87 @@ cudaError_t launch_grad_bf16(int n, int T, int d, int d_ff, const void* const* g
         maps, ep, make_shape(d, d_ff, T, kUpdBN, n, band_for(false)), status, st);
 }
 
+// The cosine of every layer from EpiGradCos's per-(tile, warp) triples: one warp per
+// layer adds its slots in a fixed order (lane-strided fp64 sums, then a fixed butterfly).
+__global__ void grad_cosine_final_kernel(const float* __restrict__ part, int slots,
+                                         double* __restrict__ out) {
+    const int layer = blockIdx.x;
+    const int lane = threadIdx.x;
+    const float* p = part + static_cast<size_t>(layer) * slots * 3;
+    double gy = 0.0, gg = 0.0, yy = 0.0;
+    for (int i = lane; i < slots; i += 32) {
+        gy += p[3 * i];
+        gg += p[3 * i + 1];
+        yy += p[3 * i + 2];
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        gy += __shfl_xor_sync(0xffffffffu, gy, o);
+        gg += __shfl_xor_sync(0xffffffffu, gg, o);
+        yy += __shfl_xor_sync(0xffffffffu, yy, o);
+    }
+    if (lane == 0) {
+        double* o = out + 4 * layer;
+        o[0] = gy;
+        o[1] = gg;
+        o[2] = yy;
+        o[3] = (gg > 0.0 && yy > 0.0) ? gy / (sqrt(gg) * sqrt(yy)) : 0.0;
+    }
+}
+
+size_t grad_cosine_partial_bytes(int n, int d, int d_ff) {
+    const size_t m256 = (static_cast<size_t>(d) + 255) / 256;
+    const size_t nb = (static_cast<size_t>(d_ff) + kUpdBN - 1) / kUpdBN;
+    return static_cast<size_t>(n) * m256 * nb * 8 * 3 * sizeof(float);
+}
+
+cudaError_t launch_grad_cosine_bf16(int n, int T, int d, int d_ff, const void* const* g,
+                                    const void* const* A, const void* const* Y,
+                                    void* const* G_out, float* part, double* out,
+                                    unsigned* status, cudaStream_t st) {
+    if (n < 1 || n > kMaxGroups) return cudaErrorInvalidValue;
+    static GemmMaps<kMaxGroups> maps;
+    static EpiGradCos::Params ep;
+    static std::mutex mu;
+    std::lock_guard<std::mutex> lock(mu);
+    for (int l = 0; l < n; ++l) {
+        if (l > 0 && g[l] == g[0])
+            maps.a[l] = maps.a[0];
+        else if (!map_mnmajor(&maps.a[l], g[l], T, d))
+            return cudaErrorInvalidValue;
+        if (!map_mnmajor(&maps.b[l], A[l], T, d_ff)) return cudaErrorInvalidValue;
+        ep.G_out[l] = static_cast<__nv_bfloat16*>(G_out[l]);
+        ep.Y[l] = static_cast<const __nv_bfloat16*>(Y[l]);
+    }
+    for (int l = n; l < kMaxGroups; ++l) {
+        maps.a[l] = maps.a[0];
+        maps.b[l] = maps.b[0];
+        ep.G_out[l] = ep.G_out[0];
+        ep.Y[l] = ep.Y[0];
+    }
+    ep.part = part;
+    ep.ld = d_ff;
+    ep.M = d;
+    ep.N = d_ff;
+    ep.m256 = (d + 255) / 256;
+    ep.n_blocks = (d_ff + kUpdBN - 1) / kUpdBN;
+    static_assert(EpiGradCos::kTileN == kUpdBN, "the cosine epilogue prefetches 256-column tiles");
+    // every slot is written by a tile (pair kernel), but single-CTA 128-row tiles leave
+    // the upper half of a last, short 256-row block unwritten: start from zeros
+    cudaError_t e = cudaMemsetAsync(part, 0, grad_cosine_partial_bytes(n, d, d_ff), st);
+    if (e != cudaSuccess) return e;
+    if (use_pair())
+        e = run_gemm_pair<kUpdBN, true, true, kPairStages, kMaxGroups, EpiGradCos>(
+            maps, ep, make_shape(d, d_ff, T, kUpdBN, n, band_for(true), kPairBM), status, st);
+    else
+        e = run_gemm<kUpdBN, true, true, kUpdStages, kMaxGroups, EpiGradCos>(
+            maps, ep, make_shape(d, d_ff, T, kUpdBN, n, band_for(false)), status, st);
+    if (e != cudaSuccess) return e;
+    grad_cosine_final_kernel<<<n, 32, 0, st>>>(part, ep.m256 * ep.n_blocks * 8, out),
+        ::fpo::note_launch();
+    return cudaGetLastError();
+}
+
 cudaError_t launch_swiglu_bf16(int T, int d, int d_ff, const void* g, const void* W3,
                                const void* a, const void* b, void* dA, void* dB, unsigned* status,
                                cudaStream_t st) {

@@ -86,6 +86,16 @@ cudaError_t launch_grad_bf16(int n, int T, int d, int d_ff, const void* const* g
                              const void* const* A, float* const* G_out, unsigned* status,
                              cudaStream_t st);
 
+// Grouped pseudogradients with the diagnostic's cosine: G_out[l] (bf16 [d, d_ff]) =
+// g[l]^T A[l], and out[4 l ..] = <G_l, Y_l>, ||G_l||^2, ||Y_l||^2, cos_l of the stored
+// G_l against Y[l] (bf16), from per-(tile, warp) partial sums in `part`
+// (grad_cosine_partial_bytes) without a second pass over G.
+size_t grad_cosine_partial_bytes(int n, int d, int d_ff);
+cudaError_t launch_grad_cosine_bf16(int n, int T, int d, int d_ff, const void* const* g,
+                                    const void* const* A, const void* const* Y,
+                                    void* const* G_out, float* part, double* out,
+                                    unsigned* status, cudaStream_t st);
+
 // SwiGLU gate / up signals: dA, dB [T, d_ff] from error_h = g W3 (W3 [d, d_ff]) and the
 // cached pre-activations a, b [T, d_ff].
 cudaError_t launch_swiglu_bf16(int T, int d, int d_ff, const void* g, const void* W3,

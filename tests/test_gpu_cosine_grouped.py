@@ -64,3 +64,64 @@ def test_cosine_grouped_diagnostic_closed_form(fpo):
         assert abs(out[l, 3] - 1.0 / math.sqrt(1.0 + sig[l] ** 2)) < 2e-3, l
     del G, Gt
     torch.cuda.empty_cache()
+
+
+def _grad_inputs(T, d, d_ff, L, dtype, seed=5):
+    gen = torch.Generator(device="cuda").manual_seed(seed)
+    g = (torch.randn(T, d, device="cuda", generator=gen) * 1e-2).to(dtype)
+    A = [torch.randn(T, d_ff, device="cuda", generator=gen).to(dtype) for _ in range(L)]
+    Y = [torch.randn(d, d_ff, device="cuda", generator=gen).to(dtype) for _ in range(L)]
+    return g, A, Y
+
+
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
+@pytest.mark.parametrize("shape", [(700, 320, 840, 3), (1024, 512, 768, 2), (300, 1032, 264, 4)])
+def test_layer_grad_cosine_matches_update_and_oracle(fpo, dtype, shape):
+    """The pseudogradients with the diagnostic's cosine in one GEMM (the sums formed in its
+    epilogue for bf16): G_l identical to the grouped update's, and each layer's sums and
+    cosine against the oracle's cosine of the same stored G_l and Y_l (ragged d, d_ff, T)."""
+    T, d, d_ff, L = shape
+    g, A, Y = _grad_inputs(T, d, d_ff, L, dtype)
+    G = [torch.full((d, d_ff), float("nan"), device="cuda").to(dtype) for _ in range(L)]
+    out = fpo.layer_grad_cosine_grouped(g, A, Y, G).cpu().numpy()
+    G_ref = [torch.empty(d, d_ff, device="cuda", dtype=dtype) for _ in range(L)]
+    ws = fpo.layer_update_grouped(g, A, 0.0, G_outs=G_ref)
+    assert fpo.get_device_status(ws) == fpo.OK
+    for l in range(L):
+        assert torch.equal(G[l], G_ref[l]), f"layer {l}"
+        ref = oracle.cosine(synth.to_numpy_exact(G[l].reshape(-1).cpu()),
+                            synth.to_numpy_exact(Y[l].reshape(-1).cpu()))
+        assert abs(out[l, 0] - ref[0]) <= 2e-5 * math.sqrt(ref[1] * ref[2]), l
+        assert abs(out[l, 1] - ref[1]) <= 2e-5 * ref[1] and abs(out[l, 2] - ref[2]) <= 2e-5 * ref[2]
+        assert abs(out[l, 3] - ref[3]) <= 2e-5, l
+    again = fpo.layer_grad_cosine_grouped(g, A, Y, G).cpu().numpy()
+    assert np.array_equal(out, again)  # deterministic
+
+
+def test_layer_grad_cosine_same_bits_under_every_kernel_variant(fpo):
+    """Single-CTA and CTA-pair tiles give the same per-(32-row x 256-column) partial sums,
+    so the cosines agree bit for bit, as G does."""
+    g, A, Y = _grad_inputs(640, 704, 520, 3, torch.bfloat16, seed=8)
+    outs = []
+    prev = fpo.set_gemm_variant(0)
+    try:
+        for v in (0, 1, 2):
+            fpo.set_gemm_variant(v)
+            G = [torch.empty(704, 520, device="cuda", dtype=torch.bfloat16) for _ in range(3)]
+            outs.append((fpo.layer_grad_cosine_grouped(g, A, Y, G).cpu(), G))
+    finally:
+        fpo.set_gemm_variant(prev)
+    for o, G in outs[1:]:
+        assert torch.equal(o, outs[0][0])
+        for a, b in zip(G, outs[0][1]):
+            assert torch.equal(a, b)
+
+
+def test_layer_grad_cosine_empty_tokens(fpo):
+    g, A, Y = _grad_inputs(0, 64, 128, 2, torch.bfloat16)
+    G = [torch.full((64, 128), 1.0, device="cuda").to(torch.bfloat16) for _ in range(2)]
+    out = fpo.layer_grad_cosine_grouped(g, A, Y, G).cpu().numpy()
+    for l in range(2):
+        assert torch.count_nonzero(G[l]).item() == 0
+        assert out[l, 0] == 0.0 and out[l, 1] == 0.0 and out[l, 3] == 0.0
+        assert out[l, 2] > 0.0

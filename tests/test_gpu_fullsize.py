@@ -17,7 +17,8 @@ GPU's own g~ feeding the GPU's own update as in a step.
   against the oracle on the GPU's g~; the cosine reduction of every layer against
   the oracle's cosine of the same bf16 G_l and synthetic 'true' gradient
   G_l + sigma_l |G_l| Z / sqrt(n), and against its closed-form expectation
-  1/sqrt(1 + sigma_l^2) (Sec. 2.2).
+  1/sqrt(1 + sigma_l^2) (Sec. 2.2); the same G_l and cosines from the one-GEMM form
+  (fpo_layer_grad_cosine_grouped) against those.
 """
 import math
 
@@ -160,22 +161,34 @@ def test_diagnostic_sweep_full_size(fpo):
         got_r, got_c = f64(G[l][ri]), f64(G[l][:, cj])
         assert rel_frob(got_r, G_rows) < TOL and cos(got_r, G_rows) >= COS_MIN, f"layer {l}"
         assert rel_frob(got_c, G_cols) < TOL and cos(got_c, G_cols) >= COS_MIN, f"layer {l}"
-    del A
-    _free()
 
+    G_true = []
     for l in range(L):
         sigma = 4.0 - 2.5 * l / (L - 1)
         Gf = G[l].float().reshape(-1)
         scale = sigma * torch.linalg.vector_norm(Gf).item() / math.sqrt(n)
         Z = synth.make_noise(n, seed=wl.seed, layer=l, device=dev)
-        G_true = (Gf + scale * Z).to(torch.bfloat16)
-        out = fpo.cosine(G[l].reshape(-1), G_true).cpu().numpy()
+        G_true.append((Gf + scale * Z).to(torch.bfloat16).view(wl.d, wl.d_ff))
+        del Gf, Z
+    # the same G_l with the cosines formed in the update GEMM's epilogue
+    G2 = [torch.empty(wl.d, wl.d_ff, dtype=torch.bfloat16, device=dev) for _ in range(L)]
+    fused = fpo.layer_grad_cosine_grouped(g, A, G_true, G2).cpu().numpy()
+    del A
+    _free()
+
+    for l in range(L):
+        sigma = 4.0 - 2.5 * l / (L - 1)
+        assert torch.equal(G2[l], G[l]), f"layer {l}"
+        out = fpo.cosine(G[l].reshape(-1), G_true[l].reshape(-1)).cpu().numpy()
+        for k in range(3):
+            assert abs(fused[l, k] - out[k]) <= 1e-5 * math.sqrt(out[1] * out[2]), (l, k)
+        assert abs(fused[l, 3] - out[3]) < 1e-5, f"layer {l}"
         assert abs(out[3] - 1.0 / math.sqrt(1.0 + sigma * sigma)) < 2e-3, f"layer {l}"
-        ref = oracle.cosine(synth.to_numpy_exact(G[l].reshape(-1)), synth.to_numpy_exact(G_true))
+        ref = oracle.cosine(synth.to_numpy_exact(G[l].reshape(-1)),
+                            synth.to_numpy_exact(G_true[l].reshape(-1)))
         assert abs(out[3] - ref[3]) < 1e-4, f"layer {l}"
         # fp32 runs of a few hundred elements per thread, fp64 after that
         assert abs(out[0] - ref[0]) <= 1e-5 * math.sqrt(ref[1] * ref[2]), f"layer {l}"
         assert abs(out[1] - ref[1]) <= 1e-5 * ref[1] and abs(out[2] - ref[2]) <= 1e-5 * ref[2]
-        del Gf, Z, G_true
-    del G, g, ws2
+    del G, G2, G_true, g, ws2
     _free()
