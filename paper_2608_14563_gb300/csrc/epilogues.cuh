@@ -407,7 +407,8 @@ struct EpiProjVjp {
         int M, N;
         int tile_n;                 // columns of the kernel's tiles (one epilogue object each)
     };
-    float a, b, inv_r, kd, pref;
+    float a;
+    float2 a2, b2, nk2;  // per row, twice: alpha pref, beta pref, -(cv / d) pref / rho
     const __nv_bfloat16* wy;
     const __nv_bfloat16* hr;
     bool valid, pair_out;
@@ -433,11 +434,15 @@ struct EpiProjVjp {
         : pair_out(false) {
         valid = row < p.M;
         a = valid ? __ldg(p.alpha + row) : 0.f;
-        b = valid ? __ldg(p.beta + row) : 0.f;
+        const float b = valid ? __ldg(p.beta + row) : 0.f;
         const float r = valid ? __ldg(p.rho + row) : 1.f;
-        inv_r = 1.0f / r;
-        kd = valid ? __ldg(p.cv + row) * p.inv_d : 0.f;
-        pref = 1.0f / fmaxf(r, p.min_rms);
+        const float kd = valid ? __ldg(p.cv + row) * p.inv_d : 0.f;
+        const float pref = 1.0f / fmaxf(r, p.min_rms);
+        // g~_j = w_j (a pref acc_j + b pref W_U[y]_j) - h_j (kd pref / rho)
+        a2 = make_float2(a * pref, a * pref);
+        b2 = make_float2(b * pref, b * pref);
+        const float nk = -(kd * (1.0f / r)) * pref;
+        nk2 = make_float2(nk, nk);
         wy = (a != 0.f && b != 0.f) ? p.W_U + static_cast<long long>(__ldg(p.y + row)) * p.N
                                     : nullptr;
         hr = p.h + static_cast<long long>(valid ? row : 0) * p.N;
@@ -459,24 +464,28 @@ struct EpiProjVjp {
         if (!second) pair_out = col0 >= p.N || io.row0 >= p.M;
         if (pair_out) return;
         uint32_t r[16];
+        if (a == 0.f) {  // s == 0 or an out-of-range target: g = 0 and cv = 0, so g~ = 0
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            const uint32_t hh[4] = {ch[q].x, ch[q].y, ch[q].z, ch[q].w};
-            const uint32_t ww[4] = {cw[q].x, cw[q].y, cw[q].z, cw[q].w};
-            const uint32_t yy[4] = {cy[q].x, cy[q].y, cy[q].z, cy[q].w};
+            for (int i = 0; i < 16; ++i) r[i] = 0u;
+        } else {
 #pragma unroll
-            for (int k = 0; k < 4; ++k) {
-                const int j = 8 * q + 2 * k;
-                float gv[2], out[2];
-                const float hv[2] = {__uint_as_float(hh[k] << 16), __uint_as_float(hh[k] & 0xffff0000u)};
-                const float wv[2] = {__uint_as_float(ww[k] << 16), __uint_as_float(ww[k] & 0xffff0000u)};
-                const float uv[2] = {__uint_as_float(yy[k] << 16), __uint_as_float(yy[k] & 0xffff0000u)};
+            for (int q = 0; q < 4; ++q) {
+                const uint32_t hh[4] = {ch[q].x, ch[q].y, ch[q].z, ch[q].w};
+                const uint32_t ww[4] = {cw[q].x, cw[q].y, cw[q].z, cw[q].w};
+                const uint32_t yy[4] = {cy[q].x, cy[q].y, cy[q].z, cy[q].w};
 #pragma unroll
-                for (int e = 0; e < 2; ++e) {
-                    gv[e] = a == 0.f ? 0.f : fmaf(a, v[j + e], b * uv[e]);
-                    out[e] = (wv[e] * gv[e] - (hv[e] * inv_r) * kd) * pref;
+                for (int k = 0; k < 4; ++k) {
+                    const int j = 8 * q + 2 * k;
+                    const float2 hv = make_float2(__uint_as_float(hh[k] << 16),
+                                                  __uint_as_float(hh[k] & 0xffff0000u));
+                    const float2 wv = make_float2(__uint_as_float(ww[k] << 16),
+                                                  __uint_as_float(ww[k] & 0xffff0000u));
+                    const float2 uv = make_float2(__uint_as_float(yy[k] << 16),
+                                                  __uint_as_float(yy[k] & 0xffff0000u));
+                    const float2 t = __ffma2_rn(b2, uv, __fmul2_rn(a2, make_float2(v[j], v[j + 1])));
+                    const float2 out = __ffma2_rn(wv, t, __fmul2_rn(nk2, hv));
+                    r[j / 2] = pack_bf16x2(out.x, out.y);
                 }
-                r[j / 2] = pack_bf16x2(out[0], out[1]);
             }
         }
         if (!second) {

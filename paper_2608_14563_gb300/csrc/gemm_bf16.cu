@@ -267,9 +267,10 @@ __global__ void __launch_bounds__(kFixupThreads)
     if (!sk_tail_sum<BN>(sh, scratch, row, n, s4)) return;
     const float a = va.alpha[row], bb = va.beta[row];
     const float rr = va.rho[row];
-    const float inv_r = 1.0f / rr;
     const float kd = va.cv[row] * va.inv_d;
     const float pref = 1.0f / fmaxf(rr, va.min_rms);
+    // the same association as EpiProjVjp: w (a pref sum + b pref W_U[y]) - h (kd pref / rho)
+    const float ap = a * pref, bp = bb * pref, nk = -(kd * (1.0f / rr)) * pref;
     const __nv_bfloat16* wy =
         (a != 0.f && bb != 0.f) ? va.W_U + static_cast<long long>(va.y[row]) * sh.N : nullptr;
     const __nv_bfloat16* hr = va.h + static_cast<long long>(row) * sh.N;
@@ -277,9 +278,10 @@ __global__ void __launch_bounds__(kFixupThreads)
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
         const float yv = wy ? __bfloat162float(wy[n + j]) : 0.f;
-        const float gv = a == 0.f ? 0.f : fmaf(a, s4[j], bb * yv);
-        o[j] = (__bfloat162float(va.w[n + j]) * gv - (__bfloat162float(hr[n + j]) * inv_r) * kd) *
-               pref;
+        const float t = fmaf(bp, yv, ap * s4[j]);
+        o[j] = a == 0.f ? 0.f
+                        : fmaf(__bfloat162float(va.w[n + j]), t,
+                               nk * __bfloat162float(hr[n + j]));
     }
     *reinterpret_cast<uint2*>(out + static_cast<size_t>(row) * sh.N + n) =
         make_uint2(pack_bf16x2(o[0], o[1]), pack_bf16x2(o[2], o[3]));
