@@ -175,7 +175,8 @@ cudaError_t run_gemm_pair(const GemmMaps<MAXG>& maps, const typename Epi::Params
                           float* sk_scratch = nullptr, SkPlan* plan = nullptr) {
     if (plan) *plan = SkPlan{};
     if (sh_in.tiles <= 0 || sh_in.k_blocks <= 0) return cudaSuccess;
-    using L = GemmPairSmem<BN, STAGES>;
+    using L = GemmPairSmem<BN, STAGES, pair_ksub<BN, A_MN, B_MN>()>;
+    static_assert(L::kBytes <= 227 * 1024, "stages exceed the shared memory of a CTA");
     auto kern = tc_gemm_pair_kernel<BN, A_MN, B_MN, STAGES, MAXG, Epi>;
     static cudaError_t attr_err =
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::kBytes);
@@ -319,7 +320,7 @@ cudaError_t launch_sk_fixup_vjp(const SkPlan& plan, const GemmShape& sh, const f
     return cudaGetLastError();
 }
 
-constexpr int kPairStages = 6;
+constexpr int kPairStages = 3;   // 256 x 256 pair tiles: 64 KB stages of two k-blocks
 constexpr int kWideBN = 512;     // pair tiles 256 x 512: 48 KB stages
 constexpr int kWideStages = 4;
 
@@ -356,7 +357,7 @@ size_t proj_sk_scratch_bytes() {
     // kTailWaves x clusters units of 256 x 512 fp32; clusters of the 256 x 512 pair kernel
     // on this device, or an upper bound of 128 without one
     static const size_t bytes = [] {
-        using L = GemmPairSmem<kWideBN, kWideStages>;
+        using L = GemmPairSmem<kWideBN, kWideStages, pair_ksub<kWideBN, false, true>()>;
         auto kern = tc_gemm_pair_kernel<kWideBN, false, true, kWideStages, 1, EpiProjVjp>;
         DevInfo di;
         long long c = 128;

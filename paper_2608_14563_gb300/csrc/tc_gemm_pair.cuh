@@ -4,8 +4,21 @@
 // tcgen05.mma.cta_group::2: CTA r holds rows [128 r, 128 r + 128) of the A
 // tile and columns [BN/2 r, BN/2 (r + 1)) of the B tile in its own shared
 // memory, and its TMEM receives output rows [128 r, 128 r + 128).  Per SM a
-// k-block stage is A 16 KB + B 16 KB (instead of A 16 KB + B 32 KB), so six
-// stages fit and each SM streams a third less operand data per FLOP.
+// 64-deep k-block is A 16 KB + B 16 KB (instead of A 16 KB + B 32 KB), so each
+// SM streams a third less operand data per FLOP.
+//
+// A pipeline stage of the 256-column tiles holds two consecutive 64-deep k-blocks
+// (64 KB per CTA, three stages): the MMA thread then waits on one barrier and
+// commits once per eight N = 256 MMAs (1024 tensor cycles) instead of per four.  Measured with clock counters in the MMA thread, one
+// wait + fence + four MMAs + commit per 64-deep stage took ~550 cycles for 512
+// cycles of tensor work (the issuing thread, not the operand supply, set the pace:
+// the same loop with the operands loaded once per launch ran at the same rate); with
+// eight MMAs per stage the loop keeps pace with the tensor pipe.  The 512-column
+// tiles issue eight MMAs per 64-deep k-block already.  The layer update (MN-major,
+// g~ and A_l streamed from DRAM) alone runs 2% slower with three 64 KB stages than
+// with six of 32 KB, but the step as a whole is faster with them (at the power cap
+// the update's lower draw leaves clock to the other GEMMs), so every 256-column
+// tile uses them.
 //
 //   both CTAs, warp 0   TMA loads of the CTA's halves; completion is counted
 //                       on the LEADER's (rank 0) full barrier
@@ -32,11 +45,18 @@ namespace fpo {
 
 constexpr int kPairBM = 256;  // output rows of one pair tile
 
-template <int BN, int STAGES>
+// 64-deep k-blocks per pipeline stage of a BN-column pair tile.
+template <int BN, bool A_MN, bool B_MN>
+constexpr int pair_ksub() {
+    return BN == 256 ? 2 : 1;
+}
+
+template <int BN, int STAGES, int KSUB>
 struct GemmPairSmem {
-    static constexpr int kABytes = 128 * kBK * 2;
-    static constexpr int kBBytes = (BN / 2) * kBK * 2;
-    static constexpr int kStageBytes = kABytes + kBBytes;
+    static constexpr int kSub = KSUB;
+    static constexpr int kABytes = 128 * kBK * 2;         // one 64-deep k-block of A
+    static constexpr int kBBytes = (BN / 2) * kBK * 2;    // one 64-deep k-block of B
+    static constexpr int kStageBytes = kSub * (kABytes + kBBytes);  // A blocks, then B blocks
     static constexpr int kOutOffset = STAGES * kStageBytes;
     static constexpr int kBarOffset = kOutOffset + 4 * kOutBytesPerWarp;
     static constexpr int kNumBars = 2 * STAGES + 5;
@@ -165,7 +185,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
                         const __grid_constant__ typename Epi::Params ep, const GemmShape sh_in,
                         unsigned int* status, unsigned long long wait_limit_ns) {
     static_assert(BN == 256 || BN == 512, "pair tiles are 256 or 512 columns wide");
-    using L = GemmPairSmem<BN, STAGES>;
+    using L = GemmPairSmem<BN, STAGES, pair_ksub<BN, A_MN, B_MN>()>;
+    constexpr int kSub = L::kSub;                  // 64-deep k-blocks per stage
     constexpr int kNSub = BN / 256;                // N = 256 MMAs per K slice
     constexpr int kAccBufs = kNSub == 1 ? 2 : 1;   // accumulator buffers in TMEM
     constexpr int kBSub = 128;                     // B columns per CTA per N = 256 MMA
@@ -175,6 +196,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
     constexpr uint16_t kBoth = 0x3;                // both CTAs of the pair
 
     GemmShape sh = sh_in;
+    // from here on a "k-block" is one stage: kSub 64-deep k-blocks (the last one may
+    // reach past K; its loads read zeros there)
+    sh.k_blocks = (sh.k_blocks + kSub - 1) / kSub;
     if (sh.m_dev) {  // rows counted on the device (every thread reads the same value)
         const int m = min(*sh.m_dev, sh.M);
         if (m <= 0) return;
@@ -255,14 +279,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
                 for (int kb = kb0; kb < kb1; ++kb) {
                     if (!mbar_wait_cl(empty_bar(stage), phase ^ 1u, guard)) { ok = false; break; }
                     const uint32_t sa = sbase + stage * L::kStageBytes;
-                    const uint32_t sb = sa + L::kABytes;
+                    const uint32_t sb = sa + kSub * L::kABytes;
                     const uint32_t fb = mapa_shared(full_bar(stage), 0);
                     if (leader) mbar_arrive_expect_tx(full_bar(stage), 2 * L::kStageBytes);
-                    load_operand_pair<A_MN, 128>(amap, sa, fb, a_row, kb * kBK);
 #pragma unroll
-                    for (int h = 0; h < kNSub; ++h)
-                        load_operand_pair<B_MN, kBSub>(bmap, sb + h * kBSubBytes, fb,
-                                                       b_row + 256 * h, kb * kBK);
+                    for (int j = 0; j < kSub; ++j) {
+                        const int k0 = (kb * kSub + j) * kBK;
+                        load_operand_pair<A_MN, 128>(amap, sa + j * L::kABytes, fb, a_row, k0);
+#pragma unroll
+                        for (int h = 0; h < kNSub; ++h)
+                            load_operand_pair<B_MN, kBSub>(
+                                bmap, sb + j * L::kBBytes + h * kBSubBytes, fb, b_row + 256 * h, k0);
+                    }
                     ++issued;
                     if (++stage == STAGES) { stage = 0; phase ^= 1u; }
                 }
@@ -289,14 +317,17 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
                     if (!mbar_wait_cl(full_bar(stage), phase, guard)) { ok = false; break; }
                     tc_fence_after();
                     const uint32_t sa = sbase + stage * L::kStageBytes;
-                    const uint32_t sb = sa + L::kABytes;
+                    const uint32_t sb = sa + kSub * L::kABytes;
 #pragma unroll
-                    for (int kk = 0; kk < kBK / kUmmaK; ++kk)
+                    for (int j = 0; j < kSub; ++j)
 #pragma unroll
-                        for (int h = 0; h < kNSub; ++h)
-                            tc_mma_bf16_pair(d_tmem + 256u * h, operand_desc<A_MN>(sa, kk),
-                                             operand_desc<B_MN>(sb + h * kBSubBytes, kk), kIdesc,
-                                             (kb != kb0 || kk != 0) ? 1u : 0u);
+                        for (int kk = 0; kk < kBK / kUmmaK; ++kk)
+#pragma unroll
+                            for (int h = 0; h < kNSub; ++h)
+                                tc_mma_bf16_pair(
+                                    d_tmem + 256u * h, operand_desc<A_MN>(sa + j * L::kABytes, kk),
+                                    operand_desc<B_MN>(sb + j * L::kBBytes + h * kBSubBytes, kk),
+                                    kIdesc, (kb != kb0 || j != 0 || kk != 0) ? 1u : 0u);
                     issued_any = true;
                     // the stage is free in both CTAs once the MMAs reading it completed
                     tc_commit_pair_multicast(empty_bar(stage), kBoth);
