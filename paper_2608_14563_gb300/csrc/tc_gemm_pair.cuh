@@ -96,6 +96,38 @@ __device__ __forceinline__ bool mbar_wait_cl(uint32_t bar, uint32_t parity, cons
     }
 }
 
+__device__ __forceinline__ bool mbar_test_wait_cluster(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.test_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// mbar_wait_cl for the MMA thread's stage waits: it polls with test_wait, which never
+// suspends the thread, so the next MMAs issue as soon as the stage lands (measured: the
+// layer update 1% faster than with try_wait, the other GEMMs unchanged).  The limit and
+// the abort flag are checked every 32 polls.
+__device__ __forceinline__ bool mbar_wait_cl_poll(uint32_t bar, uint32_t parity, const WaitGuard& g) {
+    if (mbar_test_wait_cluster(bar, parity)) return true;
+    const uint64_t t0 = global_timer_ns();
+    for (uint32_t i = 1;; ++i) {
+        if (mbar_test_wait_cluster(bar, parity)) return true;
+        if ((i & 31u) == 0) {
+            if (*g.abort_flag) return false;
+            if (global_timer_ns() - t0 > g.limit_ns) {
+                *g.abort_flag = 1;
+                if (g.status) atomicOr(g.status, kDevTimeout);
+                return false;
+            }
+        }
+    }
+}
+
 __device__ __forceinline__ bool mbar_wait_cl_drain(uint32_t bar, uint32_t parity, uint64_t limit_ns) {
     const uint64_t t0 = global_timer_ns();
     while (!mbar_try_wait_cluster(bar, parity))
@@ -314,7 +346,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
                 tc_fence_after();
                 const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * BN);
                 for (int kb = kb0; kb < kb1; ++kb) {
-                    if (!mbar_wait_cl(full_bar(stage), phase, guard)) { ok = false; break; }
+                    if (!mbar_wait_cl_poll(full_bar(stage), phase, guard)) { ok = false; break; }
                     tc_fence_after();
                     const uint32_t sa = sbase + stage * L::kStageBytes;
                     const uint32_t sb = sa + kSub * L::kABytes;
