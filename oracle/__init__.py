@@ -11,6 +11,8 @@ Each function follows one passage of the paper:
   with the min-RMS clamp.
 * :func:`rmsnorm_vjp`   App. E Eq. (rmsnorm-vjp) at any norm (the per-layer post-FFN
   norm of OLMo-2 / Gemma 3, Sec. 3.2).
+* :func:`layer_signal`  Sec. 3.1 step 4, Sec. 3.2: the layer-specific signal composed with
+  the post-feedforward and / or pre-MLP RMSNorm Jacobians.
 * :func:`gate_up_signals`  Sec. 3.1 step 5, Eq. (errh): W1/W2 signals of a SwiGLU MLP.
 * :func:`pseudograd`    Sec. 3.1 step 5, Eq. (w3update).
 * :func:`sgd_update`    App. A, fp32 master weights cast to bf16.
@@ -60,6 +62,8 @@ def _load():
     lib.oracle_error_signal.restype = i32
     lib.oracle_rmsnorm_vjp.argtypes = [i64, i64, i32, vp, i32, vp, vp, dbl, dbl, vp]
     lib.oracle_rmsnorm_vjp.restype = i32
+    lib.oracle_layer_signal.argtypes = [i64, i64, i32, vp, i32, vp, vp, vp, vp, dbl, dbl, vp]
+    lib.oracle_layer_signal.restype = i32
     lib.oracle_gate_up_signals.argtypes = [i64, i64, i64, i32, vp, vp, vp, vp, vp, vp]
     lib.oracle_gate_up_signals.restype = i32
     lib.oracle_pseudograd.argtypes = [i64, i64, i64, i32, vp, i32, vp, vp, vp, i64, vp]
@@ -154,6 +158,41 @@ def rmsnorm_vjp(g, x, gamma, *, eps=1e-6, min_rms=0.5):
                                     _ptr(out))
     if rc != 0:
         raise ValueError(f"oracle_rmsnorm_vjp failed ({rc})")
+    return out
+
+
+def layer_signal(g, m=None, gamma_post=None, x=None, gamma_pre=None, *, eps=1e-6, min_rms=0.5):
+    """Sec. 3.1 step 4 / Sec. 3.2: compose g with the post-feedforward RMSNorm Jacobian at
+    the MLP output m (weight gamma_post), then with the pre-MLP RMSNorm Jacobian at its
+    input x (weight gamma_pre); a norm given as None is not composed.
+
+    g, m, x: [T, d]; gammas: [d] (m, x and the gammas share one dtype).  Returns fp64 [T, d].
+    """
+    dtg, g = _typed(g)
+    T, d = g.shape
+    norms = [a for a in (m, gamma_post, x, gamma_pre) if a is not None]
+    if (m is None) != (gamma_post is None) or (x is None) != (gamma_pre is None):
+        raise ValueError("each norm needs both its input and its weight")
+    typed = [_typed(a) for a in norms]
+    if len({t for t, _ in typed}) > 1:
+        raise TypeError("norm inputs and weights must share one dtype")
+    dtn = typed[0][0] if typed else dtg
+    arrs = iter(a for _, a in typed)
+    mm = next(arrs) if m is not None else None
+    gp = next(arrs) if m is not None else None
+    xx = next(arrs) if x is not None else None
+    gq = next(arrs) if x is not None else None
+    for a in (mm, xx):
+        if a is not None and a.shape != (T, d):
+            raise ValueError("norm inputs must be [T, d] like g")
+    for a in (gp, gq):
+        if a is not None and a.shape != (d,):
+            raise ValueError("norm weights must be [d]")
+    out = np.zeros((T, d))
+    rc = _load().oracle_layer_signal(T, d, dtg, _ptr(g), dtn, _ptr(mm), _ptr(gp), _ptr(xx),
+                                     _ptr(gq), eps, min_rms, _ptr(out))
+    if rc != 0:
+        raise ValueError(f"oracle_layer_signal failed ({rc})")
     return out
 
 

@@ -13,6 +13,8 @@
  *   oracle_error_signal  Sec. 3.1 steps 2-4, Eq. (gproj), App. E Eq. (rmsnorm-vjp)
  *                        and the min-RMS clamp (Sec. 3.2 / App. E)
  *   oracle_rmsnorm_vjp   App. E Eq. (rmsnorm-vjp) at any norm (post-FFN, Sec. 3.2)
+ *   oracle_layer_signal  Sec. 3.1 step 4 and Sec. 3.2: the per-layer composition with the
+ *                        post-feedforward and / or pre-MLP RMSNorm Jacobians
  *   oracle_gate_up_signals  Sec. 3.1 step 5, Eq. (errh): W1/W2 signals of a SwiGLU MLP
  *   oracle_pseudograd    Sec. 3.1 step 5, Eq. (w3update): G = g~^T h_mid
  *   oracle_sgd_update    App. A (fp32 master weights, cast to bf16)
@@ -182,6 +184,69 @@ int oracle_rmsnorm_vjp(int64_t T, int64_t d, int dt_g, const void* g, int dt_x, 
         for (int64_t j = 0; j < d; ++j)
             out[t * d + j] = (orc_load(dt_x, gamma, j) * orc_load(dt_g, g, t * d + j) -
                               (orc_load(dt_x, x, t * d + j) / rh) * c / (double)d) / denom;
+    }
+    return 0;
+}
+
+/*
+ * App. E Eq. (rmsnorm-vjp) on one fp64 row u at norm input row x (element offset
+ * off of a typed [T, d] array) with weight gamma:
+ *   rho = sqrt(mean_j x_j^2 + eps), xhat = x / rho, c = <xhat, gamma (.) u>,
+ *   v   = (gamma (.) u - xhat c / d) / max(rho, rho_min)
+ */
+static void orc_vjp_row(int64_t d, const double* u, int dt, const void* x, int64_t off,
+                        const void* gamma, double eps, double min_rms, double* v) {
+    double ss = 0.0;
+    for (int64_t j = 0; j < d; ++j) {
+        double xv = orc_load(dt, x, off + j);
+        ss += xv * xv;
+    }
+    double rh = sqrt(ss / (double)d + eps);
+    double c = 0.0;
+    for (int64_t j = 0; j < d; ++j) c += (orc_load(dt, x, off + j) / rh) * orc_load(dt, gamma, j) * u[j];
+    double denom = rh > min_rms ? rh : min_rms;
+    for (int64_t j = 0; j < d; ++j)
+        v[j] = (orc_load(dt, gamma, j) * u[j] - (orc_load(dt, x, off + j) / rh) * c / (double)d) / denom;
+}
+
+/*
+ * The layer-specific signal of one target layer (Sec. 3.1 step 4, Sec. 3.2, App. E
+ * table of norms per family).  Starting from g (the signal after the final norm's
+ * Jacobian), in the paper's order:
+ *   1. post-feedforward RMSNorm (OLMo-2, Gemma 3): compose with its Jacobian at the
+ *      layer's MLP output m with weight gamma_post;
+ *   2. pre-MLP RMSNorm (Qwen3, Gemma 3): additionally compose with its Jacobian at
+ *      the norm's input x (the residual stream entering the MLP block) with weight
+ *      gamma_pre.
+ * Each is App. E Eq. (rmsnorm-vjp) with its own rho and the min-RMS clamp; a norm
+ * whose input is NULL is not composed (both NULL: out = g).  The intermediate signal
+ * stays in fp64.  g: [T, d] (dt_g); m, x: [T, d] and gammas: [d] (dt_n); out: fp64.
+ */
+int oracle_layer_signal(int64_t T, int64_t d, int dt_g, const void* g, int dt_n, const void* m,
+                        const void* gamma_post, const void* x, const void* gamma_pre, double eps,
+                        double min_rms, double* out) {
+    if (T < 0 || d <= 0 || !out || (T > 0 && !g) || (m && !gamma_post) || (x && !gamma_pre))
+        return -1;
+#pragma omp parallel
+    {
+        double* u = (double*)malloc((size_t)d * sizeof(double));
+        double* v = (double*)malloc((size_t)d * sizeof(double));
+#pragma omp for schedule(static)
+        for (int64_t t = 0; t < T; ++t) {
+            if (!u || !v) continue;
+            for (int64_t j = 0; j < d; ++j) u[j] = orc_load(dt_g, g, t * d + j);
+            if (m) {
+                orc_vjp_row(d, u, dt_n, m, t * d, gamma_post, eps, min_rms, v);
+                memcpy(u, v, (size_t)d * sizeof(double));
+            }
+            if (x) {
+                orc_vjp_row(d, u, dt_n, x, t * d, gamma_pre, eps, min_rms, v);
+                memcpy(u, v, (size_t)d * sizeof(double));
+            }
+            memcpy(out + t * d, u, (size_t)d * sizeof(double));
+        }
+        free(u);
+        free(v);
     }
     return 0;
 }

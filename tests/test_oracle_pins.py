@@ -390,6 +390,90 @@ def test_rmsnorm_vjp_matches_error_signal_final_norm_step():
 
 
 # ---------------------------------------------------------------------------
+# Per-layer composition with the post-FFN and pre-MLP norms (Sec. 3.1 step 4, Sec. 3.2)
+# ---------------------------------------------------------------------------
+def _two_norm_toy(seed, T=5, d=6, V=10, small_x_token=None):
+    rng = np.random.default_rng(seed)
+    h0 = rng.standard_normal((T, d))
+    x = rng.standard_normal((T, d))                 # input of the pre-MLP norm
+    if small_x_token is not None:
+        x[small_x_token] *= 0.05
+    gq = 0.8 + 0.1 * rng.standard_normal(d)         # pre-MLP norm weight
+    gp = 0.3 + 0.05 * rng.standard_normal(d)        # post-FFN norm weight
+    w = 1.0 + 0.1 * rng.standard_normal(d)          # final norm weight
+    W_U = 0.5 * rng.standard_normal((V, d))
+    y = rng.integers(0, V, T).astype(np.int32)
+    return h0, x, gq, gp, w, W_U, y
+
+
+def _rmsn(a, eps):
+    return a / np.sqrt(np.mean(a * a, axis=1, keepdims=True) + eps)
+
+
+def test_layer_signal_is_gradient_through_both_norms():
+    """Wire the post-FFN norm straight onto the pre-MLP norm's output (m = gq * N(x),
+    h = h0 + gp * N(m)): then composing the post-FFN Jacobian at m and the pre-MLP one
+    at x, in that order, is exactly dL/dx.  The other order, or a dropped norm, is not."""
+    h0, x, gq, gp, w, W_U, y = _two_norm_toy(30)
+    s, eps = 1.0 / len(y), 1e-6
+    m = gq * _rmsn(x, eps)
+    h = h0 + gp * _rmsn(m, eps)
+    gt = oracle.error_signal(h, w, W_U, y, eps=eps, min_rms=0.0, s=s)["g_tilde"]
+    out = oracle.layer_signal(gt, m, gp, x, gq, eps=eps, min_rms=0.0)
+    fd = fd_grad(lambda xx: forward_loss(h0 + gp * _rmsn(gq * _rmsn(xx, eps), eps), w, W_U, y,
+                                         eps, s), x.copy())
+    assert rel_err(out, fd) < 1e-7
+    swapped = oracle.rmsnorm_vjp(oracle.rmsnorm_vjp(gt, x, gq, eps=eps, min_rms=0.0), m, gp,
+                                 eps=eps, min_rms=0.0)
+    assert rel_err(swapped, fd) > 1e-2
+    assert rel_err(oracle.layer_signal(gt, x=x, gamma_pre=gq, eps=eps, min_rms=0.0), fd) > 1e-2
+
+
+def test_layer_signal_single_norm_is_that_norms_vjp():
+    """With one norm the composition is that norm's App. E VJP; with none it is g."""
+    h0, x, gq, gp, w, W_U, y = _two_norm_toy(31)
+    rng = np.random.default_rng(32)
+    g = rng.standard_normal(x.shape)
+    m = rng.standard_normal(x.shape)
+    assert rel_err(oracle.layer_signal(g, m, gp), oracle.rmsnorm_vjp(g, m, gp)) < 1e-15
+    assert rel_err(oracle.layer_signal(g, x=x, gamma_pre=gq), oracle.rmsnorm_vjp(g, x, gq)) < 1e-15
+    assert np.array_equal(oracle.layer_signal(g), g)
+
+
+def test_layer_signal_clamp_acts_per_norm():
+    """A token whose pre-MLP norm input has RMS below rho_min gets (rho/rho_min) x its
+    unclamped signal; the post-FFN stage's clamp scales its input to the linear pre-MLP
+    stage by its own factor."""
+    h0, x, gq, gp, w, W_U, y = _two_norm_toy(33, small_x_token=1)
+    rng = np.random.default_rng(34)
+    g = rng.standard_normal(x.shape)
+    m = rng.standard_normal(x.shape)
+    m[3] *= 0.1                                     # post-FFN input RMS far below 0.5
+    eps = 1e-6
+    rx = np.sqrt(np.mean(x * x, axis=1) + eps)
+    rm = np.sqrt(np.mean(m * m, axis=1) + eps)
+    assert rx[1] < 0.5 and rm[3] < 0.5
+    assert np.all(np.delete(rx, 1) > 0.5) and np.all(np.delete(rm, 3) > 0.5)
+    exact = oracle.layer_signal(g, m, gp, x, gq, eps=eps, min_rms=0.0)
+    clamped = oracle.layer_signal(g, m, gp, x, gq, eps=eps, min_rms=0.5)
+    expect = exact.copy()
+    expect[1] *= rx[1] / 0.5
+    expect[3] *= rm[3] / 0.5
+    assert rel_err(clamped, expect) < 1e-14
+
+
+def test_layer_signal_eps0_is_orthogonal_to_the_pre_mlp_input():
+    """With eps = 0 the last Jacobian's output is orthogonal to its norm input."""
+    _, x, gq, gp, _, _, _ = _two_norm_toy(35)
+    rng = np.random.default_rng(36)
+    g = rng.standard_normal(x.shape)
+    m = rng.standard_normal(x.shape)
+    out = oracle.layer_signal(g, m, gp, x, gq, eps=0.0, min_rms=0.0)
+    dots = np.abs(np.sum(out * x, axis=1)) / (np.linalg.norm(out, axis=1) * np.linalg.norm(x, axis=1))
+    assert np.all(dots < 1e-13)
+
+
+# ---------------------------------------------------------------------------
 # Optimizers on the fp32 master and the relative clip (Sec. 3.1, App. A)
 # ---------------------------------------------------------------------------
 def _opt_case(seed, n=(6, 9)):
