@@ -274,7 +274,8 @@ def workload_config(wl, args):
             "global_batch_tokens": wl.T * args.gpus,
             "error_matrix": {"auto": "direct (auto)", "recompute": "recompute",
                              "stored": "stored-logits", "direct": "direct"}[args.algo],
-            "norms_composed": "final + post-FFN per layer" if args.post_ffn_norm else "final",
+            "norms_composed": "final" + (" + post-FFN per layer" if args.post_ffn_norm else "")
+                              + (" + pre-MLP per layer" if args.pre_mlp_norm else ""),
             "weights_updated": ("W3, W1, W2 (W1/W2 via W3_init feedback, the same optimizer)"
                                 if args.gate_up else "W3"),
             "optimizer": ("plain SGD fused in the update GEMM epilogue" if args.optimizer == "fused-sgd"
@@ -322,6 +323,8 @@ def run_fpo(args, wl):
     g = torch.empty_like(h)
     loss = torch.empty(1, dtype=torch.float32, device=dev)
     post = args.post_ffn_norm
+    pre = args.pre_mlp_norm
+    layer_norms = post or pre  # per-layer signals g~^(l) (Sec. 3.2)
     gate_up = args.gate_up
     if gate_up:  # SwiGLU caches, W3_init feedback, gate/up masters and signal buffers
         gu_ab = [synth.make_gate_up(wl_r, l, dev) for l in range(wl.layers)]
@@ -332,9 +335,13 @@ def run_fpo(args, wl):
         gu_sig = [torch.empty(wl.T, wl.d_ff, dtype=torch.bfloat16, device=dev)
                   for _ in range(2 * wl.layers)]
         ws_gu = torch.empty(fpo.layer_update_workspace(), dtype=torch.uint8, device=dev)
-    if post:  # per-layer MLP outputs, post-FFN norm weights and layer-specific signals
+    if post:  # per-layer MLP outputs and post-FFN norm weights
         m_out = [synth.make_mlp_out(wl_r, l, dev) for l in range(wl.layers)]
         gp = [synth.make_post_norm_w(wl_r, l, dev) for l in range(wl.layers)]
+    if pre:  # per-layer pre-MLP norm inputs (residual stream) and weights
+        x_pre = [synth.make_pre_norm_in(wl_r, l, dev) for l in range(wl.layers)]
+        gq = [synth.make_pre_norm_w(wl_r, l, dev) for l in range(wl.layers)]
+    if layer_norms:  # the layer-specific signals
         g_l = [torch.empty_like(h) for _ in range(wl.layers)]
     algo = {"auto": fpo.ES_AUTO, "recompute": fpo.ES_RECOMPUTE,
             "stored": fpo.ES_STORED_LOGITS, "direct": fpo.ES_DIRECT}[args.algo]
@@ -368,7 +375,7 @@ def run_fpo(args, wl):
 
     # The tensors one step reads that come from the forward pass / the data: the
     # end-to-end loop below copies them from host memory every step.
-    X0 = {"h": h, "y": y, "A": A, "m": m_out if post else [],
+    X0 = {"h": h, "y": y, "A": A, "m": m_out if post else [], "xpre": x_pre if pre else [],
           "ab": [t for pair in gu_ab for t in pair] if gate_up else [],
           "x": gu_x if gate_up else []}
 
@@ -397,7 +404,7 @@ def run_fpo(args, wl):
         Go_flat = [x.view(-1) for x in Go]
     # the diagnostic's step (G_l only, no master to move) forms the cosines in the update
     # GEMM's epilogue, so G_l is not read back, unless asked to run the two calls
-    fused_cos = (cosine and wl.lr == 0.0 and not (post or optimize or ratio or gate_up)
+    fused_cos = (cosine and wl.lr == 0.0 and not (layer_norms or optimize or ratio or gate_up)
                  and not args.cosine_separate)
     if fused_cos:
         G_true_2d = [x.view(wl.d, wl.d_ff) for x in G_true]
@@ -405,12 +412,12 @@ def run_fpo(args, wl):
                             dtype=torch.uint8, device=dev)
 
     def update(X):
-        signals = g_l if post else [g] * wl.layers
+        signals = g_l if layer_norms else [g] * wl.layers
         G_outs = Go if (ratio or cosine) else None
         if optimize:
             fpo.layer_optimize_grouped(signals, X["A"], opt, Wm, W_outs=Wo, states1=st1,
                                        states2=st2, workspace=ws_up)
-        elif post:
+        elif layer_norms:
             fpo.layer_update_grouped_signals(g_l, X["A"], wl.lr, W_masters=Wm, W_outs=Wo,
                                              G_outs=G_outs, workspace=ws_up)
         elif fused_cos:
@@ -425,7 +432,7 @@ def run_fpo(args, wl):
 
     def gate_up_update(X):
         for l in range(wl.layers):
-            fpo.gate_up_signals(g_l[l] if post else g, gu_W3[l], X["ab"][2 * l],
+            fpo.gate_up_signals(g_l[l] if layer_norms else g, gu_W3[l], X["ab"][2 * l],
                                 X["ab"][2 * l + 1], gu_sig[2 * l], gu_sig[2 * l + 1],
                                 workspace=ws_gu)
         gu_act = [x for x in X["x"] for _ in range(2)]
@@ -440,11 +447,12 @@ def run_fpo(args, wl):
         fpo.error_signal(X["h"], w, W_U, X["y"], g, eps=wl.eps, min_rms=wl.min_rms,
                          t_chunk=args.t_chunk, loss_out=loss, workspace=ws_es,
                          stage_events=stage_events, algo=algo, per_chunk_events=per_chunk)
-        if post:
+        if layer_norms:
             if upd_events:
                 upd_events[2].record(stream)
-            for l in range(wl.layers):
-                fpo.rmsnorm_vjp(g, X["m"][l], gp[l], g_l[l], eps=wl.eps, min_rms=wl.min_rms)
+            fpo.layer_signals(g, g_l, m=X["m"] if post else None, gamma_post=gp if post else None,
+                              x=X["xpre"] if pre else None, gamma_pre=gq if pre else None,
+                              eps=wl.eps, min_rms=wl.min_rms)
         if upd_events:
             upd_events[0].record(stream)
         update(X)
@@ -530,9 +538,9 @@ def run_fpo(args, wl):
                 for k, n in enumerate(names)}
     stage_ms["layer_update"] = statistics.mean(uev[i][0].elapsed_time(uev[i][1])
                                                for i in range(args.steps))
-    if post:
-        stage_ms["post_ffn_vjp"] = statistics.mean(uev[i][2].elapsed_time(uev[i][0])
-                                                   for i in range(args.steps))
+    if layer_norms:
+        stage_ms["layer_signals"] = statistics.mean(uev[i][2].elapsed_time(uev[i][0])
+                                                    for i in range(args.steps))
     if gate_up:
         stage_ms["gate_up"] = statistics.mean(uev[i][1].elapsed_time(uev[i][3])
                                               for i in range(args.steps))
@@ -558,7 +566,7 @@ def run_fpo(args, wl):
                     for k, v in X.items()}
 
         def flat(X):
-            return [X["h"], X["y"]] + [t for k in ("A", "m", "ab", "x") for t in X[k]]
+            return [X["h"], X["y"]] + [t for k in ("A", "m", "xpre", "ab", "x") for t in X[k]]
 
         depth = max(2, args.e2e_depth)
         sets = [X0] + [clone_set(X0) for _ in range(depth - 1)]
@@ -727,7 +735,11 @@ def run_fpo(args, wl):
                                 / (stage_ms["norm_ratio"] / 1e3) / 1e9} if ratio else {}),
                             **({"cosine": wl.layers * wl.d * wl.d_ff * (2 + 2)
                                 / (stage_ms["cosine"] / 1e3) / 1e9}
-                               if cosine and not fused_cos else {})},
+                               if cosine and not fused_cos else {}),
+                            # per layer: g, the norm inputs and the signal, bf16 rows
+                            **({"layer_signals": wl.layers * wl.T * wl.d * 2 * (2 + post + pre)
+                                / (stage_ms["layer_signals"] / 1e3) / 1e9}
+                               if layer_norms else {})},
             "cosine": cos_out[:, 3].tolist() if cosine else None,
             "cosine_mode": (None if not cosine else
                             "fused: fpo_layer_grad_cosine_grouped forms the sums in the update "
@@ -825,6 +837,9 @@ def main():
                     help="also update W1/W2 of every layer through the cached W3_init feedback")
     ap.add_argument("--post-ffn-norm", action="store_true",
                     help="compose each layer's post-FFN RMSNorm VJP (OLMo-2 layout) in the step")
+    ap.add_argument("--pre-mlp-norm", action="store_true",
+                    help="compose each layer's pre-MLP RMSNorm VJP (Qwen3 layout; with "
+                         "--post-ffn-norm the Gemma 3 layout) in the step")
     ap.add_argument("--algo", choices=("auto", "recompute", "stored", "direct"), default="auto",
                     help="how the error matrix is formed (fpo_es_algo)")
     ap.add_argument("--cosine", action="store_true",

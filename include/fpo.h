@@ -13,8 +13,8 @@
  * and the layer-viability diagnostic of Sec. 2.2 reduces pairs of gradients
  * with fpo_cosine (one pair) or fpo_cosine_grouped (every layer in one call).
  * Further entry points cover the rest of the method around that step: the
- * post-FFN RMSNorm VJP and per-layer signals (fpo_rmsnorm_vjp,
- * fpo_layer_update_grouped_signals), optimizers with the relative clip
+ * post-FFN and pre-MLP RMSNorm VJPs and per-layer signals (fpo_rmsnorm_vjp,
+ * fpo_layer_signals, fpo_layer_update_grouped_signals), optimizers with the relative clip
  * (fpo_layer_optimize_grouped), the gate/up signals through the cached
  * W3_init (fpo_gate_up_signals) and the App. C update-magnitude ratio
  * (fpo_norm_ratio).  fpo_h2d_copy stages a step's inputs from host memory.
@@ -252,14 +252,44 @@ int32_t fpo_layer_update_grouped(int32_t n_layers, int64_t T, int64_t d, int64_t
  * fpo_layer_update_grouped_signals -- fpo_layer_update_grouped where layer l
  * has its own signal g[l] (HOST array of n_layers device pointers, [T, d]
  * each): the layer-specific g~^(l) of Sec. 3.1 step 4 for architectures with a
- * per-layer post-feedforward RMSNorm (OLMo-2, Gemma 3), obtained from g~ with
- * fpo_rmsnorm_vjp at that layer's cached MLP output.  Entries may repeat.
+ * per-layer post-feedforward and / or pre-MLP RMSNorm (OLMo-2, Qwen3, Gemma 3),
+ * obtained from g~ with fpo_layer_signals (or fpo_rmsnorm_vjp at that layer's cached
+ * MLP output).  Entries may repeat.
  */
 int32_t fpo_layer_update_grouped_signals(int32_t n_layers, int64_t T, int64_t d, int64_t d_ff,
                                          int32_t dtype, const void* const* g,
                                          const void* const* A, float lr, float* const* W_master,
                                          void* const* W_out, void* const* G_out, void* workspace,
                                          size_t workspace_bytes, void* stream);
+
+/*
+ * fpo_layer_signals -- the layer-specific signals g~^(l) (Sec. 3.1 step 4; Sec. 3.2 and
+ * the App. E table of norms per model family) for n_layers target layers in one launch
+ * (1 <= n_layers <= FPO_MAX_GROUPED_LAYERS).  For layer l and every token, starting from
+ * the shared signal g (g~ after the final norm's Jacobian, [T, d]):
+ *
+ *   u        = post-FFN RMSNorm VJP of g at m[l] with weight gamma_post[l]   (m given)
+ *   g_out[l] = pre-MLP RMSNorm VJP of u at x[l] with weight gamma_pre[l]     (x given)
+ *
+ * each the expression of fpo_rmsnorm_vjp with its own rho = sqrt(mean x^2 + eps) and
+ * the min-RMS clamp; OLMo-2 composes the post-FFN norm only, Qwen3 the pre-MLP norm
+ * only, Gemma 3 both, in this order.  m[l] is the layer's cached MLP output (the input
+ * of its post-feedforward norm), x[l] the input of its pre-MLP norm (the residual stream
+ * entering the MLP block).  The intermediate u stays in fp32 registers: each row of g,
+ * m[l] and x[l] is read once per layer (rows up to 8192 bf16 elements; longer bf16 rows
+ * and fp32 rows are read in three passes) and g_out[l] written once.
+ *
+ * m, gamma_post, x, gamma_pre and g_out are HOST arrays of n_layers device pointers
+ * ([T, d] rows and [d] weights, all in dtype).  m and gamma_post are both NULL (no
+ * post-FFN norm) or both given, likewise x and gamma_pre, and at least one norm is
+ * given (else FPO_ERR_ARG).  Entries of an input array may repeat; g_out[l] may not
+ * alias g, any input, or another g_out.  bf16 needs d % 8 == 0; every pointer 16-byte
+ * aligned (FPO_ERR_ALIGN).  fp32 accumulation; no workspace; asynchronous on `stream`.
+ */
+int32_t fpo_layer_signals(int32_t n_layers, int64_t T, int64_t d, int32_t dtype, const void* g,
+                          const void* const* m, const void* const* gamma_post,
+                          const void* const* x, const void* const* gamma_pre, float eps,
+                          float min_rms, void* const* g_out, void* stream);
 
 /*
  * fpo_rmsnorm_vjp -- the closed-form RMSNorm Jacobian applied to an upstream

@@ -74,6 +74,9 @@ _lib.fpo_layer_update_grouped_signals.argtypes = [_i32, _i64, _i64, _i64, _i32,
 _lib.fpo_layer_update_grouped_signals.restype = _i32
 _lib.fpo_rmsnorm_vjp.argtypes = [_i64, _i64, _i32, _vp, _vp, _vp, _f32, _f32, _vp, _vp]
 _lib.fpo_rmsnorm_vjp.restype = _i32
+_lib.fpo_layer_signals.argtypes = [_i32, _i64, _i64, _i32, _vp, _vp, _vp, _vp, _vp, _f32, _f32,
+                                   _vp, _vp]
+_lib.fpo_layer_signals.restype = _i32
 
 
 class OptimizerDesc(ctypes.Structure):
@@ -353,6 +356,27 @@ def gate_up_signals(g, W3_init, a, b, dA, dB, *, workspace=None, stream=None):
                                   _stream(stream))
     _check(rc, "fpo_gate_up_signals")
     return workspace
+
+
+def layer_signals(g, g_outs, *, m=None, gamma_post=None, x=None, gamma_pre=None, eps=1e-6,
+                  min_rms=0.5, stream=None):
+    """fpo_layer_signals: g_outs[l] = pre-MLP VJP at x[l] of (post-FFN VJP at m[l] of g);
+    m / gamma_post and x / gamma_pre are lists with one entry per layer, or None."""
+    n = len(g_outs)
+    T, d = g.shape
+
+    def arr(ts):
+        if ts is None:
+            return None
+        if len(ts) != n:
+            raise ValueError("one entry per layer expected")
+        return _ptr_array(ts, n)
+
+    rc = _lib.fpo_layer_signals(n, T, d, _dtype_code(g), _ptr(g), arr(m), arr(gamma_post), arr(x),
+                                arr(gamma_pre), float(eps), float(min_rms), _ptr_array(g_outs, n),
+                                _stream(stream))
+    _check(rc, "fpo_layer_signals")
+    return g_outs
 
 
 def rmsnorm_vjp(g, x, gamma, g_out, *, eps=1e-6, min_rms=0.5, stream=None):

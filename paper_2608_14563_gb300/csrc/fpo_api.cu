@@ -633,9 +633,45 @@ int32_t fpo_rmsnorm_vjp(int64_t T, int64_t d, int32_t dtype, const void* g, cons
     int32_t rc = check_arch();
     if (rc != FPO_OK) return rc;
     if (T == 0) return FPO_OK;
-    return cuda_status(launch_rmsnorm_vjp_at(dtype, g, x, gamma, static_cast<int>(T),
-                                             static_cast<int>(d), eps, min_rms, g_out,
-                                             static_cast<cudaStream_t>(stream)));
+    // one norm of fpo_layer_signals: its pre-MLP stage alone, for one layer
+    const void* xs[1] = {x};
+    const void* gs[1] = {gamma};
+    void* outs[1] = {g_out};
+    return cuda_status(launch_layer_signals(dtype, 1, g, nullptr, nullptr, xs, gs, outs,
+                                            static_cast<int>(T), static_cast<int>(d), eps, min_rms,
+                                            static_cast<cudaStream_t>(stream)));
+}
+
+int32_t fpo_layer_signals(int32_t n_layers, int64_t T, int64_t d, int32_t dtype, const void* g,
+                          const void* const* m, const void* const* gamma_post,
+                          const void* const* x, const void* const* gamma_pre, float eps,
+                          float min_rms, void* const* g_out, void* stream) {
+    if (dtype != FPO_F32 && dtype != FPO_BF16) return FPO_ERR_DTYPE;
+    if (n_layers < 1 || n_layers > FPO_MAX_GROUPED_LAYERS) return FPO_ERR_SHAPE;
+    if (T < 0 || d <= 0 || T > INT_MAX || d > INT_MAX) return FPO_ERR_SHAPE;
+    if (dtype == FPO_BF16 && d % 8 != 0) return FPO_ERR_SHAPE;
+    if (!(eps >= 0.f) || !(min_rms >= 0.f)) return FPO_ERR_ARG;
+    if ((!m) != (!gamma_post) || (!x) != (!gamma_pre) || (!m && !x)) return FPO_ERR_ARG;
+    if (!g_out) return FPO_ERR_NULL;
+    if (T > 0) {
+        if (!g || !aligned16(g)) return g ? FPO_ERR_ALIGN : FPO_ERR_NULL;
+        const void* const* arrays[4] = {m, gamma_post, x, gamma_pre};
+        for (int l = 0; l < n_layers; ++l) {
+            for (const void* const* a : arrays) {
+                if (!a) continue;
+                if (!a[l]) return FPO_ERR_NULL;
+                if (!aligned16(a[l])) return FPO_ERR_ALIGN;
+            }
+            if (!g_out[l]) return FPO_ERR_NULL;
+            if (!aligned16(g_out[l])) return FPO_ERR_ALIGN;
+        }
+    }
+    int32_t rc = check_arch();
+    if (rc != FPO_OK) return rc;
+    if (T == 0) return FPO_OK;
+    return cuda_status(launch_layer_signals(dtype, n_layers, g, m, gamma_post, x, gamma_pre, g_out,
+                                            static_cast<int>(T), static_cast<int>(d), eps, min_rms,
+                                            static_cast<cudaStream_t>(stream)));
 }
 
 int32_t fpo_layer_update(int64_t T, int64_t d, int64_t d_ff, int32_t dtype, const void* g,

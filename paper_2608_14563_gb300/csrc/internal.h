@@ -170,10 +170,12 @@ cudaError_t launch_cast_f32(int dtype, const float* src, size_t n, void* dst, cu
 cudaError_t launch_rmsnorm_vjp(int dtype, const float* g, const void* h, const void* w,
                                const float* rho, int T, int d, float min_rms, void* out,
                                cudaStream_t st);
-// RMSNorm VJP at a norm input x (rho from x itself): out = vjp(g, x, gamma), all in dtype.
-cudaError_t launch_rmsnorm_vjp_at(int dtype, const void* g, const void* x, const void* gamma,
-                                  int T, int d, float eps, float min_rms, void* out,
-                                  cudaStream_t st);
+// Layer-specific signals: out[l] = pre-MLP VJP at x[l] of (post-FFN VJP at m[l] of g), either
+// stage skipped when its array is null (not both); one launch for all layers.
+cudaError_t launch_layer_signals(int dtype, int n_layers, const void* g, const void* const* m,
+                                 const void* const* gamma_post, const void* const* x,
+                                 const void* const* gamma_pre, void* const* out, int T, int d,
+                                 float eps, float min_rms, cudaStream_t st);
 
 // One block waiting on an mbarrier nothing arrives on, bounded by limit_ns.
 cudaError_t launch_wait_timeout(unsigned* status, uint64_t limit_ns, cudaStream_t st);

@@ -12,6 +12,9 @@
 //   mean          mean of a vector in a fixed order (the mean cross-entropy)
 //   rmsnorm_vjp   App. E Eq. (rmsnorm-vjp) with the min-RMS clamp:
 //                 g~ = (w (.) g - xhat <xhat, w (.) g> / d) / max(rho, rho_min)
+//   layer_signal  the same expression at a layer's post-FFN and / or pre-MLP norm,
+//                 composed per target layer (Sec. 3.2); fpo_rmsnorm_vjp runs its
+//                 one-norm form
 //
 // bf16 rows of up to 8192 elements: one block per row, the row kept in registers
 // (each input read once); otherwise one warp per row (two passes over the row),
@@ -158,8 +161,9 @@ __global__ void __launch_bounds__(kRowThreads)
 constexpr int kBlkThreads = 256;
 
 // Block-wide sum of two values; every thread gets both results.
+template <int THREADS = kBlkThreads>
 __device__ __forceinline__ float2 block_sum2(float a, float b) {
-    __shared__ float2 red[kBlkThreads / 32];
+    __shared__ float2 red[THREADS / 32];
     a = warp_sum(a);
     b = warp_sum(b);
     const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
@@ -168,7 +172,7 @@ __device__ __forceinline__ float2 block_sum2(float a, float b) {
     __syncthreads();
     float2 t = make_float2(0.f, 0.f);
 #pragma unroll
-    for (int i = 0; i < kBlkThreads / 32; ++i) {
+    for (int i = 0; i < THREADS / 32; ++i) {
         t.x += red[i].x;
         t.y += red[i].y;
     }
@@ -287,58 +291,6 @@ __global__ void __launch_bounds__(kBlkThreads)
     }
 }
 
-template <int EPT>
-__global__ void __launch_bounds__(kBlkThreads)
-    rmsnorm_vjp_at_row_kernel(const __nv_bfloat16* __restrict__ g,
-                              const __nv_bfloat16* __restrict__ x,
-                              const __nv_bfloat16* __restrict__ gamma, int T, int d, float eps,
-                              float min_rms, __nv_bfloat16* __restrict__ out) {
-    constexpr int NV = EPT / 8;
-    for (int row = blockIdx.x; row < T; row += gridDim.x) {
-        const __nv_bfloat16* gr = g + static_cast<size_t>(row) * d;
-        const __nv_bfloat16* xr = x + static_cast<size_t>(row) * d;
-        float wg[EPT], xv[EPT];
-        float ss = 0.f, xg = 0.f;
-#pragma unroll
-        for (int v = 0; v < NV; ++v) {
-            const int k = (v * kBlkThreads + threadIdx.x) * 8;
-            float gv[8], xx[8], wv[8];
-            if (k < d) {
-                ld_vec<8>(gr + k, gv);
-                ld_vec<8>(xr + k, xx);
-                ld_vec<8>(gamma + k, wv);
-            } else {
-#pragma unroll
-                for (int q = 0; q < 8; ++q) gv[q] = xx[q] = wv[q] = 0.f;
-            }
-#pragma unroll
-            for (int q = 0; q < 8; ++q) {
-                wg[8 * v + q] = wv[q] * gv[q];
-                xv[8 * v + q] = xx[q];
-                ss = fmaf(xx[q], xx[q], ss);
-                xg = fmaf(xx[q], wg[8 * v + q], xg);
-            }
-        }
-        const float2 sums = block_sum2(ss, xg);
-        const float r = sqrtf(sums.x / static_cast<float>(d) + eps);
-        const float inv_r = 1.0f / r;
-        const float kd = (sums.y * inv_r) / static_cast<float>(d);
-        const float pref = 1.0f / fmaxf(r, min_rms);
-        __nv_bfloat16* orow = out + static_cast<size_t>(row) * d;
-#pragma unroll
-        for (int v = 0; v < NV; ++v) {
-            const int k = (v * kBlkThreads + threadIdx.x) * 8;
-            if (k < d) {
-                float o[8];
-#pragma unroll
-                for (int q = 0; q < 8; ++q)
-                    o[q] = (wg[8 * v + q] - (xv[8 * v + q] * inv_r) * kd) * pref;
-                st_vec<8>(orow + k, o);
-            }
-        }
-    }
-}
-
 // Elements per thread of the block-per-row kernels for a bf16 row of d, or 0 when
 // the row does not fit (the warp-per-row kernels take it).
 int row_ept(int d) {
@@ -386,49 +338,6 @@ __global__ void __launch_bounds__(kRowThreads)
             ld_vec<VEC>(w + j, wv);
 #pragma unroll
             for (int k = 0; k < VEC; ++k) o[k] = (wv[k] * gv[k] - (x[k] * inv_r) * kd) * pref;
-            st_vec<VEC>(orow + j, o);
-        }
-    }
-}
-
-// RMSNorm VJP at a norm input x whose rho is recomputed from x: one pass for
-// sum x^2 and sum x gamma g, then the output pass (App. E Eq. rmsnorm-vjp).
-template <typename TT, int VEC>
-__global__ void __launch_bounds__(kRowThreads)
-    rmsnorm_vjp_at_kernel(const TT* __restrict__ g, const TT* __restrict__ x,
-                          const TT* __restrict__ gamma, int T, int d, float eps, float min_rms,
-                          TT* __restrict__ out) {
-    const int lane = threadIdx.x & 31;
-    const int wpb = blockDim.x >> 5;
-    for (int row = blockIdx.x * wpb + (threadIdx.x >> 5); row < T; row += gridDim.x * wpb) {
-        const TT* gr = g + static_cast<size_t>(row) * d;
-        const TT* xr = x + static_cast<size_t>(row) * d;
-        float ss = 0.f, xg = 0.f;
-        for (int j = lane * VEC; j < d; j += 32 * VEC) {
-            float gv[VEC], xv[VEC], wv[VEC];
-            ld_vec<VEC>(gr + j, gv);
-            ld_vec<VEC>(xr + j, xv);
-            ld_vec<VEC>(gamma + j, wv);
-#pragma unroll
-            for (int k = 0; k < VEC; ++k) {
-                ss = fmaf(xv[k], xv[k], ss);
-                xg = fmaf(xv[k], wv[k] * gv[k], xg);
-            }
-        }
-        ss = warp_sum(ss);
-        xg = warp_sum(xg);
-        const float r = sqrtf(ss / static_cast<float>(d) + eps);
-        const float inv_r = 1.0f / r;
-        const float kd = (xg * inv_r) / static_cast<float>(d);
-        const float pref = 1.0f / fmaxf(r, min_rms);
-        TT* orow = out + static_cast<size_t>(row) * d;
-        for (int j = lane * VEC; j < d; j += 32 * VEC) {
-            float gv[VEC], xv[VEC], wv[VEC], o[VEC];
-            ld_vec<VEC>(gr + j, gv);
-            ld_vec<VEC>(xr + j, xv);
-            ld_vec<VEC>(gamma + j, wv);
-#pragma unroll
-            for (int k = 0; k < VEC; ++k) o[k] = (wv[k] * gv[k] - (xv[k] * inv_r) * kd) * pref;
             st_vec<VEC>(orow + j, o);
         }
     }
@@ -687,6 +596,282 @@ __global__ void wait_timeout_kernel(unsigned* status, unsigned long long limit_n
     }
 }
 
+// ---------------------------------------------------------------------------
+// Layer-specific signals (Sec. 3.1 step 4, Sec. 3.2, App. E): for target layer l and
+// token t, the shared signal g (after the final norm's Jacobian) composed with the
+// post-feedforward RMSNorm Jacobian at m_l, then with the pre-MLP one at x_l:
+//   u   = (gp (.) g - mhat <mhat, gp (.) g> / d) / max(rho_m, rho_min)    (POST)
+//   out = (gq (.) u - xhat <xhat, gq (.) u> / d) / max(rho_x, rho_min)    (PRE)
+// Each stage's sums in fp32; u stays in registers (fp32) between the stages.  Grid y
+// runs over the layers.
+constexpr int kSigThreads = 256;  // block size of the block-per-row kernel (512: slower)
+
+struct LayerSignalPtrs {
+    const void* m[kNrMaxLayers];
+    const void* gp[kNrMaxLayers];
+    const void* x[kNrMaxLayers];
+    const void* gq[kNrMaxLayers];
+    void* out[kNrMaxLayers];
+};
+
+// Block-wide sums of N values (warp butterflies, then the warps' partials in order).
+template <int N, int THREADS>
+__device__ __forceinline__ void block_sum_n(float (&v)[N]) {
+    __shared__ float red[THREADS / 32][N];
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+#pragma unroll
+    for (int i = 0; i < N; ++i) v[i] = warp_sum(v[i]);
+    __syncthreads();  // the previous call's readers are done with red
+    if (lane == 0) {
+#pragma unroll
+        for (int i = 0; i < N; ++i) red[wid][i] = v[i];
+    }
+    __syncthreads();
+#pragma unroll
+    for (int i = 0; i < N; ++i) {
+        float t = 0.f;
+#pragma unroll
+        for (int w = 0; w < THREADS / 32; ++w) t += red[w][i];
+        v[i] = t;
+    }
+}
+
+// This thread's NV 16-byte vectors of a bf16 row (elements (v THREADS + tid) 8 ..),
+// zeros past d; converted to fp32 only where used, so that every row the block needs is
+// in flight at once.
+template <int NV, int THREADS>
+__device__ __forceinline__ void ld_row_raw(const __nv_bfloat16* __restrict__ p, int d,
+                                           uint4 (&r)[NV]) {
+#pragma unroll
+    for (int v = 0; v < NV; ++v) {
+        const int k = (v * THREADS + threadIdx.x) * 8;
+        r[v] = k < d ? __ldg(reinterpret_cast<const uint4*>(p + k)) : make_uint4(0u, 0u, 0u, 0u);
+    }
+}
+
+__device__ __forceinline__ void raw_to_f32(const uint4& a, float (&v)[8]) {
+    const __nv_bfloat162* h2 = reinterpret_cast<const __nv_bfloat162*>(&a);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const float2 f = __bfloat1622float2(h2[k]);
+        v[2 * k] = f.x;
+        v[2 * k + 1] = f.y;
+    }
+}
+
+// One Jacobian stage on a register-held row (block per row): u <- VJP of u at the norm
+// input row xr with weight gam (both as loaded).
+template <int NV, int THREADS>
+__device__ __forceinline__ void vjp_stage_row(float (&u)[NV * 8], const uint4 (&xr)[NV],
+                                              const uint4 (&gam)[NV], int d, float eps,
+                                              float min_rms) {
+    float ss = 0.f, xg = 0.f;
+#pragma unroll
+    for (int v = 0; v < NV; ++v) {
+        float xx[8], wv[8];
+        raw_to_f32(xr[v], xx);
+        raw_to_f32(gam[v], wv);
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+            u[8 * v + q] *= wv[q];  // gamma (.) u
+            ss = fmaf(xx[q], xx[q], ss);
+            xg = fmaf(xx[q], u[8 * v + q], xg);
+        }
+    }
+    const float2 sums = block_sum2<THREADS>(ss, xg);
+    const float r = sqrtf(sums.x / static_cast<float>(d) + eps);
+    const float inv_r = 1.0f / r;
+    const float kd = (sums.y * inv_r) / static_cast<float>(d);
+    const float pref = 1.0f / fmaxf(r, min_rms);
+#pragma unroll
+    for (int v = 0; v < NV; ++v) {
+        float xx[8];
+        raw_to_f32(xr[v], xx);
+#pragma unroll
+        for (int q = 0; q < 8; ++q) u[8 * v + q] = (u[8 * v + q] - (xx[q] * inv_r) * kd) * pref;
+    }
+}
+
+template <int EPT, int THREADS, bool POST, bool PRE>
+__global__ void __launch_bounds__(THREADS)
+    layer_signal_row_kernel(const __nv_bfloat16* __restrict__ g,
+                            const __grid_constant__ LayerSignalPtrs p, int T, int d, float eps,
+                            float min_rms) {
+    constexpr int NV = EPT / 8;
+    const int l = blockIdx.y;
+    const auto* m = static_cast<const __nv_bfloat16*>(p.m[l]);
+    const auto* x = static_cast<const __nv_bfloat16*>(p.x[l]);
+    auto* out = static_cast<__nv_bfloat16*>(p.out[l]);
+    uint4 gp[NV], gq[NV];  // the layer's norm weights, loaded once
+    if constexpr (POST) ld_row_raw<NV, THREADS>(static_cast<const __nv_bfloat16*>(p.gp[l]), d, gp);
+    if constexpr (PRE) ld_row_raw<NV, THREADS>(static_cast<const __nv_bfloat16*>(p.gq[l]), d, gq);
+    for (int row = blockIdx.x; row < T; row += gridDim.x) {
+        const size_t off = static_cast<size_t>(row) * d;
+        uint4 graw[NV], mraw[NV], xraw[NV];
+        ld_row_raw<NV, THREADS>(g + off, d, graw);
+        if constexpr (POST) ld_row_raw<NV, THREADS>(m + off, d, mraw);
+        if constexpr (PRE) ld_row_raw<NV, THREADS>(x + off, d, xraw);
+        float u[EPT];
+        if constexpr (POST && PRE) {
+            // Both stages from one block reduction: with a = gp (.) g and
+            // u = (a - m inv1 kd1) pref1, the pre-MLP stage's sum <x, gq (.) u> is
+            // pref1 (<x gq, a> - inv1 kd1 <x gq, m>), so all five sums are taken in one
+            // pass over the loaded rows (one barrier round per row instead of two).
+            float s5[5] = {0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+            for (int v = 0; v < NV; ++v) {
+                float gv[8], mv[8], xv[8], wp[8], wq[8];
+                raw_to_f32(graw[v], gv);
+                raw_to_f32(mraw[v], mv);
+                raw_to_f32(xraw[v], xv);
+                raw_to_f32(gp[v], wp);
+                raw_to_f32(gq[v], wq);
+#pragma unroll
+                for (int q = 0; q < 8; ++q) {
+                    const float a = wp[q] * gv[q], b = xv[q] * wq[q];
+                    s5[0] = fmaf(mv[q], mv[q], s5[0]);
+                    s5[1] = fmaf(mv[q], a, s5[1]);
+                    s5[2] = fmaf(xv[q], xv[q], s5[2]);
+                    s5[3] = fmaf(b, a, s5[3]);
+                    s5[4] = fmaf(b, mv[q], s5[4]);
+                }
+            }
+            block_sum_n<5, THREADS>(s5);
+            const float r1 = sqrtf(s5[0] / static_cast<float>(d) + eps);
+            const float inv1 = 1.0f / r1;
+            const float kd1 = (s5[1] * inv1) / static_cast<float>(d);
+            const float pref1 = 1.0f / fmaxf(r1, min_rms);
+            const float r2 = sqrtf(s5[2] / static_cast<float>(d) + eps);
+            const float inv2 = 1.0f / r2;
+            const float xu = pref1 * (s5[3] - (inv1 * kd1) * s5[4]);
+            const float kd2 = (xu * inv2) / static_cast<float>(d);
+            const float pref2 = 1.0f / fmaxf(r2, min_rms);
+#pragma unroll
+            for (int v = 0; v < NV; ++v) {
+                float gv[8], mv[8], xv[8], wp[8], wq[8];
+                raw_to_f32(graw[v], gv);
+                raw_to_f32(mraw[v], mv);
+                raw_to_f32(xraw[v], xv);
+                raw_to_f32(gp[v], wp);
+                raw_to_f32(gq[v], wq);
+                float o[8];
+#pragma unroll
+                for (int q = 0; q < 8; ++q) {
+                    const float uq = (wp[q] * gv[q] - (mv[q] * inv1) * kd1) * pref1;
+                    o[q] = (wq[q] * uq - (xv[q] * inv2) * kd2) * pref2;
+                }
+                const int k = (v * THREADS + threadIdx.x) * 8;
+                if (k < d) st_vec<8>(out + off + k, o);
+            }
+            continue;
+        } else {
+#pragma unroll
+            for (int v = 0; v < NV; ++v) {
+                float gv[8];
+                raw_to_f32(graw[v], gv);
+#pragma unroll
+                for (int q = 0; q < 8; ++q) u[8 * v + q] = gv[q];
+            }
+            if constexpr (POST) vjp_stage_row<NV, THREADS>(u, mraw, gp, d, eps, min_rms);
+            if constexpr (PRE) vjp_stage_row<NV, THREADS>(u, xraw, gq, d, eps, min_rms);
+        }
+#pragma unroll
+        for (int v = 0; v < NV; ++v) {
+            const int k = (v * THREADS + threadIdx.x) * 8;
+            if (k < d) {
+                float o[8];
+#pragma unroll
+                for (int q = 0; q < 8; ++q) o[q] = u[8 * v + q];
+                st_vec<8>(out + off + k, o);
+            }
+        }
+    }
+}
+
+// Rows too long for registers, and fp32: one warp per row, three passes over the row
+// (the post-FFN sums; the pre-MLP sums over u recomputed elementwise; the output).
+template <typename TT, int VEC, bool POST, bool PRE>
+__global__ void __launch_bounds__(kRowThreads)
+    layer_signal_kernel(const TT* __restrict__ g, const __grid_constant__ LayerSignalPtrs p, int T,
+                        int d, float eps, float min_rms) {
+    const int l = blockIdx.y;
+    const TT* m = static_cast<const TT*>(p.m[l]);
+    const TT* gp = static_cast<const TT*>(p.gp[l]);
+    const TT* x = static_cast<const TT*>(p.x[l]);
+    const TT* gq = static_cast<const TT*>(p.gq[l]);
+    TT* out = static_cast<TT*>(p.out[l]);
+    const int lane = threadIdx.x & 31;
+    const int wpb = blockDim.x >> 5;
+    for (int row = blockIdx.x * wpb + (threadIdx.x >> 5); row < T; row += gridDim.x * wpb) {
+        const size_t off = static_cast<size_t>(row) * d;
+        float inv1 = 0.f, kd1 = 0.f, pref1 = 1.f;
+        if constexpr (POST) {
+            float ss = 0.f, mg = 0.f;
+            for (int j = lane * VEC; j < d; j += 32 * VEC) {
+                float gv[VEC], mv[VEC], wv[VEC];
+                ld_vec<VEC>(g + off + j, gv);
+                ld_vec<VEC>(m + off + j, mv);
+                ld_vec<VEC>(gp + j, wv);
+#pragma unroll
+                for (int k = 0; k < VEC; ++k) {
+                    ss = fmaf(mv[k], mv[k], ss);
+                    mg = fmaf(mv[k], wv[k] * gv[k], mg);
+                }
+            }
+            ss = warp_sum(ss);
+            mg = warp_sum(mg);
+            const float r = sqrtf(ss / static_cast<float>(d) + eps);
+            inv1 = 1.0f / r;
+            kd1 = (mg * inv1) / static_cast<float>(d);
+            pref1 = 1.0f / fmaxf(r, min_rms);
+        }
+        // u at elements j .. j + VEC - 1 (the post-FFN stage, or g itself)
+        auto u_at = [&](int j, float (&u)[VEC]) {
+            ld_vec<VEC>(g + off + j, u);
+            if constexpr (POST) {
+                float mv[VEC], wv[VEC];
+                ld_vec<VEC>(m + off + j, mv);
+                ld_vec<VEC>(gp + j, wv);
+#pragma unroll
+                for (int k = 0; k < VEC; ++k) u[k] = (wv[k] * u[k] - (mv[k] * inv1) * kd1) * pref1;
+            }
+        };
+        float inv2 = 0.f, kd2 = 0.f, pref2 = 1.f;
+        if constexpr (PRE) {
+            float ss = 0.f, xu = 0.f;
+            for (int j = lane * VEC; j < d; j += 32 * VEC) {
+                float u[VEC], xv[VEC], wv[VEC];
+                u_at(j, u);
+                ld_vec<VEC>(x + off + j, xv);
+                ld_vec<VEC>(gq + j, wv);
+#pragma unroll
+                for (int k = 0; k < VEC; ++k) {
+                    ss = fmaf(xv[k], xv[k], ss);
+                    xu = fmaf(xv[k], wv[k] * u[k], xu);
+                }
+            }
+            ss = warp_sum(ss);
+            xu = warp_sum(xu);
+            const float r = sqrtf(ss / static_cast<float>(d) + eps);
+            inv2 = 1.0f / r;
+            kd2 = (xu * inv2) / static_cast<float>(d);
+            pref2 = 1.0f / fmaxf(r, min_rms);
+        }
+        for (int j = lane * VEC; j < d; j += 32 * VEC) {
+            float u[VEC];
+            u_at(j, u);
+            if constexpr (PRE) {
+                float xv[VEC], wv[VEC];
+                ld_vec<VEC>(x + off + j, xv);
+                ld_vec<VEC>(gq + j, wv);
+#pragma unroll
+                for (int k = 0; k < VEC; ++k) u[k] = (wv[k] * u[k] - (xv[k] * inv2) * kd2) * pref2;
+            }
+            st_vec<VEC>(out + off + j, u);
+        }
+    }
+}
+
 int row_grid(int T) {
     DevInfo di;
     const int sms = current_device_info(&di) ? di.sm_count : 148;
@@ -850,46 +1035,71 @@ cudaError_t launch_wait_timeout(unsigned* status, uint64_t limit_ns, cudaStream_
     return cudaGetLastError();
 }
 
-cudaError_t launch_rmsnorm_vjp_at(int dtype, const void* g, const void* x, const void* gamma,
-                                  int T, int d, float eps, float min_rms, void* out,
-                                  cudaStream_t st) {
-    if (T <= 0) return cudaSuccess;
-    const int grid = row_grid(T);
-    const int ept = dtype == 1 ? row_ept(d) : 0;
+namespace {
+
+template <bool POST, bool PRE>
+cudaError_t run_layer_signals(int dtype, int n_layers, const void* g, const LayerSignalPtrs& p,
+                              int T, int d, float eps, float min_rms, cudaStream_t st) {
+    DevInfo di;
+    const int sms = current_device_info(&di) ? di.sm_count : 148;
+    const int per_layer = (sms * 8 + n_layers - 1) / n_layers;  // ~8 blocks per SM in all
+    // bf16 rows up to 32 x kSigThreads elements: block per row, the rows in registers
+    const int ept = dtype != 1             ? 0
+                    : d <= 8 * kSigThreads  ? 8
+                    : d <= 16 * kSigThreads ? 16
+                    : d <= 32 * kSigThreads ? 32
+                                            : 0;
     if (ept) {
+        const dim3 grid(static_cast<unsigned>(T < per_layer ? T : per_layer),
+                        static_cast<unsigned>(n_layers));
         const auto* gg = static_cast<const __nv_bfloat16*>(g);
-        const auto* xx = static_cast<const __nv_bfloat16*>(x);
-        const auto* ga = static_cast<const __nv_bfloat16*>(gamma);
-        auto* oo = static_cast<__nv_bfloat16*>(out);
         if (ept == 8)
-            rmsnorm_vjp_at_row_kernel<8><<<blk_grid(T), kBlkThreads, 0, st>>>(gg, xx, ga, T, d, eps,
-                                                                           min_rms, oo),
-                ::fpo::note_launch();
+            layer_signal_row_kernel<8, kSigThreads, POST, PRE><<<grid, kSigThreads, 0, st>>>(
+                gg, p, T, d, eps, min_rms);
         else if (ept == 16)
-            rmsnorm_vjp_at_row_kernel<16><<<blk_grid(T), kBlkThreads, 0, st>>>(gg, xx, ga, T, d,
-                                                                            eps, min_rms, oo),
-                ::fpo::note_launch();
+            layer_signal_row_kernel<16, kSigThreads, POST, PRE><<<grid, kSigThreads, 0, st>>>(
+                gg, p, T, d, eps, min_rms);
         else
-            rmsnorm_vjp_at_row_kernel<32><<<blk_grid(T), kBlkThreads, 0, st>>>(gg, xx, ga, T, d,
-                                                                            eps, min_rms, oo),
-                ::fpo::note_launch();
-    } else if (dtype == 1) {
-        rmsnorm_vjp_at_kernel<__nv_bfloat16, 8><<<grid, kRowThreads, 0, st>>>(
-            static_cast<const __nv_bfloat16*>(g), static_cast<const __nv_bfloat16*>(x),
-            static_cast<const __nv_bfloat16*>(gamma), T, d, eps, min_rms,
-            static_cast<__nv_bfloat16*>(out)), ::fpo::note_launch();
-    } else if (d % 4 == 0) {
-        rmsnorm_vjp_at_kernel<float, 4><<<grid, kRowThreads, 0, st>>>(
-            static_cast<const float*>(g), static_cast<const float*>(x),
-            static_cast<const float*>(gamma), T, d, eps, min_rms, static_cast<float*>(out)),
-            ::fpo::note_launch();
+            layer_signal_row_kernel<32, kSigThreads, POST, PRE><<<grid, kSigThreads, 0, st>>>(
+                gg, p, T, d, eps, min_rms);
     } else {
-        rmsnorm_vjp_at_kernel<float, 1><<<grid, kRowThreads, 0, st>>>(
-            static_cast<const float*>(g), static_cast<const float*>(x),
-            static_cast<const float*>(gamma), T, d, eps, min_rms, static_cast<float*>(out)),
-            ::fpo::note_launch();
+        const int wpb = kRowThreads / 32;
+        const int need = (T + wpb - 1) / wpb;
+        const dim3 grid(static_cast<unsigned>(need < per_layer ? need : per_layer),
+                        static_cast<unsigned>(n_layers));
+        if (dtype == 1)
+            layer_signal_kernel<__nv_bfloat16, 8, POST, PRE><<<grid, kRowThreads, 0, st>>>(
+                static_cast<const __nv_bfloat16*>(g), p, T, d, eps, min_rms);
+        else if (d % 4 == 0)
+            layer_signal_kernel<float, 4, POST, PRE><<<grid, kRowThreads, 0, st>>>(
+                static_cast<const float*>(g), p, T, d, eps, min_rms);
+        else
+            layer_signal_kernel<float, 1, POST, PRE><<<grid, kRowThreads, 0, st>>>(
+                static_cast<const float*>(g), p, T, d, eps, min_rms);
     }
+    ::fpo::note_launch();
     return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_layer_signals(int dtype, int n_layers, const void* g, const void* const* m,
+                                 const void* const* gamma_post, const void* const* x,
+                                 const void* const* gamma_pre, void* const* out, int T, int d,
+                                 float eps, float min_rms, cudaStream_t st) {
+    if (n_layers < 1 || n_layers > kNrMaxLayers || (!m && !x)) return cudaErrorInvalidValue;
+    if (T <= 0) return cudaSuccess;
+    LayerSignalPtrs p{};
+    for (int l = 0; l < n_layers; ++l) {
+        p.m[l] = m ? m[l] : nullptr;
+        p.gp[l] = m ? gamma_post[l] : nullptr;
+        p.x[l] = x ? x[l] : nullptr;
+        p.gq[l] = x ? gamma_pre[l] : nullptr;
+        p.out[l] = out[l];
+    }
+    if (m && x) return run_layer_signals<true, true>(dtype, n_layers, g, p, T, d, eps, min_rms, st);
+    if (m) return run_layer_signals<true, false>(dtype, n_layers, g, p, T, d, eps, min_rms, st);
+    return run_layer_signals<false, true>(dtype, n_layers, g, p, T, d, eps, min_rms, st);
 }
 
 cudaError_t launch_lse_combine(const float2* part, int n_tiles, int T, const float* zy, float* lse,

@@ -35,7 +35,7 @@ from dataclasses import dataclass, field
 import torch
 
 _TENSOR_IDS = {"h": 1, "w": 2, "W_U": 3, "A": 4, "W": 5, "y": 6, "noise": 7, "m": 8, "gp": 9,
-               "x": 10, "W1": 11, "W2": 12}
+               "x": 10, "W1": 11, "W2": 12, "xpre": 13, "gq": 14}
 
 
 @dataclass(frozen=True)
@@ -171,6 +171,23 @@ def make_mlp_out(wl: Workload, layer: int, device="cpu"):
 
 def make_post_norm_w(wl: Workload, layer: int, device="cpu"):
     return normal((wl.d,), std=0.05, mean=0.3, seed=wl.seed, tensor="gp", layer=layer,
+                  device=device, dtype=wl.torch_dtype)
+
+
+def make_pre_norm_in(wl: Workload, layer: int, device="cpu"):
+    """Input of a layer's pre-MLP RMSNorm (the residual stream entering the MLP block):
+    rows of log-normal scale around RMS 1, every 64th row (offset 32) at RMS ~0.2 so that
+    the min-RMS clamp acts on some tokens."""
+    g = _gen(wl.seed, "xpre", layer, device)
+    x = torch.randn((wl.T, wl.d), generator=g, device=device, dtype=torch.float32)
+    scale = torch.exp(0.3 * torch.randn((wl.T, 1), generator=g, device=device,
+                                        dtype=torch.float32))
+    scale[32::64] = 0.2
+    return (x * scale).to(wl.torch_dtype)
+
+
+def make_pre_norm_w(wl: Workload, layer: int, device="cpu"):
+    return normal((wl.d,), std=0.1, mean=1.0, seed=wl.seed, tensor="gq", layer=layer,
                   device=device, dtype=wl.torch_dtype)
 
 
