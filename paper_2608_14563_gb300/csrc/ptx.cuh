@@ -178,6 +178,21 @@ __device__ __forceinline__ void tma_load_2d_pair(const CUtensorMap* map, uint32_
         : "memory");
 }
 
+// 16-byte global -> shared copy (cp.async, L2 only), grouped per thread with
+// cp_async_commit and awaited with cp_async_wait<N> (at most N of this thread's groups
+// still pending); no mbarrier is involved.
+__device__ __forceinline__ void cp_async16(uint32_t smem_dst, const void* gmem_src) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_dst), "l"(gmem_src)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+    asm volatile("cp.async.commit_group;" ::: "memory");
+}
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
 // Complete `bytes` of the current phase's expected transaction count of an mbarrier
 // of this CTA without a copy (the accounting of a copy that will never be issued).
 __device__ __forceinline__ void mbar_complete_tx(uint32_t bar, uint32_t bytes) {

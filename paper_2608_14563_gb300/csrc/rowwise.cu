@@ -602,8 +602,8 @@ __global__ void wait_timeout_kernel(unsigned* status, unsigned long long limit_n
 // post-feedforward RMSNorm Jacobian at m_l, then with the pre-MLP one at x_l:
 //   u   = (gp (.) g - mhat <mhat, gp (.) g> / d) / max(rho_m, rho_min)    (POST)
 //   out = (gq (.) u - xhat <xhat, gq (.) u> / d) / max(rho_x, rho_min)    (PRE)
-// Each stage's sums in fp32; u stays in registers (fp32) between the stages.  Grid y
-// runs over the layers.
+// Each stage's sums in fp32; u stays in registers (fp32) between the stages.  Grid x
+// runs over the layers, grid y over the rows.
 constexpr int kSigThreads = 256;  // block size of the block-per-row kernel (512: slower)
 
 struct LayerSignalPtrs {
@@ -659,83 +659,152 @@ __device__ __forceinline__ void raw_to_f32(const uint4& a, float (&v)[8]) {
     }
 }
 
+// Elements 2k, 2k + 1 of a loaded 16-byte bf16 vector as a float pair.
+__device__ __forceinline__ float2 bf16x2_at(const uint4& a, int k) {
+    const uint32_t w = k == 0 ? a.x : k == 1 ? a.y : k == 2 ? a.z : a.w;
+    return make_float2(__uint_as_float(w << 16), __uint_as_float(w & 0xffff0000u));
+}
+
 // One Jacobian stage on a register-held row (block per row): u <- VJP of u at the norm
-// input row xr with weight gam (both as loaded).
+// input row xr with weight gam (both as loaded), in packed f32x2 arithmetic:
+//   a = gam (.) u,  sums <x, x>, <x, a>;  u = a pref - x (inv_r kd pref)
 template <int NV, int THREADS>
 __device__ __forceinline__ void vjp_stage_row(float (&u)[NV * 8], const uint4 (&xr)[NV],
                                               const uint4 (&gam)[NV], int d, float eps,
                                               float min_rms) {
-    float ss = 0.f, xg = 0.f;
+    float2 sxx = make_float2(0.f, 0.f), sxa = make_float2(0.f, 0.f);
 #pragma unroll
     for (int v = 0; v < NV; ++v) {
-        float xx[8], wv[8];
-        raw_to_f32(xr[v], xx);
-        raw_to_f32(gam[v], wv);
 #pragma unroll
-        for (int q = 0; q < 8; ++q) {
-            u[8 * v + q] *= wv[q];  // gamma (.) u
-            ss = fmaf(xx[q], xx[q], ss);
-            xg = fmaf(xx[q], u[8 * v + q], xg);
+        for (int k = 0; k < 4; ++k) {
+            const float2 x2 = bf16x2_at(xr[v], k);
+            const float2 a2 = __fmul2_rn(bf16x2_at(gam[v], k), make_float2(u[8 * v + 2 * k],
+                                                                           u[8 * v + 2 * k + 1]));
+            u[8 * v + 2 * k] = a2.x;
+            u[8 * v + 2 * k + 1] = a2.y;
+            sxx = __ffma2_rn(x2, x2, sxx);
+            sxa = __ffma2_rn(x2, a2, sxa);
         }
     }
-    const float2 sums = block_sum2<THREADS>(ss, xg);
+    const float2 sums = block_sum2<THREADS>(sxx.x + sxx.y, sxa.x + sxa.y);
     const float r = sqrtf(sums.x / static_cast<float>(d) + eps);
     const float inv_r = 1.0f / r;
     const float kd = (sums.y * inv_r) / static_cast<float>(d);
     const float pref = 1.0f / fmaxf(r, min_rms);
+    const float2 P = make_float2(pref, pref);
+    const float nc = -(inv_r * kd) * pref;
+    const float2 NC = make_float2(nc, nc);
 #pragma unroll
     for (int v = 0; v < NV; ++v) {
-        float xx[8];
-        raw_to_f32(xr[v], xx);
 #pragma unroll
-        for (int q = 0; q < 8; ++q) u[8 * v + q] = (u[8 * v + q] - (xx[q] * inv_r) * kd) * pref;
+        for (int k = 0; k < 4; ++k) {
+            const float2 o = __ffma2_rn(make_float2(u[8 * v + 2 * k], u[8 * v + 2 * k + 1]), P,
+                                        __fmul2_rn(bf16x2_at(xr[v], k), NC));
+            u[8 * v + 2 * k] = o.x;
+            u[8 * v + 2 * k + 1] = o.y;
+        }
     }
 }
 
+// Stages of rows in flight per block of the block-per-row kernel (shared memory:
+// kSigStages x (1 + POST + PRE) rows of d bf16).
+constexpr int kSigStages = 3;
+
+// Block per (row, layer), the rows staged in shared memory by cp.async kSigStages - 1
+// rows ahead of the one being computed (each thread copies, then reads, the same
+// 16-byte chunks, so its own cp.async.wait_group is all the synchronisation the staging
+// needs).  The layer's norm weights are held in registers.
 template <int EPT, int THREADS, bool POST, bool PRE>
 __global__ void __launch_bounds__(THREADS)
     layer_signal_row_kernel(const __nv_bfloat16* __restrict__ g,
                             const __grid_constant__ LayerSignalPtrs p, int T, int d, float eps,
                             float min_rms) {
     constexpr int NV = EPT / 8;
-    const int l = blockIdx.y;
+    constexpr int NT = 1 + (POST ? 1 : 0) + (PRE ? 1 : 0);  // staged rows per token
+    extern __shared__ __align__(128) uint8_t sig_smem[];
+    const int l = blockIdx.x;  // layers fastest: the blocks of all layers of a row are
+                               // resident together and share its g row in L2
     const auto* m = static_cast<const __nv_bfloat16*>(p.m[l]);
     const auto* x = static_cast<const __nv_bfloat16*>(p.x[l]);
     auto* out = static_cast<__nv_bfloat16*>(p.out[l]);
     uint4 gp[NV], gq[NV];  // the layer's norm weights, loaded once
     if constexpr (POST) ld_row_raw<NV, THREADS>(static_cast<const __nv_bfloat16*>(p.gp[l]), d, gp);
     if constexpr (PRE) ld_row_raw<NV, THREADS>(static_cast<const __nv_bfloat16*>(p.gq[l]), d, gq);
-    for (int row = blockIdx.x; row < T; row += gridDim.x) {
+    const uint32_t sbase = smem_u32(sig_smem);
+    const uint32_t row_bytes = static_cast<uint32_t>(d) * 2u;  // a multiple of 16
+    auto stage_row = [&](int s, int t) { return sbase + static_cast<uint32_t>(s * NT + t) * row_bytes; };
+    auto copy_row = [&](uint32_t dst, const __nv_bfloat16* src) {
+#pragma unroll
+        for (int v = 0; v < NV; ++v) {
+            const int k = (v * THREADS + threadIdx.x) * 8;
+            if (k < d) cp_async16(dst + static_cast<uint32_t>(k) * 2u, src + k);
+        }
+    };
+    auto issue = [&](int row, int s) {
+        const size_t off = static_cast<size_t>(row) * d;
+        copy_row(stage_row(s, 0), g + off);
+        if constexpr (POST) copy_row(stage_row(s, 1), m + off);
+        if constexpr (PRE) copy_row(stage_row(s, NT - 1), x + off);
+    };
+    auto read_row = [&](uint32_t src, uint4 (&r)[NV]) {
+#pragma unroll
+        for (int v = 0; v < NV; ++v) {
+            const int k = (v * THREADS + threadIdx.x) * 8;
+            if (k < d) {
+                asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+                             : "=r"(r[v].x), "=r"(r[v].y), "=r"(r[v].z), "=r"(r[v].w)
+                             : "r"(src + static_cast<uint32_t>(k) * 2u)
+                             : "memory");
+            } else {
+                r[v] = make_uint4(0u, 0u, 0u, 0u);
+            }
+        }
+    };
+    const int G = gridDim.y;
+#pragma unroll
+    for (int s = 0; s < kSigStages - 1; ++s) {
+        const int r = blockIdx.y + s * G;
+        if (r < T) issue(r, s);
+        cp_async_commit();
+    }
+    int k_it = 0;
+    for (int row = blockIdx.y; row < T; row += G, ++k_it) {
+        const int rn = row + (kSigStages - 1) * G;
+        if (rn < T) issue(rn, (k_it + kSigStages - 1) % kSigStages);
+        cp_async_commit();
+        cp_async_wait<kSigStages - 1>();  // this thread's copies of `row` have landed
+        const int s = k_it % kSigStages;
         const size_t off = static_cast<size_t>(row) * d;
         uint4 graw[NV], mraw[NV], xraw[NV];
-        ld_row_raw<NV, THREADS>(g + off, d, graw);
-        if constexpr (POST) ld_row_raw<NV, THREADS>(m + off, d, mraw);
-        if constexpr (PRE) ld_row_raw<NV, THREADS>(x + off, d, xraw);
+        read_row(stage_row(s, 0), graw);
+        if constexpr (POST) read_row(stage_row(s, 1), mraw);
+        if constexpr (PRE) read_row(stage_row(s, NT - 1), xraw);
         float u[EPT];
         if constexpr (POST && PRE) {
             // Both stages from one block reduction: with a = gp (.) g and
             // u = (a - m inv1 kd1) pref1, the pre-MLP stage's sum <x, gq (.) u> is
             // pref1 (<x gq, a> - inv1 kd1 <x gq, m>), so all five sums are taken in one
-            // pass over the loaded rows (one barrier round per row instead of two).
-            float s5[5] = {0.f, 0.f, 0.f, 0.f, 0.f};
+            // pass over the row (one barrier round per row instead of two).
+            float2 S[5];
+#pragma unroll
+            for (int i = 0; i < 5; ++i) S[i] = make_float2(0.f, 0.f);
 #pragma unroll
             for (int v = 0; v < NV; ++v) {
-                float gv[8], mv[8], xv[8], wp[8], wq[8];
-                raw_to_f32(graw[v], gv);
-                raw_to_f32(mraw[v], mv);
-                raw_to_f32(xraw[v], xv);
-                raw_to_f32(gp[v], wp);
-                raw_to_f32(gq[v], wq);
 #pragma unroll
-                for (int q = 0; q < 8; ++q) {
-                    const float a = wp[q] * gv[q], b = xv[q] * wq[q];
-                    s5[0] = fmaf(mv[q], mv[q], s5[0]);
-                    s5[1] = fmaf(mv[q], a, s5[1]);
-                    s5[2] = fmaf(xv[q], xv[q], s5[2]);
-                    s5[3] = fmaf(b, a, s5[3]);
-                    s5[4] = fmaf(b, mv[q], s5[4]);
+                for (int k = 0; k < 4; ++k) {
+                    const float2 m2 = bf16x2_at(mraw[v], k), x2 = bf16x2_at(xraw[v], k);
+                    const float2 a2 = __fmul2_rn(bf16x2_at(gp[v], k), bf16x2_at(graw[v], k));
+                    const float2 b2 = __fmul2_rn(x2, bf16x2_at(gq[v], k));
+                    S[0] = __ffma2_rn(m2, m2, S[0]);
+                    S[1] = __ffma2_rn(m2, a2, S[1]);
+                    S[2] = __ffma2_rn(x2, x2, S[2]);
+                    S[3] = __ffma2_rn(b2, a2, S[3]);
+                    S[4] = __ffma2_rn(b2, m2, S[4]);
                 }
             }
+            float s5[5];
+#pragma unroll
+            for (int i = 0; i < 5; ++i) s5[i] = S[i].x + S[i].y;
             block_sum_n<5, THREADS>(s5);
             const float r1 = sqrtf(s5[0] / static_cast<float>(d) + eps);
             const float inv1 = 1.0f / r1;
@@ -746,24 +815,22 @@ __global__ void __launch_bounds__(THREADS)
             const float xu = pref1 * (s5[3] - (inv1 * kd1) * s5[4]);
             const float kd2 = (xu * inv2) / static_cast<float>(d);
             const float pref2 = 1.0f / fmaxf(r2, min_rms);
+            // u = a pref1 - m (inv1 kd1 pref1);  out = (gq (.) u) pref2 - x (inv2 kd2 pref2)
+            const float2 P1 = make_float2(pref1, pref1), P2 = make_float2(pref2, pref2);
+            const float c1 = -(inv1 * kd1) * pref1, c2 = -(inv2 * kd2) * pref2;
+            const float2 C1 = make_float2(c1, c1), C2 = make_float2(c2, c2);
 #pragma unroll
             for (int v = 0; v < NV; ++v) {
-                float gv[8], mv[8], xv[8], wp[8], wq[8];
-                raw_to_f32(graw[v], gv);
-                raw_to_f32(mraw[v], mv);
-                raw_to_f32(xraw[v], xv);
-                raw_to_f32(gp[v], wp);
-                raw_to_f32(gq[v], wq);
-                float o[8];
 #pragma unroll
-                for (int q = 0; q < 8; ++q) {
-                    const float uq = (wp[q] * gv[q] - (mv[q] * inv1) * kd1) * pref1;
-                    o[q] = (wq[q] * uq - (xv[q] * inv2) * kd2) * pref2;
+                for (int k = 0; k < 4; ++k) {
+                    const float2 a2 = __fmul2_rn(bf16x2_at(gp[v], k), bf16x2_at(graw[v], k));
+                    const float2 u2 = __ffma2_rn(a2, P1, __fmul2_rn(bf16x2_at(mraw[v], k), C1));
+                    const float2 o2 = __ffma2_rn(__fmul2_rn(bf16x2_at(gq[v], k), u2), P2,
+                                                 __fmul2_rn(bf16x2_at(xraw[v], k), C2));
+                    u[8 * v + 2 * k] = o2.x;
+                    u[8 * v + 2 * k + 1] = o2.y;
                 }
-                const int k = (v * THREADS + threadIdx.x) * 8;
-                if (k < d) st_vec<8>(out + off + k, o);
             }
-            continue;
         } else {
 #pragma unroll
             for (int v = 0; v < NV; ++v) {
@@ -786,6 +853,7 @@ __global__ void __launch_bounds__(THREADS)
             }
         }
     }
+    cp_async_wait<0>();
 }
 
 // Rows too long for registers, and fp32: one warp per row, three passes over the row
@@ -794,7 +862,7 @@ template <typename TT, int VEC, bool POST, bool PRE>
 __global__ void __launch_bounds__(kRowThreads)
     layer_signal_kernel(const TT* __restrict__ g, const __grid_constant__ LayerSignalPtrs p, int T,
                         int d, float eps, float min_rms) {
-    const int l = blockIdx.y;
+    const int l = blockIdx.x;
     const TT* m = static_cast<const TT*>(p.m[l]);
     const TT* gp = static_cast<const TT*>(p.gp[l]);
     const TT* x = static_cast<const TT*>(p.x[l]);
@@ -802,7 +870,7 @@ __global__ void __launch_bounds__(kRowThreads)
     TT* out = static_cast<TT*>(p.out[l]);
     const int lane = threadIdx.x & 31;
     const int wpb = blockDim.x >> 5;
-    for (int row = blockIdx.x * wpb + (threadIdx.x >> 5); row < T; row += gridDim.x * wpb) {
+    for (int row = blockIdx.y * wpb + (threadIdx.x >> 5); row < T; row += gridDim.y * wpb) {
         const size_t off = static_cast<size_t>(row) * d;
         float inv1 = 0.f, kd1 = 0.f, pref1 = 1.f;
         if constexpr (POST) {
@@ -1037,6 +1105,20 @@ cudaError_t launch_wait_timeout(unsigned* status, uint64_t limit_ns, cudaStream_
 
 namespace {
 
+// The block-per-row kernel with its shared-memory size; the attribute is raised once per
+// instantiation to the largest staging it can need (rows of 32 x kSigThreads elements).
+template <int EPT, bool POST, bool PRE>
+cudaError_t launch_sig_rows(dim3 grid, size_t smem, cudaStream_t st, const __nv_bfloat16* g,
+                            const LayerSignalPtrs& p, int T, int d, float eps, float min_rms) {
+    auto kern = layer_signal_row_kernel<EPT, kSigThreads, POST, PRE>;
+    constexpr int kNT = 1 + (POST ? 1 : 0) + (PRE ? 1 : 0);
+    static const cudaError_t attr = cudaFuncSetAttribute(
+        kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSigStages * kNT * EPT * kSigThreads * 2);
+    if (attr != cudaSuccess) return attr;
+    kern<<<grid, kSigThreads, smem, st>>>(g, p, T, d, eps, min_rms);
+    return cudaSuccess;
+}
+
 template <bool POST, bool PRE>
 cudaError_t run_layer_signals(int dtype, int n_layers, const void* g, const LayerSignalPtrs& p,
                               int T, int d, float eps, float min_rms, cudaStream_t st) {
@@ -1050,23 +1132,24 @@ cudaError_t run_layer_signals(int dtype, int n_layers, const void* g, const Laye
                     : d <= 32 * kSigThreads ? 32
                                             : 0;
     if (ept) {
-        const dim3 grid(static_cast<unsigned>(T < per_layer ? T : per_layer),
-                        static_cast<unsigned>(n_layers));
+        const dim3 grid(static_cast<unsigned>(n_layers),
+                        static_cast<unsigned>(T < per_layer ? T : per_layer));
         const auto* gg = static_cast<const __nv_bfloat16*>(g);
+        constexpr int kNT = 1 + (POST ? 1 : 0) + (PRE ? 1 : 0);
+        const size_t smem = static_cast<size_t>(kSigStages) * kNT * d * 2;
+        cudaError_t e = cudaSuccess;
         if (ept == 8)
-            layer_signal_row_kernel<8, kSigThreads, POST, PRE><<<grid, kSigThreads, 0, st>>>(
-                gg, p, T, d, eps, min_rms);
+            e = launch_sig_rows<8, POST, PRE>(grid, smem, st, gg, p, T, d, eps, min_rms);
         else if (ept == 16)
-            layer_signal_row_kernel<16, kSigThreads, POST, PRE><<<grid, kSigThreads, 0, st>>>(
-                gg, p, T, d, eps, min_rms);
+            e = launch_sig_rows<16, POST, PRE>(grid, smem, st, gg, p, T, d, eps, min_rms);
         else
-            layer_signal_row_kernel<32, kSigThreads, POST, PRE><<<grid, kSigThreads, 0, st>>>(
-                gg, p, T, d, eps, min_rms);
+            e = launch_sig_rows<32, POST, PRE>(grid, smem, st, gg, p, T, d, eps, min_rms);
+        if (e != cudaSuccess) return e;
     } else {
         const int wpb = kRowThreads / 32;
         const int need = (T + wpb - 1) / wpb;
-        const dim3 grid(static_cast<unsigned>(need < per_layer ? need : per_layer),
-                        static_cast<unsigned>(n_layers));
+        const dim3 grid(static_cast<unsigned>(n_layers),
+                        static_cast<unsigned>(need < per_layer ? need : per_layer));
         if (dtype == 1)
             layer_signal_kernel<__nv_bfloat16, 8, POST, PRE><<<grid, kRowThreads, 0, st>>>(
                 static_cast<const __nv_bfloat16*>(g), p, T, d, eps, min_rms);
