@@ -161,3 +161,29 @@ def test_pre_mlp_step_matches_oracle(fpo, post):
         Wn, _ = oracle.sgd_update(inp["W"][l].numpy(), G, wl.lr)
         W0 = inp["W"][l].double().numpy()
         assert rel_frob(f64(Wm[l]) - W0, Wn.astype(np.float64) - W0) < 2e-2
+
+
+@pytest.mark.slow
+@pytest.mark.parametrize("post", [False, True])
+def test_layer_signals_full_size_sampled_rows(fpo, post):
+    """Qwen3-8B-shaped layers (T = 16384, d = 4096, 9 target layers; with the post-FFN
+    norm the Gemma-3 layout), one launch for all layers, 12 sampled rows of every layer's
+    signal (clamped rows 32 + 64 k of x and 64 k of m included) against the oracle."""
+    wl = synth.WORKLOADS["qwen"]
+    g = synth.normal((wl.T, wl.d), std=1e-4, seed=8, tensor="h", layer=11, device="cuda").to(
+        torch.bfloat16)
+    x = [synth.make_pre_norm_in(wl, l, device="cuda") for l in range(wl.layers)]
+    gq = [synth.make_pre_norm_w(wl, l, device="cuda") for l in range(wl.layers)]
+    m = [synth.make_mlp_out(wl, l, device="cuda") for l in range(wl.layers)] if post else None
+    gp = [synth.make_post_norm_w(wl, l, device="cuda") for l in range(wl.layers)] if post else None
+    outs = [torch.empty_like(g) for _ in range(wl.layers)]
+    fpo.layer_signals(g, outs, m=m, gamma_post=gp, x=x, gamma_pre=gq)
+    torch.cuda.synchronize()
+    rows = [0, 1, 32, 64, 96, 8191, 8192, 12345, 16352, wl.T - 2, wl.T - 1, 5000]
+    e = synth.to_numpy_exact
+    for l in range(wl.layers):
+        ref = oracle.layer_signal(e(g[rows]), e(m[l][rows]) if post else None,
+                                  e(gp[l]) if post else None, e(x[l][rows]), e(gq[l]))
+        got = f64(outs[l][rows])
+        for r in range(len(rows)):
+            assert rel_frob(got[r], ref[r]) < 2e-2
