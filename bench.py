@@ -750,8 +750,10 @@ def run_fpo(args, wl):
             "algo": algo_name,
             "direct_fixup_rows_last_chunk": fixup_rows,
             "gemm_kernel": {0: "single-cta 128x256 (tcgen05 cta_group::1)",
-                            1: "cta-pair 256x256 (tcgen05 cta_group::2)",
-                            2: "cta-pair 256x256, projection 256x512 (tcgen05 cta_group::2)",
+                            1: "cta-pair 256x256 (tcgen05 cta_group::2; three 64 KB stages of "
+                               "two k-blocks)",
+                            2: "cta-pair 256x256 (three 64 KB stages of two k-blocks), projection "
+                               "256x512 (tcgen05 cta_group::2)",
                             }[variant],
             "cpu_baseline": cpu,
             "e2e": e2e,
