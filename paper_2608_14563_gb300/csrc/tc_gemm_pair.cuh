@@ -8,20 +8,18 @@
 // SM streams a third less operand data per FLOP.
 //
 // A pipeline stage of the 256-column tiles holds two consecutive 64-deep k-blocks
-// (64 KB per CTA, three stages): the MMA thread then waits on one barrier and
-// commits once per eight N = 256 MMAs (1024 tensor cycles) instead of per four.  Measured with clock counters in the MMA thread, one
-// wait + fence + four MMAs + commit per 64-deep stage took ~550 cycles for 512
-// cycles of tensor work (the issuing thread, not the operand supply, set the pace:
-// the same loop with the operands loaded once per launch ran at the same rate); with
-// eight MMAs per stage the loop keeps pace with the tensor pipe.  Each 64-deep half of
-// a stage has its own full barrier (the commit that frees the stage stays one), so the
-// first four MMAs of a stage start as soon as its first half has landed: the layer
-// update 2.6% faster, the step 0.3% (same box).  The 512-column
-// tiles issue eight MMAs per 64-deep k-block already.  The layer update (MN-major,
-// g~ and A_l streamed from DRAM) alone runs 2% slower with three 64 KB stages than
-// with six of 32 KB, but the step as a whole is faster with them (at the power cap
-// the update's lower draw leaves clock to the other GEMMs), so every 256-column
-// tile uses them.
+// (64 KB per CTA, three stages), each with its own full barrier, and is freed by one
+// commit: the MMA thread issues eight N = 256 MMAs (1024 tensor cycles) per commit and
+// starts the first four as soon as the stage's first half has landed.  Measured with
+// clock counters in the MMA thread, one wait + fence + four MMAs + commit per 32 KB
+// stage took ~550 cycles for 512 cycles of tensor work, at the same rate with the
+// operands loaded only once per launch: the issuing thread, not the operand supply,
+// set the pace.  With eight MMAs per commit the loop keeps pace with the tensor pipe
+// (512 cycles per k-block without copies).  The 512-column tiles issue eight MMAs per
+// 64-deep k-block already and keep one k-block (48 KB) per stage.  The layer update
+// (MN-major, g~ and A_l streamed from DRAM) would alone run faster with six 32 KB
+// stages, but the step is faster with three 64 KB stages everywhere: at the power cap
+// the update's lower draw leaves clock to the other GEMMs.
 //
 //   both CTAs, warp 0   TMA loads of the CTA's halves; completion is counted
 //                       on the LEADER's (rank 0) full barrier
