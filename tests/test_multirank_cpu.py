@@ -145,3 +145,14 @@ def test_end_to_end_copy_schedule():
     assert b.copy_schedule("auto", 16.3, 16.3) == "sm"
     for m in ("sm", "sm1", "ce"):
         assert b.copy_schedule(m, 51.1, 33.4) == m
+
+
+def test_committed_traffic_summary_matches_the_gemm_sources():
+    """The bench's roofline.traffic comes from profiles/traffic.json only while its source
+    digest matches the GEMM sources: a kernel change without a new capture reads null."""
+    b = _bench()
+    cfg = {"workload": "olmo2-7b-shaped", "algo": "direct", "gemm_variant": 2, "t_chunk": 8192,
+           "window_stress": False}
+    got = {k: b.load_traffic(k, cfg) for k in ("logits_lse_pass", "projection", "layer_update")}
+    assert all(v is not None and v > 0 for v in got.values()), got
+    assert b.load_traffic("logits_lse_pass", dict(cfg, t_chunk=4096)) is None
