@@ -13,6 +13,7 @@
 #include <math.h>
 
 #include "error_math.cuh"
+#include "optim_math.cuh"
 #include "ptx.cuh"
 #include "tc_gemm.cuh"
 
@@ -698,6 +699,102 @@ struct EpiStoreGroupF32 {
     }
 
     __device__ __forceinline__ void finish(const Params&, int) {}
+};
+
+// ---------------------------------------------------------------------------
+// The optimizer's first pass in the pseudogradient GEMM's epilogue, for the relative
+// clip on the step (Sec. 3.1: SGD, SGD with momentum, AdamW on the fp32 masters; App. A:
+// ||dW|| <= clip_frac ||W||).  With G from the accumulator, each element's optimizer state
+// advances and its unclipped step d = opt_step(G, W, s1, s2) is stored (fp32, D[g]; the
+// state sees the unclipped gradient), and ||W||^2, ||d||^2 of the warp's 32 rows of the
+// tile are written as one pair per (layer, 256-row block, column tile, 32-row slot); a
+// kernel then scales each layer's steps by min(1, clip_frac ||W|| / ||d||) and applies
+// them (W is not written here, so its norm is the pre-step one).  Without a clip the
+// stand-alone passes are used: taking the whole step here made the update faster but
+// the power-capped step slower (its epilogue then held the tensor pipe back at full
+// draw).
+struct EpiOptStep {
+    struct Params {
+        const float* W_master[kMaxGroups];
+        float* s1[kMaxGroups];             // momentum / AdamW first moment (or null)
+        float* s2[kMaxGroups];             // AdamW second moment (or null)
+        float* D[kMaxGroups];              // the unclipped steps
+        float* part;                       // [groups][m256][n_blocks][8][2]
+        OptimParams op;
+        long long ld;
+        int M, N;
+        int m256, n_blocks;
+    };
+    int row, g;
+    bool valid;
+    float s_ww, s_dd;
+
+    __device__ __forceinline__ EpiOptStep(const Params& p, int g_, int row_, int)
+        : row(row_), g(g_), s_ww(0.f), s_dd(0.f) {
+        valid = row_ < p.M;
+    }
+
+    __device__ __forceinline__ void chunk(const Params& p, const float (&v)[32], int col0, int,
+                                          EpiIO&) {
+        const int lim = p.N - col0;
+        if (!valid || lim <= 0) return;
+        const long long off = row * p.ld + col0;
+        const float4* wp = reinterpret_cast<const float4*>(p.W_master[g] + off);
+        float4* p1 = p.s1[g] ? reinterpret_cast<float4*>(p.s1[g] + off) : nullptr;
+        float4* p2 = p.s2[g] ? reinterpret_cast<float4*>(p.s2[g] + off) : nullptr;
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {  // 16 columns at a time
+            if (h * 16 >= lim) break;
+            float w[16], a[16], b[16];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const int c4 = 4 * h + q;  // float4 index in the chunk
+                if (c4 * 4 < lim) {
+                    const float4 x = wp[c4];
+                    w[4 * q] = x.x; w[4 * q + 1] = x.y; w[4 * q + 2] = x.z; w[4 * q + 3] = x.w;
+                    const float4 y = p1 ? p1[c4] : make_float4(0.f, 0.f, 0.f, 0.f);
+                    a[4 * q] = y.x; a[4 * q + 1] = y.y; a[4 * q + 2] = y.z; a[4 * q + 3] = y.w;
+                    const float4 z = p2 ? p2[c4] : make_float4(0.f, 0.f, 0.f, 0.f);
+                    b[4 * q] = z.x; b[4 * q + 1] = z.y; b[4 * q + 2] = z.z; b[4 * q + 3] = z.w;
+                }
+            }
+            float out[16];
+#pragma unroll
+            for (int e = 0; e < 16; ++e) {
+                out[e] = opt_step(p.op, v[16 * h + e], w[e], a[e], b[e]);
+                if (16 * h + e < lim) {  // (columns past N were not loaded)
+                    s_ww = fmaf(w[e], w[e], s_ww);
+                    s_dd = fmaf(out[e], out[e], s_dd);
+                }
+            }
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const int c4 = 4 * h + q;
+                if (c4 * 4 >= lim) break;
+                reinterpret_cast<float4*>(p.D[g] + off)[c4] =
+                    make_float4(out[4 * q], out[4 * q + 1], out[4 * q + 2], out[4 * q + 3]);
+                if (p1) p1[c4] = make_float4(a[4 * q], a[4 * q + 1], a[4 * q + 2], a[4 * q + 3]);
+                if (p2) p2[c4] = make_float4(b[4 * q], b[4 * q + 1], b[4 * q + 2], b[4 * q + 3]);
+            }
+        }
+    }
+
+    __device__ __forceinline__ void finish(const Params& p, int nb) {
+        float ww = s_ww, dd = s_dd;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            ww += __shfl_xor_sync(0xffffffffu, ww, o);
+            dd += __shfl_xor_sync(0xffffffffu, dd, o);
+        }
+        if ((threadIdx.x & 31) == 0) {
+            const long long slot =
+                ((static_cast<long long>(g) * p.m256 + row / 256) * p.n_blocks + nb) * 8 +
+                (row % 256) / 32;
+            float* o = p.part + slot * 2;
+            o[0] = ww;
+            o[1] = dd;
+        }
+    }
 };
 
 // ---------------------------------------------------------------------------

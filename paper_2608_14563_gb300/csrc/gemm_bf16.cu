@@ -640,6 +640,51 @@ cudaError_t launch_grad_bf16(int n, int T, int d, int d_ff, const void* const* g
         maps, ep, make_shape(d, d_ff, T, kUpdBN, n, band_for(false)), status, st);
 }
 
+cudaError_t launch_opt_step_bf16(int n, int T, int d, int d_ff, const void* const* g,
+                                 const void* const* A, const OptimParams& op,
+                                 float* const* W_master, float* const* s1, float* const* s2,
+                                 float* const* D, float* part, unsigned* status, cudaStream_t st) {
+    if (n < 1 || n > kMaxGroups) return cudaErrorInvalidValue;
+    static GemmMaps<kMaxGroups> maps;
+    static EpiOptStep::Params ep;
+    static std::mutex mu;
+    std::lock_guard<std::mutex> lock(mu);
+    for (int l = 0; l < kMaxGroups; ++l) {
+        const int k = l < n ? l : 0;
+        if (l < n) {
+            if (l > 0 && g[l] == g[0])
+                maps.a[l] = maps.a[0];
+            else if (!map_mnmajor(&maps.a[l], g[l], T, d))
+                return cudaErrorInvalidValue;
+            if (!map_mnmajor(&maps.b[l], A[l], T, d_ff)) return cudaErrorInvalidValue;
+        } else {
+            maps.a[l] = maps.a[0];
+            maps.b[l] = maps.b[0];
+        }
+        ep.W_master[l] = W_master[k];
+        ep.s1[l] = s1 ? s1[k] : nullptr;
+        ep.s2[l] = s2 ? s2[k] : nullptr;
+        ep.D[l] = D ? D[k] : nullptr;
+    }
+    ep.part = part;
+    ep.op = op;
+    ep.ld = d_ff;
+    ep.M = d;
+    ep.N = d_ff;
+    ep.m256 = (d + 255) / 256;
+    ep.n_blocks = (d_ff + kUpdBN - 1) / kUpdBN;
+    if (use_pair())
+        return run_gemm_pair<kUpdBN, true, true, kPairStages, kMaxGroups, EpiOptStep>(
+            maps, ep, make_shape(d, d_ff, T, kUpdBN, n, band_for(true), kPairBM), status, st);
+    return run_gemm<kUpdBN, true, true, kUpdStages, kMaxGroups, EpiOptStep>(
+        maps, ep, make_shape(d, d_ff, T, kUpdBN, n, band_for(false)), status, st);
+}
+
+size_t opt_step_partial_bytes(int n_layers, int d, int d_ff) {
+    return static_cast<size_t>(n_layers) * ((d + 255) / 256) * ((d_ff + kUpdBN - 1) / kUpdBN) * 8 *
+           2 * sizeof(float);
+}
+
 // The cosine of every layer from EpiGradCos's per-(tile, warp) triples: one warp per
 // layer adds its slots in a fixed order (lane-strided fp64 sums, then a fixed butterfly).
 __global__ void grad_cosine_final_kernel(const float* __restrict__ part, int slots,

@@ -113,6 +113,18 @@ struct OptimParams {
     float inv_bc1, inv_sqrt_bc2;  // AdamW bias corrections 1/(1-b1^t), 1/sqrt(1-b2^t)
 };
 size_t optim_partials_bytes(int n_layers);
+// The step clip's first optimizer pass fused into the pseudogradient GEMM (bf16): the
+// state advanced, the unclipped steps in D and (||W||^2, ||d||^2) per (layer, 256 rows,
+// column tile, 32 rows) in part, for launch_opt_step_clip.
+cudaError_t launch_opt_step_bf16(int n, int T, int d, int d_ff, const void* const* g,
+                                 const void* const* A, const OptimParams& op,
+                                 float* const* W_master, float* const* s1, float* const* s2,
+                                 float* const* D, float* part, unsigned* status, cudaStream_t st);
+size_t opt_step_partial_bytes(int n_layers, int d, int d_ff);
+cudaError_t launch_opt_step_clip(int n_layers, size_t n_elem, const OptimParams& op,
+                                 const float* part, int slots, float* const* D,
+                                 float* const* W_master, void* const* W_out, float* scales,
+                                 cudaStream_t st);
 cudaError_t launch_optimizer(int dtype, int n_layers, size_t n_elem, const OptimParams& op,
                              float* const* G, float* const* W_master, void* const* W_out,
                              float* const* s1, float* const* s2, double* partials, float* scales,

@@ -3,7 +3,9 @@
 // masters cast to the working dtype, and each step's relative clip to
 // clip_frac * ||W||_F, on the step itself or on the gradient).
 //
-// From the pseudogradients G_l (fp32, written by the grouped GEMM):
+// bf16 with the step clip: the GEMM's epilogue (EpiOptStep) advances the state and leaves
+// the unclipped steps and their norm partials to opt_step_scale + opt_step_apply below.
+// Otherwise, from the pseudogradients G_l (fp32, written by the grouped GEMM):
 //   pass 1  optim_norms    per layer, partial sums of ||W||^2, ||G||^2 and
 //                          ||step||^2 (step = the unclipped optimizer step)
 //   pass 2  optim_scale    per layer, the clip factor from those sums
@@ -15,6 +17,7 @@
 #include <math.h>
 
 #include "internal.h"
+#include "optim_math.cuh"
 
 namespace fpo {
 namespace {
@@ -30,21 +33,6 @@ struct LayerPtrs {
     float* s1[kMaxLayers];
     float* s2[kMaxLayers];
 };
-
-// Optimizer state update and step for one element (gradient already scaled).
-__device__ __forceinline__ float opt_step(const OptimParams& op, float g, float w, float& s1,
-                                          float& s2) {
-    if (op.kind == 0) return -op.lr * g;
-    if (op.kind == 1) {
-        s1 = fmaf(op.momentum, s1, g);
-        return -op.lr * s1;
-    }
-    s1 = fmaf(op.beta1, s1, (1.f - op.beta1) * g);
-    s2 = fmaf(op.beta2, s2, (1.f - op.beta2) * g * g);
-    const float mhat = s1 * op.inv_bc1;
-    const float denom = sqrtf(s2) * op.inv_sqrt_bc2 + op.eps;
-    return -op.lr * (mhat / denom + op.weight_decay * w);
-}
 
 __device__ __forceinline__ double warp_sum_d(double x) {
 #pragma unroll
@@ -143,6 +131,54 @@ __global__ void __launch_bounds__(kOptThreads)
     }
 }
 
+// Step clip after the fused epilogue (EpiOptStep): one warp per layer adds the layer's
+// (||W||^2, ||d||^2) slot pairs in a fixed order (lane-strided fp64 sums, then a fixed
+// butterfly) and writes the layer's scale min(1, clip_frac ||W|| / ||d||).
+__global__ void opt_step_scale_kernel(const float* __restrict__ part, int slots,
+                                      const OptimParams op, float* __restrict__ scales) {
+    const int layer = blockIdx.x;
+    const int lane = threadIdx.x;
+    const float* p = part + static_cast<size_t>(layer) * slots * 2;
+    double ww = 0.0, dd = 0.0;
+    for (int i = lane; i < slots; i += 32) {
+        ww += p[2 * i];
+        dd += p[2 * i + 1];
+    }
+    ww = warp_sum_d(ww);
+    dd = warp_sum_d(dd);
+    if (lane != 0) return;
+    const double lim = static_cast<double>(op.clip_frac) * sqrt(ww);
+    scales[layer] = static_cast<float>(sqrt(dd) > lim ? lim / sqrt(dd) : 1.0);
+}
+
+// W <- W + s d with the layer's scale, and W_out = bf16(W) (16-byte vectors).
+__global__ void __launch_bounds__(kOptThreads)
+    opt_step_apply_kernel(const __grid_constant__ LayerPtrs lp, size_t n,
+                          const float* __restrict__ scales) {
+    const int layer = blockIdx.y;
+    const float4* D = reinterpret_cast<const float4*>(lp.G[layer]);
+    float4* W = reinterpret_cast<float4*>(lp.W[layer]);
+    uint2* Wo = static_cast<uint2*>(lp.Wo[layer]);
+    const float s = scales[layer];
+    const size_t n4 = n / 4;  // n = d d_ff, a multiple of 8
+    const size_t stride = static_cast<size_t>(gridDim.x) * kOptThreads;
+    for (size_t i = blockIdx.x * static_cast<size_t>(kOptThreads) + threadIdx.x; i < n4; i += stride) {
+        const float4 dv = D[i];
+        float4 w = W[i];
+        w.x = fmaf(s, dv.x, w.x);
+        w.y = fmaf(s, dv.y, w.y);
+        w.z = fmaf(s, dv.z, w.z);
+        w.w = fmaf(s, dv.w, w.w);
+        W[i] = w;
+        if (Wo) {
+            const __nv_bfloat162 lo = __floats2bfloat162_rn(w.x, w.y);
+            const __nv_bfloat162 hi = __floats2bfloat162_rn(w.z, w.w);
+            Wo[i] = make_uint2(*reinterpret_cast<const uint32_t*>(&lo),
+                               *reinterpret_cast<const uint32_t*>(&hi));
+        }
+    }
+}
+
 int blocks_per_layer(int n_layers) {
     DevInfo di;
     const int sms = current_device_info(&di) ? di.sm_count : 148;
@@ -192,6 +228,28 @@ cudaError_t launch_optimizer(int dtype, int n_layers, size_t n_elem, const Optim
         optim_apply_kernel<false><<<grid, kOptThreads, 0, st>>>(lp, n_elem, op,
                                                                 op.clip != 0 ? scales : nullptr),
             ::fpo::note_launch();
+    return cudaGetLastError();
+}
+
+cudaError_t launch_opt_step_clip(int n_layers, size_t n_elem, const OptimParams& op,
+                                 const float* part, int slots, float* const* D,
+                                 float* const* W_master, void* const* W_out, float* scales,
+                                 cudaStream_t st) {
+    if (n_layers < 1 || n_layers > kMaxLayers) return cudaErrorInvalidValue;
+    if (n_elem == 0) return cudaSuccess;
+    LayerPtrs lp;
+    for (int l = 0; l < kMaxLayers; ++l) {
+        const bool in = l < n_layers;
+        lp.G[l] = in ? D[l] : nullptr;
+        lp.W[l] = in ? W_master[l] : nullptr;
+        lp.Wo[l] = in && W_out ? W_out[l] : nullptr;
+        lp.s1[l] = lp.s2[l] = nullptr;
+    }
+    opt_step_scale_kernel<<<n_layers, 32, 0, st>>>(part, slots, op, scales), ::fpo::note_launch();
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    const dim3 grid(blocks_per_layer(n_layers), n_layers);
+    opt_step_apply_kernel<<<grid, kOptThreads, 0, st>>>(lp, n_elem, scales), ::fpo::note_launch();
     return cudaGetLastError();
 }
 
