@@ -346,8 +346,10 @@ size_t fpo_layer_optimize_workspace(int32_t n_layers, int64_t d, int64_t d_ff);
  * state1[l] is the momentum buffer (SGD_MOMENTUM) or the first moment (ADAMW),
  * state2[l] the second moment (ADAMW); fp32 [d, d_ff], updated in place (NULL
  * arrays when the optimizer has no such state).  W_out may be NULL.  The clip
- * needs all of G_l before any element steps, so G lives in the workspace
- * (n_layers x d x d_ff x 4 bytes).  g, A, W_out: as fpo_layer_update_grouped_signals.
+ * needs all of G_l (or of the steps) before any element steps, so the workspace
+ * holds n_layers x d x d_ff x 4 bytes: G_l, or with bf16 and FPO_CLIP_STEP the
+ * unclipped steps, which the GEMM's epilogue forms from G_l (and the state) without
+ * storing G_l.  g, A, W_out: as fpo_layer_update_grouped_signals.
  */
 int32_t fpo_layer_optimize_grouped(int32_t n_layers, int64_t T, int64_t d, int64_t d_ff,
                                    int32_t dtype, const void* const* g, const void* const* A,
