@@ -90,3 +90,44 @@ def test_clip_is_active_in_the_step_cases(fpo):
     assert r["scale"] < 1.0
     r = oracle.optimizer_step(W[0].numpy(), G, kind=0, lr=0.5, clip=2)
     assert r["scale"] < 1.0
+
+
+@pytest.mark.slow
+def test_adamw_step_clip_full_size(fpo):
+    """OLMo-2-7B-shaped layers (T = 16384, d = 4096, d_ff = 11008, 8 layers; bf16, so the
+    step clip's first pass runs in the GEMM's epilogue), AdamW's first step with the clip
+    active: every layer's ||dW|| is clip_frac ||W||, and 4 sampled rows of each dW are the
+    oracle's AdamW step rows (from the oracle's G rows over all T tokens) times one common
+    factor per layer.  AdamW's first step is lr (G / (|G| + eps) + wd W), a sign where
+    |G| >> eps: elements whose G is within the GPU's fp32 accumulation error over 16384
+    tokens of zero (|G| < 1e-4 rms(G), ~1e-4 of them; one at 9.5e-8 came out at -2.2e-8)
+    may take either sign, and are left out of the row comparison."""
+    wl = synth.WORKLOADS["olmo"]
+    L = wl.layers
+    g = synth.normal((wl.T, wl.d), std=1e-4, seed=9, tensor="h", layer=13, device="cuda").to(
+        torch.bfloat16)
+    A = [synth.make_A(wl, l, device="cuda") for l in range(L)]
+    W0 = [synth.make_W_master(wl, l, device="cuda") for l in range(L)]
+    Wm = [w.clone() for w in W0]
+    S1 = [torch.zeros_like(w) for w in W0]
+    S2 = [torch.zeros_like(w) for w in W0]
+    lr, frac = 1e-3, 0.01
+    opt = fpo.optimizer_desc(2, lr=lr, clip=1, clip_frac=frac, step=1)
+    ws = fpo.layer_optimize_grouped([g] * L, A, opt, Wm, states1=S1, states2=S2)
+    assert fpo.get_device_status(ws) == fpo.OK
+    rows = [0, 1234, 2048, wl.d - 1]
+    gcol = synth.to_numpy_exact(g[:, rows].contiguous())
+    for l in range(L):
+        dW = (Wm[l] - W0[l]).double()
+        ratio = float(dW.norm() / W0[l].double().norm())
+        assert abs(ratio - frac) < 1e-4 * frac
+        G = oracle.pseudograd(gcol, synth.to_numpy_exact(A[l]))          # [4, d_ff]
+        w_rows = W0[l][rows].double().cpu().numpy()
+        step = -lr * (G / (np.abs(G) + 1e-8) + 0.01 * w_rows)              # AdamW, t = 1
+        got = dW[rows].cpu().numpy()
+        keep = np.abs(G) > 1e-4 * np.sqrt(np.mean(G * G))
+        assert keep.mean() > 0.999
+        got, step = got[keep], step[keep]
+        s = np.sum(got * step) / np.sum(step * step)                       # common factor
+        assert 0.0 < s < 1.0
+        assert rel_frob(got, s * step) < 2e-3
