@@ -187,19 +187,34 @@ __global__ void __launch_bounds__(kBlkThreads)
                            unsigned* status, const __nv_bfloat16* __restrict__ W_U,
                            float* __restrict__ anchor) {
     constexpr int NV = EPT / 8;
-    for (int row = blockIdx.x; row < T; row += gridDim.x) {
-        const __nv_bfloat16* hr = h + static_cast<size_t>(row) * d;
-        const int t = y[row];
-        const bool t_ok = t >= 0 && t < V;
-        // the target's unembedding row, read only for an in-range target, loaded with h
-        const __nv_bfloat16* ur = (anchor && t_ok) ? W_U + static_cast<size_t>(t) * d : nullptr;
-        uint4 hx[NV], ux[NV];
+    // h row r and, for an in-range target, the target's unembedding row (the anchor's
+    // operand); the next row's are loaded before the current row is computed
+    auto load_row = [&](int r, int& t, uint4 (&hx)[NV], uint4 (&ux)[NV]) {
+        t = y[r];
+        const __nv_bfloat16* hr = h + static_cast<size_t>(r) * d;
+        const __nv_bfloat16* ur =
+            (anchor && t >= 0 && t < V) ? W_U + static_cast<size_t>(t) * d : nullptr;
 #pragma unroll
         for (int v = 0; v < NV; ++v) {
             const int k = (v * kBlkThreads + threadIdx.x) * 8;
             hx[v] = k < d ? *reinterpret_cast<const uint4*>(hr + k) : make_uint4(0, 0, 0, 0);
             ux[v] = (ur && k < d) ? *reinterpret_cast<const uint4*>(ur + k) : make_uint4(0, 0, 0, 0);
         }
+    };
+    int t_next = 0;
+    uint4 hx_next[NV], ux_next[NV];
+    if (blockIdx.x < T) load_row(blockIdx.x, t_next, hx_next, ux_next);
+    for (int row = blockIdx.x; row < T; row += gridDim.x) {
+        const int t = t_next;
+        uint4 hx[NV], ux[NV];
+#pragma unroll
+        for (int v = 0; v < NV; ++v) {
+            hx[v] = hx_next[v];
+            ux[v] = ux_next[v];
+        }
+        if (row + static_cast<int>(gridDim.x) < T)
+            load_row(row + gridDim.x, t_next, hx_next, ux_next);
+        const bool t_ok = t >= 0 && t < V;
         float ss = 0.f;
 #pragma unroll
         for (int v = 0; v < NV; ++v) {
