@@ -92,6 +92,30 @@ def test_clip_is_active_in_the_step_cases(fpo):
     assert r["scale"] < 1.0
 
 
+@pytest.mark.parametrize("clip", ["none", "step"])
+def test_optimizer_step_with_no_tokens(fpo, clip):
+    """T = 0: G = 0, and AdamW still steps (decayed moments, weight decay), through the
+    stand-alone passes whatever the clip (the fused pass needs a GEMM with tokens)."""
+    wl, gs, A, W = _case("bf16", seed=77)
+    g0 = [torch.zeros((0, wl.d), dtype=torch.bfloat16, device="cuda") for _ in range(wl.layers)]
+    A0 = [torch.zeros((0, wl.d_ff), dtype=torch.bfloat16, device="cuda") for _ in range(wl.layers)]
+    Gs = [np.zeros((wl.d, wl.d_ff)) for _ in range(wl.layers)]
+    s1, s2 = _states(wl, [np.full((wl.d, wl.d_ff), 1e-3) for _ in range(wl.layers)], "adamw", 3)
+    opt = fpo.optimizer_desc(2, lr=2e-3, clip=CLIPS[clip], step=3)
+    Wm = [w.cuda() for w in W]
+    S1 = [torch.from_numpy(x).cuda() for x in s1]
+    S2 = [torch.from_numpy(x).cuda() for x in s2]
+    ws = fpo.layer_optimize_grouped(g0, A0, opt, Wm, states1=S1, states2=S2)
+    assert fpo.get_device_status(ws) == fpo.OK
+    for l in range(wl.layers):
+        ref = oracle.optimizer_step(W[l].numpy(), Gs[l], kind=2, lr=2e-3, t=3, clip=CLIPS[clip],
+                                    s1=s1[l], s2=s2[l])
+        W0 = W[l].double().numpy()
+        assert rel_frob(f64(Wm[l]) - W0, ref["W"].astype(np.float64) - W0) < 1e-4
+        assert rel_frob(f64(S1[l]), ref["s1"]) < 1e-6
+        assert rel_frob(f64(S2[l]), ref["s2"]) < 1e-6
+
+
 @pytest.mark.slow
 def test_adamw_step_clip_full_size(fpo):
     """OLMo-2-7B-shaped layers (T = 16384, d = 4096, d_ff = 11008, 8 layers; bf16, so the
