@@ -41,6 +41,10 @@
  *   fp32 FFMA (no TF32); any positive shape is accepted.
  * - The library only runs on compute capability 10.3 (GB300); any other
  *   device returns FPO_ERR_ARCH.
+ * - Every call runs on the calling thread's current device.  One process may
+ *   drive several GPUs: a kernel's launch setup (its shared-memory limit, the
+ *   clusters resident at once) is made once per device, on that device's
+ *   first call.
  */
 #ifndef FPO_H_
 #define FPO_H_

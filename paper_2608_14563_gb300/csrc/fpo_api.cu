@@ -24,7 +24,7 @@ struct DevCache {
     DevInfo info;
     bool ok = false;
 };
-DevCache g_dev[64];
+DevCache g_dev[kMaxDevices];
 }  // namespace
 
 uint64_t wait_limit_ns() { return g_wait_limit_ns.load(std::memory_order_relaxed); }
@@ -33,9 +33,15 @@ void note_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
 
 uint64_t launches() { return g_launches.load(std::memory_order_relaxed); }
 
-bool current_device_info(DevInfo* out) {
+int current_device() {
     int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return false;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return -1;
+    return dev;
+}
+
+bool current_device_info(DevInfo* out) {
+    const int dev = current_device();
+    if (dev < 0) return false;
     DevCache& c = g_dev[dev];
     std::call_once(c.once, [&] {
         int sms = 0, maj = 0, min = 0;

@@ -106,9 +106,8 @@ cudaError_t run_gemm(const GemmMaps<MAXG>& maps, const typename Epi::Params& ep,
                      const GemmShape& sh, unsigned* status, cudaStream_t st) {
     if (sh.tiles <= 0 || sh.k_blocks <= 0) return cudaSuccess;
     using L = GemmSmem<BN, STAGES>;
-    auto kern = tc_gemm_kernel<BN, A_MN, B_MN, STAGES, MAXG, Epi>;
-    static cudaError_t attr_err =
-        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::kBytes);
+    constexpr auto kern = tc_gemm_kernel<BN, A_MN, B_MN, STAGES, MAXG, Epi>;
+    const cudaError_t attr_err = set_smem_limit<kern>(L::kBytes);
     if (attr_err != cudaSuccess) return attr_err;
     DevInfo di;
     if (!current_device_info(&di)) return cudaErrorUnknown;
@@ -132,6 +131,20 @@ int pair_clusters(Kern kern, int smem_bytes, int sm_count, int cta) {
         cudaGetLastError();
         n = sm_count / cta;
     }
+    return n;
+}
+
+// pair_clusters for the current device, computed once per device (after the kernel's
+// shared-memory limit is raised there).
+template <auto Kern>
+int resident_clusters(int smem_bytes, int sm_count, int cta) {
+    static std::atomic<int> cache[kMaxDevices];
+    const int dev = current_device();
+    if (dev < 0) return sm_count / cta;
+    int n = cache[dev].load(std::memory_order_relaxed);
+    if (n > 0) return n;
+    n = pair_clusters(Kern, smem_bytes, sm_count, cta);
+    cache[dev].store(n, std::memory_order_relaxed);
     return n;
 }
 
@@ -177,13 +190,12 @@ cudaError_t run_gemm_pair(const GemmMaps<MAXG>& maps, const typename Epi::Params
     if (sh_in.tiles <= 0 || sh_in.k_blocks <= 0) return cudaSuccess;
     using L = GemmPairSmem<BN, STAGES, pair_ksub<BN, A_MN, B_MN>()>;
     static_assert(L::kBytes <= 227 * 1024, "stages exceed the shared memory of a CTA");
-    auto kern = tc_gemm_pair_kernel<BN, A_MN, B_MN, STAGES, MAXG, Epi>;
-    static cudaError_t attr_err =
-        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::kBytes);
+    constexpr auto kern = tc_gemm_pair_kernel<BN, A_MN, B_MN, STAGES, MAXG, Epi>;
+    const cudaError_t attr_err = set_smem_limit<kern>(L::kBytes);
     if (attr_err != cudaSuccess) return attr_err;
     DevInfo di;
     if (!current_device_info(&di)) return cudaErrorUnknown;
-    static int max_clusters = pair_clusters(kern, L::kBytes, di.sm_count, 2);
+    const int max_clusters = resident_clusters<kern>(L::kBytes, di.sm_count, 2);
     const long long clusters = sh_in.tiles < max_clusters ? sh_in.tiles : max_clusters;
     GemmShape sh = sh_in;
     if (sk_scratch) {
@@ -355,20 +367,15 @@ int gemm_variant() { return g_gemm_variant.load(std::memory_order_relaxed); }
 
 size_t proj_sk_scratch_bytes() {
     // kTailWaves x clusters units of 256 x 512 fp32; clusters of the 256 x 512 pair kernel
-    // on this device, or an upper bound of 128 without one
-    static const size_t bytes = [] {
-        using L = GemmPairSmem<kWideBN, kWideStages, pair_ksub<kWideBN, false, true>()>;
-        auto kern = tc_gemm_pair_kernel<kWideBN, false, true, kWideStages, 1, EpiProjVjp>;
-        DevInfo di;
-        long long c = 128;
-        if (current_device_info(&di) &&
-            cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::kBytes) ==
-                cudaSuccess)
-            c = pair_clusters(kern, L::kBytes, di.sm_count, 2);
-        cudaGetLastError();
-        return static_cast<size_t>(kTailWaves) * c * kPairBM * kWideBN * sizeof(float);
-    }();
-    return bytes;
+    // on the current device, or an upper bound of 128 without one
+    using L = GemmPairSmem<kWideBN, kWideStages, pair_ksub<kWideBN, false, true>()>;
+    constexpr auto kern = tc_gemm_pair_kernel<kWideBN, false, true, kWideStages, 1, EpiProjVjp>;
+    DevInfo di;
+    long long c = 128;
+    if (current_device_info(&di) && set_smem_limit<kern>(L::kBytes) == cudaSuccess)
+        c = resident_clusters<kern>(L::kBytes, di.sm_count, 2);
+    cudaGetLastError();
+    return static_cast<size_t>(kTailWaves) * c * kPairBM * kWideBN * sizeof(float);
 }
 
 constexpr int kLseBN = 256;

@@ -6,6 +6,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+
 namespace fpo {
 
 // Device status bits, OR-ed into the status word at offset 0 of a workspace.
@@ -20,6 +22,25 @@ struct DevInfo {
 };
 // Cached properties of the current device; false if the query failed.
 bool current_device_info(DevInfo* out);
+
+constexpr int kMaxDevices = 64;
+// The current device's index, or -1 if it cannot be read (or is >= kMaxDevices).
+int current_device();
+
+// Raises Kern's dynamic shared-memory limit to `bytes` in the current device's context.
+// A function attribute belongs to each context's copy of the module, so this runs once
+// per device; a failed attempt is not remembered, and the next launch tries again.
+template <auto Kern>
+cudaError_t set_smem_limit(int bytes) {
+    static std::atomic<bool> done[kMaxDevices];
+    const int dev = current_device();
+    if (dev < 0) return cudaErrorInvalidDevice;
+    if (done[dev].load(std::memory_order_acquire)) return cudaSuccess;
+    const cudaError_t e =
+        cudaFuncSetAttribute(Kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e == cudaSuccess) done[dev].store(true, std::memory_order_release);
+    return e;
+}
 
 uint64_t wait_limit_ns();
 

@@ -525,8 +525,19 @@ constexpr int kMeanThreads = 1024;
 __global__ void __launch_bounds__(kMeanThreads) mean_kernel(const float* __restrict__ x, int n,
                                                             float* __restrict__ out) {
     __shared__ double buf[kMeanThreads];
+    // thread i adds x[i], x[i + kMeanThreads], ... in that order; eight loads are issued
+    // before their adds, so the loop waits once per eight elements, not once per element
+    constexpr int kBatch = 8;
     double acc = 0.0;
-    for (int i = threadIdx.x; i < n; i += kMeanThreads) acc += static_cast<double>(x[i]);
+    long long i = threadIdx.x;
+    for (; i + (kBatch - 1) * static_cast<long long>(kMeanThreads) < n; i += kBatch * kMeanThreads) {
+        float v[kBatch];
+#pragma unroll
+        for (int k = 0; k < kBatch; ++k) v[k] = x[i + k * kMeanThreads];
+#pragma unroll
+        for (int k = 0; k < kBatch; ++k) acc += static_cast<double>(v[k]);
+    }
+    for (; i < n; i += kMeanThreads) acc += static_cast<double>(x[i]);
     buf[threadIdx.x] = acc;
     __syncthreads();
     for (int s = kMeanThreads / 2; s > 0; s >>= 1) {
@@ -1120,15 +1131,15 @@ cudaError_t launch_wait_timeout(unsigned* status, uint64_t limit_ns, cudaStream_
 
 namespace {
 
-// The block-per-row kernel with its shared-memory size; the attribute is raised once per
-// instantiation to the largest staging it can need (rows of 32 x kSigThreads elements).
+// The block-per-row kernel with its shared-memory size; the limit is raised once per
+// instantiation and device to the largest staging it can need (rows of EPT x kSigThreads
+// elements).
 template <int EPT, bool POST, bool PRE>
 cudaError_t launch_sig_rows(dim3 grid, size_t smem, cudaStream_t st, const __nv_bfloat16* g,
                             const LayerSignalPtrs& p, int T, int d, float eps, float min_rms) {
-    auto kern = layer_signal_row_kernel<EPT, kSigThreads, POST, PRE>;
+    constexpr auto kern = layer_signal_row_kernel<EPT, kSigThreads, POST, PRE>;
     constexpr int kNT = 1 + (POST ? 1 : 0) + (PRE ? 1 : 0);
-    static const cudaError_t attr = cudaFuncSetAttribute(
-        kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSigStages * kNT * EPT * kSigThreads * 2);
+    const cudaError_t attr = set_smem_limit<kern>(kSigStages * kNT * EPT * kSigThreads * 2);
     if (attr != cudaSuccess) return attr;
     kern<<<grid, kSigThreads, smem, st>>>(g, p, T, d, eps, min_rms);
     return cudaSuccess;
