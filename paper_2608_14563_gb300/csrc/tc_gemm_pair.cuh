@@ -16,10 +16,11 @@
 // operands loaded only once per launch: the issuing thread, not the operand supply,
 // set the pace.  With eight MMAs per commit the loop keeps pace with the tensor pipe
 // (512 cycles per k-block without copies).  The 512-column tiles issue eight MMAs per
-// 64-deep k-block already and keep one k-block (48 KB) per stage.  The layer update
-// (MN-major, g~ and A_l streamed from DRAM) would alone run faster with six 32 KB
-// stages, but the step is faster with three 64 KB stages everywhere: at the power cap
-// the update's lower draw leaves clock to the other GEMMs.
+// 64-deep k-block already and keep one k-block (48 KB) per stage.  Six k-blocks in
+// flight is the depth that measured best in the power-capped step: four cost about a
+// quarter of the per-clock rate, six one-k-block stages (a commit per four MMAs) 3-7%,
+// and a seventh k-block (a ring of seven 32 KB slots committed in pairs) raised the
+// per-clock rates 1-2% but lowered the clock more.
 //
 //   both CTAs, warp 0   TMA loads of the CTA's halves; completion is counted
 //                       on the LEADER's (rank 0) full barrier
