@@ -692,32 +692,51 @@ size_t opt_step_partial_bytes(int n_layers, int d, int d_ff) {
            2 * sizeof(float);
 }
 
-// The cosine of every layer from EpiGradCos's per-(tile, warp) triples: one warp per
-// layer adds its slots in a fixed order (lane-strided fp64 sums, then a fixed butterfly).
-__global__ void grad_cosine_final_kernel(const float* __restrict__ part, int slots,
-                                         double* __restrict__ out) {
+// Second pass of the fused cosine: one block per layer adds the layer's slot triples in a
+// fixed order (thread-strided fp64 sums, a fixed butterfly per warp, then the warps' sums
+// in warp order) and writes <G, Y>, ||G||^2, ||Y||^2 and the cosine.
+constexpr int kCosFinalThreads = 256;
+
+__device__ __forceinline__ double warp_sum_f64(double x) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+    return x;
+}
+
+__global__ void __launch_bounds__(kCosFinalThreads)
+    grad_cosine_final_kernel(const float* __restrict__ part, int slots, double* __restrict__ out) {
     const int layer = blockIdx.x;
-    const int lane = threadIdx.x;
     const float* p = part + static_cast<size_t>(layer) * slots * 3;
     double gy = 0.0, gg = 0.0, yy = 0.0;
-    for (int i = lane; i < slots; i += 32) {
+#pragma unroll 4
+    for (int i = threadIdx.x; i < slots; i += kCosFinalThreads) {
         gy += p[3 * i];
         gg += p[3 * i + 1];
         yy += p[3 * i + 2];
     }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-        gy += __shfl_xor_sync(0xffffffffu, gy, o);
-        gg += __shfl_xor_sync(0xffffffffu, gg, o);
-        yy += __shfl_xor_sync(0xffffffffu, yy, o);
-    }
+    gy = warp_sum_f64(gy);
+    gg = warp_sum_f64(gg);
+    yy = warp_sum_f64(yy);
+    __shared__ double sh[3][kCosFinalThreads / 32];
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
     if (lane == 0) {
-        double* o = out + 4 * layer;
-        o[0] = gy;
-        o[1] = gg;
-        o[2] = yy;
-        o[3] = (gg > 0.0 && yy > 0.0) ? gy / (sqrt(gg) * sqrt(yy)) : 0.0;
+        sh[0][wid] = gy;
+        sh[1][wid] = gg;
+        sh[2][wid] = yy;
     }
+    __syncthreads();
+    if (threadIdx.x != 0) return;
+    gy = gg = yy = 0.0;
+    for (int k = 0; k < kCosFinalThreads / 32; ++k) {
+        gy += sh[0][k];
+        gg += sh[1][k];
+        yy += sh[2][k];
+    }
+    double* o = out + 4 * layer;
+    o[0] = gy;
+    o[1] = gg;
+    o[2] = yy;
+    o[3] = (gg > 0.0 && yy > 0.0) ? gy / (sqrt(gg) * sqrt(yy)) : 0.0;
 }
 
 size_t grad_cosine_partial_bytes(int n, int d, int d_ff) {
@@ -768,7 +787,7 @@ cudaError_t launch_grad_cosine_bf16(int n, int T, int d, int d_ff, const void* c
         e = run_gemm<kUpdBN, true, true, kUpdStages, kMaxGroups, EpiGradCos>(
             maps, ep, make_shape(d, d_ff, T, kUpdBN, n, band_for(false)), status, st);
     if (e != cudaSuccess) return e;
-    grad_cosine_final_kernel<<<n, 32, 0, st>>>(part, ep.m256 * ep.n_blocks * 8, out),
+    grad_cosine_final_kernel<<<n, kCosFinalThreads, 0, st>>>(part, ep.m256 * ep.n_blocks * 8, out),
         ::fpo::note_launch();
     return cudaGetLastError();
 }

@@ -131,22 +131,40 @@ __global__ void __launch_bounds__(kOptThreads)
     }
 }
 
-// Step clip after the fused epilogue (EpiOptStep): one warp per layer adds the layer's
-// (||W||^2, ||d||^2) slot pairs in a fixed order (lane-strided fp64 sums, then a fixed
-// butterfly) and writes the layer's scale min(1, clip_frac ||W|| / ||d||).
-__global__ void opt_step_scale_kernel(const float* __restrict__ part, int slots,
-                                      const OptimParams op, float* __restrict__ scales) {
+// Step clip after the fused epilogue (EpiOptStep): one block per layer adds the layer's
+// (||W||^2, ||d||^2) slot pairs in a fixed order (thread-strided fp64 sums, a fixed
+// butterfly per warp, then the warps' sums in warp order; 256 threads keep many loads
+// in flight, where one warp waited on one load at a time) and writes the layer's scale
+// min(1, clip_frac ||W|| / ||d||).
+constexpr int kScaleThreads = 256;
+
+__global__ void __launch_bounds__(kScaleThreads)
+    opt_step_scale_kernel(const float* __restrict__ part, int slots, const OptimParams op,
+                          float* __restrict__ scales) {
     const int layer = blockIdx.x;
-    const int lane = threadIdx.x;
-    const float* p = part + static_cast<size_t>(layer) * slots * 2;
+    const float2* p = reinterpret_cast<const float2*>(part) + static_cast<size_t>(layer) * slots;
     double ww = 0.0, dd = 0.0;
-    for (int i = lane; i < slots; i += 32) {
-        ww += p[2 * i];
-        dd += p[2 * i + 1];
+#pragma unroll 4
+    for (int i = threadIdx.x; i < slots; i += kScaleThreads) {
+        const float2 v = p[i];
+        ww += v.x;
+        dd += v.y;
     }
     ww = warp_sum_d(ww);
     dd = warp_sum_d(dd);
-    if (lane != 0) return;
+    __shared__ double sh[2][kScaleThreads / 32];
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    if (lane == 0) {
+        sh[0][wid] = ww;
+        sh[1][wid] = dd;
+    }
+    __syncthreads();
+    if (threadIdx.x != 0) return;
+    ww = dd = 0.0;
+    for (int k = 0; k < kScaleThreads / 32; ++k) {
+        ww += sh[0][k];
+        dd += sh[1][k];
+    }
     const double lim = static_cast<double>(op.clip_frac) * sqrt(ww);
     scales[layer] = static_cast<float>(sqrt(dd) > lim ? lim / sqrt(dd) : 1.0);
 }
@@ -245,7 +263,8 @@ cudaError_t launch_opt_step_clip(int n_layers, size_t n_elem, const OptimParams&
         lp.Wo[l] = in && W_out ? W_out[l] : nullptr;
         lp.s1[l] = lp.s2[l] = nullptr;
     }
-    opt_step_scale_kernel<<<n_layers, 32, 0, st>>>(part, slots, op, scales), ::fpo::note_launch();
+    opt_step_scale_kernel<<<n_layers, kScaleThreads, 0, st>>>(part, slots, op, scales),
+        ::fpo::note_launch();
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     const dim3 grid(blocks_per_layer(n_layers), n_layers);
